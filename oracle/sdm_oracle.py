@@ -1,0 +1,201 @@
+"""Float64 CPU oracle of the Sparse Delta Memory (SDM) hot path.
+
+TEST INFRASTRUCTURE ONLY.  Only ``tests/``, ``__graft_entry__.smoke()`` and the
+``cpu_baseline`` / ``--impl reference`` legs of ``bench.py`` may import this
+module.  The CUDA library never calls it and shares no code with it.
+
+What it computes, step by step, in the paper's order and notation
+(arXiv 2607.07386):
+
+1. Sparse key selection (Sec. 3.1 item 1; Sec. 2 "Product Key Memory"):
+   pre-PKM scores s = P x in R^{2 sqrt(N)} (PROJECTED mode; DIRECT mode takes
+   s = x), split into halves s1, s2 in R^{sqrt(N)}; the N slot scores are the
+   outer sum s1 (+) s2 flattened row-major (slot = i*sqrt(N) + j); the top-k
+   of the outer sum is taken as top_k(top_k(s1) (+) top_k(s2)) (Sec. 2).
+   Selected scores are softmax-normalised (Sec. 4, "SDM Configuration") and the
+   index list is sorted by slot (App. A.2, sort-by-index).
+2. Learned initial state (Sec. 3.1, "Learned Initial State M0"): every
+   sequence's memory starts as a copy of the per-head M0.
+3. Gated delta write (Eqs. sdm-decay, sdm-write): for the write slots only,
+   decay by alpha_t, then add beta_t * w_i * (v_t - v~_t) with the single
+   prediction v~_t = sum_i w_i * M~_t[i]  (reading of Eq. sdm-write that makes
+   the GDN reduction of Sec. 3.1 "Connection to GDN" exact; Fig. 1 draws the
+   same data flow).  Unselected slots are unchanged (Sec. 3.1 item 2).
+4. Sparse read (Eq. sdm-read) of the post-write memory M_t.
+
+Precision: every input is the float64 value of its storage-dtype number.
+Scores are accumulated in float64 in ascending d order (products of two bf16
+or two fp32 numbers are exact in float64, so the only roundings are the
+additions).  Rows written to memory and the output y are rounded to the
+storage dtype (round-to-nearest-even, directly from float64); all other
+intermediates stay in float64.
+
+Tie-breaking (the paper is silent): per half by (score desc, index asc); over
+the outer sum by (score desc, slot asc).
+
+Parity pins: see ``tests/test_oracle_pins.py`` (GDN reduction, dense masked
+form, beta = 0 closed form, single-slot recall, brute-force top-k including
+forced ties, invariants, the paper's state-size tables).
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+__all__ = [
+    "to_f64", "round_storage", "half_scores", "topk_half", "pkm_select", "address",
+    "recur", "forward_slice", "state_elements_per_layer", "n_global_layers",
+]
+
+
+# --------------------------------------------------------------------------------------
+# storage dtype helpers
+# --------------------------------------------------------------------------------------
+
+def to_f64(a: np.ndarray, dtype: str) -> np.ndarray:
+    """Storage array -> float64 values.  "bf16" arrays hold the bfloat16 bit pattern
+    as uint16; "f32" arrays are float32; "f64" arrays are returned as float64."""
+    if dtype == "bf16":
+        bits = np.asarray(a, dtype=np.uint16).astype(np.uint32) << np.uint32(16)
+        return bits.view(np.float32).astype(np.float64)
+    return np.asarray(a, dtype=np.float64 if dtype == "f64" else np.float32).astype(np.float64)
+
+
+def round_storage(x: np.ndarray, dtype: str) -> np.ndarray:
+    """R(x): float64 -> nearest storage-dtype value (ties to even), returned as float64.
+
+    bf16 has 8 significant bits: the value is snapped to the multiple of
+    2^(e-8) nearest to x, where 2^(e-1) <= |x| < 2^e (quantum clamped at the
+    subnormal step 2^-133).  "f64" is the identity (exact storage, used by pins).
+    """
+    x = np.asarray(x, dtype=np.float64)
+    if dtype == "f64":
+        return x.copy()
+    if dtype == "f32":
+        return x.astype(np.float32).astype(np.float64)
+    if dtype != "bf16":
+        raise ValueError(dtype)
+    _, e = np.frexp(x)
+    step = np.ldexp(1.0, np.maximum(e - 8, -133))
+    return np.rint(x / step) * step
+
+
+def to_bf16_bits(x64: np.ndarray) -> np.ndarray:
+    """Bit pattern of the bf16 numbers R(x) (x already representable)."""
+    return (np.asarray(x64, np.float64).astype(np.float32).view(np.uint32) >> np.uint32(16)).astype(np.uint16)
+
+
+# --------------------------------------------------------------------------------------
+# addressing (Sec. 2 Product Key Memory; Sec. 3.1 item 1)
+# --------------------------------------------------------------------------------------
+
+def half_scores(P: np.ndarray | None, X: np.ndarray) -> np.ndarray:
+    """Pre-PKM scores s = P x for every token.
+
+    P: [2S, d_k] float64 (None for DIRECT mode, where s = x), X: [T, d_k] float64.
+    Returns [T, 2S] float64, each entry summed over d = 0, 1, ..., d_k-1 in that order.
+    """
+    if P is None:
+        return np.array(X, dtype=np.float64, copy=True)
+    s = np.zeros((X.shape[0], P.shape[0]), dtype=np.float64)
+    for d in range(P.shape[1]):
+        s += X[:, d:d + 1] * P[None, :, d]
+    return s
+
+
+def topk_half(s: np.ndarray, k: int) -> np.ndarray:
+    """Indices of the top-k of each row of s under (value desc, index asc), best first."""
+    order = np.argsort(-s, axis=-1, kind="stable")
+    return order[..., :k]
+
+
+def pkm_select(s1: np.ndarray, s2: np.ndarray, k: int):
+    """top_k(top_k(s1) (+) top_k(s2)) for every token (Sec. 2, PKM identity).
+
+    s1, s2: [T, S].  Returns (idx [T, k] int64 sorted ascending by slot,
+    score [T, k] float64 combined scores in the same order, w [T, k] softmax weights).
+    Candidate order: (score desc, slot asc); slot = i * S + j (row-major outer sum).
+    """
+    T, S = s1.shape
+    i1 = topk_half(s1, k)                                   # [T, k]
+    i2 = topk_half(s2, k)
+    v1 = np.take_along_axis(s1, i1, axis=1)
+    v2 = np.take_along_axis(s2, i2, axis=1)
+    cand = (v1[:, :, None] + v2[:, None, :]).reshape(T, k * k)
+    slot = (i1[:, :, None] * S + i2[:, None, :]).reshape(T, k * k)
+    pick = np.lexsort((slot, -cand), axis=-1)[:, :k]        # primary: score desc; then slot asc
+    sel_slot = np.take_along_axis(slot, pick, axis=1)
+    sel_score = np.take_along_axis(cand, pick, axis=1)
+    by_slot = np.argsort(sel_slot, axis=1, kind="stable")
+    idx = np.take_along_axis(sel_slot, by_slot, axis=1)
+    score = np.take_along_axis(sel_score, by_slot, axis=1)
+    z = np.exp(score - score.max(axis=1, keepdims=True))
+    w = z / z.sum(axis=1, keepdims=True)
+    return idx, score, w
+
+
+def address(P: np.ndarray | None, X: np.ndarray, N: int, k: int):
+    """Sparse key selection for every token of one head: (idx, score, w), each [T, k]."""
+    S = math.isqrt(N)
+    assert S * S == N
+    s = half_scores(P, X)
+    assert s.shape[1] == 2 * S, "scores must have 2 sqrt(N) entries"
+    return pkm_select(s[:, :S], s[:, S:], k)
+
+
+# --------------------------------------------------------------------------------------
+# recurrence (Eqs. sdm-decay, sdm-write, sdm-read)
+# --------------------------------------------------------------------------------------
+
+def recur(M: np.ndarray, idx_w, w_w, idx_r, w_r, v, alpha, beta, store: str):
+    """Run the sparse gated delta recurrence over T tokens of one (b, h) slice.
+
+    M: [N, d_v] float64 memory, updated in place (values stay representable in
+    the storage dtype).  idx_*: [T, k_*] int, w_*: [T, k_*] float64,
+    v: [T, d_v], alpha, beta: [T] (float64).  Within a token the write slots
+    must be distinct.  Returns (y [T, d_v] float64 before rounding, R(y)).
+    """
+    T = v.shape[0]
+    y = np.empty((T, M.shape[1]), dtype=np.float64)
+    for t in range(T):
+        iw = idx_w[t]
+        decayed = alpha[t] * M[iw]                  # M~_t[i] = alpha_t M_{t-1}[i], i in I^w_t   (Eq. sdm-decay)
+        pred = w_w[t] @ decayed                     # v~_t = sum_i k_t^(i) M~_t[i]
+        delta = v[t] - pred                         # v_t - v~_t
+        M[iw] = round_storage(decayed + beta[t] * w_w[t][:, None] * delta[None, :], store)  # Eq. sdm-write
+        y[t] = w_r[t] @ M[idx_r[t]]                 # y_t = sum_i q_t^(i) M_t[i]   (Eq. sdm-read, post-write)
+    return y, round_storage(y, store)
+
+
+def forward_slice(M0_h: np.ndarray, P_q, P_k, q, k, v, alpha, beta, N: int, k_write: int, k_read: int,
+                  store: str, M: np.ndarray | None = None):
+    """Whole hot path for one (b, h) slice, all inputs already float64.
+
+    M0_h: [N, d_v] initial memory of head h (copied: Sec. 3.1 "Learned Initial
+    State"), unless a running memory M is given (continuing a sequence).
+    Returns dict with y (rounded), y64, M (final memory), idx_w, w_w, idx_r, w_r.
+    """
+    idx_w, _, w_w = address(P_k, k, N, k_write)
+    idx_r, _, w_r = address(P_q, q, N, k_read)
+    if M is None:
+        M = np.array(M0_h, dtype=np.float64, copy=True)
+    y64, y = recur(M, idx_w, w_w, idx_r, w_r, v, alpha, beta, store)
+    return {"y": y, "y64": y64, "M": M, "idx_w": idx_w, "w_w": w_w, "idx_r": idx_r, "w_r": w_r}
+
+
+# --------------------------------------------------------------------------------------
+# geometry (Sec. 3.2 / 3.3, Sec. 4 "SDM Configuration")
+# --------------------------------------------------------------------------------------
+
+def n_global_layers(layers: int) -> int:
+    """Global (long-range) layers in the 3:1 local:global hybrid (Sec. 4, Architecture)."""
+    return layers // 4
+
+
+def state_elements_per_layer(d: int, H: int) -> int:
+    """SDM state of one layer: H heads x N slots x d_v, with N = (d / 4H)^2 and d_v = d / H
+    (Sec. 4 "SDM Configuration"; d_qk^total = d/2 and d_v^total = d from Sec. 3.2, Eq. of Sec. 3.3)."""
+    assert d % (4 * H) == 0
+    n = (d // (4 * H)) ** 2
+    return H * n * (d // H)

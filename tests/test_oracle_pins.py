@@ -1,0 +1,339 @@
+"""Pins of the float64 oracle against facts fixed by the paper and by mathematics.
+
+Each test checks the oracle against something other than itself: a textbook
+formula (Gated DeltaNet, Eq. gdn-update), an independent dense formulation of
+the sparse update, a closed form, brute force over all N slots, a library
+routine (bf16 rounding in torch, a BLAS matmul), or numbers printed in the
+paper (Table 1, Table 3, App. A.3).  The last tests plant plausible mistakes
+in copies of the oracle and check that a pin rejects each.
+"""
+import math
+import os
+
+import numpy as np
+import pytest
+
+from oracle import sdm_oracle as O
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _golden_rows(name):
+    rows = []
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            line = line.split("#", 1)[0].strip()
+            if line:
+                rows.append(line.split())
+    return rows
+
+
+# ------------------------------------------------------------------ storage rounding
+
+def test_bf16_rounding_matches_torch_on_fp32_values():
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(7)
+    x32 = np.concatenate([rng.standard_normal(20000) * 10.0 ** rng.integers(-6, 6, 20000),
+                          np.float32(1.0) + np.arange(-64, 64) * np.float32(2.0 ** -9)]).astype(np.float32)
+    ref = torch.from_numpy(x32).to(torch.bfloat16).to(torch.float64).numpy()
+    got = O.round_storage(x32.astype(np.float64), "bf16")
+    assert np.array_equal(got, ref)
+
+
+def test_bf16_rounding_is_direct_from_float64():
+    # Just above the midpoint between 1 and 1+2^-7: nearest bf16 is 1+2^-7.
+    # Rounding through fp32 first would land exactly on the midpoint and then tie to 1.0.
+    x = 1.0 + 2.0 ** -8 + 2.0 ** -30
+    assert O.round_storage(np.array([x]), "bf16")[0] == 1.0 + 2.0 ** -7
+    assert O.round_storage(np.array([1.0 + 2.0 ** -8]), "bf16")[0] == 1.0          # tie -> even
+    assert O.round_storage(np.array([1.0 + 3 * 2.0 ** -8]), "bf16")[0] == 1.0 + 2.0 ** -6
+    bits = O.to_bf16_bits(O.round_storage(np.array([-2.5, 1.0, 0.0]), "bf16"))
+    assert list(bits) == [0xC020, 0x3F80, 0x0000]
+
+
+# ------------------------------------------------------------------ addressing
+
+def test_half_scores_against_matmul_and_exact_integers():
+    rng = np.random.default_rng(1)
+    P = rng.standard_normal((32, 24))
+    X = rng.standard_normal((5, 24))
+    np.testing.assert_allclose(O.half_scores(P, X), X @ P.T, rtol=1e-13, atol=1e-13)
+    Pi = rng.integers(-9, 10, (32, 24)).astype(np.float64)
+    Xi = rng.integers(-9, 10, (5, 24)).astype(np.float64)
+    assert np.array_equal(O.half_scores(Pi, Xi), (Xi.astype(np.int64) @ Pi.astype(np.int64).T).astype(np.float64))
+    assert np.array_equal(O.half_scores(None, Xi), Xi)
+
+
+def _brute_topk(s1, s2, k):
+    """Exact top-k over all N = S*S flattened outer-sum scores, (score desc, slot asc)."""
+    S = s1.shape[0]
+    full = (s1[:, None] + s2[None, :]).reshape(-1)
+    slot = np.arange(S * S)
+    pick = np.lexsort((slot, -full))[:k]
+    return np.sort(slot[pick])
+
+
+@pytest.mark.parametrize("S,k,integer", [(8, 3, False), (16, 8, False), (16, 8, True), (32, 16, True),
+                                         (8, 8, True), (64, 8, False), (5, 5, True)])
+def test_pkm_two_stage_equals_brute_force(S, k, integer):
+    rng = np.random.default_rng(S * 100 + k)
+    T = 200
+    if integer:   # few distinct values: many exact ties in both halves and in the outer sum
+        s1 = rng.integers(-3, 4, (T, S)).astype(np.float64)
+        s2 = rng.integers(-3, 4, (T, S)).astype(np.float64)
+    else:
+        s1 = rng.standard_normal((T, S))
+        s2 = rng.standard_normal((T, S))
+    idx, score, w = O.pkm_select(s1, s2, k)
+    for t in range(T):
+        assert np.array_equal(idx[t], _brute_topk(s1[t], s2[t], k)), t
+        assert np.all(np.diff(idx[t]) > 0)
+        np.testing.assert_array_equal(score[t], s1[t][idx[t] // S] + s2[t][idx[t] % S])
+    np.testing.assert_allclose(w.sum(axis=1), 1.0, rtol=0, atol=1e-14)
+    ref_w = np.exp(score) / np.exp(score).sum(axis=1, keepdims=True)
+    np.testing.assert_allclose(w, ref_w, rtol=1e-12)
+
+
+def test_address_projected_end_to_end_brute_force():
+    rng = np.random.default_rng(3)
+    S, dk, k, T = 16, 12, 6, 50
+    P = rng.standard_normal((2 * S, dk))
+    X = rng.standard_normal((T, dk))
+    idx, _, _ = O.address(P, X, S * S, k)
+    s = X @ P.T
+    for t in range(T):
+        assert np.array_equal(idx[t], _brute_topk(s[t, :S], s[t, S:], k))
+
+
+def test_address_direct_mode_uses_x_halves():
+    rng = np.random.default_rng(4)
+    S, k = 8, 4
+    X = rng.standard_normal((10, 2 * S))
+    idx, _, _ = O.address(None, X, S * S, k)
+    for t in range(10):
+        assert np.array_equal(idx[t], _brute_topk(X[t, :S], X[t, S:], k))
+
+
+# ------------------------------------------------------------------ recurrence
+
+def _gdn_textbook(M, K, V, Q, alpha, beta):
+    """Gated DeltaNet (Eq. gdn-update): M_t = a M + b k (v - a M^T k)^T, read y = M_t^T q."""
+    M = M.copy()
+    ys = []
+    for t in range(K.shape[0]):
+        k, v, q = K[t], V[t], Q[t]
+        M = alpha[t] * M + beta[t] * np.outer(k, v - alpha[t] * (M.T @ k))
+        ys.append(M.T @ q)
+    return M, np.array(ys)
+
+
+def test_gdn_reduction_all_slots_dense_keys():
+    """Sec. 3.1 "Connection to GDN": N = d_qk, W = R = N, dense key values -> GDN exactly."""
+    rng = np.random.default_rng(11)
+    dqk, dv, T = 6, 5, 40
+    M0 = rng.standard_normal((dqk, dv))
+    K = rng.standard_normal((T, dqk)) / np.sqrt(dqk)
+    Q = rng.standard_normal((T, dqk))
+    V = rng.standard_normal((T, dv))
+    alpha = 1 / (1 + np.exp(-rng.standard_normal(T) - 2))
+    beta = 1 / (1 + np.exp(-rng.standard_normal(T)))
+    allslots = np.tile(np.arange(dqk), (T, 1))
+    M = M0.copy()
+    y64, _ = O.recur(M, allslots, K, allslots, Q, V, alpha, beta, "f64")
+    M_ref, y_ref = _gdn_textbook(M0, K, V, Q, alpha, beta)
+    np.testing.assert_allclose(M, M_ref, rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(y64, y_ref, rtol=1e-12, atol=1e-12)
+
+
+def _dense_masked_sdm(M0, idx_w, w_w, idx_r, w_r, V, alpha, beta):
+    """The same update written densely over all N slots: decay mask D_t = I + (a-1) diag(1[i in I^w]),
+    dense write vector kappa (zero off I^w), dense read vector rho (zero off I^r)."""
+    N = M0.shape[0]
+    M = M0.copy()
+    ys = []
+    for t in range(V.shape[0]):
+        mask = np.zeros(N)
+        mask[idx_w[t]] = 1.0
+        kappa = np.zeros(N)
+        kappa[idx_w[t]] = w_w[t]
+        rho = np.zeros(N)
+        rho[idx_r[t]] = w_r[t]
+        Mt = (1.0 + (alpha[t] - 1.0) * mask)[:, None] * M
+        Mt = Mt + beta[t] * np.outer(kappa, V[t] - Mt.T @ kappa)
+        M = Mt
+        ys.append(M.T @ rho)
+    return M, np.array(ys)
+
+
+def _random_sparse_case(rng, N=40, dv=4, T=60, kw=5, kr=4):
+    idx_w = np.array([np.sort(rng.choice(N, kw, replace=False)) for _ in range(T)])
+    idx_r = np.array([np.sort(rng.choice(N, kr, replace=False)) for _ in range(T)])
+    w_w = rng.dirichlet(np.ones(kw), T)
+    w_r = rng.dirichlet(np.ones(kr), T)
+    V = rng.standard_normal((T, dv))
+    alpha = 1 / (1 + np.exp(-rng.standard_normal(T) - 1))
+    beta = 1 / (1 + np.exp(-rng.standard_normal(T)))
+    M0 = rng.standard_normal((N, dv))
+    return M0, idx_w, w_w, idx_r, w_r, V, alpha, beta
+
+
+def test_sparse_recurrence_equals_dense_masked_form():
+    rng = np.random.default_rng(12)
+    M0, idx_w, w_w, idx_r, w_r, V, alpha, beta = _random_sparse_case(rng)
+    M = M0.copy()
+    y64, _ = O.recur(M, idx_w, w_w, idx_r, w_r, V, alpha, beta, "f64")
+    M_ref, y_ref = _dense_masked_sdm(M0, idx_w, w_w, idx_r, w_r, V, alpha, beta)
+    np.testing.assert_allclose(M, M_ref, rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(y64, y_ref, rtol=1e-12, atol=1e-12)
+
+
+def test_beta_zero_closed_form():
+    """beta = 0: a slot only decays, by the product of alpha over the tokens that write it."""
+    rng = np.random.default_rng(13)
+    M0, idx_w, w_w, idx_r, w_r, V, alpha, _ = _random_sparse_case(rng)
+    T, N = V.shape[0], M0.shape[0]
+    M = M0.copy()
+    y64, _ = O.recur(M, idx_w, w_w, idx_r, w_r, V, alpha, np.zeros(T), "f64")
+    decay = np.ones(N)
+    for t in range(T):
+        decay[idx_w[t]] *= alpha[t]
+        np.testing.assert_allclose(y64[t], w_r[t] @ (decay[idx_r[t], None] * M0[idx_r[t]]), rtol=1e-13, atol=1e-15)
+    np.testing.assert_allclose(M, decay[:, None] * M0, rtol=1e-13, atol=1e-15)
+
+
+@pytest.mark.parametrize("store", ["bf16", "f32", "f64"])
+def test_single_slot_recall_exact(store):
+    """alpha = beta = 1, one slot per token (softmax weight exactly 1): the slot becomes v_t and
+    reading it returns v_t, bit for bit in the storage dtype."""
+    rng = np.random.default_rng(14)
+    N, dv, T = 64, 16, 30
+    M0 = O.round_storage(rng.standard_normal((N, dv)), store)
+    V = O.round_storage(rng.standard_normal((T, dv)), store)
+    slots = rng.choice(N, T, replace=False)[:, None]
+    M = M0.copy()
+    _, y = O.recur(M, slots, np.ones((T, 1)), slots, np.ones((T, 1)), V, np.ones(T), np.ones(T), store)
+    if store == "f64":   # r + (v - r) is only exact when v and r carry few significant bits
+        np.testing.assert_allclose(y, V, rtol=1e-15, atol=1e-15)
+        np.testing.assert_allclose(M[slots[:, 0]], V, rtol=1e-15, atol=1e-15)
+    else:
+        assert np.array_equal(y, V)
+        assert np.array_equal(M[slots[:, 0]], V)
+    untouched = np.setdiff1d(np.arange(N), slots[:, 0])
+    assert np.array_equal(M[untouched], M0[untouched])
+
+
+def test_untouched_rows_bit_identical_and_split_invariance():
+    rng = np.random.default_rng(15)
+    M0, idx_w, w_w, idx_r, w_r, V, alpha, beta = _random_sparse_case(rng, N=500, T=80)
+    M0 = O.round_storage(M0 * 0.02, "bf16")
+    V = O.round_storage(V, "bf16")
+    Ma = M0.copy()
+    _, ya = O.recur(Ma, idx_w, w_w, idx_r, w_r, V, alpha, beta, "bf16")
+    Mb = M0.copy()
+    _, yb1 = O.recur(Mb, idx_w[:33], w_w[:33], idx_r[:33], w_r[:33], V[:33], alpha[:33], beta[:33], "bf16")
+    _, yb2 = O.recur(Mb, idx_w[33:], w_w[33:], idx_r[33:], w_r[33:], V[33:], alpha[33:], beta[33:], "bf16")
+    assert np.array_equal(Ma, Mb) and np.array_equal(ya, np.concatenate([yb1, yb2]))
+    untouched = np.setdiff1d(np.arange(500), idx_w.ravel())
+    assert untouched.size > 0 and np.array_equal(Ma[untouched], M0[untouched])
+    assert np.array_equal(O.round_storage(Ma, "bf16"), Ma)
+
+
+def test_forward_slice_is_address_then_recur():
+    rng = np.random.default_rng(16)
+    S, dk, dv, T, k = 8, 10, 6, 40, 4
+    N = S * S
+    Pq, Pk = rng.standard_normal((2 * S, dk)), rng.standard_normal((2 * S, dk))
+    q, kk, v = rng.standard_normal((T, dk)), rng.standard_normal((T, dk)), rng.standard_normal((T, dv))
+    a, b = np.full(T, 0.9), np.full(T, 0.5)
+    M0 = rng.standard_normal((N, dv))
+    out = O.forward_slice(M0, Pq, Pk, q, kk, v, a, b, N, k, k, "f64")
+    iw, _, ww = O.address(Pk, kk, N, k)
+    ir, _, wr = O.address(Pq, q, N, k)
+    M_ref, y_ref = _dense_masked_sdm(M0, iw, ww, ir, wr, v, a, b)
+    np.testing.assert_allclose(out["y64"], y_ref, rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(out["M"], M_ref, rtol=1e-12, atol=1e-12)
+    assert np.array_equal(M0, O.forward_slice(M0, Pq, Pk, q, kk, v, a, b, N, k, k, "f64")["M"]) is False
+
+
+# ------------------------------------------------------------------ geometry (printed numbers)
+
+def test_table1_sdm_state_sizes():
+    for level, d, layers, H, printed in _golden_rows("table1_sdm_state.txt"):
+        d, layers, H, printed = int(d), int(layers), int(H), float(printed)
+        total = O.n_global_layers(layers) * O.state_elements_per_layer(d, H)
+        digits = 4 if printed >= 1e9 else (3 if printed >= 1e8 else 2)
+        assert float(f"{total:.{digits}g}") == printed, (level, total, printed)
+
+
+def test_table3_state_per_layer_mb():
+    for d, H, dqk, printed in _golden_rows("table3_state_per_layer.txt"):
+        d, H, dqk, printed = int(d), int(H), int(dqk), int(printed)
+        n = (dqk // (2 * H)) ** 2                # per-head key = 2 sqrt(N), d_qk per head = dqk / H
+        mib = H * n * (d // H) * 2 / 2 ** 20
+        assert round(mib) == printed, (d, H, dqk, mib)
+    assert O.state_elements_per_layer(1920, 2) * 2 / 2 ** 20 == pytest.approx(211, abs=0.5)
+
+
+def test_appendix_a3_checkpoint_sizes():
+    printed = {name: float(v) for name, v in _golden_rows("appA3_checkpoints.txt")}
+    d, H, T, C, W = 3840, 2, 16384, 128, 64
+    per_layer = O.state_elements_per_layer(d, H)
+    assert round((T // C) * per_layer * 2 / 1e9) == printed["chunk_snapshots"]
+    assert round(T * W * d * 2 / 1e9) == printed["undo_log"]
+
+
+# ------------------------------------------------------------------ planted mistakes
+
+def _recur_per_slot_delta(M, idx_w, w_w, idx_r, w_r, v, alpha, beta):
+    # Literal per-slot reading of Eq. sdm-write: v_t - M~_t[i] instead of v_t - v~_t.
+    ys = []
+    for t in range(v.shape[0]):
+        d = alpha[t] * M[idx_w[t]]
+        M[idx_w[t]] = d + beta[t] * w_w[t][:, None] * (v[t][None, :] - d)
+        ys.append(w_r[t] @ M[idx_r[t]])
+    return np.array(ys)
+
+
+def _recur_read_before_write(M, idx_w, w_w, idx_r, w_r, v, alpha, beta):
+    ys = []
+    for t in range(v.shape[0]):
+        ys.append(w_r[t] @ M[idx_r[t]])
+        d = alpha[t] * M[idx_w[t]]
+        M[idx_w[t]] = d + beta[t] * w_w[t][:, None] * (v[t] - w_w[t] @ d)[None, :]
+    return np.array(ys)
+
+
+def _recur_global_decay(M, idx_w, w_w, idx_r, w_r, v, alpha, beta):
+    ys = []
+    for t in range(v.shape[0]):
+        M *= alpha[t]
+        d = M[idx_w[t]]
+        M[idx_w[t]] = d + beta[t] * w_w[t][:, None] * (v[t] - w_w[t] @ d)[None, :]
+        ys.append(w_r[t] @ M[idx_r[t]])
+    return np.array(ys)
+
+
+def test_pins_reject_planted_mistakes():
+    rng = np.random.default_rng(17)
+    dqk, dv, T = 6, 5, 30
+    M0 = rng.standard_normal((dqk, dv))
+    K = rng.standard_normal((T, dqk)) / np.sqrt(dqk)
+    Q = rng.standard_normal((T, dqk))
+    V = rng.standard_normal((T, dv))
+    a = np.full(T, 0.9)
+    b = np.full(T, 0.7)
+    alls = np.tile(np.arange(dqk), (T, 1))
+    _, y_gdn = _gdn_textbook(M0, K, V, Q, a, b)
+    assert not np.allclose(_recur_per_slot_delta(M0.copy(), alls, K, alls, Q, V, a, b), y_gdn, atol=1e-6)
+    assert not np.allclose(_recur_read_before_write(M0.copy(), alls, K, alls, Q, V, a, b), y_gdn, atol=1e-6)
+    M0s, iw, ww, ir, wr, Vs, al, _ = _random_sparse_case(rng)
+    M = M0s.copy()
+    _recur_global_decay(M, iw, ww, ir, wr, Vs, al, np.zeros(Vs.shape[0]))
+    decay = np.ones(M0s.shape[0])
+    for t in range(Vs.shape[0]):
+        decay[iw[t]] *= al[t]
+    assert not np.allclose(M, decay[:, None] * M0s)
+    # a transposed outer-sum flattening (slot = j*S + i) fails the brute-force pin
+    s1, s2 = rng.standard_normal(8), rng.standard_normal(8)
+    idx, _, _ = O.pkm_select(s2[None], s1[None], 4)
+    assert not np.array_equal(idx[0], _brute_topk(s1, s2, 4))
