@@ -1,0 +1,148 @@
+/*
+ * sdm.h -- C ABI of the Sparse Delta Memory (SDM) hot path on one GB300 (sm_103a).
+ *
+ * Sparse Delta Memory (arXiv 2607.07386) replaces Gated DeltaNet's dense
+ * d_qk x d_v state with an explicit per-head memory M in R^{N x d_v}.  For every
+ * token t and head h:
+ *   1. sparse key selection (Sec. 3.1 item 1, Sec. 2 "Product Key Memory"):
+ *      s = P x in R^{2 sqrt(N)} is split into halves s1, s2; the N slot scores are
+ *      the outer sum s1 (+) s2 (slot = i*sqrt(N) + j); the top-k slots are found as
+ *      top_k(top_k(s1) (+) top_k(s2)) and their scores are softmax-normalised
+ *      (Sec. 4, "SDM Configuration");
+ *   2. gated delta write (Eqs. sdm-decay, sdm-write) on the k_write selected slots:
+ *      M~[i] = alpha_t M[i];  M[i] = M~[i] + beta_t w_i (v_t - v~_t),
+ *      v~_t = sum_i w_i M~[i];  unselected slots are unchanged;
+ *   3. sparse read (Eq. sdm-read) of the post-write memory: y_t = sum_i r_i M_t[i].
+ *   The memory of every sequence starts as a copy of the learned initial state M0
+ *   (Sec. 3.1, "Learned Initial State").
+ *
+ * Conventions (all entry points):
+ *   - Every buffer is caller-owned device memory (except where a host pointer is
+ *     stated), contiguous row-major, 16-byte aligned.  The library never
+ *     allocates device memory: scratch space is the caller's `workspace`.
+ *   - One dtype (shape->dtype) for every floating-point tensor: memory, M0, P_q,
+ *     P_k, q, k, v, alpha, beta and y.  Slot indices are int32, slot weights fp32.
+ *     Arithmetic is fp32 (scores, prediction, delta, read), with storage rounding
+ *     (round-to-nearest-even) of every written memory row and of y.
+ *   - Asynchronous on `stream` (a cudaStream_t; NULL = legacy default stream);
+ *     no hidden synchronisation.  Calls that overlap on the GPU must not share
+ *     `mem` or `workspace`.
+ *   - Errors: shape / pointer / workspace errors return SDM_ERR_INVALID_ARG (or
+ *     SDM_ERR_UNSUPPORTED) before anything is launched; launch failures return
+ *     SDM_ERR_CUDA.  sdm_last_error() gives a message (thread-local).  Kernels
+ *     never trap: a slot index outside [0, N) is skipped and recorded in a device
+ *     status word read by sdm_device_status().
+ *   - Index lists are ascending by slot within each token and the weights of a
+ *     token sum to 1.
+ */
+#ifndef SDM_H
+#define SDM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define SDM_ABI_VERSION 1
+
+/* Same type as cudaStream_t. */
+typedef struct CUstream_st* sdm_stream_t;
+
+typedef enum {
+    SDM_OK = 0,
+    SDM_ERR_INVALID_ARG = 1,   /* bad shape, null pointer, misalignment, aliasing, small workspace */
+    SDM_ERR_UNSUPPORTED = 2,   /* valid SDM shape this build has no kernel for (see sdm_last_error) */
+    SDM_ERR_OOM = 3,           /* reserved: the library itself never allocates */
+    SDM_ERR_CUDA = 4,          /* a CUDA runtime call or launch failed (message has cudaGetErrorString) */
+    SDM_ERR_TIMEOUT = 5,       /* reserved for bounded device waits */
+    SDM_ERR_DEVICE = 6         /* device status word reported a bad slot index (sdm_device_status) */
+} sdm_status;
+
+typedef enum { SDM_F32 = 0, SDM_BF16 = 1 } sdm_dtype;
+
+/* PROJECTED: s = P x with P [H, 2 sqrt(N), d_k] (the paper's W_k / W_q factored through d_k).
+ * DIRECT:    s = x itself; requires d_k == 2 sqrt(N) (the paper's k' in R^{2 sqrt(N)}); P unused. */
+typedef enum { SDM_ADDR_PROJECTED = 0, SDM_ADDR_DIRECT = 1 } sdm_addr_mode;
+
+typedef struct {
+    int32_t B;        /* independent sequences */
+    int32_t H;        /* SDM heads */
+    int32_t T;        /* tokens per sequence in this call (1 for sdm_decode_step) */
+    int32_t d_k;      /* key / query width */
+    int32_t d_v;      /* value width = memory row width; d_v * elem_bytes must be a multiple of 16 */
+    int64_t N;        /* memory slots per head; a perfect square S*S */
+    int32_t k_write;  /* W: slots written per token, 1 <= W <= min(S, 64) for addressing */
+    int32_t k_read;   /* R: slots read per token, 1 <= R <= min(S, 64) for addressing */
+    int32_t dtype;    /* sdm_dtype */
+    int32_t addr;     /* sdm_addr_mode */
+} sdm_shape;
+
+/* Returns SDM_ABI_VERSION of the loaded library. */
+int sdm_abi_version(void);
+
+/* Message of the last failing call on this host thread ("" if none). */
+const char* sdm_last_error(void);
+
+/* Bytes of workspace that sdm_forward / sdm_decode_step / sdm_address need for `shape`
+ * (covers slot lists the caller does not request, PKM partial lists and row norms).
+ * Returns 0 and sets sdm_last_error for an invalid shape. */
+size_t sdm_workspace_bytes(const sdm_shape* shape);
+
+/* Sec. 3.1 "Learned Initial State": mem[b, h] = M0[h] for every sequence b.
+ * M0: [H, N, d_v] (read only);  mem: [B, H, N, d_v] (written).  Must not overlap. */
+sdm_status sdm_init_memory(const sdm_shape* shape, const void* M0, void* mem, sdm_stream_t stream);
+
+/* Sparse key selection only (Sec. 3.1 item 1; Sec. 2 PKM; Sec. 4 softmax), for every
+ * (b, h, t): write slots from k with P_k, read slots from q with P_q.
+ * P_q, P_k: [H, 2 sqrt(N), d_k] (NULL allowed in DIRECT mode);  q, k: [B, H, T, d_k].
+ * idx_w/w_w: [B, H, T, k_write], idx_r/w_r: [B, H, T, k_read]; all four required here.
+ * Selected slot sets equal the exact top-k of the float64 outer-sum scores under
+ * (score desc, slot asc) order: fp32 scores are certified against an error bound and
+ * near-ties are re-decided in float64. */
+sdm_status sdm_address(const sdm_shape* shape, const void* P_q, const void* P_k,
+                       const void* q, const void* k,
+                       int32_t* idx_w, float* w_w, int32_t* idx_r, float* w_r,
+                       void* workspace, size_t workspace_bytes, sdm_stream_t stream);
+
+/* Whole hot path over T tokens: addressing (as sdm_address), then the fused
+ * recurrence (Eqs. sdm-decay, sdm-write, sdm-read) in token order, per (b, h).
+ * mem: [B, H, N, d_v] running memory, updated in place to M_T (must not alias inputs);
+ * v: [B, H, T, d_v];  alpha, beta: [B, H, T] (gates in (0,1) and [0,1]);
+ * y: [B, H, T, d_v] (written).  idx_w, w_w, idx_r, w_r may be NULL (kept in the
+ * workspace) or caller buffers that receive the selection. */
+sdm_status sdm_forward(const sdm_shape* shape, const void* P_q, const void* P_k,
+                       const void* q, const void* k, const void* v,
+                       const void* alpha, const void* beta, void* mem, void* y,
+                       int32_t* idx_w, float* w_w, int32_t* idx_r, float* w_r,
+                       void* workspace, size_t workspace_bytes, sdm_stream_t stream);
+
+/* One decode step for B independent sequences: sdm_forward with shape->T == 1 and
+ * the per-token tensors shaped [B, H, d] / [B, H]. */
+sdm_status sdm_decode_step(const sdm_shape* shape, const void* P_q, const void* P_k,
+                           const void* q, const void* k, const void* v,
+                           const void* alpha, const void* beta, void* mem, void* y,
+                           int32_t* idx_w, float* w_w, int32_t* idx_r, float* w_r,
+                           void* workspace, size_t workspace_bytes, sdm_stream_t stream);
+
+/* Recurrence with explicit addressing (Eqs. sdm-decay, sdm-write, sdm-read), no PKM:
+ * idx_w [B,H,T,k_write] / w_w fp32, idx_r [B,H,T,k_read] / w_r fp32 (any weights,
+ * e.g. dense key values for the GDN special case of Sec. 3.1; write slots distinct
+ * within a token; k_write, k_read <= 64; slots may be in any order).
+ * v, alpha, beta, mem, y as in sdm_forward.  shape->d_k and shape->addr are ignored. */
+sdm_status sdm_recur(const sdm_shape* shape, const int32_t* idx_w, const float* w_w,
+                     const int32_t* idx_r, const float* w_r, const void* v,
+                     const void* alpha, const void* beta, void* mem, void* y,
+                     sdm_stream_t stream);
+
+/* Reads (host pointer `code`, synchronising on `stream`) and clears the device
+ * status word of the current device: 0 = no fault; bit 0 = a slot index outside
+ * [0, N) was skipped.  Returns SDM_ERR_DEVICE when the word was non-zero. */
+sdm_status sdm_device_status(int32_t* code, sdm_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SDM_H */

@@ -135,13 +135,20 @@ def pkm_select(s1: np.ndarray, s2: np.ndarray, k: int):
     return idx, score, w
 
 
-def address(P: np.ndarray | None, X: np.ndarray, N: int, k: int):
-    """Sparse key selection for every token of one head: (idx, score, w), each [T, k]."""
+def address(P: np.ndarray | None, X: np.ndarray, N: int, k: int, block: int = 2048):
+    """Sparse key selection for every token of one head: (idx, score, w), each [T, k].
+    Tokens are independent; they are processed in blocks only to bound memory."""
     S = math.isqrt(N)
     assert S * S == N
-    s = half_scores(P, X)
-    assert s.shape[1] == 2 * S, "scores must have 2 sqrt(N) entries"
-    return pkm_select(s[:, :S], s[:, S:], k)
+    parts = []
+    for t0 in range(0, X.shape[0], block):
+        s = half_scores(P, X[t0:t0 + block])
+        assert s.shape[1] == 2 * S, "scores must have 2 sqrt(N) entries"
+        parts.append(pkm_select(s[:, :S], s[:, S:], k))
+    if not parts:
+        z = np.zeros((0, k))
+        return z.astype(np.int64), z, z
+    return tuple(np.concatenate([p[i] for p in parts]) for i in range(3))
 
 
 # --------------------------------------------------------------------------------------

@@ -1,0 +1,11 @@
+"""GB300-native Sparse Delta Memory (arXiv 2607.07386) hot path.
+
+A thin ctypes binding of ``libsdm.so`` (C ABI in ``include/sdm.h``): argument
+marshalling only; every step runs in the library's sm_103a kernels.  The
+library is built in-tree by ``paper_2607_07386_gb300.build.build()``; using any
+entry point without it raises ``RuntimeError`` (there is no fallback).
+"""
+from ._binding import (  # noqa: F401
+    ADDR_DIRECT, ADDR_PROJECTED, DTYPE_BF16, DTYPE_F32, SdmError, SdmShape, abi_version, address,
+    decode_step, device_status, forward, init_memory, last_error, lib, lib_path, recur, workspace_bytes,
+)

@@ -1,0 +1,162 @@
+"""ctypes binding of libsdm.so.  Functions take torch CUDA tensors (or raw integer
+device pointers) and pass their addresses, sizes and the current CUDA stream."""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+_LIB_PATH = os.path.join(HERE, "lib", "libsdm.so")
+
+DTYPE_F32, DTYPE_BF16 = 0, 1
+ADDR_PROJECTED, ADDR_DIRECT = 0, 1
+_STATUS = {0: "SDM_OK", 1: "SDM_ERR_INVALID_ARG", 2: "SDM_ERR_UNSUPPORTED", 3: "SDM_ERR_OOM",
+           4: "SDM_ERR_CUDA", 5: "SDM_ERR_TIMEOUT", 6: "SDM_ERR_DEVICE"}
+
+
+class SdmError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{_STATUS.get(status, status)}: {message}")
+        self.status = status
+
+
+class SdmShape(ctypes.Structure):
+    _fields_ = [("B", ctypes.c_int32), ("H", ctypes.c_int32), ("T", ctypes.c_int32),
+                ("d_k", ctypes.c_int32), ("d_v", ctypes.c_int32), ("N", ctypes.c_int64),
+                ("k_write", ctypes.c_int32), ("k_read", ctypes.c_int32),
+                ("dtype", ctypes.c_int32), ("addr", ctypes.c_int32)]
+
+    @classmethod
+    def make(cls, B, H, T, d_k, d_v, N, k_write, k_read, dtype="bf16", addr="projected") -> "SdmShape":
+        dt = {"f32": DTYPE_F32, "bf16": DTYPE_BF16}[dtype] if isinstance(dtype, str) else int(dtype)
+        ad = {"projected": ADDR_PROJECTED, "direct": ADDR_DIRECT}[addr] if isinstance(addr, str) else int(addr)
+        return cls(B, H, T, d_k, d_v, N, k_write, k_read, dt, ad)
+
+    def replace(self, **kw) -> "SdmShape":
+        vals = {f: getattr(self, f) for f, _ in self._fields_}
+        vals.update(kw)
+        return SdmShape(**vals)
+
+
+_lib = None
+_lock = threading.Lock()
+_VP, _SZ, _I32P = ctypes.c_void_p, ctypes.c_size_t, ctypes.c_void_p
+_SHP = ctypes.POINTER(SdmShape)
+
+
+def lib_path() -> str:
+    return _LIB_PATH
+
+
+def lib():
+    """Load libsdm.so (built in-tree); raises if it has not been built."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(_LIB_PATH):
+                raise RuntimeError(f"libsdm.so not found at {_LIB_PATH}: build it with "
+                                   "paper_2607_07386_gb300.build.build() (no fallback exists)")
+            L = ctypes.CDLL(_LIB_PATH)
+            L.sdm_abi_version.restype = ctypes.c_int
+            L.sdm_last_error.restype = ctypes.c_char_p
+            L.sdm_workspace_bytes.restype = ctypes.c_size_t
+            L.sdm_workspace_bytes.argtypes = [_SHP]
+            L.sdm_init_memory.argtypes = [_SHP, _VP, _VP, _VP]
+            fwd = [_SHP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _I32P, _VP, _I32P, _VP, _VP, _SZ, _VP]
+            L.sdm_forward.argtypes = fwd
+            L.sdm_decode_step.argtypes = fwd
+            L.sdm_address.argtypes = [_SHP, _VP, _VP, _VP, _VP, _I32P, _VP, _I32P, _VP, _VP, _SZ, _VP]
+            L.sdm_recur.argtypes = [_SHP, _I32P, _VP, _I32P, _VP, _VP, _VP, _VP, _VP, _VP, _VP]
+            L.sdm_device_status.argtypes = [ctypes.POINTER(ctypes.c_int32), _VP]
+            for f in ("sdm_init_memory", "sdm_forward", "sdm_decode_step", "sdm_address", "sdm_recur",
+                      "sdm_device_status"):
+                getattr(L, f).restype = ctypes.c_int
+            _lib = L
+    return _lib
+
+
+def abi_version() -> int:
+    return lib().sdm_abi_version()
+
+
+def last_error() -> str:
+    return lib().sdm_last_error().decode()
+
+
+def _check(status: int):
+    if status != 0:
+        raise SdmError(status, last_error())
+
+
+def _ptr(x):
+    """Address of a tensor (must be contiguous), an int, or None."""
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    if not x.is_contiguous():
+        raise ValueError("tensors passed to libsdm must be contiguous")
+    if x.device.type != "cuda":
+        raise ValueError("tensors passed to libsdm must live on a CUDA device")
+    return x.data_ptr()
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _nbytes(x):
+    return x.numel() * x.element_size() if x is not None and not isinstance(x, int) else None
+
+
+def workspace_bytes(shape: SdmShape) -> int:
+    n = lib().sdm_workspace_bytes(ctypes.byref(shape))
+    if n == 0:
+        raise SdmError(1, last_error())
+    return n
+
+
+def init_memory(shape: SdmShape, M0, mem, stream=None):
+    _check(lib().sdm_init_memory(ctypes.byref(shape), _ptr(M0), _ptr(mem), _stream(stream)))
+
+
+def address(shape: SdmShape, P_q, P_k, q, k, idx_w, w_w, idx_r, w_r, workspace, stream=None, workspace_nbytes=None):
+    nb = workspace_nbytes if workspace_nbytes is not None else (_nbytes(workspace) or 0)
+    _check(lib().sdm_address(ctypes.byref(shape), _ptr(P_q), _ptr(P_k), _ptr(q), _ptr(k), _ptr(idx_w), _ptr(w_w),
+                             _ptr(idx_r), _ptr(w_r), _ptr(workspace), nb, _stream(stream)))
+
+
+def forward(shape: SdmShape, P_q, P_k, q, k, v, alpha, beta, mem, y, workspace, idx_w=None, w_w=None,
+            idx_r=None, w_r=None, stream=None, workspace_nbytes=None):
+    nb = workspace_nbytes if workspace_nbytes is not None else (_nbytes(workspace) or 0)
+    _check(lib().sdm_forward(ctypes.byref(shape), _ptr(P_q), _ptr(P_k), _ptr(q), _ptr(k), _ptr(v), _ptr(alpha),
+                             _ptr(beta), _ptr(mem), _ptr(y), _ptr(idx_w), _ptr(w_w), _ptr(idx_r), _ptr(w_r),
+                             _ptr(workspace), nb, _stream(stream)))
+
+
+def decode_step(shape: SdmShape, P_q, P_k, q, k, v, alpha, beta, mem, y, workspace, idx_w=None, w_w=None,
+                idx_r=None, w_r=None, stream=None, workspace_nbytes=None):
+    nb = workspace_nbytes if workspace_nbytes is not None else (_nbytes(workspace) or 0)
+    _check(lib().sdm_decode_step(ctypes.byref(shape), _ptr(P_q), _ptr(P_k), _ptr(q), _ptr(k), _ptr(v),
+                                 _ptr(alpha), _ptr(beta), _ptr(mem), _ptr(y), _ptr(idx_w), _ptr(w_w), _ptr(idx_r),
+                                 _ptr(w_r), _ptr(workspace), nb, _stream(stream)))
+
+
+def recur(shape: SdmShape, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem, y, stream=None):
+    _check(lib().sdm_recur(ctypes.byref(shape), _ptr(idx_w), _ptr(w_w), _ptr(idx_r), _ptr(w_r), _ptr(v),
+                           _ptr(alpha), _ptr(beta), _ptr(mem), _ptr(y), _stream(stream)))
+
+
+def device_status(stream=None) -> int:
+    """Read and clear the device status word (0 = clean).  Raises SdmError if it was set."""
+    code = ctypes.c_int32(0)
+    st = lib().sdm_device_status(ctypes.byref(code), _stream(stream))
+    if st not in (0, 6):
+        _check(st)
+    return int(code.value)

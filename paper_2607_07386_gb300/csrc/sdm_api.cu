@@ -1,0 +1,351 @@
+// C ABI of the SDM hot path: argument validation, workspace layout, kernel launches.
+// Declarations and semantics: include/sdm.h.
+#include "sdm_internal.h"
+#include "sdm.h"
+
+#include <stdarg.h>
+#include <stdio.h>
+#include <stddef.h>
+#include <string.h>
+
+#include <atomic>
+#include <string>
+
+static_assert(sizeof(sdm_shape) == 48, "sdm_shape layout is part of the ABI");
+static_assert(offsetof(sdm_shape, N) == 24, "sdm_shape layout is part of the ABI");
+
+namespace {
+
+thread_local std::string g_last_error;
+
+sdm_status fail(sdm_status st, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    g_last_error = buf;
+    return st;
+}
+
+sdm_status ok() {
+    g_last_error.clear();
+    return SDM_OK;
+}
+
+sdm_status cuda_fail(cudaError_t e, const char* where) {
+    return fail(SDM_ERR_CUDA, "%s: %s (%s)", where, cudaGetErrorString(e), cudaGetErrorName(e));
+}
+
+// Device status word, one per device; its address is looked up once per device.
+__device__ int g_status_word;
+constexpr int kMaxDevices = 64;
+std::atomic<int*> g_status_addr[kMaxDevices];
+
+sdm_status status_word(int** out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev < 0 || dev >= kMaxDevices) return fail(SDM_ERR_UNSUPPORTED, "device ordinal %d >= %d", dev, kMaxDevices);
+    int* p = g_status_addr[dev].load(std::memory_order_acquire);
+    if (p == nullptr) {
+        e = cudaGetSymbolAddress(reinterpret_cast<void**>(&p), g_status_word);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress(status word)");
+        g_status_addr[dev].store(p, std::memory_order_release);
+    }
+    *out = p;
+    return SDM_OK;
+}
+
+int64_t isqrt64(int64_t n) {
+    if (n < 0) return -1;
+    int64_t r = 0;
+    while ((r + 1) * (r + 1) <= n) {
+        int64_t step = 1;
+        while ((r + 2 * step) * (r + 2 * step) <= n) step *= 2;
+        r += step;
+    }
+    return r;
+}
+
+size_t elem_bytes(int dtype) { return dtype == SDM_F32 ? 4 : 2; }
+
+size_t align256(size_t x) { return (x + 255) & ~static_cast<size_t>(255); }
+
+bool aligned(const void* p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+struct Range {
+    const void* p;
+    size_t n;
+    const char* name;
+};
+
+bool overlaps(const Range& a, const Range& b) {
+    if (!a.p || !b.p || !a.n || !b.n) return false;
+    const uintptr_t a0 = reinterpret_cast<uintptr_t>(a.p), b0 = reinterpret_cast<uintptr_t>(b.p);
+    return a0 < b0 + b.n && b0 < a0 + a.n;
+}
+
+// Common shape checks.  need_pkm: the call runs PKM addressing (N square, k <= sqrt(N), d_k bounds).
+sdm_status check_shape(const sdm_shape* s, bool need_pkm, int64_t* S_out) {
+    if (!s) return fail(SDM_ERR_INVALID_ARG, "shape is NULL");
+    if (s->B < 0 || s->H < 0 || s->T < 0) return fail(SDM_ERR_INVALID_ARG, "B, H, T must be >= 0 (got %d, %d, %d)", s->B, s->H, s->T);
+    if (s->dtype != SDM_F32 && s->dtype != SDM_BF16) return fail(SDM_ERR_INVALID_ARG, "unknown dtype %d", s->dtype);
+    if (s->N < 1 || s->N > INT32_MAX) return fail(SDM_ERR_INVALID_ARG, "N must be in [1, 2^31-1] (got %lld)", (long long)s->N);
+    if (s->d_v < 1) return fail(SDM_ERR_INVALID_ARG, "d_v must be >= 1 (got %d)", s->d_v);
+    if ((static_cast<size_t>(s->d_v) * elem_bytes(s->dtype)) % 16 != 0)
+        return fail(SDM_ERR_UNSUPPORTED, "d_v * element size must be a multiple of 16 bytes (d_v=%d)", s->d_v);
+    if (s->k_write < 1 || s->k_read < 1 || s->k_write > 64 || s->k_read > 64)
+        return fail(SDM_ERR_UNSUPPORTED, "k_write and k_read must be in [1, 64] (got %d, %d)", s->k_write, s->k_read);
+    if (s->k_write > s->N || s->k_read > s->N) return fail(SDM_ERR_INVALID_ARG, "k exceeds N");
+    if (need_pkm) {
+        const int64_t S = isqrt64(s->N);
+        if (S * S != s->N) return fail(SDM_ERR_INVALID_ARG, "N=%lld is not a perfect square", (long long)s->N);
+        if (S > 46340) return fail(SDM_ERR_UNSUPPORTED, "sqrt(N) too large");
+        if (s->k_write > S || s->k_read > S)
+            return fail(SDM_ERR_INVALID_ARG, "k_write, k_read must be <= sqrt(N)=%lld", (long long)S);
+        if (s->addr != SDM_ADDR_PROJECTED && s->addr != SDM_ADDR_DIRECT) return fail(SDM_ERR_INVALID_ARG, "unknown addr mode %d", s->addr);
+        if (s->d_k < 1) return fail(SDM_ERR_INVALID_ARG, "d_k must be >= 1");
+        if (s->addr == SDM_ADDR_DIRECT && s->d_k != 2 * S)
+            return fail(SDM_ERR_INVALID_ARG, "DIRECT addressing needs d_k == 2*sqrt(N) (d_k=%d, sqrt(N)=%lld)", s->d_k, (long long)S);
+        if (s->d_k > 256) return fail(SDM_ERR_UNSUPPORTED, "d_k > 256 is not supported");
+        if (S_out) *S_out = S;
+    }
+    return SDM_OK;
+}
+
+struct Layout {
+    size_t idx_w, w_w, idx_r, w_r, pnorm, part_v, part_i, total;
+    sdm::AddrPlan plan;
+};
+
+Layout layout_for(const sdm_shape* s, int64_t S) {
+    Layout L{};
+    const size_t bht = static_cast<size_t>(s->B) * s->H * s->T;
+    const int kmax = s->k_write > s->k_read ? s->k_write : s->k_read;
+    L.plan = sdm::addr_plan(s->B, s->H, s->T, static_cast<int>(S), kmax);
+    size_t off = 0;
+    L.idx_w = off; off = align256(off + bht * s->k_write * 4);
+    L.w_w = off;   off = align256(off + bht * s->k_write * 4);
+    L.idx_r = off; off = align256(off + bht * s->k_read * 4);
+    L.w_r = off;   off = align256(off + bht * s->k_read * 4);
+    L.pnorm = off; off = align256(off + 2 * static_cast<size_t>(s->H) * 4);
+    const size_t part = sdm::addr_partial_bytes(L.plan, s->B, s->H, s->T) / 2;
+    L.part_v = off; off = align256(off + part);
+    L.part_i = off; off = align256(off + part);
+    L.total = off;
+    return L;
+}
+
+// Addressing into the given (or workspace) index/weight buffers.
+sdm_status run_address(const sdm_shape* s, int64_t S, const Layout& L, const void* P_q, const void* P_k, const void* q,
+                       const void* k, int32_t* idx_w, float* w_w, int32_t* idx_r, float* w_r, char* ws,
+                       int* err, cudaStream_t stream) {
+    sdm::AddrArgs a{};
+    const bool direct = s->addr == SDM_ADDR_DIRECT;
+    a.P[0] = direct ? nullptr : P_q;
+    a.P[1] = direct ? nullptr : P_k;
+    a.X[0] = q;
+    a.X[1] = k;
+    a.idx[0] = idx_r; a.w[0] = w_r; a.kk[0] = s->k_read;
+    a.idx[1] = idx_w; a.w[1] = w_w; a.kk[1] = s->k_write;
+    a.B = s->B; a.H = s->H; a.T = s->T; a.dk = s->d_k; a.S = static_cast<int>(S);
+    a.ncc = L.plan.ncc;
+    a.cw = L.plan.cw;
+    a.cbound = static_cast<float>((s->d_k + 4) * 0x1p-24);
+    a.part_v = reinterpret_cast<float*>(ws + L.part_v);
+    a.part_i = reinterpret_cast<int*>(ws + L.part_i);
+    a.pnorm = reinterpret_cast<float*>(ws + L.pnorm);
+    a.err = err;
+    cudaError_t e = sdm::launch_address(s->dtype, L.plan, a, stream);
+    if (e != cudaSuccess) return cuda_fail(e, "addressing launch");
+    return SDM_OK;
+}
+
+sdm_status check_vec(const void* p, const char* name, size_t align) {
+    if (!p) return fail(SDM_ERR_INVALID_ARG, "%s is NULL", name);
+    if (!aligned(p, align)) return fail(SDM_ERR_INVALID_ARG, "%s is not %zu-byte aligned", name, align);
+    return SDM_OK;
+}
+
+#define SDM_TRY(expr)                  \
+    do {                               \
+        sdm_status _st = (expr);       \
+        if (_st != SDM_OK) return _st; \
+    } while (0)
+
+sdm_status forward_impl(const char* who, const sdm_shape* s, const void* P_q, const void* P_k, const void* q,
+                        const void* k, const void* v, const void* alpha, const void* beta, void* mem, void* y,
+                        int32_t* idx_w, float* w_w, int32_t* idx_r, float* w_r, void* workspace,
+                        size_t workspace_bytes, cudaStream_t stream, bool run_recurrence) {
+    int64_t S = 0;
+    SDM_TRY(check_shape(s, true, &S));
+    const size_t es = elem_bytes(s->dtype);
+    const size_t bht = static_cast<size_t>(s->B) * s->H * s->T;
+    if (bht == 0) return ok();
+    if (s->addr == SDM_ADDR_PROJECTED) {
+        SDM_TRY(check_vec(P_q, "P_q", es));
+        SDM_TRY(check_vec(P_k, "P_k", es));
+    }
+    SDM_TRY(check_vec(q, "q", es));
+    SDM_TRY(check_vec(k, "k", es));
+    if (run_recurrence) {
+        SDM_TRY(check_vec(v, "v", 16));
+        SDM_TRY(check_vec(alpha, "alpha", es));
+        SDM_TRY(check_vec(beta, "beta", es));
+        SDM_TRY(check_vec(mem, "mem", 16));
+        SDM_TRY(check_vec(y, "y", 16));
+    } else {
+        SDM_TRY(check_vec(idx_w, "idx_w", 4));
+        SDM_TRY(check_vec(w_w, "w_w", 4));
+        SDM_TRY(check_vec(idx_r, "idx_r", 4));
+        SDM_TRY(check_vec(w_r, "w_r", 4));
+    }
+    const Layout L = layout_for(s, S);
+    if (!workspace) return fail(SDM_ERR_INVALID_ARG, "%s: workspace is NULL (need %zu bytes)", who, L.total);
+    if (!aligned(workspace, 256)) return fail(SDM_ERR_INVALID_ARG, "%s: workspace must be 256-byte aligned", who);
+    if (workspace_bytes < L.total)
+        return fail(SDM_ERR_INVALID_ARG, "%s: workspace too small (%zu < %zu bytes)", who, workspace_bytes, L.total);
+    const size_t rowb = static_cast<size_t>(s->d_v) * es;
+    if (run_recurrence) {
+        const Range rm{mem, static_cast<size_t>(s->B) * s->H * static_cast<size_t>(s->N) * rowb, "mem"};
+        const Range others[] = {
+            {P_q, s->addr == SDM_ADDR_PROJECTED ? static_cast<size_t>(s->H) * 2 * S * s->d_k * es : 0, "P_q"},
+            {P_k, s->addr == SDM_ADDR_PROJECTED ? static_cast<size_t>(s->H) * 2 * S * s->d_k * es : 0, "P_k"},
+            {q, bht * s->d_k * es, "q"}, {k, bht * s->d_k * es, "k"}, {v, bht * rowb, "v"},
+            {alpha, bht * es, "alpha"}, {beta, bht * es, "beta"}, {y, bht * rowb, "y"},
+            {idx_w, idx_w ? bht * s->k_write * 4 : 0, "idx_w"}, {w_w, w_w ? bht * s->k_write * 4 : 0, "w_w"},
+            {idx_r, idx_r ? bht * s->k_read * 4 : 0, "idx_r"}, {w_r, w_r ? bht * s->k_read * 4 : 0, "w_r"},
+            {workspace, L.total, "workspace"}};
+        for (const Range& r : others)
+            if (overlaps(rm, r)) return fail(SDM_ERR_INVALID_ARG, "%s: mem overlaps %s", who, r.name);
+        const Range ry{y, bht * rowb, "y"};
+        for (int i = 0; i < 7; ++i)
+            if (overlaps(ry, others[i])) return fail(SDM_ERR_INVALID_ARG, "%s: y overlaps %s", who, others[i].name);
+    }
+    char* ws = static_cast<char*>(workspace);
+    int32_t* iw = idx_w ? idx_w : reinterpret_cast<int32_t*>(ws + L.idx_w);
+    float* ww = w_w ? w_w : reinterpret_cast<float*>(ws + L.w_w);
+    int32_t* ir = idx_r ? idx_r : reinterpret_cast<int32_t*>(ws + L.idx_r);
+    float* wr = w_r ? w_r : reinterpret_cast<float*>(ws + L.w_r);
+    int* err = nullptr;
+    SDM_TRY(status_word(&err));
+    SDM_TRY(run_address(s, S, L, P_q, P_k, q, k, iw, ww, ir, wr, ws, err, stream));
+    if (run_recurrence) {
+        sdm::RecArgs r{};
+        r.idx_w = iw; r.w_w = ww; r.idx_r = ir; r.w_r = wr;
+        r.v = v; r.alpha = alpha; r.beta = beta; r.mem = mem; r.y = y;
+        r.B = s->B; r.H = s->H; r.T = s->T; r.dv = s->d_v; r.kw = s->k_write; r.kr = s->k_read;
+        r.N = s->N;
+        r.err = err;
+        cudaError_t e = sdm::launch_recur(s->dtype, r, stream);
+        if (e != cudaSuccess) return cuda_fail(e, "recurrence launch");
+    }
+    return ok();
+}
+
+}  // namespace
+
+extern "C" {
+
+int sdm_abi_version(void) { return SDM_ABI_VERSION; }
+
+const char* sdm_last_error(void) { return g_last_error.c_str(); }
+
+size_t sdm_workspace_bytes(const sdm_shape* shape) {
+    int64_t S = 0;
+    if (check_shape(shape, true, &S) != SDM_OK) return 0;
+    return layout_for(shape, S).total;
+}
+
+sdm_status sdm_init_memory(const sdm_shape* s, const void* M0, void* mem, sdm_stream_t stream) {
+    SDM_TRY(check_shape(s, false, nullptr));
+    const size_t per_seq = static_cast<size_t>(s->H) * static_cast<size_t>(s->N) * s->d_v * elem_bytes(s->dtype);
+    if (per_seq == 0 || s->B == 0) return ok();
+    SDM_TRY(check_vec(M0, "M0", 16));
+    SDM_TRY(check_vec(mem, "mem", 16));
+    if (overlaps(Range{M0, per_seq, "M0"}, Range{mem, per_seq * s->B, "mem"}))
+        return fail(SDM_ERR_INVALID_ARG, "sdm_init_memory: M0 overlaps mem");
+    cudaError_t e = sdm::launch_init_memory(M0, mem, static_cast<int64_t>(per_seq), s->B, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "init_memory launch");
+    return ok();
+}
+
+sdm_status sdm_address(const sdm_shape* s, const void* P_q, const void* P_k, const void* q, const void* k,
+                       int32_t* idx_w, float* w_w, int32_t* idx_r, float* w_r, void* workspace,
+                       size_t workspace_bytes, sdm_stream_t stream) {
+    return forward_impl("sdm_address", s, P_q, P_k, q, k, nullptr, nullptr, nullptr, nullptr, nullptr, idx_w, w_w,
+                        idx_r, w_r, workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream), false);
+}
+
+sdm_status sdm_forward(const sdm_shape* s, const void* P_q, const void* P_k, const void* q, const void* k,
+                       const void* v, const void* alpha, const void* beta, void* mem, void* y, int32_t* idx_w,
+                       float* w_w, int32_t* idx_r, float* w_r, void* workspace, size_t workspace_bytes,
+                       sdm_stream_t stream) {
+    return forward_impl("sdm_forward", s, P_q, P_k, q, k, v, alpha, beta, mem, y, idx_w, w_w, idx_r, w_r, workspace,
+                        workspace_bytes, reinterpret_cast<cudaStream_t>(stream), true);
+}
+
+sdm_status sdm_decode_step(const sdm_shape* s, const void* P_q, const void* P_k, const void* q, const void* k,
+                           const void* v, const void* alpha, const void* beta, void* mem, void* y, int32_t* idx_w,
+                           float* w_w, int32_t* idx_r, float* w_r, void* workspace, size_t workspace_bytes,
+                           sdm_stream_t stream) {
+    if (s && s->T != 1) return fail(SDM_ERR_INVALID_ARG, "sdm_decode_step needs shape->T == 1 (got %d)", s->T);
+    return forward_impl("sdm_decode_step", s, P_q, P_k, q, k, v, alpha, beta, mem, y, idx_w, w_w, idx_r, w_r,
+                        workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream), true);
+}
+
+sdm_status sdm_recur(const sdm_shape* s, const int32_t* idx_w, const float* w_w, const int32_t* idx_r,
+                     const float* w_r, const void* v, const void* alpha, const void* beta, void* mem, void* y,
+                     sdm_stream_t stream) {
+    SDM_TRY(check_shape(s, false, nullptr));
+    const size_t es = elem_bytes(s->dtype);
+    const size_t bht = static_cast<size_t>(s->B) * s->H * s->T;
+    if (bht == 0) return ok();
+    SDM_TRY(check_vec(idx_w, "idx_w", 4));
+    SDM_TRY(check_vec(w_w, "w_w", 4));
+    SDM_TRY(check_vec(idx_r, "idx_r", 4));
+    SDM_TRY(check_vec(w_r, "w_r", 4));
+    SDM_TRY(check_vec(v, "v", 16));
+    SDM_TRY(check_vec(alpha, "alpha", es));
+    SDM_TRY(check_vec(beta, "beta", es));
+    SDM_TRY(check_vec(mem, "mem", 16));
+    SDM_TRY(check_vec(y, "y", 16));
+    const size_t rowb = static_cast<size_t>(s->d_v) * es;
+    const Range rm{mem, static_cast<size_t>(s->B) * s->H * static_cast<size_t>(s->N) * rowb, "mem"};
+    const Range others[] = {{idx_w, bht * s->k_write * 4, "idx_w"}, {w_w, bht * s->k_write * 4, "w_w"},
+                            {idx_r, bht * s->k_read * 4, "idx_r"},  {w_r, bht * s->k_read * 4, "w_r"},
+                            {v, bht * rowb, "v"}, {alpha, bht * es, "alpha"}, {beta, bht * es, "beta"},
+                            {y, bht * rowb, "y"}};
+    for (const Range& r : others)
+        if (overlaps(rm, r)) return fail(SDM_ERR_INVALID_ARG, "sdm_recur: mem overlaps %s", r.name);
+    int* err = nullptr;
+    SDM_TRY(status_word(&err));
+    sdm::RecArgs r{};
+    r.idx_w = idx_w; r.w_w = w_w; r.idx_r = idx_r; r.w_r = w_r;
+    r.v = v; r.alpha = alpha; r.beta = beta; r.mem = mem; r.y = y;
+    r.B = s->B; r.H = s->H; r.T = s->T; r.dv = s->d_v; r.kw = s->k_write; r.kr = s->k_read;
+    r.N = s->N;
+    r.err = err;
+    cudaError_t e = sdm::launch_recur(s->dtype, r, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "recurrence launch");
+    return ok();
+}
+
+sdm_status sdm_device_status(int32_t* code, sdm_stream_t stream) {
+    if (!code) return fail(SDM_ERR_INVALID_ARG, "code is NULL");
+    int* w = nullptr;
+    SDM_TRY(status_word(&w));
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    int host = 0;
+    cudaError_t e = cudaMemcpyAsync(&host, w, sizeof(int), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(w, 0, sizeof(int), st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(e, "sdm_device_status");
+    *code = host;
+    if (host != 0) return fail(SDM_ERR_DEVICE, "device status word = 0x%x (bit 0: slot index outside [0, N) skipped)", host);
+    return ok();
+}
+
+}  // extern "C"

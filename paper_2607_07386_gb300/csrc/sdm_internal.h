@@ -1,0 +1,56 @@
+// Host-side interface between the C ABI (sdm_api.cu) and the kernel translation units.
+#pragma once
+#include <cuda_runtime.h>
+#include <stdint.h>
+#include <stddef.h>
+
+#include "sdm_common.cuh"
+
+namespace sdm {
+
+// ---------------------------------------------------------------- K-INIT
+cudaError_t launch_init_memory(const void* M0, void* mem, int64_t bytes_per_seq, int B, cudaStream_t stream);
+
+// ---------------------------------------------------------------- K-ADDR
+// "which" 0 = read side (q with P_q -> idx_r, w_r), 1 = write side (k with P_k -> idx_w, w_w).
+struct AddrArgs {
+    const void* P[2];      // [H, 2S, dk] per side, or nullptr (DIRECT mode: scores are x)
+    const void* X[2];      // [B, H, T, dk]
+    int32_t* idx[2];       // [B, H, T, k_side]
+    float* w[2];           // [B, H, T, k_side]
+    int kk[2];             // k_read, k_write
+    int B, H, T, dk, S;
+    int ncc;               // column chunks per half
+    int cw;                // columns per chunk (the last one may be shorter)
+    float cbound;          // |fp32 score - float64 score| <= cbound * max_j ||P_j|| * ||x||
+    float* part_v;         // workspace [2H][2 ncc][L][B*T]: per-chunk top-L scores
+    int* part_i;           //   ... and their column index within the half
+    float* pnorm;          // workspace [2H]: max row norm of P per side and head
+    int* err;              // device status word
+};
+
+// Geometry of the PKM partial lists for a shape (depends only on the shape).
+struct AddrPlan {
+    int L;      // list length kept per chunk (>= k + 4)
+    int ncc;    // column chunks per half
+    int cw;     // columns per chunk
+};
+AddrPlan addr_plan(int B, int H, int T, int S, int kmax);
+size_t addr_partial_bytes(const AddrPlan& plan, int B, int H, int T);
+cudaError_t launch_address(int dtype, const AddrPlan& plan, const AddrArgs& a, cudaStream_t stream);
+
+// ---------------------------------------------------------------- K-REC
+struct RecArgs {
+    const int32_t* idx_w; const float* w_w;   // [B, H, T, kw]
+    const int32_t* idx_r; const float* w_r;   // [B, H, T, kr]
+    const void* v;                            // [B, H, T, dv]
+    const void* alpha; const void* beta;      // [B, H, T]
+    void* mem;                                // [B, H, N, dv]
+    void* y;                                  // [B, H, T, dv]
+    int B, H, T, dv, kw, kr;
+    int64_t N;
+    int* err;
+};
+cudaError_t launch_recur(int dtype, const RecArgs& a, cudaStream_t stream);
+
+}  // namespace sdm

@@ -1,0 +1,61 @@
+"""GPU-side helpers for the parity tests: build device inputs from the seeded
+generator, run the library through its C ABI, fetch results."""
+from __future__ import annotations
+
+import numpy as np
+
+import synth
+from synth.torch_io import from_torch, to_torch, torch_dtype
+
+
+def shape_of(cfg: synth.SdmConfig, T: int | None = None):
+    import paper_2607_07386_gb300 as sdm
+    return sdm.SdmShape.make(cfg.B, cfg.H, cfg.T if T is None else T, cfg.d_k, cfg.d_v, cfg.N, cfg.k_write,
+                             cfg.k_read, cfg.dtype, cfg.addr)
+
+
+def device_inputs(cfg: synth.SdmConfig, full: dict | None = None) -> dict:
+    full = full if full is not None else synth.full_inputs(cfg)
+    return {name: to_torch(a, cfg.dtype) for name, a in full.items()}
+
+
+def alloc_outputs(cfg: synth.SdmConfig, T: int):
+    import torch
+    dt = torch_dtype(cfg.dtype)
+    o = {
+        "y": torch.empty((cfg.B, cfg.H, T, cfg.d_v), dtype=dt, device="cuda"),
+        "idx_w": torch.empty((cfg.B, cfg.H, T, cfg.k_write), dtype=torch.int32, device="cuda"),
+        "w_w": torch.empty((cfg.B, cfg.H, T, cfg.k_write), dtype=torch.float32, device="cuda"),
+        "idx_r": torch.empty((cfg.B, cfg.H, T, cfg.k_read), dtype=torch.int32, device="cuda"),
+        "w_r": torch.empty((cfg.B, cfg.H, T, cfg.k_read), dtype=torch.float32, device="cuda"),
+    }
+    return o
+
+
+def workspace(shape):
+    import torch
+    import paper_2607_07386_gb300 as sdm
+    return torch.empty(sdm.workspace_bytes(shape), dtype=torch.uint8, device="cuda")
+
+
+def run_forward(cfg: synth.SdmConfig, dev: dict, T0: int = 0, T1: int | None = None, mem=None, ws=None):
+    """sdm_forward over tokens [T0, T1) (memory initialised from M0 unless `mem` is given)."""
+    import torch
+    import paper_2607_07386_gb300 as sdm
+    T1 = cfg.tokens_per_seq if T1 is None else T1
+    T = T1 - T0
+    shape = shape_of(cfg, T)
+    if mem is None:
+        mem = torch.empty((cfg.B, cfg.H, cfg.N, cfg.d_v), dtype=torch_dtype(cfg.dtype), device="cuda")
+        sdm.init_memory(shape, dev["M0"], mem)
+    sl = lambda name: dev[name][:, :, T0:T1].contiguous()
+    out = alloc_outputs(cfg, T)
+    ws = ws if ws is not None else workspace(shape)
+    sdm.forward(shape, dev.get("P_q"), dev.get("P_k"), sl("q"), sl("k"), sl("v"), sl("alpha"), sl("beta"), mem,
+                out["y"], ws, idx_w=out["idx_w"], w_w=out["w_w"], idx_r=out["idx_r"], w_r=out["w_r"])
+    out["mem"] = mem
+    return out
+
+
+def host(t, dtype: str) -> np.ndarray:
+    return from_torch(t, dtype)

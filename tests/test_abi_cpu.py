@@ -1,0 +1,130 @@
+"""Host-side checks of libsdm.so: it builds, loads, exports every entry point that
+include/sdm.h declares, and rejects bad arguments before launching anything.
+
+No call here reaches a kernel launch: every argument set fails validation first
+(the fake device addresses below are never dereferenced)."""
+import ctypes
+import os
+import re
+import shutil
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "sdm.h")
+
+
+@pytest.fixture(scope="module")
+def sdm():
+    import paper_2607_07386_gb300 as sdm
+    from paper_2607_07386_gb300 import build as B
+    if not os.path.exists(sdm.lib_path()):
+        if shutil.which("nvcc") is None and not os.path.exists("/usr/local/cuda/bin/nvcc"):
+            pytest.skip("nvcc not available to build libsdm.so")
+        B.build()
+    return sdm
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:sdm_status|int|size_t|const\s+char\s*\*)\s+(sdm_\w+)\s*\(", text, flags=re.M)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("sdm_abi_version", "sdm_last_error", "sdm_workspace_bytes", "sdm_init_memory",
+                     "sdm_forward", "sdm_decode_step", "sdm_recur", "sdm_address", "sdm_device_status"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(sdm):
+    L = sdm.lib()
+    for name in declared_functions():
+        assert hasattr(L, name), name
+    assert sdm.abi_version() == 1
+
+
+def test_shape_struct_layout_matches_header(sdm):
+    S = sdm.SdmShape
+    assert ctypes.sizeof(S) == 48
+    assert S.N.offset == 24 and S.k_write.offset == 32 and S.addr.offset == 44
+
+
+def _shape(sdm, **kw):
+    base = dict(B=2, H=2, T=16, d_k=32, d_v=32, N=1024, k_write=8, k_read=8, dtype="bf16", addr="projected")
+    base.update(kw)
+    return sdm.SdmShape.make(**base)
+
+
+@pytest.mark.parametrize("kw,frag", [
+    (dict(N=1000), "perfect square"),
+    (dict(k_write=33), "sqrt(N)"),
+    (dict(k_read=0), "[1, 64]"),
+    (dict(d_v=3), "multiple of 16"),
+    (dict(addr="direct"), "DIRECT"),
+    (dict(B=-1), ">= 0"),
+    (dict(d_k=300), "d_k > 256"),
+])
+def test_workspace_bytes_rejects_bad_shapes(sdm, kw, frag):
+    n = sdm.lib().sdm_workspace_bytes(ctypes.byref(_shape(sdm, **kw)))
+    assert n == 0
+    assert frag in sdm.last_error()
+
+
+def test_workspace_bytes_covers_selection_buffers(sdm):
+    s = sdm.SdmShape.make(8, 16, 4096, 128, 128, 262144, 32, 32, "bf16")
+    n = sdm.workspace_bytes(s)
+    assert n >= 4 * 8 * 16 * 4096 * 32 * 4
+    assert sdm.workspace_bytes(s) == n   # deterministic
+
+
+FAKE = 0x7F0000000000   # never dereferenced: each call below fails validation first
+
+
+def _fwd(sdm, shape, **over):
+    L = sdm.lib()
+    args = dict(P_q=FAKE, P_k=FAKE + 0x100000, q=FAKE + 0x200000, k=FAKE + 0x300000, v=FAKE + 0x400000,
+                alpha=FAKE + 0x500000, beta=FAKE + 0x600000, mem=FAKE + 0x10000000, y=FAKE + 0x700000,
+                ws=FAKE + 0x40000000, ws_bytes=0)
+    args.update(over)
+    return L.sdm_forward(ctypes.byref(shape), args["P_q"], args["P_k"], args["q"], args["k"], args["v"],
+                         args["alpha"], args["beta"], args["mem"], args["y"], None, None, None, None, args["ws"],
+                         args["ws_bytes"], None)
+
+
+def test_forward_rejects_null_misaligned_small_workspace_and_aliasing(sdm):
+    s = _shape(sdm)
+    assert _fwd(sdm, s, q=None) == 1 and "q is NULL" in sdm.last_error()
+    assert _fwd(sdm, s, q=FAKE + 1) == 1 and "aligned" in sdm.last_error()
+    assert _fwd(sdm, s, v=FAKE + 8) == 1 and "v is not 16-byte aligned" in sdm.last_error()
+    assert _fwd(sdm, s, ws_bytes=16) == 1 and "workspace too small" in sdm.last_error()
+    need = sdm.workspace_bytes(s)
+    assert _fwd(sdm, s, ws_bytes=need, y=FAKE + 0x10000000 + 4096) == 1 and "mem overlaps y" in sdm.last_error()
+    assert _fwd(sdm, s, ws_bytes=need, ws=FAKE + 0x10000000) == 1 and "overlaps workspace" in sdm.last_error()
+    assert sdm.lib().sdm_forward(None, *([None] * 14), 0, None) == 1
+
+
+def test_decode_step_requires_T_equal_1(sdm):
+    s = _shape(sdm, T=2)
+    L = sdm.lib()
+    st = L.sdm_decode_step(ctypes.byref(s), *([FAKE] * 9), None, None, None, None, FAKE, 1 << 30, None)
+    assert st == 1 and "T == 1" in sdm.last_error()
+
+
+def test_init_memory_and_recur_reject_overlap(sdm):
+    s = _shape(sdm)
+    L = sdm.lib()
+    assert L.sdm_init_memory(ctypes.byref(s), FAKE, FAKE + 64, None) == 1 and "overlaps" in sdm.last_error()
+    assert L.sdm_init_memory(ctypes.byref(s), None, FAKE, None) == 1
+    st = L.sdm_recur(ctypes.byref(s), FAKE + 0x10000000, FAKE + 0x100000, FAKE + 0x200000, FAKE + 0x300000,
+                     FAKE + 0x400000, FAKE + 0x500000, FAKE + 0x600000, FAKE + 0x10000000, FAKE + 0x700000, None)
+    assert st == 1 and "mem overlaps idx_w" in sdm.last_error()
+
+
+def test_binding_fails_loudly_without_library(tmp_path, monkeypatch):
+    import paper_2607_07386_gb300._binding as b
+    monkeypatch.setattr(b, "_LIB_PATH", str(tmp_path / "missing.so"))
+    monkeypatch.setattr(b, "_lib", None)
+    with pytest.raises(RuntimeError, match="not found"):
+        b.lib()

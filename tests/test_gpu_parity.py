@@ -1,0 +1,360 @@
+"""Parity of the CUDA path (through the C ABI) with the float64 oracle.
+
+Bars: selected slot indices bit-exact; y, the rows the sequence wrote and the
+slot weights within max relative error (per (b, h) slice, Frobenius norm)
+TOL["bf16"] = 2e-3 or TOL["f32"] = 1e-5; untouched memory rows bit-identical to
+M0; kernels that must agree with each other (split runs, decode steps, batch
+slices) agree bit for bit.
+"""
+import numpy as np
+import pytest
+
+import synth
+from oracle import sdm_oracle as O
+from oracle.reference_run import oracle_slice, oracle_slices, rel_fro
+
+torch = pytest.importorskip("torch")
+pytestmark = [pytest.mark.gpu,
+              pytest.mark.skipif(not torch.cuda.is_available(), reason="needs a CUDA GPU")]
+
+from tests import gpu_harness as G  # noqa: E402
+
+TOL = {"bf16": 2e-3, "f32": 1e-5}
+
+
+@pytest.fixture(scope="module")
+def sdm():
+    import paper_2607_07386_gb300 as sdm
+    from paper_2607_07386_gb300 import build as B
+    B.build()
+    return sdm
+
+
+def _check_slices(cfg, out, slices, T=None, check_untouched=True):
+    tol = TOL[cfg.dtype]
+    ref = oracle_slices(cfg, slices, T=T)
+    y = out["y"]
+    for (b, h), r in ref.items():
+        assert np.array_equal(out["idx_w"][b, h].cpu().numpy(), r["idx_w"]), ("idx_w", b, h)
+        assert np.array_equal(out["idx_r"][b, h].cpu().numpy(), r["idx_r"]), ("idx_r", b, h)
+        assert rel_fro(out["w_w"][b, h].cpu().numpy(), r["w_w"]) <= tol
+        assert rel_fro(out["w_r"][b, h].cpu().numpy(), r["w_r"]) <= tol
+        ey = rel_fro(O.to_f64(G.host(y[b, h], cfg.dtype), cfg.dtype), r["y"])
+        mem_bh = G.host(out["mem"][b, h], cfg.dtype)
+        em = rel_fro(O.to_f64(mem_bh[r["touched"]], cfg.dtype), r["M_touched"])
+        assert ey <= tol and em <= tol, (b, h, ey, em)
+        if check_untouched:
+            M0 = synth.head_inputs(cfg, h, which=("M0",))["M0"]
+            mask = np.ones(cfg.N, bool)
+            mask[r["touched"]] = False
+            assert np.array_equal(mem_bh[mask], M0[mask]), ("untouched rows changed", b, h)
+
+
+# ------------------------------------------------------------------ K-INIT
+
+@pytest.mark.parametrize("dtype,B,H,N,dv", [("bf16", 3, 2, 1000, 64), ("f32", 2, 3, 4096, 32), ("bf16", 1, 1, 7, 8)])
+def test_init_memory_bit_exact(sdm, dtype, B, H, N, dv):
+    g = torch.Generator().manual_seed(1)
+    dt = synth.torch_io.torch_dtype(dtype)
+    M0 = torch.randn((H, N, dv), generator=g).to(dt).cuda()
+    mem = torch.full((B, H, N, dv), 7.0, dtype=dt, device="cuda")
+    sdm.init_memory(sdm.SdmShape.make(B, H, 1, 8, dv, N, 1, 1, dtype), M0, mem)
+    torch.cuda.synchronize()
+    for b in range(B):
+        assert torch.equal(mem[b], M0)
+
+
+# ------------------------------------------------------------------ K-ADDR
+
+ADDR_CASES = {
+    "tiny_fp32": synth.TINY_FP32,
+    "ragged_tokens_bf16": synth.SMALL_BF16.with_(B=2, H=2, T=300),
+    "layer_geometry": synth.LAYER_1P4B.with_(B=1, H=2, T=200),
+    "decode_chunked": synth.DECODE.with_(B=256, H=2, prefill_steps=0, decode_steps=1),
+    "direct_mode": synth.SdmConfig("direct", B=2, H=2, T=100, d_k=128, d_v=64, N=4096, k_write=8, k_read=8,
+                                   dtype="bf16", seed=21, alpha_mu=3.0, addr="direct"),
+    "odd_S_uneven_k": synth.SdmConfig("odd", B=1, H=3, T=77, d_k=48, d_v=32, N=48 * 48, k_write=5, k_read=3,
+                                      dtype="bf16", seed=22, alpha_mu=3.0),
+    "k_equals_S": synth.SdmConfig("keqS", B=1, H=1, T=50, d_k=16, d_v=16, N=64, k_write=8, k_read=8,
+                                  dtype="f32", seed=23, alpha_mu=3.0),
+}
+
+
+def _run_address(sdm, cfg, dev, T):
+    shape = G.shape_of(cfg, T)
+    out = G.alloc_outputs(cfg, T)
+    ws = G.workspace(shape)
+    sdm.address(shape, dev.get("P_q"), dev.get("P_k"), dev["q"][:, :, :T].contiguous(),
+                dev["k"][:, :, :T].contiguous(), out["idx_w"], out["w_w"], out["idx_r"], out["w_r"], ws)
+    torch.cuda.synchronize()
+    return out
+
+
+@pytest.mark.parametrize("name", list(ADDR_CASES))
+def test_address_matches_oracle(sdm, name):
+    cfg = ADDR_CASES[name]
+    T = cfg.tokens_per_seq
+    full = synth.full_inputs(cfg)
+    dev = G.device_inputs(cfg, full)
+    out = _run_address(sdm, cfg, dev, T)
+    tol = TOL[cfg.dtype]
+    f = lambda a: O.to_f64(a, cfg.dtype)
+    bs = range(cfg.B) if cfg.B <= 4 else [0, 1, cfg.B // 2, cfg.B - 1]
+    for b in bs:
+        for h in range(cfg.H):
+            Pq = f(full["P_q"][h]) if "P_q" in full else None
+            Pk = f(full["P_k"][h]) if "P_k" in full else None
+            iw, _, ww = O.address(Pk, f(full["k"][b, h]), cfg.N, cfg.k_write)
+            ir, _, wr = O.address(Pq, f(full["q"][b, h]), cfg.N, cfg.k_read)
+            assert np.array_equal(out["idx_w"][b, h].cpu().numpy(), iw), (name, b, h)
+            assert np.array_equal(out["idx_r"][b, h].cpu().numpy(), ir), (name, b, h)
+            assert rel_fro(out["w_w"][b, h].cpu().numpy(), ww) <= tol
+            assert rel_fro(out["w_r"][b, h].cpu().numpy(), wr) <= tol
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_address_integer_ties(sdm, dtype):
+    """Small-integer keys and projections: many exactly equal scores, so the selection
+    rests on the (score desc, index asc) / (score desc, slot asc) tie-breaks."""
+    cfg = synth.SdmConfig("ties", B=1, H=2, T=64, d_k=8, d_v=16, N=256, k_write=8, k_read=4,
+                          dtype=dtype, seed=31, alpha_mu=3.0)
+    rng = np.random.default_rng(5)
+    full = {"P_q": rng.integers(-2, 3, (2, 32, 8)), "P_k": rng.integers(-2, 3, (2, 32, 8)),
+            "q": rng.integers(-2, 3, (1, 2, 64, 8)), "k": rng.integers(-2, 3, (1, 2, 64, 8))}
+    full = {n: synth.round_f64_to_storage(a.astype(np.float64), dtype) for n, a in full.items()}
+    dev = {n: synth.torch_io.to_torch(a, dtype) for n, a in full.items()}
+    out = _run_address(sdm, cfg, dev, 64)
+    f = lambda a: O.to_f64(a, dtype)
+    for h in range(2):
+        iw, _, _ = O.address(f(full["P_k"][h]), f(full["k"][0, h]), 256, 8)
+        ir, _, _ = O.address(f(full["P_q"][h]), f(full["q"][0, h]), 256, 4)
+        assert np.array_equal(out["idx_w"][0, h].cpu().numpy(), iw)
+        assert np.array_equal(out["idx_r"][0, h].cpu().numpy(), ir)
+
+
+# ------------------------------------------------------------------ K-REC with explicit addressing
+
+def _recur(sdm, dtype, idx_w, w_w, idx_r, w_r, v, alpha, beta, M0, B=1, H=1):
+    """Run sdm_recur on float64 host inputs (v, alpha, beta, M0 already representable)."""
+    T, kw = idx_w.shape
+    kr = idx_r.shape[1]
+    N, dv = M0.shape
+    tt = lambda a: synth.torch_io.to_torch(synth.round_f64_to_storage(a, dtype), dtype)
+    mem = tt(M0).reshape(1, 1, N, dv).contiguous()
+    y = torch.empty((1, 1, T, dv), dtype=synth.torch_io.torch_dtype(dtype), device="cuda")
+    shape = sdm.SdmShape.make(1, 1, T, 8, dv, N, kw, kr, dtype)
+    i32 = lambda a: torch.from_numpy(np.ascontiguousarray(a, np.int32)).cuda()
+    f32 = lambda a: torch.from_numpy(np.ascontiguousarray(a, np.float32)).cuda()
+    sdm.recur(shape, i32(idx_w), f32(w_w), i32(idx_r), f32(w_r), tt(v).contiguous(), tt(alpha), tt(beta), mem, y)
+    torch.cuda.synchronize()
+    return (O.to_f64(G.host(y[0, 0], dtype), dtype), O.to_f64(G.host(mem[0, 0], dtype), dtype))
+
+
+def test_recur_gdn_special_case(sdm):
+    """Sec. 3.1 "Connection to GDN" on the GPU: N = d_qk = 64 slots, every slot selected,
+    dense key values as write weights and dense queries as read weights."""
+    rng = np.random.default_rng(41)
+    dqk, dv, T = 64, 32, 64
+    K = rng.standard_normal((T, dqk)) / np.sqrt(dqk)
+    Q = rng.standard_normal((T, dqk)) / np.sqrt(dqk)
+    V = O.round_storage(rng.standard_normal((T, dv)), "f32")
+    a = O.round_storage(1 / (1 + np.exp(-rng.standard_normal(T) - 3)), "f32")
+    b = O.round_storage(1 / (1 + np.exp(-rng.standard_normal(T))), "f32")
+    M0 = O.round_storage(rng.standard_normal((dqk, dv)) * 0.1, "f32")
+    K32, Q32 = K.astype(np.float32).astype(np.float64), Q.astype(np.float32).astype(np.float64)
+    alls = np.tile(np.arange(dqk), (T, 1))
+    y_gpu, M_gpu = _recur(sdm, "f32", alls, K32, alls, Q32, V, a, b, M0)
+    M = M0.copy()
+    y_or, _ = O.recur(M, alls, K32, alls, Q32, V, a, b, "f32")
+    assert rel_fro(y_gpu, y_or) <= 1e-5 and rel_fro(M_gpu, M) <= 1e-5
+    Mg = M0.copy()   # textbook GDN (Eq. gdn-update) in float64
+    ys = []
+    for t in range(T):
+        Mg = a[t] * Mg + b[t] * np.outer(K32[t], V[t] - a[t] * (Mg.T @ K32[t]))
+        ys.append(Mg.T @ Q32[t])
+    assert rel_fro(y_gpu, np.array(ys)) <= 1e-5
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_recur_single_slot_recall_bit_exact(sdm, dtype):
+    rng = np.random.default_rng(42)
+    N, dv, T = 512, 64, 100
+    M0 = O.round_storage(rng.standard_normal((N, dv)) * 0.02, dtype)
+    V = O.round_storage(rng.standard_normal((T, dv)), dtype)
+    slots = rng.choice(N, T, replace=False)[:, None]
+    one = np.ones((T, 1))
+    y, M = _recur(sdm, dtype, slots, one, slots, one, V, np.ones(T), np.ones(T), M0)
+    assert np.array_equal(y, V)
+    assert np.array_equal(M[slots[:, 0]], V)
+    rest = np.setdiff1d(np.arange(N), slots[:, 0])
+    assert np.array_equal(M[rest], M0[rest])
+
+
+def test_recur_beta_zero_closed_form(sdm):
+    rng = np.random.default_rng(43)
+    N, dv, T, k = 300, 32, 80, 6
+    M0 = O.round_storage(rng.standard_normal((N, dv)), "f32")
+    iw = np.array([np.sort(rng.choice(N, k, replace=False)) for _ in range(T)])
+    ir = np.array([np.sort(rng.choice(N, k, replace=False)) for _ in range(T)])
+    ww = rng.dirichlet(np.ones(k), T).astype(np.float32).astype(np.float64)
+    wr = rng.dirichlet(np.ones(k), T).astype(np.float32).astype(np.float64)
+    a = O.round_storage(1 / (1 + np.exp(-rng.standard_normal(T) - 2)), "f32")
+    V = O.round_storage(rng.standard_normal((T, dv)), "f32")
+    y, M = _recur(sdm, "f32", iw, ww, ir, wr, V, a, np.zeros(T), M0)
+    decay = np.ones(N)
+    for t in range(T):
+        decay[iw[t]] *= a[t]
+    assert rel_fro(M, decay[:, None] * M0) <= 1e-5
+
+
+def test_recur_matches_oracle_random_sparse(sdm):
+    rng = np.random.default_rng(44)
+    for dtype in ("bf16", "f32"):
+        N, dv, T, kw, kr = 2000, 128 if dtype == "bf16" else 64, 150, 12, 20
+        M0 = O.round_storage(rng.standard_normal((N, dv)) * 0.02, dtype)
+        iw = np.array([rng.permutation(rng.choice(N, kw, replace=False)) for _ in range(T)])  # any order
+        ir = np.array([np.sort(rng.choice(N, kr, replace=False)) for _ in range(T)])
+        ww = rng.dirichlet(np.ones(kw), T).astype(np.float32).astype(np.float64)
+        wr = rng.dirichlet(np.ones(kr), T).astype(np.float32).astype(np.float64)
+        a = O.round_storage(1 / (1 + np.exp(-rng.standard_normal(T) - 3)), dtype)
+        b = O.round_storage(1 / (1 + np.exp(-rng.standard_normal(T))), dtype)
+        V = O.round_storage(rng.standard_normal((T, dv)), dtype)
+        y, M = _recur(sdm, dtype, iw, ww, ir, wr, V, a, b, M0)
+        Mo = M0.copy()
+        _, yo = O.recur(Mo, iw, ww, ir, wr, V, a, b, dtype)
+        assert rel_fro(y, yo) <= TOL[dtype] and rel_fro(M, Mo) <= TOL[dtype]
+
+
+def test_bad_slot_index_is_skipped_and_reported(sdm):
+    N, dv, T = 64, 32, 4
+    idx = np.array([[0, 1], [2, N], [3, -1], [4, 5]])
+    w = np.full((T, 2), 0.5)
+    z = np.zeros((N, dv))
+    sdm.device_status()   # clear
+    y, M = _recur(sdm, "f32", idx, w, idx, w, np.ones((T, dv)), np.ones(T), np.ones(T), z)
+    assert sdm.device_status() == 1
+    assert sdm.device_status() == 0   # cleared
+    assert np.all(np.isfinite(y))
+
+
+# ------------------------------------------------------------------ whole path
+
+@pytest.mark.parametrize("name", ["tiny_fp32", "small_bf16"])
+def test_forward_config_parity(sdm, name):
+    cfg = synth.get_config(name)
+    dev = G.device_inputs(cfg)
+    out = G.run_forward(cfg, dev)
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    slices = [(b, h) for b in range(cfg.B) for h in range(cfg.H)]
+    if len(slices) > 8:
+        rng = np.random.default_rng(0)
+        slices = [slices[i] for i in sorted(rng.choice(len(slices), 8, replace=False))]
+    _check_slices(cfg, out, slices)
+
+
+def test_forward_empty_T_is_a_no_op(sdm):
+    cfg = synth.TINY_FP32
+    shape = G.shape_of(cfg, 0)
+    sdm.forward(shape, None, None, None, None, None, None, None, None, None, None)
+
+
+def test_split_invariance_and_decode_equivalence(sdm):
+    """forward(T) == forward(T1) then forward(T - T1) == T decode steps, bit for bit."""
+    cfg = synth.SdmConfig("split", B=3, H=2, T=64, d_k=64, d_v=64, N=4096, k_write=8, k_read=8,
+                          dtype="bf16", seed=51, alpha_mu=3.0)
+    dev = G.device_inputs(cfg)
+    whole = G.run_forward(cfg, dev)
+    part1 = G.run_forward(cfg, dev, 0, 25)
+    part2 = G.run_forward(cfg, dev, 25, 64, mem=part1["mem"])
+    torch.cuda.synchronize()
+    assert torch.equal(whole["mem"], part2["mem"])
+    assert torch.equal(whole["y"], torch.cat([part1["y"], part2["y"]], dim=2))
+    mem = torch.empty_like(whole["mem"])
+    shape1 = G.shape_of(cfg, 1)
+    sdm.init_memory(shape1, dev["M0"], mem)
+    ws = G.workspace(shape1)
+    ys = []
+    for t in range(cfg.T):
+        y = torch.empty((cfg.B, cfg.H, cfg.d_v), dtype=torch.bfloat16, device="cuda")
+        sl = lambda n: dev[n][:, :, t].contiguous()
+        sdm.decode_step(shape1, dev["P_q"], dev["P_k"], sl("q"), sl("k"), sl("v"), sl("alpha"), sl("beta"),
+                        mem, y, ws)
+        ys.append(y)
+    torch.cuda.synchronize()
+    assert torch.equal(mem, whole["mem"])
+    assert torch.equal(torch.stack(ys, dim=2), whole["y"])
+
+
+def test_batch_slices_are_independent(sdm):
+    cfg = synth.SdmConfig("indep", B=4, H=2, T=40, d_k=32, d_v=32, N=1024, k_write=8, k_read=8,
+                          dtype="bf16", seed=52, alpha_mu=3.0)
+    full = synth.full_inputs(cfg)
+    dev = G.device_inputs(cfg, full)
+    outB = G.run_forward(cfg, dev)
+    one = cfg.with_(B=1)
+    sub = dict(full)
+    for n in ("q", "k", "v", "alpha", "beta"):
+        sub[n] = np.ascontiguousarray(full[n][2:3])
+    out1 = G.run_forward(one, G.device_inputs(one, sub))
+    torch.cuda.synchronize()
+    assert torch.equal(out1["y"][0], outB["y"][2]) and torch.equal(out1["mem"][0], outB["mem"][2])
+
+
+# ------------------------------------------------------------------ full-size workloads
+
+@pytest.mark.fullsize
+def test_layer_1p4b_full_size_sampled_slices(sdm):
+    cfg = synth.LAYER_1P4B
+    dev = G.device_inputs(cfg)
+    out = G.run_forward(cfg, dev)
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    _check_slices(cfg, out, [(0, 0), (3, 7), (5, 12), (7, 15)])
+
+
+@pytest.mark.fullsize
+def test_long_context_full_size_sampled_slices(sdm):
+    cfg = synth.LONG_CTX
+    dev = G.device_inputs(cfg)
+    out = G.run_forward(cfg, dev)
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    del dev
+    _check_slices(cfg, out, [(0, 3), (1, 14)])
+
+
+@pytest.mark.fullsize
+def test_decode_full_size_prefill_then_steps(sdm):
+    """B = 256 sequences x H = 16, 1024 untimed + 1000 timed decode steps from M0 (274.9 GB state);
+    sampled slices replayed by the oracle over all 2024 tokens."""
+    cfg = synth.DECODE
+    full = synth.full_inputs(cfg)
+    dev_params = {n: synth.torch_io.to_torch(full[n], cfg.dtype) for n in ("M0", "P_q", "P_k")}
+    mem = torch.empty((cfg.B, cfg.H, cfg.N, cfg.d_v), dtype=torch.bfloat16, device="cuda")
+    shape = G.shape_of(cfg, 1)
+    sdm.init_memory(shape, dev_params["M0"], mem)
+    ws = G.workspace(shape)
+    steps = cfg.tokens_per_seq
+    slices = [(0, 0), (100, 5), (255, 15)]
+    ys = {s: [] for s in slices}
+    iws = {s: [] for s in slices}
+    iw = torch.empty((cfg.B, cfg.H, cfg.k_write), dtype=torch.int32, device="cuda")
+    y = torch.empty((cfg.B, cfg.H, cfg.d_v), dtype=torch.bfloat16, device="cuda")
+    for s in range(steps):
+        st = {n: synth.torch_io.to_torch(np.ascontiguousarray(full[n][:, :, s]), cfg.dtype)
+              for n in ("q", "k", "v", "alpha", "beta")}
+        sdm.decode_step(shape, dev_params["P_q"], dev_params["P_k"], st["q"], st["k"], st["v"], st["alpha"],
+                        st["beta"], mem, y, ws, idx_w=iw)
+        for (b, h) in slices:
+            ys[(b, h)].append(y[b, h].clone())
+            iws[(b, h)].append(iw[b, h].clone())
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    ref = oracle_slices(cfg, slices)
+    for (b, h), r in ref.items():
+        assert np.array_equal(torch.stack(iws[(b, h)]).cpu().numpy(), r["idx_w"])
+        yg = O.to_f64(G.host(torch.stack(ys[(b, h)]), cfg.dtype), cfg.dtype)
+        assert rel_fro(yg, r["y"]) <= TOL["bf16"]
+        mem_bh = O.to_f64(G.host(mem[b, h], cfg.dtype), cfg.dtype)
+        assert rel_fro(mem_bh[r["touched"]], r["M_touched"]) <= TOL["bf16"]
