@@ -1,0 +1,338 @@
+"""Benchmark of the Sparse Delta Memory hot path on GB300.
+
+One step = one pass of the whole hot path over the 1.4B-scale global-layer
+workload (B=8, H=16, T=4096, d_k=d_v=128, N=262144 slots/head, k=32, bf16):
+learned-initial-state broadcast (sdm_init_memory), then sdm_forward (PKM
+addressing for the write keys and read queries of every token, then the fused
+recurrence), all inputs resident in HBM.  Prints one JSON line.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+--impl reference times the float64 CPU oracle on this machine's cores on a
+bounded sample of the same workload (the comparison arm; no GPU use).
+Multi-GPU (torchrun): every rank runs an independent shard of sequences (weak
+scaling); only the timing uses a collective.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import synth  # noqa: E402
+
+METRIC = "SDM recurrence tokens/s per layer (1 GB300) and achieved HBM GB/s vs ~8 TB/s"
+UNIT = "tokens/s"
+
+
+def _peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return {"hbm_gbs": float(p["hbm_gbs"]), "bf16_tflops": float(p.get("bf16_tflops", 1931.2)),
+                "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "source": "fallback"}
+
+
+def _workload_desc(cfg) -> str:
+    return (f"{cfg.name}: B={cfg.B} H={cfg.H} T={cfg.T} d_k={cfg.d_k} d_v={cfg.d_v} N={cfg.N} "
+            f"k_write={cfg.k_write} k_read={cfg.k_read} {cfg.dtype} seed={cfg.seed}")
+
+
+# ----------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.idx = gpu_id
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.idx}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200", "-f", self.path],
+                                         stdout=subprocess.DEVNULL, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        if not self.path or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower().startswith("active"):
+                        reasons.add(n)
+        os.unlink(self.path)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- CPU oracle arm
+
+def _oracle_pool(n):
+    import multiprocessing as mp
+    return mp.get_context("spawn").Pool(n)
+
+
+def _oracle_step(pool, cfg, slices, T):
+    """Slices run one per worker in parallel; the step time is the slowest worker's
+    oracle compute time (input generation excluded)."""
+    from oracle.reference_run import timed_worker
+    return max(pool.map(timed_worker, [(cfg, b, h, T) for b, h in slices]))
+
+
+def cpu_baseline(cfg, T=1024):
+    """Oracle throughput on a bounded sample: one (b, h) slice x T tokens per core; tokens/s
+    per layer = slice-tokens / H / time (slices are independent, so per-core work adds up)."""
+    cores = os.cpu_count() or 1
+    rng = np.random.default_rng(0)
+    slices = [(int(rng.integers(cfg.B)), int(rng.integers(cfg.H))) for _ in range(cores)]
+    with _oracle_pool(cores) as pool:
+        dt = _oracle_step(pool, cfg, slices, T)
+    return {"value": cores * T / cfg.H / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{cores} (b,h) slices x first {T} tokens of {cfg.name}, one float64 worker per core, "
+                      f"{dt:.1f} s (slowest worker, input generation excluded)"}
+
+
+def run_reference(args, cfg):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    cores = os.cpu_count() or 1
+    T = 256
+    rng = np.random.default_rng(1)
+    times = []
+    with _oracle_pool(cores) as pool:
+        for _ in range(args.warmup):
+            _oracle_step(pool, cfg, [(0, 0)], 32)
+        for _ in range(args.steps):
+            slices = [(int(rng.integers(cfg.B)), int(rng.integers(cfg.H))) for _ in range(cores)]
+            times.append(_oracle_step(pool, cfg, slices, T))
+    value = cores * T / cfg.H * len(times) / sum(times)
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * sum(times) / len(times),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": _workload_desc(cfg), "global_batch": cfg.B,
+                                            "seq_len": cfg.T, "parallelism": "none (host cores)"},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                             "sample": f"each step: {cores} (b,h) slices x first {T} tokens, float64 oracle, "
+                                       "one worker per core, input generation excluded"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------- GPU arm
+
+def run_ours(args, cfg):
+    import torch
+    import paper_2607_07386_gb300 as sdm
+    from paper_2607_07386_gb300.build import build
+    from synth.torch_io import to_torch, torch_dtype
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    if rank == 0:
+        build()
+    if world > 1:
+        dist.barrier()
+    build()   # no-op when up to date; loads in every rank
+
+    # ---- inputs (rank r owns sequences [r*B, (r+1)*B) of the global batch), resident in HBM
+    full = synth.full_inputs(cfg, b0=rank * cfg.B)
+    dt = torch_dtype(cfg.dtype)
+    dev = {n: to_torch(a, cfg.dtype) for n, a in full.items()}
+    host_pinned = {n: torch.from_numpy(np.ascontiguousarray(full[n]).view(np.int16 if cfg.dtype == "bf16" else np.float32))
+                   .view(dt).pin_memory() for n in ("q", "k", "v", "alpha", "beta")}
+    del full
+    B, H, T, N, dv = cfg.B, cfg.H, cfg.T, cfg.N, cfg.d_v
+    shape = sdm.SdmShape.make(B, H, T, cfg.d_k, dv, N, cfg.k_write, cfg.k_read, cfg.dtype)
+    mem = torch.empty((B, H, N, dv), dtype=dt, device="cuda")
+    y = torch.empty((B, H, T, dv), dtype=dt, device="cuda")
+    ws = torch.empty(sdm.workspace_bytes(shape), dtype=torch.uint8, device="cuda")
+    idx_w = torch.empty((B, H, T, cfg.k_write), dtype=torch.int32, device="cuda")
+    w_w = torch.empty((B, H, T, cfg.k_write), dtype=torch.float32, device="cuda")
+    idx_r = torch.empty((B, H, T, cfg.k_read), dtype=torch.int32, device="cuda")
+    w_r = torch.empty((B, H, T, cfg.k_read), dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    def step():
+        sdm.init_memory(shape, dev["M0"], mem, stream)
+        sdm.forward(shape, dev["P_q"], dev["P_k"], dev["q"], dev["k"], dev["v"], dev["alpha"], dev["beta"],
+                    mem, y, ws, stream=stream)
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    def max_over_ranks(x: float) -> float:
+        if world == 1:
+            return x
+        t = torch.tensor([x], device="cuda", dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    for _ in range(args.warmup):
+        step()
+    barrier()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    try:
+        gpu_id = "GPU-" + str(torch.cuda.get_device_properties(local).uuid)
+    except Exception:
+        gpu_id = str(local)
+    with ClockSampler(gpu_id) as clk:
+        barrier()
+        ev0.record(stream)
+        for _ in range(args.steps):
+            step()
+        ev1.record(stream)
+        barrier()
+    ms_total = max_over_ranks(ev0.elapsed_time(ev1))
+    ms_step = ms_total / args.steps
+    clocks = clk.summary()
+    if sdm.device_status(stream) != 0:
+        raise RuntimeError("device status word set during the benchmark")
+
+    # ---- per-phase timing (same work split at the C ABI: init / addressing / recurrence)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    barrier()
+    for s in range(args.steps):
+        e = evs[s]
+        e[0].record(stream)
+        sdm.init_memory(shape, dev["M0"], mem, stream)
+        e[1].record(stream)
+        sdm.address(shape, dev["P_q"], dev["P_k"], dev["q"], dev["k"], idx_w, w_w, idx_r, w_r, ws, stream=stream)
+        e[2].record(stream)
+        sdm.recur(shape, idx_w, w_w, idx_r, w_r, dev["v"], dev["alpha"], dev["beta"], mem, y, stream)
+        e[3].record(stream)
+    barrier()
+    ph = {"init_memory": 0.0, "address": 0.0, "recurrence": 0.0}
+    for e in evs:
+        ph["init_memory"] += e[0].elapsed_time(e[1]) / args.steps
+        ph["address"] += e[1].elapsed_time(e[2]) / args.steps
+        ph["recurrence"] += e[2].elapsed_time(e[3]) / args.steps
+
+    # ---- end to end through the public API with host buffers (pinned), copies inside the region
+    h2d = sum(t.numel() * t.element_size() for t in host_pinned.values())
+    y_host = torch.empty(y.shape, dtype=dt, pin_memory=True)
+    d2h = y_host.numel() * y_host.element_size()
+
+    def e2e_step():
+        for n, t in host_pinned.items():
+            dev[n].copy_(t, non_blocking=True)
+        step()
+        y_host.copy_(y, non_blocking=True)
+
+    e2e_step()
+    barrier()
+    ev0.record(stream)
+    for _ in range(args.steps):
+        e2e_step()
+    ev1.record(stream)
+    barrier()
+    ms_e2e = max_over_ranks(ev0.elapsed_time(ev1)) / args.steps
+
+    tokens_step = B * T * world
+    peaks = _peaks()
+    rec_bytes = cfg.recurrence_bytes_per_token_head() * B * H * T
+    rec_ms = max_over_ranks(ph["recurrence"])
+    achieved = rec_bytes / (rec_ms * 1e-3) / 1e9
+    step_bytes = cfg.algorithmic_bytes_per_token_head() * B * H * T + (1 + B) * H * N * dv * cfg.elem_bytes
+    kernels_per_step = 5   # init, P row norms, scores, finalize, recurrence
+    line = {
+        "metric": METRIC, "value": tokens_step / (ms_step * 1e-3), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": cfg.dtype, "data": "synthetic",
+        "config": {"workload": _workload_desc(cfg), "global_batch": B * world, "seq_len": T,
+                   "parallelism": f"independent sequence shards x{world}" if world > 1 else "single GPU",
+                   "step": "sdm_init_memory (M0 broadcast) + sdm_forward (addressing + recurrence)",
+                   "l2": f"inputs larger than L2: {B * H * N * dv * cfg.elem_bytes / 1e9:.2f} GB memory state"},
+        "e2e": {"value": tokens_step / (ms_e2e * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h},
+        "gpu_launches": kernels_per_step * args.steps,
+        "roofline": {"bound": "hbm", "kernel": "k_recur", "achieved": achieved, "peak": peaks["hbm_gbs"],
+                     "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "traffic": None,
+                     "peak_source": peaks["source"], "bytes_per_launch": rec_bytes, "ms_per_launch": rec_ms},
+        "phase_ms": ph,
+        "step_hbm": {"algorithmic_bytes": step_bytes, "gbs": step_bytes / (ms_step * 1e-3) / 1e9,
+                     "frac_of_measured": step_bytes / (ms_step * 1e-3) / 1e9 / peaks["hbm_gbs"],
+                     "frac_of_8tbs": step_bytes / (ms_step * 1e-3) / 1e9 / 8000.0},
+        "clocks": clocks,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(cfg)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", default="layer_1p4b", choices=sorted(synth.CONFIGS))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    cfg = synth.get_config(args.config)
+    if cfg.is_decode:
+        raise SystemExit("the decode workload is exercised by the tests; bench.py times the scan workloads")
+    if args.impl == "reference":
+        run_reference(args, cfg)
+    else:
+        run_ours(args, cfg)
+
+
+if __name__ == "__main__":
+    main()

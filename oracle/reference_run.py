@@ -64,3 +64,16 @@ def rel_fro(got: np.ndarray, ref: np.ndarray) -> float:
     den = np.linalg.norm(ref)
     num = np.linalg.norm(got - ref)
     return float(num / den) if den > 0 else float(num)
+
+
+def timed_worker(args) -> float:
+    """Oracle forward of one slice over its first T tokens; returns the compute seconds
+    (input generation and float64 conversion excluded)."""
+    import time
+    cfg, b, h, T = args
+    x = slice_f64(cfg, b, h)
+    cut = lambda a: a[:T]
+    t0 = time.perf_counter()
+    O.forward_slice(x["M0"], x["P_q"], x["P_k"], cut(x["q"]), cut(x["k"]), cut(x["v"]), cut(x["alpha"]),
+                    cut(x["beta"]), cfg.N, cfg.k_write, cfg.k_read, cfg.dtype)
+    return time.perf_counter() - t0

@@ -92,9 +92,10 @@ def slice_inputs(cfg: SdmConfig, b: int, h: int) -> dict:
     return {"q": r(q), "k": r(k), "v": r(v), "alpha": r(alpha), "beta": r(beta)}
 
 
-def full_inputs(cfg: SdmConfig) -> dict:
+def full_inputs(cfg: SdmConfig, b0: int = 0) -> dict:
     """Whole-workload inputs as storage arrays: M0 [H,N,dv], P_* [H,2S,dk], q/k [B,H,T,dk],
-    v [B,H,T,dv], alpha/beta [B,H,T] (T = tokens per sequence)."""
+    v [B,H,T,dv], alpha/beta [B,H,T] (T = tokens per sequence).  Sequence b of the result
+    is global sequence b0 + b (a rank's shard of a larger batch)."""
     T = cfg.tokens_per_seq
     nd = storage_np_dtype(cfg.dtype)
     out = {"M0": np.empty((cfg.H, cfg.N, cfg.d_v), nd)}
@@ -109,7 +110,7 @@ def full_inputs(cfg: SdmConfig) -> dict:
         out[name] = np.empty((cfg.B, cfg.H, T) + tail, nd)
     for b in range(cfg.B):
         for h in range(cfg.H):
-            for name, arr in slice_inputs(cfg, b, h).items():
+            for name, arr in slice_inputs(cfg, b0 + b, h).items():
                 out[name][b, h] = arr
     return out
 

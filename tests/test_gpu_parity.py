@@ -184,8 +184,12 @@ def test_recur_single_slot_recall_bit_exact(sdm, dtype):
     slots = rng.choice(N, T, replace=False)[:, None]
     one = np.ones((T, 1))
     y, M = _recur(sdm, dtype, slots, one, slots, one, V, np.ones(T), np.ones(T), M0)
-    assert np.array_equal(y, V)
-    assert np.array_equal(M[slots[:, 0]], V)
+    assert np.array_equal(y, M[slots[:, 0]])          # weight exactly 1: the read returns the row
+    if dtype == "bf16":   # v - r and r + (v - r) are exact in fp32 for bf16 operands
+        assert np.array_equal(M[slots[:, 0]], V)
+    else:                 # fp32 arithmetic on fp32 operands: within one ulp of v
+        ulp = np.spacing(np.abs(V).astype(np.float32)).astype(np.float64)
+        assert np.all(np.abs(M[slots[:, 0]] - V) <= ulp)
     rest = np.setdiff1d(np.arange(N), slots[:, 0])
     assert np.array_equal(M[rest], M0[rest])
 
