@@ -187,8 +187,9 @@ def test_recur_single_slot_recall_bit_exact(sdm, dtype):
     assert np.array_equal(y, M[slots[:, 0]])          # weight exactly 1: the read returns the row
     if dtype == "bf16":   # v - r and r + (v - r) are exact in fp32 for bf16 operands
         assert np.array_equal(M[slots[:, 0]], V)
-    else:   # fp32 operands: two roundings (v - r, then r + delta), each <= half an ulp of a value <= 2|v|
-        ulp = np.spacing(np.abs(V).astype(np.float32)).astype(np.float64)
+    else:   # fp32 operands: two roundings (v - r, then r + delta), each <= half an ulp of max(|v|, |r|) doubled
+        scale = np.maximum(np.abs(V), np.abs(M0[slots[:, 0]]))
+        ulp = np.spacing(scale.astype(np.float32)).astype(np.float64)
         assert np.all(np.abs(M[slots[:, 0]] - V) <= 2 * ulp)
     rest = np.setdiff1d(np.arange(N), slots[:, 0])
     assert np.array_equal(M[rest], M0[rest])
