@@ -250,7 +250,7 @@ def run_ours(args, cfg):
         e[1].record(stream)
         sdm.address(shape, dev["P_q"], dev["P_k"], dev["q"], dev["k"], idx_w, w_w, idx_r, w_r, ws, stream=stream)
         e[2].record(stream)
-        sdm.recur(shape, idx_w, w_w, idx_r, w_r, dev["v"], dev["alpha"], dev["beta"], mem, y, stream)
+        sdm.recur(shape, idx_w, w_w, idx_r, w_r, dev["v"], dev["alpha"], dev["beta"], mem, y, ws, stream=stream)
         e[3].record(stream)
     barrier()
     ph = {"init_memory": 0.0, "address": 0.0, "recurrence": 0.0}

@@ -126,19 +126,26 @@ sdm_status sdm_decode_step(const sdm_shape* shape, const void* P_q, const void* 
                            int32_t* idx_w, float* w_w, int32_t* idx_r, float* w_r,
                            void* workspace, size_t workspace_bytes, sdm_stream_t stream);
 
+/* Bytes of workspace sdm_recur needs for `shape` (its hazard table); 0 if invalid. */
+size_t sdm_recur_workspace_bytes(const sdm_shape* shape);
+
 /* Recurrence with explicit addressing (Eqs. sdm-decay, sdm-write, sdm-read), no PKM:
  * idx_w [B,H,T,k_write] / w_w fp32, idx_r [B,H,T,k_read] / w_r fp32 (any weights,
- * e.g. dense key values for the GDN special case of Sec. 3.1; write slots distinct
- * within a token; k_write, k_read <= 64; slots may be in any order).
- * v, alpha, beta, mem, y as in sdm_forward.  shape->d_k and shape->addr are ignored. */
+ * e.g. dense key values for the GDN special case of Sec. 3.1; k_write, k_read <= 64).
+ * Slot lists must be strictly ascending within each token, as sdm_address produces
+ * them (App. A.2 sorts the selected indices); a violation is recorded in bit 1 of the
+ * device status word and its results are undefined.  N need not be a square here.
+ * v, alpha, beta, mem, y as in sdm_forward; shape->d_k and shape->addr are ignored.
+ * workspace: >= sdm_recur_workspace_bytes(shape) bytes, 256-byte aligned. */
 sdm_status sdm_recur(const sdm_shape* shape, const int32_t* idx_w, const float* w_w,
                      const int32_t* idx_r, const float* w_r, const void* v,
                      const void* alpha, const void* beta, void* mem, void* y,
-                     sdm_stream_t stream);
+                     void* workspace, size_t workspace_bytes, sdm_stream_t stream);
 
 /* Reads (host pointer `code`, synchronising on `stream`) and clears the device
  * status word of the current device: 0 = no fault; bit 0 = a slot index outside
- * [0, N) was skipped.  Returns SDM_ERR_DEVICE when the word was non-zero. */
+ * [0, N) was skipped; bit 1 = a slot list given to the recurrence was not strictly
+ * ascending.  Returns SDM_ERR_DEVICE when the word was non-zero. */
 sdm_status sdm_device_status(int32_t* code, sdm_stream_t stream);
 
 #ifdef __cplusplus

@@ -67,7 +67,9 @@ def lib():
             L.sdm_forward.argtypes = fwd
             L.sdm_decode_step.argtypes = fwd
             L.sdm_address.argtypes = [_SHP, _VP, _VP, _VP, _VP, _I32P, _VP, _I32P, _VP, _VP, _SZ, _VP]
-            L.sdm_recur.argtypes = [_SHP, _I32P, _VP, _I32P, _VP, _VP, _VP, _VP, _VP, _VP, _VP]
+            L.sdm_recur.argtypes = [_SHP, _I32P, _VP, _I32P, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP]
+            L.sdm_recur_workspace_bytes.restype = ctypes.c_size_t
+            L.sdm_recur_workspace_bytes.argtypes = [_SHP]
             L.sdm_device_status.argtypes = [ctypes.POINTER(ctypes.c_int32), _VP]
             for f in ("sdm_init_memory", "sdm_forward", "sdm_decode_step", "sdm_address", "sdm_recur",
                       "sdm_device_status"):
@@ -148,9 +150,18 @@ def decode_step(shape: SdmShape, P_q, P_k, q, k, v, alpha, beta, mem, y, workspa
                                  _ptr(w_r), _ptr(workspace), nb, _stream(stream)))
 
 
-def recur(shape: SdmShape, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem, y, stream=None):
+def recur_workspace_bytes(shape: SdmShape) -> int:
+    n = lib().sdm_recur_workspace_bytes(ctypes.byref(shape))
+    if n == 0:
+        raise SdmError(1, last_error())
+    return n
+
+
+def recur(shape: SdmShape, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem, y, workspace, stream=None,
+          workspace_nbytes=None):
+    nb = workspace_nbytes if workspace_nbytes is not None else (_nbytes(workspace) or 0)
     _check(lib().sdm_recur(ctypes.byref(shape), _ptr(idx_w), _ptr(w_w), _ptr(idx_r), _ptr(w_r), _ptr(v),
-                           _ptr(alpha), _ptr(beta), _ptr(mem), _ptr(y), _stream(stream)))
+                           _ptr(alpha), _ptr(beta), _ptr(mem), _ptr(y), _ptr(workspace), nb, _stream(stream)))
 
 
 def device_status(stream=None) -> int:

@@ -115,7 +115,7 @@ sdm_status check_shape(const sdm_shape* s, bool need_pkm, int64_t* S_out) {
 }
 
 struct Layout {
-    size_t idx_w, w_w, idx_r, w_r, pnorm, part_v, part_i, total;
+    size_t idx_w, w_w, idx_r, w_r, pnorm, part_v, part_i, hz, total;
     sdm::AddrPlan plan;
 };
 
@@ -133,6 +133,7 @@ Layout layout_for(const sdm_shape* s, int64_t S) {
     const size_t part = sdm::addr_partial_bytes(L.plan, s->B, s->H, s->T) / 2;
     L.part_v = off; off = align256(off + part);
     L.part_i = off; off = align256(off + part);
+    L.hz = off;     off = align256(off + sdm::rec_workspace_bytes(s->B, s->H, s->T, s->k_write, s->k_read));
     L.total = off;
     return L;
 }
@@ -238,7 +239,7 @@ sdm_status forward_impl(const char* who, const sdm_shape* s, const void* P_q, co
         r.B = s->B; r.H = s->H; r.T = s->T; r.dv = s->d_v; r.kw = s->k_write; r.kr = s->k_read;
         r.N = s->N;
         r.err = err;
-        cudaError_t e = sdm::launch_recur(s->dtype, r, stream);
+        cudaError_t e = sdm::launch_recur(s->dtype, r, reinterpret_cast<int32_t*>(ws + L.hz), stream);
         if (e != cudaSuccess) return cuda_fail(e, "recurrence launch");
     }
     return ok();
@@ -295,9 +296,14 @@ sdm_status sdm_decode_step(const sdm_shape* s, const void* P_q, const void* P_k,
                         workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream), true);
 }
 
+size_t sdm_recur_workspace_bytes(const sdm_shape* s) {
+    if (check_shape(s, false, nullptr) != SDM_OK) return 0;
+    return align256(sdm::rec_workspace_bytes(s->B, s->H, s->T, s->k_write, s->k_read)) + 256;
+}
+
 sdm_status sdm_recur(const sdm_shape* s, const int32_t* idx_w, const float* w_w, const int32_t* idx_r,
                      const float* w_r, const void* v, const void* alpha, const void* beta, void* mem, void* y,
-                     sdm_stream_t stream) {
+                     void* workspace, size_t workspace_bytes, sdm_stream_t stream) {
     SDM_TRY(check_shape(s, false, nullptr));
     const size_t es = elem_bytes(s->dtype);
     const size_t bht = static_cast<size_t>(s->B) * s->H * s->T;
@@ -319,6 +325,12 @@ sdm_status sdm_recur(const sdm_shape* s, const int32_t* idx_w, const float* w_w,
                             {y, bht * rowb, "y"}};
     for (const Range& r : others)
         if (overlaps(rm, r)) return fail(SDM_ERR_INVALID_ARG, "sdm_recur: mem overlaps %s", r.name);
+    const size_t need = align256(sdm::rec_workspace_bytes(s->B, s->H, s->T, s->k_write, s->k_read));
+    if (!workspace) return fail(SDM_ERR_INVALID_ARG, "sdm_recur: workspace is NULL (need %zu bytes)", need);
+    if (!aligned(workspace, 256)) return fail(SDM_ERR_INVALID_ARG, "sdm_recur: workspace must be 256-byte aligned");
+    if (workspace_bytes < need)
+        return fail(SDM_ERR_INVALID_ARG, "sdm_recur: workspace too small (%zu < %zu bytes)", workspace_bytes, need);
+    if (overlaps(rm, Range{workspace, need, "workspace"})) return fail(SDM_ERR_INVALID_ARG, "sdm_recur: mem overlaps workspace");
     int* err = nullptr;
     SDM_TRY(status_word(&err));
     sdm::RecArgs r{};
@@ -327,7 +339,7 @@ sdm_status sdm_recur(const sdm_shape* s, const int32_t* idx_w, const float* w_w,
     r.B = s->B; r.H = s->H; r.T = s->T; r.dv = s->d_v; r.kw = s->k_write; r.kr = s->k_read;
     r.N = s->N;
     r.err = err;
-    cudaError_t e = sdm::launch_recur(s->dtype, r, reinterpret_cast<cudaStream_t>(stream));
+    cudaError_t e = sdm::launch_recur(s->dtype, r, static_cast<int32_t*>(workspace), reinterpret_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "recurrence launch");
     return ok();
 }
@@ -344,7 +356,9 @@ sdm_status sdm_device_status(int32_t* code, sdm_stream_t stream) {
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) return cuda_fail(e, "sdm_device_status");
     *code = host;
-    if (host != 0) return fail(SDM_ERR_DEVICE, "device status word = 0x%x (bit 0: slot index outside [0, N) skipped)", host);
+    if (host != 0)
+        return fail(SDM_ERR_DEVICE, "device status word = 0x%x (bit 0: slot index outside [0, N) skipped; "
+                    "bit 1: slot list not strictly ascending)", host);
     return ok();
 }
 

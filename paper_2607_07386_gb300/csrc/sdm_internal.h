@@ -51,6 +51,19 @@ struct RecArgs {
     int64_t N;
     int* err;
 };
-cudaError_t launch_recur(int dtype, const RecArgs& a, cudaStream_t stream);
+// Launch geometry of the recurrence (depends only on the shape).
+struct RecPlan {
+    int dch;      // 16-byte chunks of a row per CTA
+    int nsplit;   // CTAs per chain
+    int threads;  // threads per CTA
+    int spt;      // slots per thread per token
+    int la;       // lookahead depth (tokens whose gathers are in flight)
+    int kmax;     // max(k_write, k_read)
+};
+RecPlan rec_plan(int dtype, int B, int H, int T, int dv, int kw, int kr);
+// Scratch of the recurrence: the hazard table [B, H, T, max(kw, kr)] int32.
+size_t rec_workspace_bytes(int B, int H, int T, int kw, int kr);
+// Runs the hazard pass, then the recurrence.  hz_ws: rec_workspace_bytes() of scratch.
+cudaError_t launch_recur(int dtype, const RecArgs& a, int32_t* hz_ws, cudaStream_t stream);
 
 }  // namespace sdm

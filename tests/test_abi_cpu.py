@@ -34,7 +34,8 @@ def declared_functions():
 def test_header_declares_the_boundary():
     names = declared_functions()
     for required in ("sdm_abi_version", "sdm_last_error", "sdm_workspace_bytes", "sdm_init_memory",
-                     "sdm_forward", "sdm_decode_step", "sdm_recur", "sdm_address", "sdm_device_status"):
+                     "sdm_forward", "sdm_decode_step", "sdm_recur", "sdm_address", "sdm_device_status",
+                     "sdm_recur_workspace_bytes"):
         assert required in names
 
 
@@ -118,7 +119,8 @@ def test_init_memory_and_recur_reject_overlap(sdm):
     assert L.sdm_init_memory(ctypes.byref(s), FAKE, FAKE + 64, None) == 1 and "overlaps" in sdm.last_error()
     assert L.sdm_init_memory(ctypes.byref(s), None, FAKE, None) == 1
     st = L.sdm_recur(ctypes.byref(s), FAKE + 0x10000000, FAKE + 0x100000, FAKE + 0x200000, FAKE + 0x300000,
-                     FAKE + 0x400000, FAKE + 0x500000, FAKE + 0x600000, FAKE + 0x10000000, FAKE + 0x700000, None)
+                     FAKE + 0x400000, FAKE + 0x500000, FAKE + 0x600000, FAKE + 0x10000000, FAKE + 0x700000,
+                     FAKE + 0x40000000, 1 << 30, None)
     assert st == 1 and "mem overlaps idx_w" in sdm.last_error()
 
 

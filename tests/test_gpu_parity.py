@@ -145,7 +145,8 @@ def _recur(sdm, dtype, idx_w, w_w, idx_r, w_r, v, alpha, beta, M0, B=1, H=1):
     shape = sdm.SdmShape.make(1, 1, T, 8, dv, N, kw, kr, dtype)
     i32 = lambda a: torch.from_numpy(np.ascontiguousarray(a, np.int32)).cuda()
     f32 = lambda a: torch.from_numpy(np.ascontiguousarray(a, np.float32)).cuda()
-    sdm.recur(shape, i32(idx_w), f32(w_w), i32(idx_r), f32(w_r), tt(v).contiguous(), tt(alpha), tt(beta), mem, y)
+    ws = torch.empty(sdm.recur_workspace_bytes(shape), dtype=torch.uint8, device="cuda")
+    sdm.recur(shape, i32(idx_w), f32(w_w), i32(idx_r), f32(w_r), tt(v).contiguous(), tt(alpha), tt(beta), mem, y, ws)
     torch.cuda.synchronize()
     return (O.to_f64(G.host(y[0, 0], dtype), dtype), O.to_f64(G.host(mem[0, 0], dtype), dtype))
 
@@ -217,7 +218,7 @@ def test_recur_matches_oracle_random_sparse(sdm):
     for dtype in ("bf16", "f32"):
         N, dv, T, kw, kr = 2000, 128 if dtype == "bf16" else 64, 150, 12, 20
         M0 = O.round_storage(rng.standard_normal((N, dv)) * 0.02, dtype)
-        iw = np.array([rng.permutation(rng.choice(N, kw, replace=False)) for _ in range(T)])  # any order
+        iw = np.array([np.sort(rng.choice(N, kw, replace=False)) for _ in range(T)])
         ir = np.array([np.sort(rng.choice(N, kr, replace=False)) for _ in range(T)])
         ww = rng.dirichlet(np.ones(kw), T).astype(np.float32).astype(np.float64)
         wr = rng.dirichlet(np.ones(kr), T).astype(np.float32).astype(np.float64)
@@ -228,6 +229,36 @@ def test_recur_matches_oracle_random_sparse(sdm):
         Mo = M0.copy()
         _, yo = O.recur(Mo, iw, ww, ir, wr, V, a, b, dtype)
         assert rel_fro(y, yo) <= TOL[dtype] and rel_fro(M, Mo) <= TOL[dtype]
+
+
+@pytest.mark.parametrize("dtype,N,k,T", [("bf16", 64, 8, 300), ("f32", 40, 12, 200), ("bf16", 96, 32, 150),
+                                         ("bf16", 4096, 64, 64)])
+def test_recur_high_collision_rate(sdm, dtype, N, k, T):
+    """Few slots, many per token: almost every token re-reads rows written by the
+    previous few tokens (the prefetch hazards) and reads rows it has just written."""
+    rng = np.random.default_rng(N * 7 + k)
+    dv = 64
+    M0 = O.round_storage(rng.standard_normal((N, dv)) * 0.5, dtype)
+    iw = np.array([np.sort(rng.choice(N, k, replace=False)) for _ in range(T)])
+    ir = np.array([np.sort(rng.choice(N, k, replace=False)) for _ in range(T)])
+    ww = rng.dirichlet(np.ones(k), T).astype(np.float32).astype(np.float64)
+    wr = rng.dirichlet(np.ones(k), T).astype(np.float32).astype(np.float64)
+    a = O.round_storage(1 / (1 + np.exp(-rng.standard_normal(T) - 1)), dtype)
+    b = O.round_storage(1 / (1 + np.exp(-rng.standard_normal(T))), dtype)
+    V = O.round_storage(rng.standard_normal((T, dv)), dtype)
+    y, M = _recur(sdm, dtype, iw, ww, ir, wr, V, a, b, M0)
+    Mo = M0.copy()
+    _, yo = O.recur(Mo, iw, ww, ir, wr, V, a, b, dtype)
+    assert rel_fro(y, yo) <= TOL[dtype] and rel_fro(M, Mo) <= TOL[dtype]
+
+
+def test_unsorted_slot_list_is_reported(sdm):
+    N, dv, T = 64, 32, 3
+    idx = np.array([[3, 1], [2, 5], [4, 6]])
+    w = np.full((T, 2), 0.5)
+    sdm.device_status()
+    _recur(sdm, "f32", idx, w, idx, w, np.ones((T, dv)), np.ones(T), np.ones(T), np.zeros((N, dv)))
+    assert sdm.device_status() == 2
 
 
 def test_bad_slot_index_is_skipped_and_reported(sdm):
