@@ -59,6 +59,7 @@ struct RecPlan {
     int spt;      // slots per thread per token
     int la;       // lookahead depth (tokens whose gathers are in flight)
     int kmax;     // max(k_write, k_read)
+    size_t smem;  // dynamic shared memory per CTA
 };
 RecPlan rec_plan(int dtype, int B, int H, int T, int dv, int kw, int kr);
 // Scratch of the recurrence: the hazard table [B, H, T, max(kw, kr)] int32.

@@ -263,7 +263,7 @@ def test_unsorted_slot_list_is_reported(sdm):
 
 def test_bad_slot_index_is_skipped_and_reported(sdm):
     N, dv, T = 64, 32, 4
-    idx = np.array([[0, 1], [2, N], [3, -1], [4, 5]])
+    idx = np.array([[0, 1], [2, N], [-1, 3], [4, 5]])   # ascending, two entries out of range
     w = np.full((T, 2), 0.5)
     z = np.zeros((N, dv))
     sdm.device_status()   # clear
