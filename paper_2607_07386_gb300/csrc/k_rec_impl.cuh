@@ -62,6 +62,20 @@ __host__ __device__ inline size_t rec_smem_bytes(int la, int ks, int dch) {
          + static_cast<size_t>(2 * la + 1) * rec_meta_stride(ks, dch);
 }
 
+// Shared-memory address helpers (32-bit shared-window addresses).
+__device__ __forceinline__ uint4 lds128(uint32_t addr) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];\n" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr));
+    return v;
+}
+__device__ __forceinline__ void sts128(uint32_t addr, const uint4& v, bool pred) {
+    if (pred) asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};\n" ::"r"(addr), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w) : "memory");
+}
+// 16-byte async copy global -> shared through L2 only; src_bytes = 0 writes zeros.
+__device__ __forceinline__ void cp_async16z(uint32_t dst, const void* src, int src_bytes) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+
 template <class D, int DCH, int SPT, int LA>
 __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const int32_t* __restrict__ hz, int kmax,
                                               int vec_lists) {
@@ -70,10 +84,14 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
     constexpr int KS = G * SPT;
     constexpr int KP = rec_ks_pad(KS);
     constexpr int MR = 2 * LA + 1;
+    constexpr int RING = LA + 1;
+    constexpr uint32_t SLOTB = DCH * 16;                 // bytes of one slot's d-range in a ring
     extern __shared__ __align__(16) unsigned char smR[];
-    uint4* rows = reinterpret_cast<uint4*>(smR);                                  // [LA][2][KS][DCH]
-    uint4* wring = rows + LA * 2 * KS * DCH;                                        // [LA+1][KS][DCH]
-    unsigned char* meta = reinterpret_cast<unsigned char*>(wring + (LA + 1) * KS * DCH);   // [MR][stride]
+    const uint32_t sm0 = static_cast<uint32_t>(__cvta_generic_to_shared(smR));
+    const uint32_t rows0 = sm0;                                              // [LA][2][KS][DCH] x 16 B
+    const uint32_t wring0 = rows0 + LA * 2 * KS * SLOTB;                     // [RING][KS][DCH] x 16 B
+    const uint32_t meta0 = wring0 + RING * KS * SLOTB;                       // [MR][stride]
+    unsigned char* meta_gen = smR + (meta0 - sm0);
     const int meta_stride = static_cast<int>(rec_meta_stride(KS, DCH));
 
     const int lane = threadIdx.x;
@@ -82,35 +100,54 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
     const int kw = a.kw, kr = a.kr;
     const int64_t chain = blockIdx.x / nsplit;
     const int split = blockIdx.x - static_cast<int>(chain) * nsplit;
-    const int64_t rowbytes = static_cast<int64_t>(a.dv) * D::BYTES;
+    const uint32_t rowbytes = static_cast<uint32_t>(a.dv) * D::BYTES;
     const int64_t dbyte = static_cast<int64_t>(split * DCH) * 16;
-    char* Mb = static_cast<char*>(a.mem) + chain * a.N * rowbytes + dbyte + c * 16;
-    const char* vrange = static_cast<const char*>(a.v) + chain * a.T * rowbytes + dbyte;
-    char* yb = static_cast<char*>(a.y) + chain * a.T * rowbytes + dbyte + c * 16;
+    const char* Mc = static_cast<const char*>(a.mem) + chain * a.N * static_cast<int64_t>(rowbytes) + dbyte + c * 16;
+    char* Mw = const_cast<char*>(Mc);
+    const char* vrange = static_cast<const char*>(a.v) + chain * a.T * static_cast<int64_t>(rowbytes) + dbyte;
+    char* yb = static_cast<char*>(a.y) + chain * a.T * static_cast<int64_t>(rowbytes) + dbyte + c * 16;
     const int T = a.T;
     const int64_t tok0 = chain * T;
-    const int N = static_cast<int>(a.N);
+    const uint32_t N = static_cast<uint32_t>(a.N);
+    // my slots n = g*SPT + j: rows-ring / written-ring offsets of slot j = 0, chunk c
+    const uint32_t my_rows = rows0 + (g * SPT * DCH + c) * 16;
+    const uint32_t my_wring = wring0 + (g * SPT * DCH + c) * 16;
+    const uint32_t wring_c = wring0 + c * 16;
+    bool my_w[SPT], my_r[SPT];
+#pragma unroll
+    for (int j = 0; j < SPT; ++j) { my_w[j] = g * SPT + j < kw; my_r[j] = g * SPT + j < kr; }
 
-    auto mptr = [&](int slot) { return reinterpret_cast<int*>(meta + slot * meta_stride); };
+    // per-lane pieces of a token's lists (16-byte copies when vec_lists): source base, stride, offset
+    const int qw = kw / 4, qr = kr / 4, qm = kmax / 4;
+    const int npieces = 2 * qw + 2 * qr + qm;
+    const char* psrc[3];
+    uint32_t pstride[3], poff[3];
+    bool pvalid[3];
+#pragma unroll
+    for (int q = 0; q < 3; ++q) {
+        const int p = lane + 32 * q;
+        pvalid[q] = vec_lists && p < npieces;
+        const char* src = reinterpret_cast<const char*>(a.idx_w);
+        uint32_t stride = kw * 4, off = 0, sub = 0;
+        if (p < qw) { src = reinterpret_cast<const char*>(a.idx_w); stride = kw * 4; off = 0; sub = p; }
+        else if (p < 2 * qw) { src = reinterpret_cast<const char*>(a.w_w); stride = kw * 4; off = KP * 4; sub = p - qw; }
+        else if (p < 2 * qw + qr) { src = reinterpret_cast<const char*>(a.idx_r); stride = kr * 4; off = 2 * KP * 4; sub = p - 2 * qw; }
+        else if (p < 2 * qw + 2 * qr) { src = reinterpret_cast<const char*>(a.w_r); stride = kr * 4; off = 3 * KP * 4; sub = p - 2 * qw - qr; }
+        else { src = reinterpret_cast<const char*>(hz); stride = kmax * 4; off = 4 * KP * 4; sub = p - 2 * qw - 2 * qr; }
+        psrc[q] = src + tok0 * stride + sub * 16;
+        pstride[q] = stride;
+        poff[q] = off + sub * 16;
+    }
 
-    // copy token t's lists (and v chunk) into meta slot t % MR
-    auto copy_meta = [&](int t) {
+    auto copy_meta = [&](int t, uint32_t slot_addr) {
         if (t >= T) return;
-        int* dst = mptr(t % MR);
-        const int64_t tok = tok0 + t;
-        if (vec_lists) {   // k multiple of 4 and 16-byte aligned arrays: 16-byte pieces
-            const int qw = kw / 4, qr = kr / 4, qm = kmax / 4;
-            for (int p = lane; p < 2 * qw + 2 * qr + qm; p += 32) {
-                const void* src;
-                int* d;
-                if (p < qw) { src = a.idx_w + tok * kw + 4 * p; d = dst + 4 * p; }
-                else if (p < 2 * qw) { src = a.w_w + tok * kw + 4 * (p - qw); d = dst + KP + 4 * (p - qw); }
-                else if (p < 2 * qw + qr) { src = a.idx_r + tok * kr + 4 * (p - 2 * qw); d = dst + 2 * KP + 4 * (p - 2 * qw); }
-                else if (p < 2 * qw + 2 * qr) { src = a.w_r + tok * kr + 4 * (p - 2 * qw - qr); d = dst + 3 * KP + 4 * (p - 2 * qw - qr); }
-                else { src = hz + tok * kmax + 4 * (p - 2 * qw - 2 * qr); d = dst + 4 * KP + 4 * (p - 2 * qw - 2 * qr); }
-                cp_async16(d, src);
-            }
+        if (vec_lists) {
+#pragma unroll
+            for (int q = 0; q < 3; ++q)
+                if (pvalid[q]) cp_async16z(slot_addr + poff[q], psrc[q] + static_cast<int64_t>(t) * pstride[q], 16);
         } else {
+            int* dst = reinterpret_cast<int*>(meta_gen + (slot_addr - meta0));
+            const int64_t tok = tok0 + t;
             for (int p = lane; p < 2 * kw + 2 * kr + kmax; p += 32) {
                 const void* src;
                 int* d;
@@ -122,21 +159,21 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
                 cp_async4(d, src);
             }
         }
-        if (lane < DCH) cp_async16(reinterpret_cast<unsigned char*>(dst) + 5 * KP * 4 + lane * 16, vrange + t * rowbytes + lane * 16);
+        if (lane < DCH) cp_async16z(slot_addr + 5 * KP * 4 + lane * 16, vrange + static_cast<int64_t>(t) * rowbytes + lane * 16, 16);
     };
-    // rows that token t gathers (own slots, own chunk) -> rows slot t % LA
-    auto copy_rows = [&](int t) {
+    // rows that token t gathers (own slots, own chunk), zero-filled for invalid slots
+    auto copy_rows = [&](int t, uint32_t meta_addr, uint32_t rows_slot) {
         if (t >= T) return;
-        const int* m = mptr(t % MR);
-        const int slot = t % LA;
+        const int* m = reinterpret_cast<const int*>(meta_gen + (meta_addr - meta0));
         int iw[SPT], ir[SPT];
         lds_vec<SPT>(m + g * SPT, iw);
         lds_vec<SPT>(m + 2 * KP + g * SPT, ir);
 #pragma unroll
         for (int j = 0; j < SPT; ++j) {
-            const int n = g * SPT + j;
-            if (n < kw && iw[j] >= 0 && iw[j] < N) cp_async16(&rows[((slot * 2 + 0) * KS + n) * DCH + c], Mb + iw[j] * rowbytes);
-            if (n < kr && ir[j] >= 0 && ir[j] < N) cp_async16(&rows[((slot * 2 + 1) * KS + n) * DCH + c], Mb + ir[j] * rowbytes);
+            const bool ow = my_w[j] && static_cast<uint32_t>(iw[j]) < N;
+            const bool orr = my_r[j] && static_cast<uint32_t>(ir[j]) < N;
+            cp_async16z(rows_slot + j * SLOTB, Mc + static_cast<uint64_t>(ow ? iw[j] : 0) * rowbytes, ow ? 16 : 0);
+            cp_async16z(rows_slot + KS * SLOTB + j * SLOTB, Mc + static_cast<uint64_t>(orr ? ir[j] : 0) * rowbytes, orr ? 16 : 0);
         }
     };
 
@@ -145,16 +182,18 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
     if (lane < T) { a_nxt = load_elem<D>(a.alpha, tok0 + lane); b_nxt = load_elem<D>(a.beta, tok0 + lane); }
 
     // prologue: lists of tokens [0, LA); then rows of [0, LA) with lists of [LA, 2LA)
-    for (int u = 0; u < LA; ++u) copy_meta(u);
+    for (int u = 0; u < LA; ++u) copy_meta(u, meta0 + u * meta_stride);
     cp_async_commit();
     cp_async_wait<0>();
     __syncwarp();
     for (int u = 0; u < LA; ++u) {
-        copy_rows(u);
-        copy_meta(u + LA);
+        copy_rows(u, meta0 + u * meta_stride, my_rows + u * 2 * KS * SLOTB);
+        copy_meta(u + LA, meta0 + (u + LA) * meta_stride);
         cp_async_commit();
     }
 
+    bool bad = false;
+    int ms = 0, rs = 0, ws = 0;                  // ring positions of token t: t % MR, t % LA, t % RING
     for (int t = 0; t < T; ++t) {
         if ((t & 31) == 0) {
             a_cur = a_nxt; b_cur = b_nxt;
@@ -165,8 +204,9 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
         const float beta = __shfl_sync(0xffffffffu, b_cur, t & 31);
         cp_async_wait<LA - 1>();        // own rows of token t and lists of token t+LA have landed
         __syncwarp();                   // ... and everyone's; written ring of earlier tokens visible
-        const int* m = mptr(t % MR);
-        const int rs = t % LA, wsl = t % (LA + 1);
+        const uint32_t mslot = meta0 + ms * meta_stride;
+        const int* m = reinterpret_cast<const int*>(meta_gen + ms * meta_stride);
+        const uint32_t rslot = my_rows + rs * 2 * KS * SLOTB;
         int iw[SPT], ir[SPT], hzv[SPT];
         float ww[SPT], wr[SPT];
         lds_vec<SPT>(m + g * SPT, iw);
@@ -175,56 +215,40 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
         lds_vec<SPT>(m + 3 * KP + g * SPT, *reinterpret_cast<int(*)[SPT]>(wr));
         lds_vec<SPT>(m + 4 * KP + g * SPT, hzv);
 
-        // ---- gathers (stale rows from the ring), decay, partial prediction and partial read
+        // ---- gathers (stale rows replaced from the written ring), decay, partial sums
         float r[SPT][E];
         float pp[E], yp[E];
 #pragma unroll
         for (int e = 0; e < E; ++e) { pp[e] = 0.f; yp[e] = 0.f; }
         bool fix = false;
+        bool okw[SPT];
 #pragma unroll
         for (int j = 0; j < SPT; ++j) {
-            const int n = g * SPT + j;
-            const bool okw = n < kw && iw[j] >= 0 && iw[j] < N;
-            const bool okr = n < kr && ir[j] >= 0 && ir[j] < N;
-            if ((n < kw && !okw) || (n < kr && !okr)) flag_error(a.err, ERR_BAD_INDEX);
-            // entries of unused or invalid slots are never filled: they are not read at all
-            uint4 mw = make_uint4(0, 0, 0, 0);
-            if (okw) {
-                mw = rows[((rs * 2 + 0) * KS + n) * DCH + c];
-                const int hw = hzv[j] & 0xffff;
-                if (hw) {
-                    const int d = (hw - 1) >> 6, np = (hw - 1) & 63;
-                    mw = wring[(((t - d) % (LA + 1)) * KS + np) * DCH + c];
-                }
-            }
-            float f[E];
+            okw[j] = my_w[j] && static_cast<uint32_t>(iw[j]) < N;
+            const bool okr = my_r[j] && static_cast<uint32_t>(ir[j]) < N;
+            bad |= (my_w[j] && !okw[j]) || (my_r[j] && !okr);
+            const int hw = hzv[j] & 0xffff;
+            const int hr = (hzv[j] >> 16) & 0xffff;
+            const int dw = (hw - 1) >> 6, dr = (hr - 1) >> 6;
+            int rw = ws - dw; rw += rw < 0 ? RING : 0;
+            int rr = ws - dr; rr += rr < 0 ? RING : 0;
+            const uint32_t aw = hw ? wring_c + (rw * KS + ((hw - 1) & 63)) * SLOTB : rslot + j * SLOTB;
+            const bool rfix = hr && dr == 0;             // slot written by this token: added after the write
+            const uint32_t ar = (hr && !rfix) ? wring_c + (rr * KS + ((hr - 1) & 63)) * SLOTB : rslot + (KS + j) * SLOTB;
+            fix |= rfix && okr;
+            const uint4 mw = lds128(aw);
+            const uint4 mr = lds128(ar);
+            float f[E], h[E];
             unpack16<D>(mw, f);
-            const float wj = okw ? ww[j] : 0.f;
+            unpack16<D>(mr, h);
+            const float wj = okw[j] ? ww[j] : 0.f;
+            const float rho = (okr && !rfix) ? wr[j] : 0.f;
 #pragma unroll
             for (int e = 0; e < E; ++e) {
                 r[j][e] = alpha * f[e];
                 pp[e] = fmaf(wj, r[j][e], pp[e]);
+                yp[e] = fmaf(rho, h[e], yp[e]);
             }
-            uint4 mr = make_uint4(0, 0, 0, 0);
-            float rho = 0.f;
-            if (okr) {
-                const int hr = (hzv[j] >> 16) & 0xffff;
-                rho = wr[j];
-                mr = rows[((rs * 2 + 1) * KS + n) * DCH + c];
-                if (hr) {
-                    const int d = (hr - 1) >> 6, np = (hr - 1) & 63;
-                    if (d > 0) {
-                        mr = wring[(((t - d) % (LA + 1)) * KS + np) * DCH + c];
-                    } else {
-                        fix = true;     // value written by this token: added after the write
-                        rho = 0.f;
-                        mr = make_uint4(0, 0, 0, 0);
-                    }
-                }
-            }
-            unpack16<D>(mr, f);
-#pragma unroll
-            for (int e = 0; e < E; ++e) yp[e] = fmaf(rho, f[e], yp[e]);
         }
 #pragma unroll
         for (int off = DCH; off < 32; off <<= 1) {
@@ -236,21 +260,19 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
         }
         // ---- delta = v - v~ and the write
         float delta[E];
-        unpack16<D>(*reinterpret_cast<const uint4*>(reinterpret_cast<const unsigned char*>(m) + 5 * KP * 4 + c * 16), delta);
+        unpack16<D>(lds128(mslot + 5 * KP * 4 + c * 16), delta);
 #pragma unroll
         for (int e = 0; e < E; ++e) delta[e] -= pp[e];
+        const uint32_t wslot = my_wring + ws * KS * SLOTB;
 #pragma unroll
         for (int j = 0; j < SPT; ++j) {
-            const int n = g * SPT + j;
-            if (n < kw && iw[j] >= 0 && iw[j] < N) {
-                const float bw = beta * ww[j];
-                float o[E];
+            const float bw = beta * ww[j];
+            float o[E];
 #pragma unroll
-                for (int e = 0; e < E; ++e) o[e] = fmaf(bw, delta[e], r[j][e]);
-                const uint4 packed = pack16<D>(o);
-                *reinterpret_cast<uint4*>(Mb + iw[j] * rowbytes) = packed;
-                wring[(wsl * KS + n) * DCH + c] = packed;
-            }
+            for (int e = 0; e < E; ++e) o[e] = fmaf(bw, delta[e], r[j][e]);
+            const uint4 packed = pack16<D>(o);
+            if (okw[j]) *reinterpret_cast<uint4*>(Mw + static_cast<uint64_t>(iw[j]) * rowbytes) = packed;
+            sts128(wslot + j * SLOTB, packed, okw[j]);
         }
         // ---- reads of slots this token wrote (rare): recompute the writer's value
         if (__any_sync(0xffffffffu, fix)) {
@@ -259,18 +281,18 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
             for (int e = 0; e < E; ++e) yc[e] = 0.f;
 #pragma unroll
             for (int j = 0; j < SPT; ++j) {
-                const int n = g * SPT + j;
                 const int hr = (hzv[j] >> 16) & 0xffff;
-                if (n < kr && ir[j] >= 0 && ir[j] < N && hr && ((hr - 1) >> 6) == 0) {
+                const bool okr = my_r[j] && static_cast<uint32_t>(ir[j]) < N;
+                if (okr && hr && ((hr - 1) >> 6) == 0) {
                     const int np = (hr - 1) & 63;
                     const int hwn = m[4 * KP + np] & 0xffff;        // the writer's own hazard code
-                    uint4 base = rows[((rs * 2 + 1) * KS + n) * DCH + c];   // same prefetch as the writer's
+                    uint32_t ab = rslot + (KS + j) * SLOTB;       // same prefetch as the writer's
                     if (hwn) {
-                        const int d2 = (hwn - 1) >> 6, np2 = (hwn - 1) & 63;
-                        base = wring[(((t - d2) % (LA + 1)) * KS + np2) * DCH + c];
+                        int rw = ws - ((hwn - 1) >> 6); rw += rw < 0 ? RING : 0;
+                        ab = wring_c + (rw * KS + ((hwn - 1) & 63)) * SLOTB;
                     }
                     float f[E], o[E];
-                    unpack16<D>(base, f);
+                    unpack16<D>(lds128(ab), f);
                     const float bw = beta * __int_as_float(m[KP + np]);
 #pragma unroll
                     for (int e = 0; e < E; ++e) o[e] = fmaf(bw, delta[e], alpha * f[e]);
@@ -288,13 +310,21 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
 #pragma unroll
             for (int e = 0; e < E; ++e) yp[e] += yc[e];
         }
-        if (g == 0) *reinterpret_cast<uint4*>(yb + t * rowbytes) = pack16<D>(yp);
-        // ---- prefetch: rows of token t+LA, lists of token t+2LA (the slot of token t-1)
-        copy_rows(t + LA);
-        copy_meta(t + 2 * LA);
-        cp_async_commit();
+        if (g == 0) *reinterpret_cast<uint4*>(yb + static_cast<int64_t>(t) * rowbytes) = pack16<D>(yp);
+        // ---- prefetch: rows of token t+LA (rows slot of token t), lists of token t+2LA (slot of t-1)
+        {
+            int mfut = ms + LA; mfut -= mfut >= MR ? MR : 0;
+            copy_rows(t + LA, meta0 + mfut * meta_stride, rslot);
+            int mnew = ms + 2 * LA; mnew -= mnew >= MR ? MR : 0;
+            copy_meta(t + 2 * LA, meta0 + mnew * meta_stride);
+            cp_async_commit();
+        }
+        ms = ms + 1 == MR ? 0 : ms + 1;
+        rs = rs + 1 == LA ? 0 : rs + 1;
+        ws = ws + 1 == RING ? 0 : ws + 1;
     }
     cp_async_wait<0>();
+    if (__any_sync(0xffffffffu, bad) && lane == 0) flag_error(a.err, ERR_BAD_INDEX);
 }
 
 template <class D, int DCH, int SPT, int LA>
