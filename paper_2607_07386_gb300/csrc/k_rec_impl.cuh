@@ -227,8 +227,9 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
             okw[j] = my_w[j] && static_cast<uint32_t>(iw[j]) < N;
             const bool okr = my_r[j] && static_cast<uint32_t>(ir[j]) < N;
             bad |= (my_w[j] && !okw[j]) || (my_r[j] && !okr);
-            const int hw = hzv[j] & 0xffff;
-            const int hr = (hzv[j] >> 16) & 0xffff;
+            // hazard codes of unused or invalid slots are garbage: never decode them
+            const int hw = okw[j] ? (hzv[j] & 0xffff) : 0;
+            const int hr = okr ? ((hzv[j] >> 16) & 0xffff) : 0;
             const int dw = (hw - 1) >> 6, dr = (hr - 1) >> 6;
             int rw = ws - dw; rw += rw < 0 ? RING : 0;
             int rr = ws - dr; rr += rr < 0 ? RING : 0;
