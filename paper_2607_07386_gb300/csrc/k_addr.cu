@@ -293,10 +293,213 @@ __device__ __noinline__ void resolve_combined(const float* cv, const int* cf, in
 }
 
 // ------------------------------------------------------------------------------------------
-// Kernel B: merge, certify, combine, softmax, sort by slot
+// Kernel B (k <= 32): merge, certify, combine, softmax, sort by slot -- branch-free common path
 // ------------------------------------------------------------------------------------------
+// Bitonic networks on per-thread register arrays (descending by value / ascending by key).
+template <int N>
+__device__ __forceinline__ void net_desc(float (&v)[N], int (&ix)[N]) {
+#pragma unroll
+    for (int size = 2; size <= N; size <<= 1)
+#pragma unroll
+        for (int stride = size >> 1; stride > 0; stride >>= 1)
+#pragma unroll
+            for (int i = 0; i < N; ++i) {
+                const int j = i ^ stride;
+                if (j > i) {
+                    const bool up = (i & size) == 0;
+                    const bool sw = up ? (v[i] < v[j]) : (v[i] > v[j]);
+                    const float x = v[i];
+                    const int xi = ix[i];
+                    v[i] = sw ? v[j] : x;   ix[i] = sw ? ix[j] : xi;
+                    v[j] = sw ? x : v[j];   ix[j] = sw ? xi : ix[j];
+                }
+            }
+}
+template <int N>
+__device__ __forceinline__ void net_asc_key(int (&key)[N], float (&val)[N]) {
+#pragma unroll
+    for (int size = 2; size <= N; size <<= 1)
+#pragma unroll
+        for (int stride = size >> 1; stride > 0; stride >>= 1)
+#pragma unroll
+            for (int i = 0; i < N; ++i) {
+                const int j = i ^ stride;
+                if (j > i) {
+                    const bool up = (i & size) == 0;
+                    const bool sw = up ? (key[i] > key[j]) : (key[i] < key[j]);
+                    const int x = key[i];
+                    const float xv = val[i];
+                    key[i] = sw ? key[j] : x;   val[i] = sw ? val[j] : xv;
+                    key[j] = sw ? x : key[j];   val[j] = sw ? xv : val[j];
+                }
+            }
+}
+
+constexpr int CBUF = 64;   // candidate buffer per thread (= network size)
+
+// Sort the first CBUF entries of a per-thread buffer (value desc); entries >= cnt count as -inf.
+__device__ __forceinline__ void sort_buffer(float* bv, int* bi, int cnt) {
+    float v[CBUF];
+    int ix[CBUF];
+#pragma unroll
+    for (int i = 0; i < CBUF; ++i) {
+        v[i] = i < cnt ? bv[i * F_THREADS] : -INFINITY;
+        ix[i] = i < cnt ? bi[i * F_THREADS] : INT_MAX;
+    }
+    net_desc<CBUF>(v, ix);
+#pragma unroll
+    for (int i = 0; i < CBUF; ++i) { bv[i * F_THREADS] = v[i]; bi[i * F_THREADS] = ix[i]; }
+}
+
 template <class D, int L>
 __global__ void __launch_bounds__(F_THREADS) k_addr_finalize(const AddrArgs a) {
+    static_assert(L <= 36, "network finalize handles k <= 32");
+    extern __shared__ __align__(16) float smB[];
+    const int tid = threadIdx.x;
+    // per-thread regions, pitch F_THREADS: half lists H1, H2 (L), merge scratch M (L),
+    // candidates C (CBUF), final selection F (L)
+    float* H1v = smB + tid;                 int* H1i = reinterpret_cast<int*>(H1v + L * F_THREADS);
+    float* H2v = smB + 2 * L * F_THREADS + tid; int* H2i = reinterpret_cast<int*>(H2v + L * F_THREADS);
+    float* Mv = smB + 4 * L * F_THREADS + tid;  int* Mi = reinterpret_cast<int*>(Mv + L * F_THREADS);
+    float* Cv = smB + 6 * L * F_THREADS + tid;  int* Ci = reinterpret_cast<int*>(Cv + CBUF * F_THREADS);
+    float* Fv = smB + (6 * L + 2 * CBUF) * F_THREADS + tid; int* Fi = reinterpret_cast<int*>(Fv + L * F_THREADS);
+
+    const int side = blockIdx.y / a.H, h = blockIdx.y % a.H;
+    const int64_t BT = static_cast<int64_t>(a.B) * a.T;
+    const int64_t u = static_cast<int64_t>(blockIdx.x) * F_THREADS + tid;
+    const bool live = u < BT;            // dead lanes run along (warp votes below) but store nothing
+    const int k = a.kk[side];
+    const int S = a.S;
+    const int64_t uu = live ? u : 0;
+    const int64_t b = uu / a.T, t = uu - b * a.T;
+    TokenCtx c;
+    c.P = a.P[side];
+    c.X = a.X[side];
+    c.xoff = ((b * a.H + h) * a.T + t) * a.dk;
+    c.prow0 = static_cast<int64_t>(h) * 2 * S;
+    c.dk = a.dk;
+    c.S = S;
+
+    double eps = 0.0;
+    if (c.P != nullptr) {
+        float ss = 0.f;
+        for (int d = 0; d < a.dk; ++d) {
+            const float xv = load_elem<D>(c.X, c.xoff + d);
+            ss = fmaf(xv, xv, ss);
+        }
+        eps = static_cast<double>(a.cbound) * static_cast<double>(a.pnorm[side * a.H + h]) *
+              static_cast<double>(sqrtf(ss)) * (1.0 + 0x1p-12);
+    }
+
+    float amax[2];
+#pragma unroll 1
+    for (int hf = 0; hf < 2; ++hf) {
+        float* Hv = hf ? H2v : H1v;
+        int* Hi = hf ? H2i : H1i;
+        // chunk lists of this half (each sorted desc) merged with two pointers
+        for (int cc = 0; cc < a.ncc; ++cc) {
+            const int64_t base = ((static_cast<int64_t>(blockIdx.y) * (2 * a.ncc) + hf * a.ncc + cc) * L) * BT + uu;
+            float* dv = cc == 0 ? Hv : Mv;
+            int* di = cc == 0 ? Hi : Mi;
+            for (int p = 0; p < L; ++p) { dv[p * F_THREADS] = a.part_v[base + p * BT]; di[p * F_THREADS] = a.part_i[base + p * BT]; }
+            if (cc > 0) {
+                int ia = 0, ib = 0;
+                for (int p = 0; p < L; ++p) {
+                    const float va = ia < L ? Hv[ia * F_THREADS] : -INFINITY;
+                    const float vb = ib < L ? Mv[ib * F_THREADS] : -INFINITY;
+                    const bool ta = va >= vb;        // ties: the earlier chunk (smaller columns)
+                    Cv[p * F_THREADS] = ta ? va : vb;
+                    Ci[p * F_THREADS] = ta ? Hi[ia * F_THREADS] : Mi[ib * F_THREADS];
+                    ia += ta ? 1 : 0;
+                    ib += ta ? 0 : 1;
+                }
+                for (int p = 0; p < L; ++p) { Hv[p * F_THREADS] = Cv[p * F_THREADS]; Hi[p * F_THREADS] = Ci[p * F_THREADS]; }
+            }
+        }
+        bool certified = (S <= k);
+        if (!certified) certified = static_cast<double>(Hv[(k - 1) * F_THREADS]) - static_cast<double>(Hv[k * F_THREADS]) > 2.0 * eps;
+        if (!certified && live) {
+            float lv[L];
+            int li[L];
+            for (int p = 0; p < L; ++p) { lv[p] = Hv[p * F_THREADS]; li[p] = Hi[p * F_THREADS]; }
+            resolve_half<D, L>(lv, li, k, eps, c, hf, Hv, Hi);
+        }
+        amax[hf] = fmaxf(fabsf(Hv[0]), fabsf(Hv[(k - 1) * F_THREADS]));
+    }
+
+    // Outer-sum candidates.  theta = max over a of H1[a-1] + H2[ceil(k/a)-1]: the first a
+    // rows times the first ceil(k/a) columns give >= k sums >= it (rounding is monotone).
+    const double epsc = 2.0 * eps + 0x1p-22 * (static_cast<double>(amax[0]) + static_cast<double>(amax[1]));
+    float theta = -INFINITY;
+    for (int aa = 1; aa <= k; ++aa) theta = fmaxf(theta, H1v[(aa - 1) * F_THREADS] + H2v[((k + aa - 1) / aa - 1) * F_THREADS]);
+    const float lo = __double2float_rd(static_cast<double>(theta) - 2.0 * epsc);
+    int cnt = 0;
+    for (int p1 = 0; p1 < k; ++p1) {                        // k is warp-uniform per side
+        const float a1 = H1v[p1 * F_THREADS];
+        const int i1 = H1i[p1 * F_THREADS];
+        bool act = live && a1 + H2v[0] >= lo;
+        if (!__any_sync(0xffffffffu, act)) break;          // rows are sorted: the rest are below lo
+        for (int p2 = 0; p2 < k; ++p2) {
+            const float cs = a1 + H2v[p2 * F_THREADS];
+            act = act && cs >= lo;
+            if (!__any_sync(0xffffffffu, act)) break;
+            if (act) {
+                Cv[cnt * F_THREADS] = cs;
+                Ci[cnt * F_THREADS] = i1 * S + H2i[p2 * F_THREADS];
+                ++cnt;
+            }
+            if (__any_sync(0xffffffffu, cnt == CBUF)) {      // flush: keep the best L
+                sort_buffer(Cv, Ci, cnt);
+                cnt = min(cnt, L);
+            }
+        }
+    }
+    sort_buffer(Cv, Ci, cnt);
+    bool certified = (k == 1) || (cnt <= k);
+    if (!certified) certified = static_cast<double>(Cv[(k - 1) * F_THREADS]) - static_cast<double>(Cv[k * F_THREADS]) > 2.0 * epsc;
+    if (certified) {
+        for (int p = 0; p < k; ++p) { Fv[p * F_THREADS] = Cv[p * F_THREADS]; Fi[p * F_THREADS] = Ci[p * F_THREADS]; }
+    } else if (live) {
+        float cv[L];
+        int cf[L];
+        for (int p = 0; p < L; ++p) {
+            cv[p] = p < cnt ? Cv[p * F_THREADS] : -INFINITY;
+            cf[p] = p < cnt ? Ci[p * F_THREADS] : INT_MAX;
+        }
+        resolve_combined<D, L>(cv, cf, k, epsc, c, H1v, H1i, H2v, H2i, Fv, Fi);
+    }
+
+    // softmax over the selected scores, then ascending slot order (network on <= 32 pairs)
+    float m = -INFINITY;
+    for (int p = 0; p < k; ++p) m = fmaxf(m, Fv[p * F_THREADS]);
+    int key[32];
+    float val[32];
+    float z = 0.f;
+#pragma unroll
+    for (int p = 0; p < 32; ++p) {
+        const bool in = p < k;
+        const float e = in ? expf(Fv[p * F_THREADS] - m) : 0.f;
+        key[p] = in ? Fi[p * F_THREADS] : INT_MAX;
+        val[p] = e;
+        z += e;
+    }
+    net_asc_key<32>(key, val);
+    if (live) {
+        const float rz = 1.f / z;
+        const int64_t tokoff = ((b * a.H + h) * a.T + t) * k;     // [B, H, T, k] layout
+        int32_t* oi = a.idx[side] + tokoff;
+        float* ow = a.w[side] + tokoff;
+#pragma unroll
+        for (int p = 0; p < 32; ++p)
+            if (p < k) { oi[p] = key[p]; ow[p] = val[p] * rz; }
+    }
+}
+
+// ------------------------------------------------------------------------------------------
+// Kernel B, wide lists (k > 32): insertion-based merge and candidate selection
+// ------------------------------------------------------------------------------------------
+template <class D, int L>
+__global__ void __launch_bounds__(F_THREADS) k_addr_finalize_wide(const AddrArgs a) {
     extern __shared__ __align__(16) float smB[];
     const int tid = threadIdx.x;
     float* A1v = smB + tid;                       // exact top-k of half 1 (fp32 value, column), pitch F_THREADS
@@ -459,13 +662,15 @@ __global__ void __launch_bounds__(256) k_pnorm(const AddrArgs a) {
 // ------------------------------------------------------------------------------------------
 // host side
 // ------------------------------------------------------------------------------------------
-AddrPlan addr_plan(int B, int H, int T, int S, int kmax) {
+AddrPlan addr_plan(int dtype, int direct, int B, int H, int T, int dk, int S, int kmax) {
     AddrPlan p;
     p.L = (kmax <= 8 ? 8 : kmax <= 16 ? 16 : kmax <= 32 ? 32 : 64) + 4;
+    p.mma = mma_path_supported(dtype, direct, dk, S, kmax);
     const int64_t tiles = (static_cast<int64_t>(B) * T + A_TOK - 1) / A_TOK;
     const int64_t base = 2LL * H * tiles * 2;   // sides x heads x token tiles x halves
     int ncc = 1;
-    while (base * ncc < 512 && (S / (2 * ncc)) >= A_SUB) ncc *= 2;
+    while ((S + ncc - 1) / ncc > 512) ncc *= 2;                      // chunks of <= 512 columns
+    while (base * ncc < 512 && (S / (2 * ncc)) >= 64) ncc *= 2;      // enough CTAs, chunks >= 64 columns
     p.ncc = ncc;
     p.cw = (S + ncc - 1) / ncc;
     return p;
@@ -476,22 +681,41 @@ size_t addr_partial_bytes(const AddrPlan& plan, int B, int H, int T) {
 }
 
 template <class D, int L>
+static cudaError_t launch_finalize(const AddrArgs& a, cudaStream_t stream) {
+    const int64_t BT = static_cast<int64_t>(a.B) * a.T;
+    dim3 gB(static_cast<unsigned>((BT + F_THREADS - 1) / F_THREADS), 2 * a.H);
+    cudaError_t e;
+    if constexpr (L <= 36) {
+        const size_t smB = static_cast<size_t>(2) * (4 * L + 2 * CBUF) * F_THREADS * sizeof(float);
+        e = cudaFuncSetAttribute(k_addr_finalize<D, L>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smB));
+        if (e != cudaSuccess) return e;
+        k_addr_finalize<D, L><<<gB, F_THREADS, smB, stream>>>(a);
+    } else {
+        const size_t smB = static_cast<size_t>(6) * L * F_THREADS * sizeof(float);
+        e = cudaFuncSetAttribute(k_addr_finalize_wide<D, L>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smB));
+        if (e != cudaSuccess) return e;
+        k_addr_finalize_wide<D, L><<<gB, F_THREADS, smB, stream>>>(a);
+    }
+    return cudaGetLastError();
+}
+
+template <class D, int L>
 static cudaError_t launch_typed(const AddrPlan& plan, const AddrArgs& a, cudaStream_t stream) {
     const int64_t BT = static_cast<int64_t>(a.B) * a.T;
     if (a.P[0] != nullptr) {
         k_pnorm<D><<<2 * a.H, 256, 0, stream>>>(a);
+    }
+    if (plan.mma) {
+        cudaError_t e = launch_address_mma(plan, a, stream);
+        if (e != cudaSuccess) return e;
+        return launch_finalize<D, L>(a, stream);
     }
     const size_t smA = (static_cast<size_t>(a.dk) * A_TOK + (a.P[0] ? static_cast<size_t>(a.dk) * A_PPITCH : 0)) * sizeof(float);
     cudaError_t e = cudaFuncSetAttribute(k_addr_scores<D, L>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smA));
     if (e != cudaSuccess) return e;
     dim3 gA(static_cast<unsigned>((BT + A_TOK - 1) / A_TOK), 2 * plan.ncc, 2 * a.H);
     k_addr_scores<D, L><<<gA, A_TOK, smA, stream>>>(a);
-    const size_t smB = static_cast<size_t>(6) * L * F_THREADS * sizeof(float);
-    e = cudaFuncSetAttribute(k_addr_finalize<D, L>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smB));
-    if (e != cudaSuccess) return e;
-    dim3 gB(static_cast<unsigned>((BT + F_THREADS - 1) / F_THREADS), 2 * a.H);
-    k_addr_finalize<D, L><<<gB, F_THREADS, smB, stream>>>(a);
-    return cudaGetLastError();
+    return launch_finalize<D, L>(a, stream);
 }
 
 template <class D>

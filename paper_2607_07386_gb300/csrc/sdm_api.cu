@@ -123,7 +123,7 @@ Layout layout_for(const sdm_shape* s, int64_t S) {
     Layout L{};
     const size_t bht = static_cast<size_t>(s->B) * s->H * s->T;
     const int kmax = s->k_write > s->k_read ? s->k_write : s->k_read;
-    L.plan = sdm::addr_plan(s->B, s->H, s->T, static_cast<int>(S), kmax);
+    L.plan = sdm::addr_plan(s->dtype, s->addr == SDM_ADDR_DIRECT, s->B, s->H, s->T, s->d_k, static_cast<int>(S), kmax);
     size_t off = 0;
     L.idx_w = off; off = align256(off + bht * s->k_write * 4);
     L.w_w = off;   off = align256(off + bht * s->k_write * 4);
@@ -153,7 +153,10 @@ sdm_status run_address(const sdm_shape* s, int64_t S, const Layout& L, const voi
     a.B = s->B; a.H = s->H; a.T = s->T; a.dk = s->d_k; a.S = static_cast<int>(S);
     a.ncc = L.plan.ncc;
     a.cw = L.plan.cw;
-    a.cbound = static_cast<float>((s->d_k + 4) * 0x1p-24);
+    // |fp32 score - float64 score| <= cbound * max_j ||P_j|| * ||x||: (d_k + 4) * 2^-24 covers sequential
+    // fp32 FMA accumulation plus the float64 reference's own rounding; the tensor-core path
+    // (blocked accumulation, truncating adds) is given 4x that margin.
+    a.cbound = static_cast<float>((s->d_k + 4) * 0x1p-24 * (L.plan.mma ? 4.0 : 1.0));
     a.part_v = reinterpret_cast<float*>(ws + L.part_v);
     a.part_i = reinterpret_cast<int*>(ws + L.part_i);
     a.pnorm = reinterpret_cast<float*>(ws + L.pnorm);

@@ -59,7 +59,7 @@ template <> __device__ __forceinline__ float load_elem<BF16>(const void* base, i
 }
 
 // Device status word bits (read and cleared by sdm_device_status).
-enum : int { ERR_BAD_INDEX = 1, ERR_UNSORTED = 2 };
+enum : int { ERR_BAD_INDEX = 1, ERR_UNSORTED = 2, ERR_TIMEOUT = 4, ERR_SELECT = 8 };
 
 __device__ __forceinline__ void flag_error(int* err, int bit) {
     if (err) atomicOr(err, bit);

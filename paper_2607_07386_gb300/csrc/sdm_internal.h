@@ -33,9 +33,12 @@ struct AddrArgs {
 struct AddrPlan {
     int L;      // list length kept per chunk (>= k + 4)
     int ncc;    // column chunks per half
-    int cw;     // columns per chunk
+    int cw;     // columns per chunk (<= 512)
+    bool mma;   // scores on the tensor cores (bf16, PROJECTED, d_k <= 128, k <= 32)
 };
-AddrPlan addr_plan(int B, int H, int T, int S, int kmax);
+AddrPlan addr_plan(int dtype, int direct, int B, int H, int T, int dk, int S, int kmax);
+bool mma_path_supported(int dtype, int direct, int dk, int S, int kmax);
+cudaError_t launch_address_mma(const AddrPlan& plan, const AddrArgs& a, cudaStream_t stream);
 size_t addr_partial_bytes(const AddrPlan& plan, int B, int H, int T);
 cudaError_t launch_address(int dtype, const AddrPlan& plan, const AddrArgs& a, cudaStream_t stream);
 
