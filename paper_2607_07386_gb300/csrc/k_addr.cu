@@ -32,7 +32,14 @@ namespace sdm {
 constexpr int A_TOK = 128;     // tokens per score CTA (one per thread)
 constexpr int A_SUB = 32;      // columns accumulated per pass
 constexpr int A_PPITCH = 36;   // fp32 pitch of the staged P sub-chunk (16-byte aligned, fewer bank conflicts)
-constexpr int F_THREADS = 64;  // tokens per finalize CTA
+constexpr int F_THREADS = 64;  // tokens per finalize CTA (wide lists)
+constexpr int FW_WARPS = 8;    // warps (= token-sides) per finalize CTA (k <= 32)
+
+// Per-chunk top-L lists: entry p of token u, chunk `chunk` of (side, head) z is at
+// ((z * 2 ncc + chunk) * BT + u) * L + p  (a token's L entries are contiguous).
+__host__ __device__ __forceinline__ int64_t part_at(int z, int ncc, int chunk, int64_t BT, int64_t u, int L, int p) {
+    return ((static_cast<int64_t>(z) * (2 * ncc) + chunk) * BT + u) * L + p;
+}
 
 // Sorted (value desc, index asc) list of the L best entries seen so far; empty = -inf.
 template <int L>
@@ -152,11 +159,11 @@ __global__ void __launch_bounds__(A_TOK) k_addr_scores(const AddrArgs a) {
 
     const int64_t u = u0 + tid;
     if (u < BT) {
-        const int64_t base = ((static_cast<int64_t>(blockIdx.z) * (2 * a.ncc) + chunk) * L) * BT + u;
+        const int64_t base = part_at(blockIdx.z, a.ncc, chunk, BT, u, L, 0);
 #pragma unroll
         for (int p = 0; p < L; ++p) {
-            a.part_v[base + p * BT] = top.v[p];
-            a.part_i[base + p * BT] = top.i[p];
+            a.part_v[base + p] = top.v[p];
+            a.part_i[base + p] = top.i[p];
         }
     }
 }
@@ -189,7 +196,7 @@ __device__ __forceinline__ bool beats64(double a, int ia, double b, int ib) { re
 // Writes the exact top-k (ordered by fp32 value, desc) to Av/Ai with pitch F_THREADS.
 template <class D, int L>
 __device__ __noinline__ void resolve_half(const float* lv, const int* li, int k, double eps, const TokenCtx& c, int hf,
-                                          float* Av, int* Ai) {
+                                          float* Av, int* Ai, int pitch) {
     const double lo = static_cast<double>(lv[k - 1]) - 2.0 * eps;
     const double hi = static_cast<double>(lv[k]) + 2.0 * eps;
     if (c.S > L && static_cast<double>(lv[L - 1]) >= lo) {
@@ -204,7 +211,7 @@ __device__ __noinline__ void resolve_half(const float* lv, const int* li, int k,
             while (p > 0 && beats64(s, j, bv[p - 1], bi[p - 1])) { bv[p] = bv[p - 1]; bi[p] = bi[p - 1]; --p; }
             bv[p] = s; bi[p] = j;
         }
-        for (int p = 0; p < k; ++p) { Av[p * F_THREADS] = static_cast<float>(bv[p]); Ai[p * F_THREADS] = bi[p]; }
+        for (int p = 0; p < k; ++p) { Av[p * pitch] = static_cast<float>(bv[p]); Ai[p * pitch] = bi[p]; }
         return;
     }
     int cin = 0;
@@ -214,7 +221,7 @@ __device__ __noinline__ void resolve_half(const float* lv, const int* li, int k,
     double s64[L];
     bool used[L];
     for (int p = cin; p < pend; ++p) { s64[p] = score64<D>(c, hf, li[p]); used[p] = false; }
-    for (int p = 0; p < cin; ++p) { Av[p * F_THREADS] = lv[p]; Ai[p * F_THREADS] = li[p]; }
+    for (int p = 0; p < cin; ++p) { Av[p * pitch] = lv[p]; Ai[p * pitch] = li[p]; }
     // choose k - cin entries of the band by (float64 desc, index asc) ...
     int chosen[L];
     const int need = k - cin;
@@ -232,8 +239,8 @@ __device__ __noinline__ void resolve_half(const float* lv, const int* li, int k,
             const int p = chosen[q];
             if (p >= 0 && (best < 0 || TopList<L>::beats(lv[p], li[p], lv[chosen[best]], li[chosen[best]]))) best = q;
         }
-        Av[(cin + r) * F_THREADS] = lv[chosen[best]];
-        Ai[(cin + r) * F_THREADS] = li[chosen[best]];
+        Av[(cin + r) * pitch] = lv[chosen[best]];
+        Ai[(cin + r) * pitch] = li[chosen[best]];
         chosen[best] = -1;
     }
 }
@@ -243,21 +250,21 @@ __device__ __noinline__ void resolve_half(const float* lv, const int* li, int k,
 template <class D, int L>
 __device__ __noinline__ void resolve_combined(const float* cv, const int* cf, int k, double epsc, const TokenCtx& c,
                                               const float* A1v, const int* A1i, const float* A2v, const int* A2i,
-                                              float* Fv, int* Fi) {
+                                              float* Fv, int* Fi, int pitch) {
     const int S = c.S;
     const double lo = static_cast<double>(cv[k - 1]) - 2.0 * epsc;
     const double hi = static_cast<double>(cv[k]) + 2.0 * epsc;
     if (cv[L - 1] != -INFINITY && static_cast<double>(cv[L - 1]) >= lo) {
         // All k^2 candidates in float64.
         double s1[64], s2[64];
-        for (int p = 0; p < k; ++p) { s1[p] = score64<D>(c, 0, A1i[p * F_THREADS]); s2[p] = score64<D>(c, 1, A2i[p * F_THREADS]); }
+        for (int p = 0; p < k; ++p) { s1[p] = score64<D>(c, 0, A1i[p * pitch]); s2[p] = score64<D>(c, 1, A2i[p * pitch]); }
         double bv[64];
         int bf[64], bp1[64], bp2[64];
         int n = 0;
         for (int p1 = 0; p1 < k; ++p1)
             for (int p2 = 0; p2 < k; ++p2) {
                 const double s = s1[p1] + s2[p2];
-                const int f = A1i[p1 * F_THREADS] * S + A2i[p2 * F_THREADS];
+                const int f = A1i[p1 * pitch] * S + A2i[p2 * pitch];
                 if (n == k && !beats64(s, f, bv[k - 1], bf[k - 1])) continue;
                 int p = (n < k) ? n++ : k - 1;
                 while (p > 0 && beats64(s, f, bv[p - 1], bf[p - 1])) {
@@ -266,8 +273,8 @@ __device__ __noinline__ void resolve_combined(const float* cv, const int* cf, in
                 bv[p] = s; bf[p] = f; bp1[p] = p1; bp2[p] = p2;
             }
         for (int p = 0; p < k; ++p) {
-            Fv[p * F_THREADS] = A1v[bp1[p] * F_THREADS] + A2v[bp2[p] * F_THREADS];
-            Fi[p * F_THREADS] = bf[p];
+            Fv[p * pitch] = A1v[bp1[p] * pitch] + A2v[bp2[p] * pitch];
+            Fi[p * pitch] = bf[p];
         }
         return;
     }
@@ -281,97 +288,66 @@ __device__ __noinline__ void resolve_combined(const float* cv, const int* cf, in
         s64[p] = score64<D>(c, 0, cf[p] / S) + score64<D>(c, 1, cf[p] % S);
         used[p] = false;
     }
-    for (int p = 0; p < cin; ++p) { Fv[p * F_THREADS] = cv[p]; Fi[p * F_THREADS] = cf[p]; }
+    for (int p = 0; p < cin; ++p) { Fv[p * pitch] = cv[p]; Fi[p * pitch] = cf[p]; }
     for (int r = cin; r < k; ++r) {
         int best = -1;
         for (int p = cin; p < pend; ++p)
             if (!used[p] && (best < 0 || beats64(s64[p], cf[p], s64[best], cf[best]))) best = p;
         used[best] = true;
-        Fv[r * F_THREADS] = cv[best];
-        Fi[r * F_THREADS] = cf[best];
+        Fv[r * pitch] = cv[best];
+        Fi[r * pitch] = cf[best];
     }
 }
 
 // ------------------------------------------------------------------------------------------
-// Kernel B (k <= 32): merge, certify, combine, softmax, sort by slot -- branch-free common path
+// Kernel B (k <= 32): one warp per token-side.  Lane p holds entry p (and p + 32) of a list.
+//   merge of chunk lists: output rank = own position + number of entries of the other list
+//     that come first (binary search across lanes), scattered through shared memory;
+//   combined top-(k+4): exact k-way merge of the k rows i of the outer sum (lane i owns row
+//     i, its head s1[i] + s2[j_i]); each step takes the largest head by a warp max-reduce of
+//     order-preserving integer keys, ties to the smallest slot by a min-reduce;
+//   softmax by warp reductions; ascending slot order by a 32-lane bitonic shuffle network.
 // ------------------------------------------------------------------------------------------
-// Bitonic networks on per-thread register arrays (descending by value / ascending by key).
-template <int N>
-__device__ __forceinline__ void net_desc(float (&v)[N], int (&ix)[N]) {
-#pragma unroll
-    for (int size = 2; size <= N; size <<= 1)
-#pragma unroll
-        for (int stride = size >> 1; stride > 0; stride >>= 1)
-#pragma unroll
-            for (int i = 0; i < N; ++i) {
-                const int j = i ^ stride;
-                if (j > i) {
-                    const bool up = (i & size) == 0;
-                    const bool sw = up ? (v[i] < v[j]) : (v[i] > v[j]);
-                    const float x = v[i];
-                    const int xi = ix[i];
-                    v[i] = sw ? v[j] : x;   ix[i] = sw ? ix[j] : xi;
-                    v[j] = sw ? x : v[j];   ix[j] = sw ? xi : ix[j];
-                }
-            }
+__device__ __forceinline__ uint32_t f2key(float f) {
+    const uint32_t u = __float_as_uint(f);
+    return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
 }
-template <int N>
-__device__ __forceinline__ void net_asc_key(int (&key)[N], float (&val)[N]) {
-#pragma unroll
-    for (int size = 2; size <= N; size <<= 1)
-#pragma unroll
-        for (int stride = size >> 1; stride > 0; stride >>= 1)
-#pragma unroll
-            for (int i = 0; i < N; ++i) {
-                const int j = i ^ stride;
-                if (j > i) {
-                    const bool up = (i & size) == 0;
-                    const bool sw = up ? (key[i] > key[j]) : (key[i] < key[j]);
-                    const int x = key[i];
-                    const float xv = val[i];
-                    key[i] = sw ? key[j] : x;   val[i] = sw ? val[j] : xv;
-                    key[j] = sw ? x : key[j];   val[j] = sw ? xv : val[j];
-                }
-            }
+__device__ __forceinline__ float key2f(uint32_t k) {
+    return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
 }
-
-constexpr int CBUF = 64;   // candidate buffer per thread (= network size)
-
-// Sort the first CBUF entries of a per-thread buffer (value desc); entries >= cnt count as -inf.
-__device__ __forceinline__ void sort_buffer(float* bv, int* bi, int cnt) {
-    float v[CBUF];
-    int ix[CBUF];
+// entry idx (< 64) of a list held two entries per lane (v0: idx < 32, v1: idx >= 32)
+__device__ __forceinline__ float lane_get(float v0, float v1, int idx) {
+    const float a = __shfl_sync(0xffffffffu, v0, idx & 31);
+    const float b = __shfl_sync(0xffffffffu, v1, idx & 31);
+    return idx < 32 ? a : b;
+}
+// number of the first L entries of a descending list that are > x (strict) or >= x
+__device__ __forceinline__ int lane_count_before(float v0, float v1, int L, float x, bool strict) {
+    int pos = 0;
 #pragma unroll
-    for (int i = 0; i < CBUF; ++i) {
-        v[i] = i < cnt ? bv[i * F_THREADS] : -INFINITY;
-        ix[i] = i < cnt ? bi[i * F_THREADS] : INT_MAX;
+    for (int step = 32; step >= 1; step >>= 1) {
+        const int idx = pos + step - 1;
+        const float v = lane_get(v0, v1, idx);
+        const bool before = strict ? (v > x) : (v >= x);
+        if (idx < L && before) pos += step;
     }
-    net_desc<CBUF>(v, ix);
-#pragma unroll
-    for (int i = 0; i < CBUF; ++i) { bv[i * F_THREADS] = v[i]; bi[i * F_THREADS] = ix[i]; }
+    return pos;
 }
 
 template <class D, int L>
-__global__ void __launch_bounds__(F_THREADS) k_addr_finalize(const AddrArgs a) {
-    static_assert(L <= 36, "network finalize handles k <= 32");
-    extern __shared__ __align__(16) float smB[];
-    const int tid = threadIdx.x;
-    // per-thread regions, pitch F_THREADS: half lists H1, H2 (L), merge scratch M (L),
-    // candidates C (CBUF), final selection F (L)
-    float* H1v = smB + tid;                 int* H1i = reinterpret_cast<int*>(H1v + L * F_THREADS);
-    float* H2v = smB + 2 * L * F_THREADS + tid; int* H2i = reinterpret_cast<int*>(H2v + L * F_THREADS);
-    float* Mv = smB + 4 * L * F_THREADS + tid;  int* Mi = reinterpret_cast<int*>(Mv + L * F_THREADS);
-    float* Cv = smB + 6 * L * F_THREADS + tid;  int* Ci = reinterpret_cast<int*>(Cv + CBUF * F_THREADS);
-    float* Fv = smB + (6 * L + 2 * CBUF) * F_THREADS + tid; int* Fi = reinterpret_cast<int*>(Fv + L * F_THREADS);
-
-    const int side = blockIdx.y / a.H, h = blockIdx.y % a.H;
+__global__ void __launch_bounds__(FW_WARPS * 32) k_addr_finalize(const AddrArgs a) {
+    static_assert(L <= 36, "warp finalize handles k <= 32");
+    __shared__ float wv[FW_WARPS][3][64];
+    __shared__ int wi[FW_WARPS][3][64];
+    const int lane = threadIdx.x & 31, wq = threadIdx.x >> 5;
+    const int z = blockIdx.y;
+    const int side = z / a.H, h = z % a.H;
     const int64_t BT = static_cast<int64_t>(a.B) * a.T;
-    const int64_t u = static_cast<int64_t>(blockIdx.x) * F_THREADS + tid;
-    const bool live = u < BT;            // dead lanes run along (warp votes below) but store nothing
+    const int64_t u = static_cast<int64_t>(blockIdx.x) * FW_WARPS + wq;
+    if (u >= BT) return;                                   // whole warp
     const int k = a.kk[side];
     const int S = a.S;
-    const int64_t uu = live ? u : 0;
-    const int64_t b = uu / a.T, t = uu - b * a.T;
+    const int64_t b = u / a.T, t = u - b * a.T;
     TokenCtx c;
     c.P = a.P[side];
     c.X = a.X[side];
@@ -379,122 +355,161 @@ __global__ void __launch_bounds__(F_THREADS) k_addr_finalize(const AddrArgs a) {
     c.prow0 = static_cast<int64_t>(h) * 2 * S;
     c.dk = a.dk;
     c.S = S;
+    float* sv0 = wv[wq][0]; int* si0 = wi[wq][0];          // staging / merge output / A1
+    float* sv1 = wv[wq][1]; int* si1 = wi[wq][1];          // A2
+    float* sv2 = wv[wq][2]; int* si2 = wi[wq][2];          // candidates / final
 
     double eps = 0.0;
     if (c.P != nullptr) {
         float ss = 0.f;
-        for (int d = 0; d < a.dk; ++d) {
+        for (int d = lane; d < a.dk; d += 32) {
             const float xv = load_elem<D>(c.X, c.xoff + d);
             ss = fmaf(xv, xv, ss);
         }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
         eps = static_cast<double>(a.cbound) * static_cast<double>(a.pnorm[side * a.H + h]) *
               static_cast<double>(sqrtf(ss)) * (1.0 + 0x1p-12);
     }
 
+    float av[2], bv[2];      // A1 and A2 after certification: lane p holds entry p (p < k)
+    int ai[2], bi[2];
     float amax[2];
 #pragma unroll 1
     for (int hf = 0; hf < 2; ++hf) {
-        float* Hv = hf ? H2v : H1v;
-        int* Hi = hf ? H2i : H1i;
-        // chunk lists of this half (each sorted desc) merged with two pointers
-        for (int cc = 0; cc < a.ncc; ++cc) {
-            const int64_t base = ((static_cast<int64_t>(blockIdx.y) * (2 * a.ncc) + hf * a.ncc + cc) * L) * BT + uu;
-            float* dv = cc == 0 ? Hv : Mv;
-            int* di = cc == 0 ? Hi : Mi;
-            for (int p = 0; p < L; ++p) { dv[p * F_THREADS] = a.part_v[base + p * BT]; di[p * F_THREADS] = a.part_i[base + p * BT]; }
-            if (cc > 0) {
-                int ia = 0, ib = 0;
-                for (int p = 0; p < L; ++p) {
-                    const float va = ia < L ? Hv[ia * F_THREADS] : -INFINITY;
-                    const float vb = ib < L ? Mv[ib * F_THREADS] : -INFINITY;
-                    const bool ta = va >= vb;        // ties: the earlier chunk (smaller columns)
-                    Cv[p * F_THREADS] = ta ? va : vb;
-                    Ci[p * F_THREADS] = ta ? Hi[ia * F_THREADS] : Mi[ib * F_THREADS];
-                    ia += ta ? 1 : 0;
-                    ib += ta ? 0 : 1;
-                }
-                for (int p = 0; p < L; ++p) { Hv[p * F_THREADS] = Cv[p * F_THREADS]; Hi[p * F_THREADS] = Ci[p * F_THREADS]; }
+        // chunk 0 of this half
+        int64_t base = part_at(z, a.ncc, hf * a.ncc, BT, u, L, 0);
+        float v0 = lane < L ? a.part_v[base + lane] : -INFINITY;
+        float v1 = lane + 32 < L ? a.part_v[base + lane + 32] : -INFINITY;
+        int i0 = lane < L ? a.part_i[base + lane] : INT_MAX;
+        int i1 = lane + 32 < L ? a.part_i[base + lane + 32] : INT_MAX;
+        for (int cc = 1; cc < a.ncc; ++cc) {                  // merge later chunks (larger columns)
+            base = part_at(z, a.ncc, hf * a.ncc + cc, BT, u, L, 0);
+            const float w0 = lane < L ? a.part_v[base + lane] : -INFINITY;
+            const float w1 = lane + 32 < L ? a.part_v[base + lane + 32] : -INFINITY;
+            const int j0 = lane < L ? a.part_i[base + lane] : INT_MAX;
+            const int j1 = lane + 32 < L ? a.part_i[base + lane + 32] : INT_MAX;
+            // ties: the earlier chunk first
+            const int ra0 = lane + lane_count_before(w0, w1, L, v0, true);
+            const int ra1 = lane + 32 + lane_count_before(w0, w1, L, v1, true);
+            const int rb0 = lane + lane_count_before(v0, v1, L, w0, false);
+            const int rb1 = lane + 32 + lane_count_before(v0, v1, L, w1, false);
+            __syncwarp();
+            if (lane < L && ra0 < L) { sv0[ra0] = v0; si0[ra0] = i0; }
+            if (lane + 32 < L && ra1 < L) { sv0[ra1] = v1; si0[ra1] = i1; }
+            if (lane < L && rb0 < L) { sv0[rb0] = w0; si0[rb0] = j0; }
+            if (lane + 32 < L && rb1 < L) { sv0[rb1] = w1; si0[rb1] = j1; }
+            __syncwarp();
+            v0 = lane < L ? sv0[lane] : -INFINITY;       i0 = lane < L ? si0[lane] : INT_MAX;
+            v1 = lane + 32 < L ? sv0[lane + 32] : -INFINITY; i1 = lane + 32 < L ? si0[lane + 32] : INT_MAX;
+        }
+        // certify the boundary between entries k-1 and k (warp-uniform decision)
+        bool certified = S <= k;
+        if (!certified) {
+            const float vk = lane_get(v0, v1, k - 1), vk1 = lane_get(v0, v1, k);
+            certified = static_cast<double>(vk) - static_cast<double>(vk1) > 2.0 * eps;
+        }
+        if (!certified) {
+            __syncwarp();
+            if (lane < L) { sv0[lane] = v0; si0[lane] = i0; }
+            if (lane + 32 < L) { sv0[lane + 32] = v1; si0[lane + 32] = i1; }
+            __syncwarp();
+            if (lane == 0) {
+                float lv[L];
+                int li[L];
+                for (int p = 0; p < L; ++p) { lv[p] = sv0[p]; li[p] = si0[p]; }
+                resolve_half<D, L>(lv, li, k, eps, c, hf, sv0, si0, 1);
             }
+            __syncwarp();
+            v0 = lane < k ? sv0[lane] : -INFINITY;
+            i0 = lane < k ? si0[lane] : INT_MAX;
         }
-        bool certified = (S <= k);
-        if (!certified) certified = static_cast<double>(Hv[(k - 1) * F_THREADS]) - static_cast<double>(Hv[k * F_THREADS]) > 2.0 * eps;
-        if (!certified && live) {
-            float lv[L];
-            int li[L];
-            for (int p = 0; p < L; ++p) { lv[p] = Hv[p * F_THREADS]; li[p] = Hi[p * F_THREADS]; }
-            resolve_half<D, L>(lv, li, k, eps, c, hf, Hv, Hi);
-        }
-        amax[hf] = fmaxf(fabsf(Hv[0]), fabsf(Hv[(k - 1) * F_THREADS]));
+        if (hf == 0) { av[0] = lane < k ? v0 : -INFINITY; ai[0] = i0; }
+        else { bv[0] = lane < k ? v0 : -INFINITY; bi[0] = i0; }
+        amax[hf] = fmaxf(fabsf(lane_get(v0, v1, 0)), fabsf(lane_get(v0, v1, k - 1)));
     }
 
-    // Outer-sum candidates.  theta = max over a of H1[a-1] + H2[ceil(k/a)-1]: the first a
-    // rows times the first ceil(k/a) columns give >= k sums >= it (rounding is monotone).
+    // combined: k-way merge of the rows (lane i: row i; head = A1[i] + A2[j])
     const double epsc = 2.0 * eps + 0x1p-22 * (static_cast<double>(amax[0]) + static_cast<double>(amax[1]));
-    float theta = -INFINITY;
-    for (int aa = 1; aa <= k; ++aa) theta = fmaxf(theta, H1v[(aa - 1) * F_THREADS] + H2v[((k + aa - 1) / aa - 1) * F_THREADS]);
-    const float lo = __double2float_rd(static_cast<double>(theta) - 2.0 * epsc);
-    int cnt = 0;
-    for (int p1 = 0; p1 < k; ++p1) {                        // k is warp-uniform per side
-        const float a1 = H1v[p1 * F_THREADS];
-        const int i1 = H1i[p1 * F_THREADS];
-        bool act = live && a1 + H2v[0] >= lo;
-        if (!__any_sync(0xffffffffu, act)) break;          // rows are sorted: the rest are below lo
-        for (int p2 = 0; p2 < k; ++p2) {
-            const float cs = a1 + H2v[p2 * F_THREADS];
-            act = act && cs >= lo;
-            if (!__any_sync(0xffffffffu, act)) break;
-            if (act) {
-                Cv[cnt * F_THREADS] = cs;
-                Ci[cnt * F_THREADS] = i1 * S + H2i[p2 * F_THREADS];
-                ++cnt;
-            }
-            if (__any_sync(0xffffffffu, cnt == CBUF)) {      // flush: keep the best L
-                sort_buffer(Cv, Ci, cnt);
-                cnt = min(cnt, L);
-            }
+    int j = 0;
+    const float b0v = __shfl_sync(0xffffffffu, bv[0], 0);
+    const int b0i = __shfl_sync(0xffffffffu, bi[0], 0);
+    float head = lane < k ? av[0] + b0v : -INFINITY;
+    int flat = ai[0] * S + b0i;
+    float cv0 = -INFINITY, cv1 = -INFINITY;    // candidate r in lane r (r < 32) / lane r-32
+    int cf0 = INT_MAX, cf1 = INT_MAX;
+    for (int r = 0; r < L; ++r) {
+        const uint32_t key = f2key(head);
+        const uint32_t kmax = __reduce_max_sync(0xffffffffu, key);
+        const bool tie = key == kmax;
+        const uint32_t fmin = __reduce_min_sync(0xffffffffu, tie ? static_cast<uint32_t>(flat) : 0xffffffffu);
+        const bool win = tie && static_cast<uint32_t>(flat) == fmin;
+        const float val = key2f(kmax);
+        if (lane == (r & 31)) {
+            if (r < 32) { cv0 = val; cf0 = static_cast<int>(fmin); }
+            else { cv1 = val; cf1 = static_cast<int>(fmin); }
+        }
+        if (win) ++j;
+        const float nv = __shfl_sync(0xffffffffu, bv[0], j & 31);
+        const int ni = __shfl_sync(0xffffffffu, bi[0], j & 31);
+        if (win) {
+            head = (j < k && lane < k) ? av[0] + nv : -INFINITY;
+            flat = ai[0] * S + ni;
         }
     }
-    sort_buffer(Cv, Ci, cnt);
-    bool certified = (k == 1) || (cnt <= k);
-    if (!certified) certified = static_cast<double>(Cv[(k - 1) * F_THREADS]) - static_cast<double>(Cv[k * F_THREADS]) > 2.0 * epsc;
-    if (certified) {
-        for (int p = 0; p < k; ++p) { Fv[p * F_THREADS] = Cv[p * F_THREADS]; Fi[p * F_THREADS] = Ci[p * F_THREADS]; }
-    } else if (live) {
-        float cv[L];
-        int cf[L];
-        for (int p = 0; p < L; ++p) {
-            cv[p] = p < cnt ? Cv[p * F_THREADS] : -INFINITY;
-            cf[p] = p < cnt ? Ci[p * F_THREADS] : INT_MAX;
-        }
-        resolve_combined<D, L>(cv, cf, k, epsc, c, H1v, H1i, H2v, H2i, Fv, Fi);
+    bool certified = (k == 1);
+    if (!certified) {
+        const float ck = lane_get(cv0, cv1, k - 1), ck1 = lane_get(cv0, cv1, k);
+        certified = (ck1 == -INFINITY) || (static_cast<double>(ck) - static_cast<double>(ck1) > 2.0 * epsc);
     }
-
-    // softmax over the selected scores, then ascending slot order (network on <= 32 pairs)
-    float m = -INFINITY;
-    for (int p = 0; p < k; ++p) m = fmaxf(m, Fv[p * F_THREADS]);
-    int key[32];
-    float val[32];
-    float z = 0.f;
+    float fv = cv0;
+    int fi = cf0;
+    if (!certified) {
+        __syncwarp();
+        sv0[lane] = av[0]; si0[lane] = ai[0];            // A1
+        sv1[lane] = bv[0]; si1[lane] = bi[0];            // A2
+        sv2[lane] = cv0; si2[lane] = cf0;                // candidates 0..31
+        if (lane + 32 < L) { sv2[lane + 32] = cv1; si2[lane + 32] = cf1; }
+        __syncwarp();
+        if (lane == 0) {
+            float cvl[L];
+            int cfl[L];
+            for (int p = 0; p < L; ++p) { cvl[p] = sv2[p]; cfl[p] = si2[p]; }
+            resolve_combined<D, L>(cvl, cfl, k, epsc, c, sv0, si0, sv1, si1, sv2, si2, 1);
+        }
+        __syncwarp();
+        fv = lane < k ? sv2[lane] : -INFINITY;
+        fi = lane < k ? si2[lane] : INT_MAX;
+    }
+    // softmax over the k selected scores
+    if (lane >= k) { fv = -INFINITY; fi = INT_MAX; }
+    const float m = key2f(__reduce_max_sync(0xffffffffu, f2key(fv)));
+    float e = lane < k ? expf(fv - m) : 0.f;
+    float zsum = e;
 #pragma unroll
-    for (int p = 0; p < 32; ++p) {
-        const bool in = p < k;
-        const float e = in ? expf(Fv[p * F_THREADS] - m) : 0.f;
-        key[p] = in ? Fi[p * F_THREADS] : INT_MAX;
-        val[p] = e;
-        z += e;
+    for (int off = 16; off > 0; off >>= 1) zsum += __shfl_xor_sync(0xffffffffu, zsum, off);
+    // ascending slot order: bitonic network across the 32 lanes
+    int key = fi;
+#pragma unroll
+    for (int size = 2; size <= 32; size <<= 1) {
+#pragma unroll
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            const int pk = __shfl_xor_sync(0xffffffffu, key, stride);
+            const float pe = __shfl_xor_sync(0xffffffffu, e, stride);
+            const bool up = (lane & size) == 0;
+            const bool lower = (lane & stride) == 0;
+            const bool take_min = (up == lower);
+            const bool mine = take_min ? (key <= pk) : (key >= pk);
+            key = mine ? key : pk;
+            e = mine ? e : pe;
+        }
     }
-    net_asc_key<32>(key, val);
-    if (live) {
-        const float rz = 1.f / z;
+    if (lane < k) {
         const int64_t tokoff = ((b * a.H + h) * a.T + t) * k;     // [B, H, T, k] layout
-        int32_t* oi = a.idx[side] + tokoff;
-        float* ow = a.w[side] + tokoff;
-#pragma unroll
-        for (int p = 0; p < 32; ++p)
-            if (p < k) { oi[p] = key[p]; ow[p] = val[p] * rz; }
+        a.idx[side][tokoff + lane] = key;
+        a.w[side][tokoff + lane] = e / zsum;
     }
 }
-
 // ------------------------------------------------------------------------------------------
 // Kernel B, wide lists (k > 32): insertion-based merge and candidate selection
 // ------------------------------------------------------------------------------------------
@@ -541,10 +556,10 @@ __global__ void __launch_bounds__(F_THREADS) k_addr_finalize_wide(const AddrArgs
         TopList<L> top;
         top.clear();
         for (int cc = 0; cc < a.ncc; ++cc) {
-            const int64_t base = ((static_cast<int64_t>(blockIdx.y) * (2 * a.ncc) + hf * a.ncc + cc) * L) * BT + u;
+            const int64_t base = part_at(blockIdx.y, a.ncc, hf * a.ncc + cc, BT, u, L, 0);
             for (int p = 0; p < L; ++p) {
-                const float v = a.part_v[base + p * BT];
-                const int i = a.part_i[base + p * BT];
+                const float v = a.part_v[base + p];
+                const int i = a.part_i[base + p];
                 if (!top.admits(v, i)) break;
                 top.push(v, i);
             }
@@ -562,7 +577,7 @@ __global__ void __launch_bounds__(F_THREADS) k_addr_finalize_wide(const AddrArgs
             int li[L];
 #pragma unroll
             for (int p = 0; p < L; ++p) { lv[p] = top.v[p]; li[p] = top.i[p]; }
-            resolve_half<D, L>(lv, li, k, eps, c, hf, Av, Ai);
+            resolve_half<D, L>(lv, li, k, eps, c, hf, Av, Ai, F_THREADS);
         }
         amax[hf] = fmaxf(fabsf(Av[0]), fabsf(Av[(k - 1) * F_THREADS]));
     }
@@ -602,7 +617,7 @@ __global__ void __launch_bounds__(F_THREADS) k_addr_finalize_wide(const AddrArgs
         int cf[L];
 #pragma unroll
         for (int p = 0; p < L; ++p) { cv[p] = cand.v[p]; cf[p] = cand.i[p]; }
-        resolve_combined<D, L>(cv, cf, k, epsc, c, A1v, A1i, A2v, A2i, Fv, Fi);
+        resolve_combined<D, L>(cv, cf, k, epsc, c, A1v, A1i, A2v, A2i, Fv, Fi, F_THREADS);
     }
 
     // softmax over the selected scores, then ascending slot order
@@ -686,10 +701,8 @@ static cudaError_t launch_finalize(const AddrArgs& a, cudaStream_t stream) {
     dim3 gB(static_cast<unsigned>((BT + F_THREADS - 1) / F_THREADS), 2 * a.H);
     cudaError_t e;
     if constexpr (L <= 36) {
-        const size_t smB = static_cast<size_t>(2) * (4 * L + 2 * CBUF) * F_THREADS * sizeof(float);
-        e = cudaFuncSetAttribute(k_addr_finalize<D, L>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smB));
-        if (e != cudaSuccess) return e;
-        k_addr_finalize<D, L><<<gB, F_THREADS, smB, stream>>>(a);
+        dim3 gW(static_cast<unsigned>((BT + FW_WARPS - 1) / FW_WARPS), 2 * a.H);
+        k_addr_finalize<D, L><<<gW, FW_WARPS * 32, 0, stream>>>(a);
     } else {
         const size_t smB = static_cast<size_t>(6) * L * F_THREADS * sizeof(float);
         e = cudaFuncSetAttribute(k_addr_finalize_wide<D, L>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smB));

@@ -331,12 +331,17 @@ __global__ void __launch_bounds__(MM_THREADS, 1) k_addr_mma(const __grid_constan
             for (int i = 0; i < MM_BUF; ++i) { outv[i] = lv[i]; outi[i] = li[i]; }
         }
     }
-    if (valid) {
+    if (valid) {   // the token's L entries are contiguous (L % 4 == 0): 16-byte stores
         const int64_t u = static_cast<int64_t>(b) * a.T + t;
-        const int64_t lbase = ((static_cast<int64_t>(blockIdx.z) * (2 * a.ncc) + chunk) * L) * BT + u;
+        const int64_t lbase = ((static_cast<int64_t>(blockIdx.z) * (2 * a.ncc) + chunk) * BT + u) * L;
+        float4* pv = reinterpret_cast<float4*>(a.part_v + lbase);
+        int4* pi = reinterpret_cast<int4*>(a.part_i + lbase);
 #pragma unroll
-        for (int i = 0; i < MM_BUF; ++i)
-            if (i < L) { a.part_v[lbase + i * BT] = outv[i]; a.part_i[lbase + i * BT] = outi[i]; }
+        for (int i = 0; i < MM_BUF; i += 4)
+            if (i < L) {
+                pv[i / 4] = make_float4(outv[i], outv[i + 1], outv[i + 2], outv[i + 3]);
+                pi[i / 4] = make_int4(outi[i], outi[i + 1], outi[i + 2], outi[i + 3]);
+            }
     }
     if (!ok && tid == 0) flag_error(a.err, ERR_TIMEOUT);
 
