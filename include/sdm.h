@@ -148,6 +148,19 @@ sdm_status sdm_recur(const sdm_shape* shape, const int32_t* idx_w, const float* 
  * ascending.  Returns SDM_ERR_DEVICE when the word was non-zero. */
 sdm_status sdm_device_status(int32_t* code, sdm_stream_t stream);
 
+/* Reads into host array `counts` (synchronising on `stream`) and clears the first n
+ * (<= 15) event counters of the current device's selection diagnostics:
+ *   [0] a per-half top-k boundary not certified by the fp32 scores (scores closer than
+ *       their error bound): the band is re-ranked by compensated rescoring
+ *   [1] a whole half rescored in float64 (band wider than the kept list)
+ *   [2] the outer-sum boundary not certified by the fp32 scores
+ *   [3] all k^2 outer-sum candidates rescored in float64
+ *   [4] a survivor-buffer overflow retried on the tensor-core score path
+ *   [5] an outer-sum candidate set too large for the sort network (exact merge used)
+ *   [6] a band decided by the serial float64 rescoring (compensated scores too close)
+ * Counters wrap modulo 2^32. */
+sdm_status sdm_device_stats(uint32_t* counts, int n, sdm_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

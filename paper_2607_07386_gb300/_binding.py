@@ -71,6 +71,8 @@ def lib():
             L.sdm_recur_workspace_bytes.restype = ctypes.c_size_t
             L.sdm_recur_workspace_bytes.argtypes = [_SHP]
             L.sdm_device_status.argtypes = [ctypes.POINTER(ctypes.c_int32), _VP]
+            L.sdm_device_stats.argtypes = [ctypes.POINTER(ctypes.c_uint32), ctypes.c_int, _VP]
+            L.sdm_device_stats.restype = ctypes.c_int
             for f in ("sdm_init_memory", "sdm_forward", "sdm_decode_step", "sdm_address", "sdm_recur",
                       "sdm_device_status"):
                 getattr(L, f).restype = ctypes.c_int
@@ -171,3 +173,14 @@ def device_status(stream=None) -> int:
     if st not in (0, 6):
         _check(st)
     return int(code.value)
+
+
+STAT_NAMES = ("half_band", "half_full", "comb_band", "comb_full", "select_retry", "comb_merge", "band_f64")
+
+
+def device_stats(stream=None) -> dict:
+    """Read and clear the selection event counters (see sdm_device_stats in include/sdm.h)."""
+    n = len(STAT_NAMES)
+    arr = (ctypes.c_uint32 * n)()
+    _check(lib().sdm_device_stats(arr, n, _stream(stream)))
+    return {name: int(arr[i]) for i, name in enumerate(STAT_NAMES)}

@@ -172,6 +172,7 @@ __global__ void __launch_bounds__(A_TOK) k_addr_scores(const AddrArgs a) {
 // Kernel B helpers
 // ------------------------------------------------------------------------------------------
 struct TokenCtx {
+    int* err;           // device status word / counters
     const void* P;      // P of this side (nullptr = DIRECT)
     const void* X;
     int64_t xoff;       // element offset of the token's x row
@@ -201,6 +202,7 @@ __device__ __noinline__ void resolve_half(const float* lv, const int* li, int k,
     const double hi = static_cast<double>(lv[k]) + 2.0 * eps;
     if (c.S > L && static_cast<double>(lv[L - 1]) >= lo) {
         // Band may extend past the list: exact top-k of the whole half in float64.
+        stat_add(c.err, STAT_HALF_FULL);
         double bv[64 + 4];
         int bi[64 + 4];
         int n = 0;
@@ -214,6 +216,7 @@ __device__ __noinline__ void resolve_half(const float* lv, const int* li, int k,
         for (int p = 0; p < k; ++p) { Av[p * pitch] = static_cast<float>(bv[p]); Ai[p * pitch] = bi[p]; }
         return;
     }
+    stat_add(c.err, STAT_BAND_F64);
     int cin = 0;
     while (cin < L && static_cast<double>(lv[cin]) > hi) ++cin;
     int pend = cin;
@@ -256,6 +259,7 @@ __device__ __noinline__ void resolve_combined(const float* cv, const int* cf, in
     const double hi = static_cast<double>(cv[k]) + 2.0 * epsc;
     if (cv[L - 1] != -INFINITY && static_cast<double>(cv[L - 1]) >= lo) {
         // All k^2 candidates in float64.
+        stat_add(c.err, STAT_COMB_FULL);
         double s1[64], s2[64];
         for (int p = 0; p < k; ++p) { s1[p] = score64<D>(c, 0, A1i[p * pitch]); s2[p] = score64<D>(c, 1, A2i[p * pitch]); }
         double bv[64];
@@ -278,6 +282,7 @@ __device__ __noinline__ void resolve_combined(const float* cv, const int* cf, in
         }
         return;
     }
+    stat_add(c.err, STAT_BAND_F64);
     int cin = 0;
     while (cin < L && static_cast<double>(cv[cin]) > hi) ++cin;
     int pend = cin;
@@ -334,6 +339,145 @@ __device__ __forceinline__ int lane_count_before(float v0, float v1, int L, floa
     return pos;
 }
 
+__device__ __forceinline__ int lane_geti(int i0, int i1, int idx) {
+    const int a = __shfl_sync(0xffffffffu, i0, idx & 31);
+    const int b = __shfl_sync(0xffffffffu, i1, idx & 31);
+    return idx < 32 ? a : b;
+}
+
+// Compensated fp32 score of column j of half hf (one lane, one column).  Every product is
+// split exactly (p + pe = P x, pe = 0 for bf16 operands) and every addition exactly by
+// TwoSum (s + err = s_old + p); the error terms are summed in plain fp32.  With n = d_k
+// terms and u = 2^-24 the result val = s + e differs from the exact dot product by at
+// most 2 n (n + 1) u^2 (1.03) sum|P x| <= 2^-31 sum|P x| for n <= 256.  The float64
+// sequential sum of the definition lies within (n - 1) 2^-53 sum|P x| of the exact value,
+// so `bound` = 2^-28 sum|P x| (+ 2^-50 |val| for the conversion to double) covers the
+// distance to it with margin.  DIRECT addressing: the score is x itself, exact (bound 0).
+template <class D>
+__device__ void ff_score(const TokenCtx& c, int hf, int j, double& val, double& bound) {
+    if (c.P == nullptr) {
+        val = static_cast<double>(load_elem<D>(c.X, c.xoff + static_cast<int64_t>(hf) * c.S + j));
+        bound = 0.0;
+        return;
+    }
+    const int64_t prow = (c.prow0 + static_cast<int64_t>(hf) * c.S + j) * c.dk;
+    float sum = 0.f, err = 0.f, mag = 0.f;
+#pragma unroll 8
+    for (int d = 0; d < c.dk; ++d) {
+        const float pv = load_elem<D>(c.P, prow + d);
+        const float xv = load_elem<D>(c.X, c.xoff + d);
+        const float p = __fmul_rn(pv, xv);
+        const float pe = __fmaf_rn(pv, xv, -p);
+        const float t = __fadd_rn(sum, p);
+        const float bp = __fsub_rn(t, sum);
+        const float e2 = __fadd_rn(__fsub_rn(sum, __fsub_rn(t, bp)), __fsub_rn(p, bp));
+        sum = t;
+        err = __fadd_rn(err, __fadd_rn(e2, pe));
+        mag = __fadd_rn(mag, fabsf(p));
+    }
+    val = static_cast<double>(sum) + static_cast<double>(err);
+    bound = 0x1p-28 * static_cast<double>(mag) + 0x1p-50 * fabs(val);
+}
+
+// Band entries [cin, cin + m) of a list sorted by fp32 score are re-ranked by their
+// compensated scores (one lane per entry).  Returns false when two entries are closer
+// than their bounds (the float64 definition must decide) -- otherwise the ranks are
+// those of the float64 definition under (score desc, index asc).
+__device__ __forceinline__ bool rank_band(double cd, double eb, int id, int m, int lane, int& rank) {
+    rank = 0;
+    bool unsure = false;
+    for (int f = 0; f < m; ++f) {
+        const double cf = __shfl_sync(0xffffffffu, cd, f);
+        const double ef = __shfl_sync(0xffffffffu, eb, f);
+        const int jf = __shfl_sync(0xffffffffu, id, f);
+        if (lane < m && f != lane) {
+            const double tol = ef + eb;
+            const double diff = cf - cd;
+            if (tol > 0.0 && fabs(diff) <= tol) unsure = true;
+            else rank += (diff > 0.0 || (diff == 0.0 && jf < id)) ? 1 : 0;
+        }
+    }
+    return !__any_sync(0xffffffffu, unsure);
+}
+
+// Warp-cooperative resolution of an uncertified half boundary (list: lane p holds entry p
+// in v0/i0 and entry p + 32 in v1/i1).  On success writes the exact top-k, in fp32-list
+// order, to ov/oi[0, k) and returns true; returns false when the serial float64 path must
+// decide (band past the list, more than 32 band entries, or an unresolved near-tie).
+template <class D, int L>
+__device__ bool warp_band_half(float v0, int i0, float v1, int i1, int k, double eps, const TokenCtx& c, int hf,
+                               float* ov, int* oi, int lane) {
+    const double lo = static_cast<double>(lane_get(v0, v1, k - 1)) - 2.0 * eps;
+    const double hi = static_cast<double>(lane_get(v0, v1, k)) + 2.0 * eps;
+    if (c.S > L && static_cast<double>(lane_get(v0, v1, L - 1)) >= lo) return false;
+    const double d0 = static_cast<double>(v0), d1 = static_cast<double>(v1);
+    const int cin = __popc(__ballot_sync(0xffffffffu, lane < L && d0 > hi)) +
+                    __popc(__ballot_sync(0xffffffffu, lane + 32 < L && d1 > hi));
+    const int m = __popc(__ballot_sync(0xffffffffu, lane < L && d0 >= lo && d0 <= hi)) +
+                  __popc(__ballot_sync(0xffffffffu, lane + 32 < L && d1 >= lo && d1 <= hi));
+    if (m > 32) return false;
+    const int p = min(cin + lane, L - 1);
+    const float bv = lane_get(v0, v1, p);
+    const int bi = lane_geti(i0, i1, p);
+    double cd = 0.0, eb = 0.0;
+    if (lane < m) ff_score<D>(c, hf, bi, cd, eb);
+    int rank;
+    if (!rank_band(cd, eb, bi, m, lane, rank)) return false;
+    const bool chosen = lane < m && rank < k - cin;
+    const unsigned ch = __ballot_sync(0xffffffffu, chosen);
+    __syncwarp();
+    if (lane < cin) { ov[lane] = v0; oi[lane] = i0; }
+    if (chosen) {
+        const int q = cin + __popc(ch & ((1u << lane) - 1u));
+        ov[q] = bv;
+        oi[q] = bi;
+    }
+    __syncwarp();
+    return true;
+}
+
+// Same for the outer-sum boundary: candidate slot f = i S + j is rescored as the sum of
+// the compensated half scores of column i (half 0) and column j (half 1).  The float64
+// definition adds its two half scores with one more rounding (<= 2^-53 of the sum).
+template <class D, int L>
+__device__ bool warp_band_comb(float v0, int f0, float v1, int f1, int k, double epsc, const TokenCtx& c,
+                               float* ov, int* oi, int lane) {
+    const double lo = static_cast<double>(lane_get(v0, v1, k - 1)) - 2.0 * epsc;
+    const double hi = static_cast<double>(lane_get(v0, v1, k)) + 2.0 * epsc;
+    const float vl = lane_get(v0, v1, L - 1);
+    if (vl != -INFINITY && static_cast<double>(vl) >= lo) return false;
+    const double d0 = static_cast<double>(v0), d1 = static_cast<double>(v1);
+    const int cin = __popc(__ballot_sync(0xffffffffu, lane < L && d0 > hi)) +
+                    __popc(__ballot_sync(0xffffffffu, lane + 32 < L && d1 > hi));
+    const int m = __popc(__ballot_sync(0xffffffffu, lane < L && d0 >= lo && d0 <= hi)) +
+                  __popc(__ballot_sync(0xffffffffu, lane + 32 < L && d1 >= lo && d1 <= hi));
+    if (m > 32) return false;
+    const int p = min(cin + lane, L - 1);
+    const float bv = lane_get(v0, v1, p);
+    const int bf = lane_geti(f0, f1, p);
+    double cd = 0.0, eb = 0.0;
+    if (lane < m) {
+        double c1, e1, c2, e2;
+        ff_score<D>(c, 0, bf / c.S, c1, e1);
+        ff_score<D>(c, 1, bf % c.S, c2, e2);
+        cd = c1 + c2;
+        eb = (c.P == nullptr) ? 0.0 : e1 + e2 + 0x1p-50 * fabs(cd);
+    }
+    int rank;
+    if (!rank_band(cd, eb, bf, m, lane, rank)) return false;
+    const bool chosen = lane < m && rank < k - cin;
+    const unsigned ch = __ballot_sync(0xffffffffu, chosen);
+    __syncwarp();
+    if (lane < cin) { ov[lane] = v0; oi[lane] = f0; }
+    if (chosen) {
+        const int q = cin + __popc(ch & ((1u << lane) - 1u));
+        ov[q] = bv;
+        oi[q] = bf;
+    }
+    __syncwarp();
+    return true;
+}
+
 template <class D, int L>
 __global__ void __launch_bounds__(FW_WARPS * 32) k_addr_finalize(const AddrArgs a) {
     static_assert(L <= 36, "warp finalize handles k <= 32");
@@ -349,6 +493,7 @@ __global__ void __launch_bounds__(FW_WARPS * 32) k_addr_finalize(const AddrArgs 
     const int S = a.S;
     const int64_t b = u / a.T, t = u - b * a.T;
     TokenCtx c;
+    c.err = a.err;
     c.P = a.P[side];
     c.X = a.X[side];
     c.xoff = ((b * a.H + h) * a.T + t) * a.dk;
@@ -410,15 +555,18 @@ __global__ void __launch_bounds__(FW_WARPS * 32) k_addr_finalize(const AddrArgs 
             certified = static_cast<double>(vk) - static_cast<double>(vk1) > 2.0 * eps;
         }
         if (!certified) {
-            __syncwarp();
-            if (lane < L) { sv0[lane] = v0; si0[lane] = i0; }
-            if (lane + 32 < L) { sv0[lane + 32] = v1; si0[lane + 32] = i1; }
-            __syncwarp();
-            if (lane == 0) {
-                float lv[L];
-                int li[L];
-                for (int p = 0; p < L; ++p) { lv[p] = sv0[p]; li[p] = si0[p]; }
-                resolve_half<D, L>(lv, li, k, eps, c, hf, sv0, si0, 1);
+            if (lane == 0) stat_add(c.err, STAT_HALF_BAND);
+            if (!warp_band_half<D, L>(v0, i0, v1, i1, k, eps, c, hf, sv0, si0, lane)) {
+                __syncwarp();
+                if (lane < L) { sv0[lane] = v0; si0[lane] = i0; }
+                if (lane + 32 < L) { sv0[lane + 32] = v1; si0[lane + 32] = i1; }
+                __syncwarp();
+                if (lane == 0) {
+                    float lv[L];
+                    int li[L];
+                    for (int p = 0; p < L; ++p) { lv[p] = sv0[p]; li[p] = si0[p]; }
+                    resolve_half<D, L>(lv, li, k, eps, c, hf, sv0, si0, 1);
+                }
             }
             __syncwarp();
             v0 = lane < k ? sv0[lane] : -INFINITY;
@@ -465,17 +613,20 @@ __global__ void __launch_bounds__(FW_WARPS * 32) k_addr_finalize(const AddrArgs 
     float fv = cv0;
     int fi = cf0;
     if (!certified) {
-        __syncwarp();
-        sv0[lane] = av[0]; si0[lane] = ai[0];            // A1
-        sv1[lane] = bv[0]; si1[lane] = bi[0];            // A2
-        sv2[lane] = cv0; si2[lane] = cf0;                // candidates 0..31
-        if (lane + 32 < L) { sv2[lane + 32] = cv1; si2[lane + 32] = cf1; }
-        __syncwarp();
-        if (lane == 0) {
-            float cvl[L];
-            int cfl[L];
-            for (int p = 0; p < L; ++p) { cvl[p] = sv2[p]; cfl[p] = si2[p]; }
-            resolve_combined<D, L>(cvl, cfl, k, epsc, c, sv0, si0, sv1, si1, sv2, si2, 1);
+        if (lane == 0) stat_add(c.err, STAT_COMB_BAND);
+        if (!warp_band_comb<D, L>(cv0, cf0, cv1, cf1, k, epsc, c, sv2, si2, lane)) {
+            __syncwarp();
+            sv0[lane] = av[0]; si0[lane] = ai[0];            // A1
+            sv1[lane] = bv[0]; si1[lane] = bi[0];            // A2
+            sv2[lane] = cv0; si2[lane] = cf0;                // candidates 0..31
+            if (lane + 32 < L) { sv2[lane + 32] = cv1; si2[lane + 32] = cf1; }
+            __syncwarp();
+            if (lane == 0) {
+                float cvl[L];
+                int cfl[L];
+                for (int p = 0; p < L; ++p) { cvl[p] = sv2[p]; cfl[p] = si2[p]; }
+                resolve_combined<D, L>(cvl, cfl, k, epsc, c, sv0, si0, sv1, si1, sv2, si2, 1);
+            }
         }
         __syncwarp();
         fv = lane < k ? sv2[lane] : -INFINITY;
@@ -532,6 +683,7 @@ __global__ void __launch_bounds__(F_THREADS) k_addr_finalize_wide(const AddrArgs
     const int S = a.S;
     const int64_t b = u / a.T, t = u - b * a.T;
     TokenCtx c;
+    c.err = a.err;
     c.P = a.P[side];
     c.X = a.X[side];
     c.xoff = ((b * a.H + h) * a.T + t) * a.dk;
@@ -577,6 +729,7 @@ __global__ void __launch_bounds__(F_THREADS) k_addr_finalize_wide(const AddrArgs
             int li[L];
 #pragma unroll
             for (int p = 0; p < L; ++p) { lv[p] = top.v[p]; li[p] = top.i[p]; }
+            stat_add(c.err, STAT_HALF_BAND);
             resolve_half<D, L>(lv, li, k, eps, c, hf, Av, Ai, F_THREADS);
         }
         amax[hf] = fmaxf(fabsf(Av[0]), fabsf(Av[(k - 1) * F_THREADS]));
@@ -617,6 +770,7 @@ __global__ void __launch_bounds__(F_THREADS) k_addr_finalize_wide(const AddrArgs
         int cf[L];
 #pragma unroll
         for (int p = 0; p < L; ++p) { cv[p] = cand.v[p]; cf[p] = cand.i[p]; }
+        stat_add(c.err, STAT_COMB_BAND);
         resolve_combined<D, L>(cv, cf, k, epsc, c, A1v, A1i, A2v, A2i, Fv, Fi, F_THREADS);
     }
 

@@ -302,6 +302,7 @@ __global__ void __launch_bounds__(MM_THREADS, 1) k_addr_mma(const __grid_constan
         bitonic_desc<MM_BUF>(outv, outi);
         const bool overflow = cnt > MM_BUF;
         if (!__any_sync(0xffffffffu, overflow)) break;
+        if ((tid & 31) == 0) stat_add(a.err, STAT_SELECT_RETRY);
         if (overflow) {
             float th = outv[0];
 #pragma unroll

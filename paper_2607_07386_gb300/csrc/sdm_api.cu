@@ -37,8 +37,9 @@ sdm_status cuda_fail(cudaError_t e, const char* where) {
     return fail(SDM_ERR_CUDA, "%s: %s (%s)", where, cudaGetErrorString(e), cudaGetErrorName(e));
 }
 
-// Device status word, one per device; its address is looked up once per device.
-__device__ int g_status_word;
+// Device status word followed by event counters (index 1..), one array per device; its
+// address is looked up once per device.
+__device__ int g_status_word[16];
 constexpr int kMaxDevices = 64;
 std::atomic<int*> g_status_addr[kMaxDevices];
 
@@ -344,6 +345,20 @@ sdm_status sdm_recur(const sdm_shape* s, const int32_t* idx_w, const float* w_w,
     r.err = err;
     cudaError_t e = sdm::launch_recur(s->dtype, r, static_cast<int32_t*>(workspace), reinterpret_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "recurrence launch");
+    return ok();
+}
+
+sdm_status sdm_device_stats(uint32_t* counts, int n, sdm_stream_t stream) {
+    if (!counts || n < 0 || n > 15) return fail(SDM_ERR_INVALID_ARG, "counts must be non-NULL and n in [0, 15]");
+    if (n == 0) return ok();
+    int* w = nullptr;
+    SDM_TRY(status_word(&w));
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaMemcpyAsync(counts, w + 1, sizeof(uint32_t) * n, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e == cudaSuccess) e = cudaMemsetAsync(w + 1, 0, sizeof(uint32_t) * n, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(e, "sdm_device_stats");
     return ok();
 }
 

@@ -65,4 +65,19 @@ __device__ __forceinline__ void flag_error(int* err, int bit) {
     if (err) atomicOr(err, bit);
 }
 
+// Event counters stored after the status word (read and cleared by sdm_device_stats).
+enum : int {
+    STAT_HALF_BAND = 1,      // a half's top-k boundary was not certified by the fp32 scores
+    STAT_HALF_FULL = 2,      // ... and the whole half had to be rescored in float64
+    STAT_COMB_BAND = 3,      // the outer-sum boundary was not certified by the fp32 scores
+    STAT_COMB_FULL = 4,      // ... and all k^2 candidates were rescored in float64
+    STAT_SELECT_RETRY = 5,   // a warp's survivor buffer overflowed once (tensor-core path)
+    STAT_COMB_MERGE = 6,     // too many outer-sum candidates: exact k-way merge instead
+    STAT_BAND_F64 = 7,       // a band was decided by the serial float64 rescoring
+    STAT_COUNT = 8
+};
+__device__ __forceinline__ void stat_add(int* err, int which) {
+    if (err) atomicAdd(reinterpret_cast<unsigned*>(err) + which, 1u);
+}
+
 }  // namespace sdm
