@@ -148,6 +148,23 @@ sdm_status sdm_recur(const sdm_shape* shape, const int32_t* idx_w, const float* 
  * ascending.  Returns SDM_ERR_DEVICE when the word was non-zero. */
 sdm_status sdm_device_status(int32_t* code, sdm_stream_t stream);
 
+/* Size of the fixed device scratch behind sdm_recur_noalloc (its hazard table). */
+#define SDM_RECUR_NOALLOC_SCRATCH_BYTES ((size_t)16 << 20)
+
+/* sdm_recur without a workspace argument: the hazard table lives in a device array of
+ * SDM_RECUR_NOALLOC_SCRATCH_BYTES reserved by the library (the paper has no counterpart;
+ * this serves callers that cannot provide device memory, e.g. a runtime whose own pool
+ * owns the device, or a serving loop that must not call an allocator).  Same arguments,
+ * layouts and results as sdm_recur.  Needs B*H*T*max(k_write,k_read)*4 bytes of that
+ * scratch; larger shapes return SDM_ERR_UNSUPPORTED before launching anything.  Allocates
+ * nothing.  The first call on a device looks the array's address up (host-side set-up;
+ * make that first call before any stream capture).  One array per device: calls that
+ * overlap on the GPU race on it and must be serialised by the caller. */
+sdm_status sdm_recur_noalloc(const sdm_shape* shape, const int32_t* idx_w, const float* w_w,
+                             const int32_t* idx_r, const float* w_r, const void* v,
+                             const void* alpha, const void* beta, void* mem, void* y,
+                             sdm_stream_t stream);
+
 /* Reads into host array `counts` (synchronising on `stream`) and clears the first n
  * (<= 15) event counters of the current device's selection diagnostics:
  *   [0] a per-half top-k boundary not certified by the fp32 scores (scores closer than

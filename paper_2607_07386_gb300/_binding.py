@@ -71,6 +71,8 @@ def lib():
             L.sdm_recur_workspace_bytes.restype = ctypes.c_size_t
             L.sdm_recur_workspace_bytes.argtypes = [_SHP]
             L.sdm_device_status.argtypes = [ctypes.POINTER(ctypes.c_int32), _VP]
+            L.sdm_recur_noalloc.argtypes = [_SHP, _I32P, _VP, _I32P, _VP, _VP, _VP, _VP, _VP, _VP, _VP]
+            L.sdm_recur_noalloc.restype = ctypes.c_int
             L.sdm_device_stats.argtypes = [ctypes.POINTER(ctypes.c_uint32), ctypes.c_int, _VP]
             L.sdm_device_stats.restype = ctypes.c_int
             for f in ("sdm_init_memory", "sdm_forward", "sdm_decode_step", "sdm_address", "sdm_recur",
@@ -164,6 +166,16 @@ def recur(shape: SdmShape, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem, y, works
     nb = workspace_nbytes if workspace_nbytes is not None else (_nbytes(workspace) or 0)
     _check(lib().sdm_recur(ctypes.byref(shape), _ptr(idx_w), _ptr(w_w), _ptr(idx_r), _ptr(w_r), _ptr(v),
                            _ptr(alpha), _ptr(beta), _ptr(mem), _ptr(y), _ptr(workspace), nb, _stream(stream)))
+
+
+# Fixed device scratch behind recur_noalloc (SDM_RECUR_NOALLOC_SCRATCH_BYTES in include/sdm.h).
+RECUR_NOALLOC_SCRATCH_BYTES = 16 << 20
+
+
+def recur_noalloc(shape: SdmShape, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem, y, stream=None):
+    """sdm_recur_noalloc: the recurrence without a workspace (fixed device scratch, no allocation)."""
+    _check(lib().sdm_recur_noalloc(ctypes.byref(shape), _ptr(idx_w), _ptr(w_w), _ptr(idx_r), _ptr(w_r), _ptr(v),
+                                   _ptr(alpha), _ptr(beta), _ptr(mem), _ptr(y), _stream(stream)))
 
 
 def device_status(stream=None) -> int:

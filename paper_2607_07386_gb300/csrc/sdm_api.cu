@@ -381,3 +381,50 @@ sdm_status sdm_device_status(int32_t* code, sdm_stream_t stream) {
 }
 
 }  // extern "C"
+
+// Internal helpers for entry points defined in other translation units.
+namespace sdm {
+
+sdm_status api_error(sdm_status st, const char* msg) { return fail(st, "%s", msg); }
+
+sdm_status api_ok() { return ok(); }
+
+// The argument checks of sdm_recur without its workspace; fills `r` (including the status
+// word) and sets *empty when B H T == 0 (nothing to launch).
+sdm_status recur_args(const char* who, const sdm_shape* s, const int32_t* idx_w, const float* w_w,
+                      const int32_t* idx_r, const float* w_r, const void* v, const void* alpha, const void* beta,
+                      void* mem, void* y, RecArgs* r, bool* empty) {
+    SDM_TRY(check_shape(s, false, nullptr));
+    const size_t es = elem_bytes(s->dtype);
+    const size_t bht = static_cast<size_t>(s->B) * s->H * s->T;
+    *empty = bht == 0;
+    if (*empty) return ok();
+    SDM_TRY(check_vec(idx_w, "idx_w", 4));
+    SDM_TRY(check_vec(w_w, "w_w", 4));
+    SDM_TRY(check_vec(idx_r, "idx_r", 4));
+    SDM_TRY(check_vec(w_r, "w_r", 4));
+    SDM_TRY(check_vec(v, "v", 16));
+    SDM_TRY(check_vec(alpha, "alpha", es));
+    SDM_TRY(check_vec(beta, "beta", es));
+    SDM_TRY(check_vec(mem, "mem", 16));
+    SDM_TRY(check_vec(y, "y", 16));
+    const size_t rowb = static_cast<size_t>(s->d_v) * es;
+    const Range rm{mem, static_cast<size_t>(s->B) * s->H * static_cast<size_t>(s->N) * rowb, "mem"};
+    const Range others[] = {{idx_w, bht * s->k_write * 4, "idx_w"}, {w_w, bht * s->k_write * 4, "w_w"},
+                            {idx_r, bht * s->k_read * 4, "idx_r"},  {w_r, bht * s->k_read * 4, "w_r"},
+                            {v, bht * rowb, "v"}, {alpha, bht * es, "alpha"}, {beta, bht * es, "beta"},
+                            {y, bht * rowb, "y"}};
+    for (const Range& q : others)
+        if (overlaps(rm, q)) return fail(SDM_ERR_INVALID_ARG, "%s: mem overlaps %s", who, q.name);
+    int* err = nullptr;
+    SDM_TRY(status_word(&err));
+    *r = RecArgs{};
+    r->idx_w = idx_w; r->w_w = w_w; r->idx_r = idx_r; r->w_r = w_r;
+    r->v = v; r->alpha = alpha; r->beta = beta; r->mem = mem; r->y = y;
+    r->B = s->B; r->H = s->H; r->T = s->T; r->dv = s->d_v; r->kw = s->k_write; r->kr = s->k_read;
+    r->N = s->N;
+    r->err = err;
+    return SDM_OK;
+}
+
+}  // namespace sdm

@@ -4,6 +4,7 @@
 #include <stdint.h>
 #include <stddef.h>
 
+#include "sdm.h"
 #include "sdm_common.cuh"
 
 namespace sdm {
@@ -69,5 +70,13 @@ RecPlan rec_plan(int dtype, int B, int H, int T, int dv, int kw, int kr);
 size_t rec_workspace_bytes(int B, int H, int T, int kw, int kr);
 // Runs the hazard pass, then the recurrence.  hz_ws: rec_workspace_bytes() of scratch.
 cudaError_t launch_recur(int dtype, const RecArgs& a, int32_t* hz_ws, cudaStream_t stream);
+
+// Error reporting and the checks of sdm_recur (minus its workspace), for entry points
+// in other translation units (sdm_api.cu).
+sdm_status api_error(sdm_status st, const char* msg);
+sdm_status api_ok();
+sdm_status recur_args(const char* who, const sdm_shape* s, const int32_t* idx_w, const float* w_w,
+                      const int32_t* idx_r, const float* w_r, const void* v, const void* alpha, const void* beta,
+                      void* mem, void* y, RecArgs* r, bool* empty);
 
 }  // namespace sdm
