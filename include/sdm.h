@@ -169,12 +169,13 @@ sdm_status sdm_recur_noalloc(const sdm_shape* shape, const int32_t* idx_w, const
  * (<= 15) event counters of the current device's selection diagnostics:
  *   [0] a per-half top-k boundary not certified by the fp32 scores (scores closer than
  *       their error bound): the band is re-ranked by compensated rescoring
- *   [1] a whole half rescored in float64 (band wider than the kept list)
- *   [2] the outer-sum boundary not certified by the fp32 scores
- *   [3] all k^2 outer-sum candidates rescored in float64
+ *   [1] ... whose band reached past the kept list (the whole half is rescanned)
+ *   [2] an outer-sum boundary not certified by the fp32 scores
+ *   [3] ... whose band reached past 64 candidates (serial float64 resolution)
  *   [4] a survivor-buffer overflow retried on the tensor-core score path
- *   [5] an outer-sum candidate set too large for the sort network (exact merge used)
- *   [6] a band decided by the serial float64 rescoring (compensated scores too close)
+ *   [5] an outer-sum band that reached the last kept candidate (list extended to 64)
+ *   [6] a band near-tie decided by float64 rescoring of its entries
+ *   [7] the serial float64 fallback (heavy ties)
  * Counters wrap modulo 2^32. */
 sdm_status sdm_device_stats(uint32_t* counts, int n, sdm_stream_t stream);
 

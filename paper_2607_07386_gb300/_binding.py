@@ -187,7 +187,7 @@ def device_status(stream=None) -> int:
     return int(code.value)
 
 
-STAT_NAMES = ("half_band", "half_full", "comb_band", "comb_full", "select_retry", "comb_merge", "band_f64")
+STAT_NAMES = ("half_band", "half_full", "comb_band", "comb_full", "select_retry", "comb_merge", "band_f64", "serial")
 
 
 def device_stats(stream=None) -> dict:

@@ -202,7 +202,6 @@ __device__ __noinline__ void resolve_half(const float* lv, const int* li, int k,
     const double hi = static_cast<double>(lv[k]) + 2.0 * eps;
     if (c.S > L && static_cast<double>(lv[L - 1]) >= lo) {
         // Band may extend past the list: exact top-k of the whole half in float64.
-        stat_add(c.err, STAT_HALF_FULL);
         double bv[64 + 4];
         int bi[64 + 4];
         int n = 0;
@@ -216,7 +215,6 @@ __device__ __noinline__ void resolve_half(const float* lv, const int* li, int k,
         for (int p = 0; p < k; ++p) { Av[p * pitch] = static_cast<float>(bv[p]); Ai[p * pitch] = bi[p]; }
         return;
     }
-    stat_add(c.err, STAT_BAND_F64);
     int cin = 0;
     while (cin < L && static_cast<double>(lv[cin]) > hi) ++cin;
     int pend = cin;
@@ -259,7 +257,6 @@ __device__ __noinline__ void resolve_combined(const float* cv, const int* cf, in
     const double hi = static_cast<double>(cv[k]) + 2.0 * epsc;
     if (cv[L - 1] != -INFINITY && static_cast<double>(cv[L - 1]) >= lo) {
         // All k^2 candidates in float64.
-        stat_add(c.err, STAT_COMB_FULL);
         double s1[64], s2[64];
         for (int p = 0; p < k; ++p) { s1[p] = score64<D>(c, 0, A1i[p * pitch]); s2[p] = score64<D>(c, 1, A2i[p * pitch]); }
         double bv[64];
@@ -282,7 +279,6 @@ __device__ __noinline__ void resolve_combined(const float* cv, const int* cf, in
         }
         return;
     }
-    stat_add(c.err, STAT_BAND_F64);
     int cin = 0;
     while (cin < L && static_cast<double>(cv[cin]) > hi) ++cin;
     int pend = cin;
@@ -345,85 +341,135 @@ __device__ __forceinline__ int lane_geti(int i0, int i1, int idx) {
     return idx < 32 ? a : b;
 }
 
-// Compensated fp32 score of column j of half hf (one lane, one column).  Every product is
-// split exactly (p + pe = P x, pe = 0 for bf16 operands) and every addition exactly by
-// TwoSum (s + err = s_old + p); the error terms are summed in plain fp32.  With n = d_k
-// terms and u = 2^-24 the result val = s + e differs from the exact dot product by at
-// most 2 n (n + 1) u^2 (1.03) sum|P x| <= 2^-31 sum|P x| for n <= 256.  The float64
-// sequential sum of the definition lies within (n - 1) 2^-53 sum|P x| of the exact value,
-// so `bound` = 2^-28 sum|P x| (+ 2^-50 |val| for the conversion to double) covers the
-// distance to it with margin.  DIRECT addressing: the score is x itself, exact (bound 0).
-template <class D>
-__device__ void ff_score(const TokenCtx& c, int hf, int j, double& val, double& bound) {
-    if (c.P == nullptr) {
-        val = static_cast<double>(load_elem<D>(c.X, c.xoff + static_cast<int64_t>(hf) * c.S + j));
-        bound = 0.0;
-        return;
-    }
-    const int64_t prow = (c.prow0 + static_cast<int64_t>(hf) * c.S + j) * c.dk;
-    float sum = 0.f, err = 0.f, mag = 0.f;
-#pragma unroll 8
-    for (int d = 0; d < c.dk; ++d) {
-        const float pv = load_elem<D>(c.P, prow + d);
-        const float xv = load_elem<D>(c.X, c.xoff + d);
-        const float p = __fmul_rn(pv, xv);
-        const float pe = __fmaf_rn(pv, xv, -p);
-        const float t = __fadd_rn(sum, p);
-        const float bp = __fsub_rn(t, sum);
-        const float e2 = __fadd_rn(__fsub_rn(sum, __fsub_rn(t, bp)), __fsub_rn(p, bp));
-        sum = t;
-        err = __fadd_rn(err, __fadd_rn(e2, pe));
-        mag = __fadd_rn(mag, fabsf(p));
-    }
-    val = static_cast<double>(sum) + static_cast<double>(err);
-    bound = 0x1p-28 * static_cast<double>(mag) + 0x1p-50 * fabs(val);
+// All decisions of the warp finalize run in fp32 (GB300's float64 rate is a small
+// fraction of its fp32 rate): error bounds are rounded up and differences rounded down
+// (directed-rounding intrinsics), so every "certain" decision is also certain in exact
+// arithmetic.  float64 remains only in the serial fallbacks.
+
+// Float-float value h + l (|l| <= ulp(h)/2) with an error bound b on its distance to the
+// float64 score of the definition.
+struct FF {
+    float h, l, b;
+};
+
+__device__ __forceinline__ void two_sum(float a, float b, float& s, float& e) {
+    s = __fadd_rn(a, b);
+    const float bp = __fsub_rn(s, a);
+    e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bp)), __fsub_rn(b, bp));
 }
 
-// Band entries [cin, cin + m) of a list sorted by fp32 score are re-ranked by their
-// compensated scores (one lane per entry).  Returns false when two entries are closer
-// than their bounds (the float64 definition must decide) -- otherwise the ranks are
-// those of the float64 definition under (score desc, index asc).
-__device__ __forceinline__ bool rank_band(double cd, double eb, int id, int m, int lane, int& rank) {
+// Compensated score of column j of half hf, computed by the whole warp (every lane gets
+// the result).  Lane l owns the terms d = l + 32 r (its x values are in xr).  Every product
+// is split exactly (p + pe = P x; pe = 0 for bf16 operands) and every addition of the main
+// sum -- within a lane and across the butterfly -- exactly by TwoSum; only the error terms
+// are summed in plain fp32.  With n = d_k terms and u = 2^-24 the result s + e differs
+// from the exact dot product by at most 2 n (n + 1) u^2 (1.03) sum|P x| <= 2^-31 sum|P x|
+// for n <= 256, whatever the order of the additions.  The float64 sequential sum of the
+// definition lies within (n - 1) 2^-53 sum|P x| of the exact value, so b = 2^-28 sum|P x|
+// covers the distance to it with margin (also for the rounding of sum|P x| itself).
+// DIRECT addressing: the score is x itself, exact.
+template <class D>
+__device__ FF ff_score_warp(const TokenCtx& c, const float (&xr)[8], int hf, int j, int lane) {
+    if (c.P == nullptr) return FF{load_elem<D>(c.X, c.xoff + static_cast<int64_t>(hf) * c.S + j), 0.f, 0.f};
+    const int64_t prow = (c.prow0 + static_cast<int64_t>(hf) * c.S + j) * c.dk;
+    float pv[8];
+#pragma unroll
+    for (int r = 0; r < 8; ++r) {
+        const int d = lane + 32 * r;
+        pv[r] = (r * 32 < c.dk && d < c.dk) ? load_elem<D>(c.P, prow + d) : 0.f;
+    }
+    float sum = 0.f, err = 0.f, mag = 0.f;
+#pragma unroll
+    for (int r = 0; r < 8; ++r) {
+        if (r * 32 < c.dk) {
+            const float p = __fmul_rn(pv[r], xr[r]);
+            const float pe = __fmaf_rn(pv[r], xr[r], -p);
+            float t, e2;
+            two_sum(sum, p, t, e2);
+            sum = t;
+            err = __fadd_rn(err, __fadd_rn(e2, pe));
+            mag = __fadd_rn(mag, fabsf(p));
+        }
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+        const float so = __shfl_xor_sync(0xffffffffu, sum, off);
+        const float eo = __shfl_xor_sync(0xffffffffu, err, off);
+        const float mo = __shfl_xor_sync(0xffffffffu, mag, off);
+        float t, e2;
+        two_sum(sum, so, t, e2);                   // same t and e2 in both lanes of the pair
+        sum = t;
+        err = __fadd_rn(__fadd_rn(err, eo), e2);   // (err + eo) is the same in both lanes
+        mag = __fadd_rn(mag, mo);
+    }
+    FF r;
+    r.h = __fadd_rn(sum, err);                      // FastTwoSum: |err| << |sum|
+    r.l = __fsub_rn(err, __fsub_rn(r.h, sum));
+    r.b = __fmul_ru(0x1p-28f, mag);
+    return r;
+}
+
+// a + b for two compensated half scores (the float64 definition adds its two half scores
+// with one more rounding of at most 2^-53 of the sum; 2^-44 |sum| covers that and ours).
+__device__ __forceinline__ FF ff_add(const FF& a, const FF& b, bool direct) {
+    float h, r;
+    two_sum(a.h, b.h, h, r);
+    const float l = __fadd_rn(__fadd_rn(a.l, b.l), r);
+    FF o;
+    o.h = __fadd_rn(h, l);
+    o.l = __fsub_rn(l, __fsub_rn(o.h, h));
+    const float slack = direct ? __fmul_ru(0x1p-52f, fabsf(o.h)) : __fmul_ru(0x1p-44f, fabsf(o.h));
+    o.b = __fadd_ru(__fadd_ru(a.b, b.b), slack);
+    return o;
+}
+
+// Band entries (lane e < m holds entry e: compensated score v, index id) are ranked under
+// (score desc, index asc).  Returns false when two entries are closer than their bounds
+// (the float64 definition must decide); otherwise the ranks are those of the float64
+// definition.  The difference (hf + lf) - (h + l) is formed with TwoSum on the leading
+// parts; the roundings of the rest are covered by `slack`.
+__device__ __forceinline__ bool rank_band(const FF& v, int id, int m, int lane, int& rank) {
     rank = 0;
     bool unsure = false;
     for (int f = 0; f < m; ++f) {
-        const double cf = __shfl_sync(0xffffffffu, cd, f);
-        const double ef = __shfl_sync(0xffffffffu, eb, f);
+        const float hf = __shfl_sync(0xffffffffu, v.h, f);
+        const float lf = __shfl_sync(0xffffffffu, v.l, f);
+        const float bf = __shfl_sync(0xffffffffu, v.b, f);
         const int jf = __shfl_sync(0xffffffffu, id, f);
         if (lane < m && f != lane) {
-            const double tol = ef + eb;
-            const double diff = cf - cd;
-            if (tol > 0.0 && fabs(diff) <= tol) unsure = true;
-            else rank += (diff > 0.0 || (diff == 0.0 && jf < id)) ? 1 : 0;
+            float t, r;
+            two_sum(hf, -v.h, t, r);
+            const float w = __fadd_rn(__fsub_rn(lf, v.l), r);
+            const float diff = __fadd_rn(t, w);
+            const float slack = __fmul_ru(0x1p-21f, __fadd_ru(__fadd_ru(fabsf(t), fabsf(r)), __fadd_ru(fabsf(lf), fabsf(v.l))));
+            const float tol = __fadd_ru(__fadd_ru(bf, v.b), slack);
+            if (tol > 0.f && fabsf(diff) <= tol) unsure = true;
+            else rank += (diff > 0.f || (diff == 0.f && jf < id)) ? 1 : 0;
         }
     }
     return !__any_sync(0xffffffffu, unsure);
 }
 
-// Warp-cooperative resolution of an uncertified half boundary (list: lane p holds entry p
-// in v0/i0 and entry p + 32 in v1/i1).  On success writes the exact top-k, in fp32-list
-// order, to ov/oi[0, k) and returns true; returns false when the serial float64 path must
-// decide (band past the list, more than 32 band entries, or an unresolved near-tie).
-template <class D, int L>
-__device__ bool warp_band_half(float v0, int i0, float v1, int i1, int k, double eps, const TokenCtx& c, int hf,
-                               float* ov, int* oi, int lane) {
-    const double lo = static_cast<double>(lane_get(v0, v1, k - 1)) - 2.0 * eps;
-    const double hi = static_cast<double>(lane_get(v0, v1, k)) + 2.0 * eps;
-    if (c.S > L && static_cast<double>(lane_get(v0, v1, L - 1)) >= lo) return false;
-    const double d0 = static_cast<double>(v0), d1 = static_cast<double>(v1);
-    const int cin = __popc(__ballot_sync(0xffffffffu, lane < L && d0 > hi)) +
-                    __popc(__ballot_sync(0xffffffffu, lane + 32 < L && d1 > hi));
-    const int m = __popc(__ballot_sync(0xffffffffu, lane < L && d0 >= lo && d0 <= hi)) +
-                  __popc(__ballot_sync(0xffffffffu, lane + 32 < L && d1 >= lo && d1 <= hi));
-    if (m > 32) return false;
-    const int p = min(cin + lane, L - 1);
-    const float bv = lane_get(v0, v1, p);
-    const int bi = lane_geti(i0, i1, p);
-    double cd = 0.0, eb = 0.0;
-    if (lane < m) ff_score<D>(c, hf, bi, cd, eb);
-    int rank;
-    if (!rank_band(cd, eb, bi, m, lane, rank)) return false;
-    const bool chosen = lane < m && rank < k - cin;
+// Band of an uncertified top-k boundary in a list of `len` (<= 64) entries sorted by fp32
+// value (lane p: entry p in v0/i0, entry p + 32 in v1/i1): entries [cin, cin + m) lie
+// within e2 (twice the error bound, rounded up) of the boundary.  False if the band may
+// continue past the list or holds more than 32 entries.
+__device__ __forceinline__ bool band_of(float v0, float v1, int len, int k, float e2, bool list_is_all, int lane,
+                                        int& cin, int& m) {
+    const float lo = __fsub_rd(lane_get(v0, v1, k - 1), e2);
+    const float hi = __fadd_ru(lane_get(v0, v1, k), e2);
+    const float vl = lane_get(v0, v1, len - 1);
+    if (!list_is_all && vl != -INFINITY && vl >= lo) return false;
+    cin = __popc(__ballot_sync(0xffffffffu, lane < len && v0 > hi)) +
+          __popc(__ballot_sync(0xffffffffu, lane + 32 < len && v1 > hi));
+    m = __popc(__ballot_sync(0xffffffffu, lane < len && v0 >= lo && v0 <= hi)) +
+        __popc(__ballot_sync(0xffffffffu, lane + 32 < len && v1 >= lo && v1 <= hi));
+    return m <= 32;
+}
+
+// Writes the certain entries [0, cin) and the chosen band entries (in list order) to ov/oi.
+__device__ __forceinline__ void emit_band(float v0, int i0, float bv, int bi, bool chosen, int cin, float* ov, int* oi,
+                                          int lane) {
     const unsigned ch = __ballot_sync(0xffffffffu, chosen);
     __syncwarp();
     if (lane < cin) { ov[lane] = v0; oi[lane] = i0; }
@@ -433,62 +479,203 @@ __device__ bool warp_band_half(float v0, int i0, float v1, int i1, int k, double
         oi[q] = bi;
     }
     __syncwarp();
-    return true;
 }
 
-// Same for the outer-sum boundary: candidate slot f = i S + j is rescored as the sum of
-// the compensated half scores of column i (half 0) and column j (half 1).  The float64
-// definition adds its two half scores with one more rounding (<= 2^-53 of the sum).
+// Warp-cooperative resolution of an uncertified half boundary (e2 = twice the fp32 error
+// bound of the scores).  On success writes the exact top-k, in fp32-list order, to
+// ov/oi[0, k) and returns true; false when the serial float64 path must decide (band past
+// the list, more than 32 band entries, or a near-tie).
+enum : int { BAND_DONE = 0, BAND_NEAR_TIE = 1, BAND_OUTSIDE = 2 };
+
 template <class D, int L>
-__device__ bool warp_band_comb(float v0, int f0, float v1, int f1, int k, double epsc, const TokenCtx& c,
-                               float* ov, int* oi, int lane) {
-    const double lo = static_cast<double>(lane_get(v0, v1, k - 1)) - 2.0 * epsc;
-    const double hi = static_cast<double>(lane_get(v0, v1, k)) + 2.0 * epsc;
-    const float vl = lane_get(v0, v1, L - 1);
-    if (vl != -INFINITY && static_cast<double>(vl) >= lo) return false;
-    const double d0 = static_cast<double>(v0), d1 = static_cast<double>(v1);
-    const int cin = __popc(__ballot_sync(0xffffffffu, lane < L && d0 > hi)) +
-                    __popc(__ballot_sync(0xffffffffu, lane + 32 < L && d1 > hi));
-    const int m = __popc(__ballot_sync(0xffffffffu, lane < L && d0 >= lo && d0 <= hi)) +
-                  __popc(__ballot_sync(0xffffffffu, lane + 32 < L && d1 >= lo && d1 <= hi));
-    if (m > 32) return false;
+__device__ int warp_band_half(float v0, int i0, float v1, int i1, int k, float e2, const TokenCtx& c,
+                              const float (&xr)[8], int hf, float* ov, int* oi, int lane) {
+    int cin, m;
+    if (!band_of(v0, v1, L, k, e2, c.S <= L, lane, cin, m)) return BAND_OUTSIDE;
     const int p = min(cin + lane, L - 1);
     const float bv = lane_get(v0, v1, p);
-    const int bf = lane_geti(f0, f1, p);
-    double cd = 0.0, eb = 0.0;
-    if (lane < m) {
-        double c1, e1, c2, e2;
-        ff_score<D>(c, 0, bf / c.S, c1, e1);
-        ff_score<D>(c, 1, bf % c.S, c2, e2);
-        cd = c1 + c2;
-        eb = (c.P == nullptr) ? 0.0 : e1 + e2 + 0x1p-50 * fabs(cd);
+    const int bi = lane_geti(i0, i1, p);
+    FF mine{0.f, 0.f, 0.f};
+    for (int e = 0; e < m; ++e) {
+        const FF sc = ff_score_warp<D>(c, xr, hf, __shfl_sync(0xffffffffu, bi, e), lane);
+        if (lane == e) mine = sc;
     }
     int rank;
-    if (!rank_band(cd, eb, bf, m, lane, rank)) return false;
-    const bool chosen = lane < m && rank < k - cin;
-    const unsigned ch = __ballot_sync(0xffffffffu, chosen);
-    __syncwarp();
-    if (lane < cin) { ov[lane] = v0; oi[lane] = f0; }
-    if (chosen) {
-        const int q = cin + __popc(ch & ((1u << lane) - 1u));
-        ov[q] = bv;
-        oi[q] = bf;
+    if (!rank_band(mine, bi, m, lane, rank)) return BAND_NEAR_TIE;
+    emit_band(v0, i0, bv, bi, lane < m && rank < k - cin, cin, ov, oi, lane);
+    return BAND_DONE;
+}
+
+// Near-tie in the band: float64 scores of the definition (sequential d order, so equal to
+// it bit for bit), one lane per band entry; the ranking is then exact.
+template <class D>
+__device__ void warp_band64(float v0, int i0, float v1, int i1, int len, int k, float e2, bool all, bool comb,
+                            const TokenCtx& c, int hf, float* ov, int* oi, int lane) {
+    int cin, m;
+    band_of(v0, v1, len, k, e2, all, lane, cin, m);       // succeeded before with the same arguments
+    const int p = min(cin + lane, len - 1);
+    const float bv = lane_get(v0, v1, p);
+    const int bi = lane_geti(i0, i1, p);
+    double s64 = 0.0;
+    if (lane < m) s64 = comb ? score64<D>(c, 0, bi / c.S) + score64<D>(c, 1, bi % c.S) : score64<D>(c, hf, bi);
+    int rank = 0;
+    for (int f = 0; f < m; ++f) {
+        const double sf = __shfl_sync(0xffffffffu, s64, f);
+        const int jf = __shfl_sync(0xffffffffu, bi, f);
+        if (lane < m && f != lane && beats64(sf, jf, s64, bi)) ++rank;
     }
+    emit_band(v0, i0, bv, bi, lane < m && rank < k - cin, cin, ov, oi, lane);
+}
+
+// Descending bitonic sort of 64 floats held two per lane (element lane in a, lane + 32 in b).
+__device__ __forceinline__ void warp_sort64_desc(float& a, float& b, int lane) {
+#pragma unroll
+    for (int size = 2; size <= 64; size <<= 1) {
+#pragma unroll
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+            if (stride == 32) {                                 // elements lane and lane + 32
+                const float hi = fmaxf(a, b), lo = fminf(a, b);
+                a = hi; b = lo;                                 // size == 64: descending
+            } else {
+                const float pa = __shfl_xor_sync(0xffffffffu, a, stride);
+                const float pb = __shfl_xor_sync(0xffffffffu, b, stride);
+                const bool lower = (lane & stride) == 0;
+                // element e = lane (+ 32): its block of `size` sorts descending iff (e & size) == 0
+                const bool desc_a = (lane & size) == 0;
+                const bool desc_b = ((lane + 32) & size) == 0;
+                a = (lower == desc_a) ? fmaxf(a, pa) : fminf(a, pa);
+                b = (lower == desc_b) ? fmaxf(b, pb) : fminf(b, pb);
+            }
+        }
+    }
+}
+
+// The band of a half boundary reaches past the kept list: exact top-k over the whole half.
+//   pass 1: fp32 scores (warp tree sum, error <= eps), each lane keeps the top 2 of the
+//           columns j = lane (mod 32); theta = k-th largest of those 64 values (>= k columns
+//           reach it, so the k-th largest exact score is >= theta - eps);
+//   pass 2: columns with fp32 score >= theta - 2 eps (a superset of the exact top-k) are
+//           collected (at most 64, else false), rescored compensated and ranked.
+// Writes the top-k in order (value fl32 of the compensated score, index) to ov/oi.
+template <class D>
+__device__ bool warp_full_half(int k, float e2, const TokenCtx& c, const float (&xr)[8], int hf, float* ov, int* oi,
+                               int* scratch, int lane) {
+    const int S = c.S;
+    auto fp32_score = [&](int j) -> float {
+        const int64_t prow = (c.prow0 + static_cast<int64_t>(hf) * S + j) * c.dk;
+        float acc = 0.f;
+#pragma unroll
+        for (int r = 0; r < 8; ++r) {
+            const int d = lane + 32 * r;
+            if (r * 32 < c.dk && d < c.dk) acc = fmaf(load_elem<D>(c.P, prow + d), xr[r], acc);
+        }
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+        return acc;
+    };
+    float t1 = -INFINITY, t2 = -INFINITY;
+    for (int j = 0; j < S; ++j) {
+        const float sc = fp32_score(j);
+        if ((j & 31) == lane) { t2 = fmaxf(t2, fminf(t1, sc)); t1 = fmaxf(t1, sc); }
+    }
+    warp_sort64_desc(t1, t2, lane);
+    const float theta = lane_get(t1, t2, k - 1);
+    const float lo = __fsub_rd(theta, e2);
+    int m = 0;
+    for (int j = 0; j < S; ++j) {
+        const float sc = fp32_score(j);
+        if (sc >= lo) {                                          // warp-uniform
+            if (m < 64 && lane == 0) scratch[m] = j;
+            ++m;
+        }
+    }
+    if (m > 64) return false;
+    __syncwarp();
+    const int j0 = lane < m ? scratch[lane] : 0;
+    const int j1 = lane + 32 < m ? scratch[lane + 32] : 0;
+    __syncwarp();
+    FF f0{0.f, 0.f, 0.f}, f1{0.f, 0.f, 0.f};
+    for (int e = 0; e < m; ++e) {
+        const FF sc = ff_score_warp<D>(c, xr, hf, lane_geti(j0, j1, e), lane);
+        if (e == lane) f0 = sc;
+        if (e == lane + 32) f1 = sc;
+    }
+    // rank both own entries against all m (pairs closer than their bounds: give up)
+    int r0 = 0, r1 = 0;
+    bool unsure = false;
+    for (int f = 0; f < m; ++f) {
+        const int src = f & 31;
+        const bool hi = f >= 32;
+        const float hA = __shfl_sync(0xffffffffu, f0.h, src), hB = __shfl_sync(0xffffffffu, f1.h, src);
+        const float lA = __shfl_sync(0xffffffffu, f0.l, src), lB = __shfl_sync(0xffffffffu, f1.l, src);
+        const float bA = __shfl_sync(0xffffffffu, f0.b, src), bB = __shfl_sync(0xffffffffu, f1.b, src);
+        const FF ff{hi ? hB : hA, hi ? lB : lA, hi ? bB : bA};
+        const int jf = lane_geti(j0, j1, f);
+#pragma unroll
+        for (int q = 0; q < 2; ++q) {
+            const int e = lane + 32 * q;
+            const FF& mine = q ? f1 : f0;
+            const int je = q ? j1 : j0;
+            if (e < m && e != f) {
+                float t, r;
+                two_sum(ff.h, -mine.h, t, r);
+                const float w = __fadd_rn(__fsub_rn(ff.l, mine.l), r);
+                const float diff = __fadd_rn(t, w);
+                const float slack = __fmul_ru(0x1p-21f, __fadd_ru(__fadd_ru(fabsf(t), fabsf(r)), __fadd_ru(fabsf(ff.l), fabsf(mine.l))));
+                const float tol = __fadd_ru(__fadd_ru(ff.b, mine.b), slack);
+                if (tol > 0.f && fabsf(diff) <= tol) unsure = true;
+                else if (diff > 0.f || (diff == 0.f && jf < je)) { if (q) ++r1; else ++r0; }
+            }
+        }
+    }
+    if (__any_sync(0xffffffffu, unsure)) return false;
+    __syncwarp();
+    if (lane < m && r0 < k) { ov[r0] = f0.h; oi[r0] = j0; }
+    if (lane + 32 < m && r1 < k) { ov[r1] = f1.h; oi[r1] = j1; }
     __syncwarp();
     return true;
 }
 
+// Same for the outer-sum boundary over a candidate list of `len` (<= 64) entries: slot
+// f = i S + j is rescored as the sum of the compensated half scores of column i (half 0)
+// and column j (half 1).
+template <class D>
+__device__ int warp_band_comb(float v0, int f0, float v1, int f1, int len, int k, float e2c, const TokenCtx& c,
+                              const float (&xr)[8], bool all, float* ov, int* oi, int lane) {
+    int cin, m;
+    if (!band_of(v0, v1, len, k, e2c, all, lane, cin, m)) return BAND_OUTSIDE;
+    const int p = min(cin + lane, len - 1);
+    const float bv = lane_get(v0, v1, p);
+    const int bf = lane_geti(f0, f1, p);
+    FF mine{0.f, 0.f, 0.f};
+    for (int e = 0; e < m; ++e) {
+        const int fe = __shfl_sync(0xffffffffu, bf, e);
+        const FF s1 = ff_score_warp<D>(c, xr, 0, fe / c.S, lane);
+        const FF s2 = ff_score_warp<D>(c, xr, 1, fe % c.S, lane);
+        const FF sum = ff_add(s1, s2, c.P == nullptr);
+        if (lane == e) mine = sum;
+    }
+    int rank;
+    if (!rank_band(mine, bf, m, lane, rank)) return BAND_NEAR_TIE;
+    emit_band(v0, f0, bv, bf, lane < m && rank < k - cin, cin, ov, oi, lane);
+    return BAND_DONE;
+}
+
 template <class D, int L>
-__global__ void __launch_bounds__(FW_WARPS * 32) k_addr_finalize(const AddrArgs a) {
+__global__ void __launch_bounds__(FW_WARPS * 32, 4) k_addr_finalize(const AddrArgs a) {
     static_assert(L <= 36, "warp finalize handles k <= 32");
     __shared__ float wv[FW_WARPS][3][64];
     __shared__ int wi[FW_WARPS][3][64];
     const int lane = threadIdx.x & 31, wq = threadIdx.x >> 5;
-    const int z = blockIdx.y;
-    const int side = z / a.H, h = z % a.H;
     const int64_t BT = static_cast<int64_t>(a.B) * a.T;
-    const int64_t u = static_cast<int64_t>(blockIdx.x) * FW_WARPS + wq;
-    if (u >= BT) return;                                   // whole warp
+    const int64_t items = 2 * a.H * BT;
+    // persistent warps: a warp takes token-sides item, item + (all warps), ... so that slow
+    // token-sides (band rescoring) do not hold a whole CTA's slot
+    for (int64_t item = static_cast<int64_t>(blockIdx.x) * FW_WARPS + wq; item < items;
+         item += static_cast<int64_t>(gridDim.x) * FW_WARPS) {
+    const int z = static_cast<int>(item / BT);
+    const int64_t u = item - z * BT;
+    const int side = z / a.H, h = z % a.H;
     const int k = a.kk[side];
     const int S = a.S;
     const int64_t b = u / a.T, t = u - b * a.T;
@@ -504,18 +691,22 @@ __global__ void __launch_bounds__(FW_WARPS * 32) k_addr_finalize(const AddrArgs 
     float* sv1 = wv[wq][1]; int* si1 = wi[wq][1];          // A2
     float* sv2 = wv[wq][2]; int* si2 = wi[wq][2];          // candidates / final
 
-    double eps = 0.0;
+    float e2 = 0.f;                                        // 2 x the fp32 score error bound, rounded up
+    float xr[8];                                           // x[lane + 32 r] (projected mode)
     if (c.P != nullptr) {
         float ss = 0.f;
-        for (int d = lane; d < a.dk; d += 32) {
-            const float xv = load_elem<D>(c.X, c.xoff + d);
-            ss = fmaf(xv, xv, ss);
+#pragma unroll
+        for (int r = 0; r < 8; ++r) {
+            const int d = lane + 32 * r;
+            xr[r] = (r * 32 < a.dk && d < a.dk) ? load_elem<D>(c.X, c.xoff + d) : 0.f;
+            ss = fmaf(xr[r], xr[r], ss);
         }
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
-        eps = static_cast<double>(a.cbound) * static_cast<double>(a.pnorm[side * a.H + h]) *
-              static_cast<double>(sqrtf(ss)) * (1.0 + 0x1p-12);
+        // (1 + 2^-12) covers the roundings of ||x||^2, its square root and the products
+        e2 = __fmul_ru(__fmul_ru(__fmul_ru(2.f * a.cbound, a.pnorm[side * a.H + h]), sqrtf(ss)), 1.f + 0x1p-12f);
     }
+    const double eps = 0.5 * static_cast<double>(e2);    // for the serial float64 fallbacks
 
     float av[2], bv[2];      // A1 and A2 after certification: lane p holds entry p (p < k)
     int ai[2], bi[2];
@@ -552,11 +743,22 @@ __global__ void __launch_bounds__(FW_WARPS * 32) k_addr_finalize(const AddrArgs 
         bool certified = S <= k;
         if (!certified) {
             const float vk = lane_get(v0, v1, k - 1), vk1 = lane_get(v0, v1, k);
-            certified = static_cast<double>(vk) - static_cast<double>(vk1) > 2.0 * eps;
+            certified = __fsub_rd(vk, vk1) > e2;
         }
         if (!certified) {
             if (lane == 0) stat_add(c.err, STAT_HALF_BAND);
-            if (!warp_band_half<D, L>(v0, i0, v1, i1, k, eps, c, hf, sv0, si0, lane)) {
+            const int res = warp_band_half<D, L>(v0, i0, v1, i1, k, e2, c, xr, hf, sv0, si0, lane);
+            bool done = res == BAND_DONE;
+            if (res == BAND_NEAR_TIE) {
+                if (lane == 0) stat_add(c.err, STAT_BAND_F64);
+                warp_band64<D>(v0, i0, v1, i1, L, k, e2, S <= L, false, c, hf, sv0, si0, lane);
+                done = true;
+            } else if (res == BAND_OUTSIDE) {
+                if (lane == 0) stat_add(c.err, STAT_HALF_FULL);
+                done = c.P != nullptr && warp_full_half<D>(k, e2, c, xr, hf, sv0, si0, si2, lane);
+            }
+            if (!done) {
+                if (lane == 0) stat_add(c.err, STAT_SERIAL);
                 __syncwarp();
                 if (lane < L) { sv0[lane] = v0; si0[lane] = i0; }
                 if (lane + 32 < L) { sv0[lane + 32] = v1; si0[lane + 32] = i1; }
@@ -578,7 +780,9 @@ __global__ void __launch_bounds__(FW_WARPS * 32) k_addr_finalize(const AddrArgs 
     }
 
     // combined: k-way merge of the rows (lane i: row i; head = A1[i] + A2[j])
-    const double epsc = 2.0 * eps + 0x1p-22 * (static_cast<double>(amax[0]) + static_cast<double>(amax[1]));
+    // outer-sum bound: both half errors plus the fp32 rounding of A1 + A2 (rounded up, x2)
+    const float e2c = __fadd_ru(__fmul_ru(2.f, e2), __fmul_ru(0x1p-21f, __fadd_ru(amax[0], amax[1])));
+    const double epsc = 0.5 * static_cast<double>(e2c);  // for the serial float64 fallback
     int j = 0;
     const float b0v = __shfl_sync(0xffffffffu, bv[0], 0);
     const int b0i = __shfl_sync(0xffffffffu, bi[0], 0);
@@ -586,35 +790,52 @@ __global__ void __launch_bounds__(FW_WARPS * 32) k_addr_finalize(const AddrArgs 
     int flat = ai[0] * S + b0i;
     float cv0 = -INFINITY, cv1 = -INFINITY;    // candidate r in lane r (r < 32) / lane r-32
     int cf0 = INT_MAX, cf1 = INT_MAX;
-    for (int r = 0; r < L; ++r) {
-        const uint32_t key = f2key(head);
-        const uint32_t kmax = __reduce_max_sync(0xffffffffu, key);
-        const bool tie = key == kmax;
-        const uint32_t fmin = __reduce_min_sync(0xffffffffu, tie ? static_cast<uint32_t>(flat) : 0xffffffffu);
-        const bool win = tie && static_cast<uint32_t>(flat) == fmin;
-        const float val = key2f(kmax);
-        if (lane == (r & 31)) {
-            if (r < 32) { cv0 = val; cf0 = static_cast<int>(fmin); }
-            else { cv1 = val; cf1 = static_cast<int>(fmin); }
+    auto merge_steps = [&](int r0, int r1) {
+        for (int r = r0; r < r1; ++r) {
+            const uint32_t key = f2key(head);
+            const uint32_t kmax = __reduce_max_sync(0xffffffffu, key);
+            const bool tie = key == kmax;
+            const uint32_t fmin = __reduce_min_sync(0xffffffffu, tie ? static_cast<uint32_t>(flat) : 0xffffffffu);
+            const bool win = tie && static_cast<uint32_t>(flat) == fmin;
+            const float val = key2f(kmax);
+            if (lane == (r & 31)) {
+                if (r < 32) { cv0 = val; cf0 = static_cast<int>(fmin); }
+                else { cv1 = val; cf1 = static_cast<int>(fmin); }
+            }
+            if (win) ++j;
+            const float nv = __shfl_sync(0xffffffffu, bv[0], j & 31);
+            const int ni = __shfl_sync(0xffffffffu, bi[0], j & 31);
+            if (win) {
+                head = (j < k && lane < k) ? av[0] + nv : -INFINITY;
+                flat = ai[0] * S + ni;
+            }
         }
-        if (win) ++j;
-        const float nv = __shfl_sync(0xffffffffu, bv[0], j & 31);
-        const int ni = __shfl_sync(0xffffffffu, bi[0], j & 31);
-        if (win) {
-            head = (j < k && lane < k) ? av[0] + nv : -INFINITY;
-            flat = ai[0] * S + ni;
-        }
-    }
+    };
+    merge_steps(0, L);
     bool certified = (k == 1);
     if (!certified) {
         const float ck = lane_get(cv0, cv1, k - 1), ck1 = lane_get(cv0, cv1, k);
-        certified = (ck1 == -INFINITY) || (static_cast<double>(ck) - static_cast<double>(ck1) > 2.0 * epsc);
+        certified = (ck1 == -INFINITY) || (__fsub_rd(ck, ck1) > e2c);
     }
     float fv = cv0;
     int fi = cf0;
     if (!certified) {
         if (lane == 0) stat_add(c.err, STAT_COMB_BAND);
-        if (!warp_band_comb<D, L>(cv0, cf0, cv1, cf1, k, epsc, c, sv2, si2, lane)) {
+        // band may continue past the L candidates: extend the merge to 64 (or all k^2)
+        int len = L;
+        const float vl = lane_get(cv0, cv1, L - 1);
+        if (k * k > L && vl != -INFINITY &&
+            vl >= __fsub_rd(lane_get(cv0, cv1, k - 1), e2c)) {
+            if (lane == 0) stat_add(c.err, STAT_COMB_MERGE);
+            len = min(64, k * k);
+            merge_steps(L, len);
+        }
+        const int res = warp_band_comb<D>(cv0, cf0, cv1, cf1, len, k, e2c, c, xr, len >= k * k, sv2, si2, lane);
+        if (res == BAND_NEAR_TIE) {
+            if (lane == 0) stat_add(c.err, STAT_BAND_F64);
+            warp_band64<D>(cv0, cf0, cv1, cf1, len, k, e2c, len >= k * k, true, c, 0, sv2, si2, lane);
+        } else if (res == BAND_OUTSIDE) {
+            if (lane == 0) { stat_add(c.err, STAT_COMB_FULL); stat_add(c.err, STAT_SERIAL); }
             __syncwarp();
             sv0[lane] = av[0]; si0[lane] = ai[0];            // A1
             sv1[lane] = bv[0]; si1[lane] = bi[0];            // A2
@@ -659,6 +880,8 @@ __global__ void __launch_bounds__(FW_WARPS * 32) k_addr_finalize(const AddrArgs 
         const int64_t tokoff = ((b * a.H + h) * a.T + t) * k;     // [B, H, T, k] layout
         a.idx[side][tokoff + lane] = key;
         a.w[side][tokoff + lane] = e / zsum;
+    }
+    __syncwarp();                                           // per-warp staging is reused
     }
 }
 // ------------------------------------------------------------------------------------------
@@ -855,8 +1078,14 @@ static cudaError_t launch_finalize(const AddrArgs& a, cudaStream_t stream) {
     dim3 gB(static_cast<unsigned>((BT + F_THREADS - 1) / F_THREADS), 2 * a.H);
     cudaError_t e;
     if constexpr (L <= 36) {
-        dim3 gW(static_cast<unsigned>((BT + FW_WARPS - 1) / FW_WARPS), 2 * a.H);
-        k_addr_finalize<D, L><<<gW, FW_WARPS * 32, 0, stream>>>(a);
+        int dev = 0, sms = 0, per_sm = 0;
+        e = cudaGetDevice(&dev);
+        if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_addr_finalize<D, L>, FW_WARPS * 32, 0);
+        if (e != cudaSuccess) return e;
+        const int64_t need = (2 * a.H * BT + FW_WARPS - 1) / FW_WARPS;
+        const int64_t full = static_cast<int64_t>(sms) * (per_sm > 0 ? per_sm : 1);
+        k_addr_finalize<D, L><<<static_cast<unsigned>(need < full ? need : full), FW_WARPS * 32, 0, stream>>>(a);
     } else {
         const size_t smB = static_cast<size_t>(6) * L * F_THREADS * sizeof(float);
         e = cudaFuncSetAttribute(k_addr_finalize_wide<D, L>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smB));

@@ -68,13 +68,14 @@ __device__ __forceinline__ void flag_error(int* err, int bit) {
 // Event counters stored after the status word (read and cleared by sdm_device_stats).
 enum : int {
     STAT_HALF_BAND = 1,      // a half's top-k boundary was not certified by the fp32 scores
-    STAT_HALF_FULL = 2,      // ... and the whole half had to be rescored in float64
+    STAT_HALF_FULL = 2,      // ... and its band reached past the kept list (whole half rescanned)
     STAT_COMB_BAND = 3,      // the outer-sum boundary was not certified by the fp32 scores
-    STAT_COMB_FULL = 4,      // ... and all k^2 candidates were rescored in float64
+    STAT_COMB_FULL = 4,      // ... and its band reached past 64 candidates (serial float64)
     STAT_SELECT_RETRY = 5,   // a warp's survivor buffer overflowed once (tensor-core path)
-    STAT_COMB_MERGE = 6,     // too many outer-sum candidates: exact k-way merge instead
-    STAT_BAND_F64 = 7,       // a band was decided by the serial float64 rescoring
-    STAT_COUNT = 8
+    STAT_COMB_MERGE = 6,     // the outer-sum band reached the L-th candidate: merge extended to 64
+    STAT_BAND_F64 = 7,       // a band near-tie was decided by float64 rescoring
+    STAT_SERIAL = 8,         // the serial float64 fallback ran (heavy ties)
+    STAT_COUNT = 9
 };
 __device__ __forceinline__ void stat_add(int* err, int which) {
     if (err) atomicAdd(reinterpret_cast<unsigned*>(err) + which, 1u);

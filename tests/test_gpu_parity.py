@@ -132,6 +132,61 @@ def test_address_integer_ties(sdm, dtype):
         assert np.array_equal(out["idx_r"][0, h].cpu().numpy(), ir)
 
 
+def _clustered_projection(rng, S, dk, x0, n_hi, cluster, dup):
+    """P rows of one half for a query x = (x0, 1, 0, ...): n_hi rows score about 2, the
+    `cluster` rows score 1 + c_j x0 with distinct steps c_j (each repeated `dup` times),
+    the rest score at most 0.  The cluster spacing (c step times x0) is far below the fp32
+    error bound of the scores, far above the compensated bound."""
+    P = np.zeros((S, dk))
+    P[:, 1] = -rng.integers(0, 4, S)
+    perm = rng.permutation(S)
+    hi, cl = perm[:n_hi], perm[n_hi:n_hi + cluster * dup]
+    P[hi, 1] = 2.0
+    P[hi, 0] = rng.integers(0, 8, n_hi)
+    P[cl, 1] = 1.0
+    P[cl, 0] = np.repeat(1.0 + np.arange(cluster) / 128.0, dup)
+    return P
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_address_clustered_scores_take_every_band_path(sdm, dtype):
+    """Scores clustered within the fp32 error bound around the top-k boundary.  Head 0: a
+    cluster wide enough that the band leaves the kept list (whole-half rescan); head 1:
+    duplicated rows inside the band (exact ties, decided in float64).  Indices must equal
+    the float64 definition's; the event counters show which paths decided."""
+    S, dk, T = 64, 64, 48
+    x0 = 2.0 ** -10 if dtype == "bf16" else 2.0 ** -14
+    cfg = synth.SdmConfig("clustered", B=1, H=2, T=T, d_k=dk, d_v=16, N=S * S, k_write=16, k_read=8,
+                          dtype=dtype, seed=7, alpha_mu=3.0)
+    rng = np.random.default_rng(11)
+    full = {}
+    for name in ("P_q", "P_k"):
+        heads = []
+        for h in range(2):
+            halves = [_clustered_projection(rng, S, dk, x0, 6, 40, 1) if h == 0 else
+                      _clustered_projection(rng, S, dk, x0, 13, 3, 2) for _ in range(2)]
+            heads.append(np.concatenate(halves))
+        full[name] = np.stack(heads)
+    X = np.zeros((1, 2, T, dk))
+    X[..., 0] = x0
+    X[..., 1] = 1.0
+    X[..., 2:] = rng.standard_normal((1, 2, T, dk - 2)) * 0.0     # keep the scores exact
+    full["q"], full["k"] = X.copy(), X.copy()
+    full = {n: synth.round_f64_to_storage(a, dtype) for n, a in full.items()}
+    dev = {n: synth.torch_io.to_torch(a, dtype) for n, a in full.items()}
+    sdm.device_stats()
+    out = _run_address(sdm, cfg, dev, T)
+    torch.cuda.synchronize()
+    st = sdm.device_stats()
+    f = lambda a: O.to_f64(a, dtype)
+    for h in range(2):
+        iw, _, _ = O.address(f(full["P_k"][h]), f(full["k"][0, h]), S * S, 16)
+        ir, _, _ = O.address(f(full["P_q"][h]), f(full["q"][0, h]), S * S, 8)
+        assert np.array_equal(out["idx_w"][0, h].cpu().numpy(), iw), h
+        assert np.array_equal(out["idx_r"][0, h].cpu().numpy(), ir), h
+    assert st["half_band"] > 0 and st["half_full"] > 0 and st["band_f64"] > 0, st
+
+
 # ------------------------------------------------------------------ K-REC with explicit addressing
 
 def _recur(sdm, dtype, idx_w, w_w, idx_r, w_r, v, alpha, beta, M0, B=1, H=1):
