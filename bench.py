@@ -285,7 +285,7 @@ def run_ours(args, cfg):
     rec_ms = max_over_ranks(ph["recurrence"])
     achieved = rec_bytes / (rec_ms * 1e-3) / 1e9
     step_bytes = cfg.algorithmic_bytes_per_token_head() * B * H * T + (1 + B) * H * N * dv * cfg.elem_bytes
-    kernels_per_step = 6   # init, P row norms, scores, finalize, hazard pass, recurrence
+    kernels_per_step = 8   # init, P row norms, scores, finalize (3 passes), hazard pass, recurrence
     line = {
         "metric": METRIC, "value": tokens_step / (ms_step * 1e-3), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,

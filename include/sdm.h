@@ -145,7 +145,10 @@ sdm_status sdm_recur(const sdm_shape* shape, const int32_t* idx_w, const float* 
 /* Reads (host pointer `code`, synchronising on `stream`) and clears the device
  * status word of the current device: 0 = no fault; bit 0 = a slot index outside
  * [0, N) was skipped; bit 1 = a slot list given to the recurrence was not strictly
- * ascending.  Returns SDM_ERR_DEVICE when the word was non-zero. */
+ * ascending; bit 2 = a bounded wait of the tensor-core score kernel gave up (its
+ * results are undefined); bit 3 = a selection invariant failed (a candidate list not
+ * ordered by score; results undefined).  Returns SDM_ERR_DEVICE when the word was
+ * non-zero. */
 sdm_status sdm_device_status(int32_t* code, sdm_stream_t stream);
 
 /* Size of the fixed device scratch behind sdm_recur_noalloc (its hazard table). */
@@ -176,6 +179,8 @@ sdm_status sdm_recur_noalloc(const sdm_shape* shape, const int32_t* idx_w, const
  *   [5] an outer-sum band that reached the last kept candidate (list extended to 64)
  *   [6] a band near-tie decided by float64 rescoring of its entries
  *   [7] the serial float64 fallback (heavy ties)
+ *   [8] total entries of the half bands re-ranked ([0] bands)
+ *   [9] total entries of the outer-sum bands re-ranked ([2] bands)
  * Counters wrap modulo 2^32. */
 sdm_status sdm_device_stats(uint32_t* counts, int n, sdm_stream_t stream);
 

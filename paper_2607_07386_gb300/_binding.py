@@ -187,7 +187,8 @@ def device_status(stream=None) -> int:
     return int(code.value)
 
 
-STAT_NAMES = ("half_band", "half_full", "comb_band", "comb_full", "select_retry", "comb_merge", "band_f64", "serial")
+STAT_NAMES = ("half_band", "half_full", "comb_band", "comb_full", "select_retry", "comb_merge", "band_f64", "serial",
+              "half_band_entries", "comb_band_entries")
 
 
 def device_stats(stream=None) -> dict:

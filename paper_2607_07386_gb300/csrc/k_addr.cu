@@ -173,12 +173,21 @@ __global__ void __launch_bounds__(A_TOK) k_addr_scores(const AddrArgs a) {
 // ------------------------------------------------------------------------------------------
 struct TokenCtx {
     int* err;           // device status word / counters
+    unsigned* stat;     // per-warp event counters in shared memory (nullptr: count in err directly)
+    bool count_band;    // count band events (false when an earlier pass counted them)
     const void* P;      // P of this side (nullptr = DIRECT)
     const void* X;
     int64_t xoff;       // element offset of the token's x row
     int64_t prow0;      // row of P for column 0 of half 0 (= h * 2S)
     int dk, S;
 };
+
+// Event counter (called by one lane): per-warp shared counters, flushed once per warp,
+// keep the diagnostics off the global atomic unit.
+__device__ __forceinline__ void tstat(const TokenCtx& c, int which, unsigned n = 1u) {
+    if (c.stat) c.stat[which] += n;
+    else stat_add(c.err, which, n);
+}
 
 // Float64 score of column j of half hf, summed over d in ascending order.
 template <class D>
@@ -230,6 +239,11 @@ __device__ __noinline__ void resolve_half(const float* lv, const int* li, int k,
         int best = -1;
         for (int p = cin; p < pend; ++p)
             if (!used[p] && (best < 0 || beats64(s64[p], li[p], s64[best], li[best]))) best = p;
+        if (best < 0) {                 // list not sorted by value: never for the lists built here
+            flag_error(c.err, ERR_SELECT);
+            chosen[r] = -1;
+            continue;
+        }
         used[best] = true;
         chosen[r] = best;
     }
@@ -239,6 +253,11 @@ __device__ __noinline__ void resolve_half(const float* lv, const int* li, int k,
         for (int q = 0; q < need; ++q) {
             const int p = chosen[q];
             if (p >= 0 && (best < 0 || TopList<L>::beats(lv[p], li[p], lv[chosen[best]], li[chosen[best]]))) best = q;
+        }
+        if (best < 0) {
+            Av[(cin + r) * pitch] = -INFINITY;
+            Ai[(cin + r) * pitch] = 0;
+            continue;
         }
         Av[(cin + r) * pitch] = lv[chosen[best]];
         Ai[(cin + r) * pitch] = li[chosen[best]];
@@ -294,6 +313,12 @@ __device__ __noinline__ void resolve_combined(const float* cv, const int* cf, in
         int best = -1;
         for (int p = cin; p < pend; ++p)
             if (!used[p] && (best < 0 || beats64(s64[p], cf[p], s64[best], cf[best]))) best = p;
+        if (best < 0) {                 // candidate list not sorted by value: never here
+            flag_error(c.err, ERR_SELECT);
+            Fv[r * pitch] = -INFINITY;
+            Fi[r * pitch] = 0;
+            continue;
+        }
         used[best] = true;
         Fv[r * pitch] = cv[best];
         Fi[r * pitch] = cf[best];
@@ -487,11 +512,25 @@ __device__ __forceinline__ void emit_band(float v0, int i0, float bv, int bi, bo
 // the list, more than 32 band entries, or a near-tie).
 enum : int { BAND_DONE = 0, BAND_NEAR_TIE = 1, BAND_OUTSIDE = 2 };
 
+// x[lane + 32 r] of the token (projected mode) for the warp-cooperative rescoring
+template <class D>
+__device__ __forceinline__ void load_xr(const TokenCtx& c, int lane, float (&xr)[8]) {
+#pragma unroll
+    for (int r = 0; r < 8; ++r) {
+        const int d = lane + 32 * r;
+        xr[r] = (c.P != nullptr && r * 32 < c.dk && d < c.dk) ? load_elem<D>(c.X, c.xoff + d) : 0.f;
+    }
+}
+
+// Band resolvers.  The common-path kernel (MODE 0) does not contain them.
 template <class D, int L>
-__device__ int warp_band_half(float v0, int i0, float v1, int i1, int k, float e2, const TokenCtx& c,
-                              const float (&xr)[8], int hf, float* ov, int* oi, int lane) {
+__device__ __forceinline__ int warp_band_half(float v0, int i0, float v1, int i1, int k, float e2, const TokenCtx& c,
+                                           int hf, float* ov, int* oi, int lane) {
+    float xr[8];
+    load_xr<D>(c, lane, xr);
     int cin, m;
     if (!band_of(v0, v1, L, k, e2, c.S <= L, lane, cin, m)) return BAND_OUTSIDE;
+    if (lane == 0 && c.count_band) tstat(c, STAT_HALF_BAND_ENTRIES, static_cast<unsigned>(m));
     const int p = min(cin + lane, L - 1);
     const float bv = lane_get(v0, v1, p);
     const int bi = lane_geti(i0, i1, p);
@@ -509,8 +548,8 @@ __device__ int warp_band_half(float v0, int i0, float v1, int i1, int k, float e
 // Near-tie in the band: float64 scores of the definition (sequential d order, so equal to
 // it bit for bit), one lane per band entry; the ranking is then exact.
 template <class D>
-__device__ void warp_band64(float v0, int i0, float v1, int i1, int len, int k, float e2, bool all, bool comb,
-                            const TokenCtx& c, int hf, float* ov, int* oi, int lane) {
+__device__ __noinline__ void warp_band64(float v0, int i0, float v1, int i1, int len, int k, float e2, bool all,
+                                         bool comb, const TokenCtx& c, int hf, float* ov, int* oi, int lane) {
     int cin, m;
     band_of(v0, v1, len, k, e2, all, lane, cin, m);       // succeeded before with the same arguments
     const int p = min(cin + lane, len - 1);
@@ -550,44 +589,68 @@ __device__ __forceinline__ void warp_sort64_desc(float& a, float& b, int lane) {
     }
 }
 
-// The band of a half boundary reaches past the kept list: exact top-k over the whole half.
-//   pass 1: fp32 scores (warp tree sum, error <= eps), each lane keeps the top 2 of the
+// Compensated score of column j of half hf by one lane (sequential d; same splitting and
+// the same 2^-28 sum|P x| bound as ff_score_warp).
+template <class D>
+__device__ FF ff_score_lane(const TokenCtx& c, int hf, int j) {
+    if (c.P == nullptr) return FF{load_elem<D>(c.X, c.xoff + static_cast<int64_t>(hf) * c.S + j), 0.f, 0.f};
+    const int64_t prow = (c.prow0 + static_cast<int64_t>(hf) * c.S + j) * c.dk;
+    float sum = 0.f, err = 0.f, mag = 0.f;
+#pragma unroll 4
+    for (int d = 0; d < c.dk; ++d) {
+        const float pv = load_elem<D>(c.P, prow + d), xv = load_elem<D>(c.X, c.xoff + d);
+        const float p = __fmul_rn(pv, xv);
+        const float pe = __fmaf_rn(pv, xv, -p);
+        float t, e2;
+        two_sum(sum, p, t, e2);
+        sum = t;
+        err = __fadd_rn(err, __fadd_rn(e2, pe));
+        mag = __fadd_rn(mag, fabsf(p));
+    }
+    FF r;
+    r.h = __fadd_rn(sum, err);
+    r.l = __fsub_rn(err, __fsub_rn(r.h, sum));
+    r.b = __fmul_ru(0x1p-28f, mag);
+    return r;
+}
+
+// The band of a half boundary reaches past the kept list: exact top-k over the whole half,
+// one column per lane at a time.
+//   pass 1: fp32 scores (sequential FMA, error <= eps), each lane keeps the top 2 of its
 //           columns j = lane (mod 32); theta = k-th largest of those 64 values (>= k columns
 //           reach it, so the k-th largest exact score is >= theta - eps);
 //   pass 2: columns with fp32 score >= theta - 2 eps (a superset of the exact top-k) are
 //           collected (at most 64, else false), rescored compensated and ranked.
 // Writes the top-k in order (value fl32 of the compensated score, index) to ov/oi.
 template <class D>
-__device__ bool warp_full_half(int k, float e2, const TokenCtx& c, const float (&xr)[8], int hf, float* ov, int* oi,
-                               int* scratch, int lane) {
+__device__ __noinline__ bool warp_full_half(int k, float e2, const TokenCtx& c, int hf, float* ov, int* oi,
+                                            int* scratch, int lane) {
     const int S = c.S;
     auto fp32_score = [&](int j) -> float {
         const int64_t prow = (c.prow0 + static_cast<int64_t>(hf) * S + j) * c.dk;
         float acc = 0.f;
-#pragma unroll
-        for (int r = 0; r < 8; ++r) {
-            const int d = lane + 32 * r;
-            if (r * 32 < c.dk && d < c.dk) acc = fmaf(load_elem<D>(c.P, prow + d), xr[r], acc);
-        }
-#pragma unroll
-        for (int off = 16; off > 0; off >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, off);
+#pragma unroll 8
+        for (int d = 0; d < c.dk; ++d) acc = fmaf(load_elem<D>(c.P, prow + d), load_elem<D>(c.X, c.xoff + d), acc);
         return acc;
     };
     float t1 = -INFINITY, t2 = -INFINITY;
-    for (int j = 0; j < S; ++j) {
-        const float sc = fp32_score(j);
-        if ((j & 31) == lane) { t2 = fmaxf(t2, fminf(t1, sc)); t1 = fmaxf(t1, sc); }
+    for (int j0 = 0; j0 < S; j0 += 32) {
+        const int j = j0 + lane;
+        const float sc = j < S ? fp32_score(j) : -INFINITY;
+        t2 = fmaxf(t2, fminf(t1, sc));
+        t1 = fmaxf(t1, sc);
     }
     warp_sort64_desc(t1, t2, lane);
     const float theta = lane_get(t1, t2, k - 1);
     const float lo = __fsub_rd(theta, e2);
     int m = 0;
-    for (int j = 0; j < S; ++j) {
-        const float sc = fp32_score(j);
-        if (sc >= lo) {                                          // warp-uniform
-            if (m < 64 && lane == 0) scratch[m] = j;
-            ++m;
-        }
+    for (int j0 = 0; j0 < S; j0 += 32) {
+        const int j = j0 + lane;
+        const bool keep = j < S && fp32_score(j) >= lo;
+        const unsigned mask = __ballot_sync(0xffffffffu, keep);
+        const int pos = m + __popc(mask & ((1u << lane) - 1u));
+        if (keep && pos < 64) scratch[pos] = j;
+        m += __popc(mask);
     }
     if (m > 64) return false;
     __syncwarp();
@@ -595,11 +658,8 @@ __device__ bool warp_full_half(int k, float e2, const TokenCtx& c, const float (
     const int j1 = lane + 32 < m ? scratch[lane + 32] : 0;
     __syncwarp();
     FF f0{0.f, 0.f, 0.f}, f1{0.f, 0.f, 0.f};
-    for (int e = 0; e < m; ++e) {
-        const FF sc = ff_score_warp<D>(c, xr, hf, lane_geti(j0, j1, e), lane);
-        if (e == lane) f0 = sc;
-        if (e == lane + 32) f1 = sc;
-    }
+    if (lane < m) f0 = ff_score_lane<D>(c, hf, j0);
+    if (lane + 32 < m) f1 = ff_score_lane<D>(c, hf, j1);
     // rank both own entries against all m (pairs closer than their bounds: give up)
     int r0 = 0, r1 = 0;
     bool unsure = false;
@@ -640,10 +700,13 @@ __device__ bool warp_full_half(int k, float e2, const TokenCtx& c, const float (
 // f = i S + j is rescored as the sum of the compensated half scores of column i (half 0)
 // and column j (half 1).
 template <class D>
-__device__ int warp_band_comb(float v0, int f0, float v1, int f1, int len, int k, float e2c, const TokenCtx& c,
-                              const float (&xr)[8], bool all, float* ov, int* oi, int lane) {
+__device__ __forceinline__ int warp_band_comb(float v0, int f0, float v1, int f1, int len, int k, float e2c,
+                                           const TokenCtx& c, bool all, float* ov, int* oi, int lane) {
+    float xr[8];
+    load_xr<D>(c, lane, xr);
     int cin, m;
     if (!band_of(v0, v1, len, k, e2c, all, lane, cin, m)) return BAND_OUTSIDE;
+    if (lane == 0 && c.count_band) tstat(c, STAT_COMB_BAND_ENTRIES, static_cast<unsigned>(m));
     const int p = min(cin + lane, len - 1);
     const float bv = lane_get(v0, v1, p);
     const int bf = lane_geti(f0, f1, p);
@@ -661,26 +724,57 @@ __device__ int warp_band_comb(float v0, int f0, float v1, int f1, int len, int k
     return BAND_DONE;
 }
 
-template <class D, int L>
+// Three passes over token-sides, each kernel holding only the code its cases need (the
+// band code's registers and instruction footprint would otherwise slow the common path):
+//   MODE 0: every token-side; those whose two half boundaries and outer-sum boundary are
+//           all certified are finished, the others go to queue A (nothing written);
+//   MODE 1: queue A, with band resolution by compensated rescoring; near-ties and bands
+//           that leave the kept lists go to queue B;
+//   MODE 2: queue B (or every token-side when there is no queue) with every path.
+enum : int { FIN_FAST = 0, FIN_BAND = 1, FIN_FULL = 2 };
+
+template <class D, int L, int MODE>
 __global__ void __launch_bounds__(FW_WARPS * 32, 4) k_addr_finalize(const AddrArgs a) {
     static_assert(L <= 36, "warp finalize handles k <= 32");
     __shared__ float wv[FW_WARPS][3][64];
     __shared__ int wi[FW_WARPS][3][64];
+    __shared__ unsigned wstat[FW_WARPS][STAT_COUNT];
     const int lane = threadIdx.x & 31, wq = threadIdx.x >> 5;
+    if (lane < STAT_COUNT) wstat[wq][lane] = 0u;
+    __syncwarp();
     const int64_t BT = static_cast<int64_t>(a.B) * a.T;
-    const int64_t items = 2 * a.H * BT;
-    // persistent warps: a warp takes token-sides item, item + (all warps), ... so that slow
-    // token-sides (band rescoring) do not hold a whole CTA's slot
-    for (int64_t item = static_cast<int64_t>(blockIdx.x) * FW_WARPS + wq; item < items;
-         item += static_cast<int64_t>(gridDim.x) * FW_WARPS) {
-    const int z = static_cast<int>(item / BT);
-    const int64_t u = item - z * BT;
+    const int64_t all = 2 * a.H * BT;
+    const bool queued = a.queue != nullptr;               // then all < 2^31
+    int* const qa = queued ? a.queue + 2 : nullptr;        // queue A items
+    int* const qb = queued ? a.queue + 2 + all : nullptr;  // queue B items
+    const int64_t items = MODE == FIN_FAST || !queued ? all
+                        : static_cast<int64_t>(reinterpret_cast<volatile int*>(a.queue)[MODE == FIN_BAND ? 0 : 1]);
+    // persistent warps: a warp takes token-sides it, it + (all warps), ...
+    for (int64_t it = static_cast<int64_t>(blockIdx.x) * FW_WARPS + wq; it < items;
+         it += static_cast<int64_t>(gridDim.x) * FW_WARPS) {
+    int64_t item, u, b, t;
+    int z;
+    if (queued) {                                          // 32-bit index arithmetic
+        const uint32_t it32 = MODE == FIN_FAST ? static_cast<uint32_t>(it)
+                            : static_cast<uint32_t>((MODE == FIN_BAND ? qa : qb)[it]);
+        const uint32_t z32 = it32 / static_cast<uint32_t>(BT);
+        const uint32_t u32 = it32 - z32 * static_cast<uint32_t>(BT);
+        const uint32_t b32 = u32 / static_cast<uint32_t>(a.T);
+        item = it32; z = static_cast<int>(z32); u = u32; b = b32; t = u32 - b32 * static_cast<uint32_t>(a.T);
+    } else {
+        item = it;
+        z = static_cast<int>(item / BT);
+        u = item - z * BT;
+        b = u / a.T;
+        t = u - b * a.T;
+    }
     const int side = z / a.H, h = z % a.H;
     const int k = a.kk[side];
     const int S = a.S;
-    const int64_t b = u / a.T, t = u - b * a.T;
     TokenCtx c;
     c.err = a.err;
+    c.stat = wstat[wq];
+    c.count_band = MODE != FIN_FULL || !queued;
     c.P = a.P[side];
     c.X = a.X[side];
     c.xoff = ((b * a.H + h) * a.T + t) * a.dk;
@@ -692,14 +786,11 @@ __global__ void __launch_bounds__(FW_WARPS * 32, 4) k_addr_finalize(const AddrAr
     float* sv2 = wv[wq][2]; int* si2 = wi[wq][2];          // candidates / final
 
     float e2 = 0.f;                                        // 2 x the fp32 score error bound, rounded up
-    float xr[8];                                           // x[lane + 32 r] (projected mode)
     if (c.P != nullptr) {
         float ss = 0.f;
-#pragma unroll
-        for (int r = 0; r < 8; ++r) {
-            const int d = lane + 32 * r;
-            xr[r] = (r * 32 < a.dk && d < a.dk) ? load_elem<D>(c.X, c.xoff + d) : 0.f;
-            ss = fmaf(xr[r], xr[r], ss);
+        for (int d = lane; d < a.dk; d += 32) {
+            const float xv = load_elem<D>(c.X, c.xoff + d);
+            ss = fmaf(xv, xv, ss);
         }
 #pragma unroll
         for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
@@ -711,6 +802,7 @@ __global__ void __launch_bounds__(FW_WARPS * 32, 4) k_addr_finalize(const AddrAr
     float av[2], bv[2];      // A1 and A2 after certification: lane p holds entry p (p < k)
     int ai[2], bi[2];
     float amax[2];
+    bool deferred = false;
 #pragma unroll 1
     for (int hf = 0; hf < 2; ++hf) {
         // chunk 0 of this half
@@ -745,20 +837,28 @@ __global__ void __launch_bounds__(FW_WARPS * 32, 4) k_addr_finalize(const AddrAr
             const float vk = lane_get(v0, v1, k - 1), vk1 = lane_get(v0, v1, k);
             certified = __fsub_rd(vk, vk1) > e2;
         }
+        if (MODE == FIN_FAST && !certified) {
+            deferred = true;
+            break;
+        }
         if (!certified) {
-            if (lane == 0) stat_add(c.err, STAT_HALF_BAND);
-            const int res = warp_band_half<D, L>(v0, i0, v1, i1, k, e2, c, xr, hf, sv0, si0, lane);
+            if (lane == 0 && c.count_band) tstat(c, STAT_HALF_BAND);
+            const int res = warp_band_half<D, L>(v0, i0, v1, i1, k, e2, c, hf, sv0, si0, lane);
             bool done = res == BAND_DONE;
+            if (MODE == FIN_BAND && !done) {
+                deferred = true;
+                break;
+            }
             if (res == BAND_NEAR_TIE) {
-                if (lane == 0) stat_add(c.err, STAT_BAND_F64);
+                if (lane == 0) tstat(c, STAT_BAND_F64);
                 warp_band64<D>(v0, i0, v1, i1, L, k, e2, S <= L, false, c, hf, sv0, si0, lane);
                 done = true;
             } else if (res == BAND_OUTSIDE) {
-                if (lane == 0) stat_add(c.err, STAT_HALF_FULL);
-                done = c.P != nullptr && warp_full_half<D>(k, e2, c, xr, hf, sv0, si0, si2, lane);
+                if (lane == 0) tstat(c, STAT_HALF_FULL);
+                done = c.P != nullptr && warp_full_half<D>(k, e2, c, hf, sv0, si0, si2, lane);
             }
             if (!done) {
-                if (lane == 0) stat_add(c.err, STAT_SERIAL);
+                if (lane == 0) tstat(c, STAT_SERIAL);
                 __syncwarp();
                 if (lane < L) { sv0[lane] = v0; si0[lane] = i0; }
                 if (lane + 32 < L) { sv0[lane + 32] = v1; si0[lane + 32] = i1; }
@@ -777,6 +877,14 @@ __global__ void __launch_bounds__(FW_WARPS * 32, 4) k_addr_finalize(const AddrAr
         if (hf == 0) { av[0] = lane < k ? v0 : -INFINITY; ai[0] = i0; }
         else { bv[0] = lane < k ? v0 : -INFINITY; bi[0] = i0; }
         amax[hf] = fmaxf(fabsf(lane_get(v0, v1, 0)), fabsf(lane_get(v0, v1, k - 1)));
+    }
+    if (MODE != FIN_FULL && deferred) {
+        if (lane == 0) {
+            if (MODE == FIN_FAST) qa[atomicAdd(a.queue, 1)] = static_cast<int>(item);
+            else qb[atomicAdd(a.queue + 1, 1)] = static_cast<int>(item);
+        }
+        __syncwarp();
+        continue;
     }
 
     // combined: k-way merge of the rows (lane i: row i; head = A1[i] + A2[j])
@@ -811,7 +919,7 @@ __global__ void __launch_bounds__(FW_WARPS * 32, 4) k_addr_finalize(const AddrAr
             }
         }
     };
-    merge_steps(0, L);
+    merge_steps(0, MODE == FIN_FAST ? k + 1 : L);           // certification needs entries k-1 and k
     bool certified = (k == 1);
     if (!certified) {
         const float ck = lane_get(cv0, cv1, k - 1), ck1 = lane_get(cv0, cv1, k);
@@ -819,23 +927,33 @@ __global__ void __launch_bounds__(FW_WARPS * 32, 4) k_addr_finalize(const AddrAr
     }
     float fv = cv0;
     int fi = cf0;
+    if (MODE == FIN_FAST && !certified) {
+        if (lane == 0) qa[atomicAdd(a.queue, 1)] = static_cast<int>(item);
+        __syncwarp();
+        continue;
+    }
     if (!certified) {
-        if (lane == 0) stat_add(c.err, STAT_COMB_BAND);
+        if (lane == 0 && c.count_band) tstat(c, STAT_COMB_BAND);
         // band may continue past the L candidates: extend the merge to 64 (or all k^2)
         int len = L;
         const float vl = lane_get(cv0, cv1, L - 1);
         if (k * k > L && vl != -INFINITY &&
             vl >= __fsub_rd(lane_get(cv0, cv1, k - 1), e2c)) {
-            if (lane == 0) stat_add(c.err, STAT_COMB_MERGE);
+            if (lane == 0 && c.count_band) tstat(c, STAT_COMB_MERGE);
             len = min(64, k * k);
             merge_steps(L, len);
         }
-        const int res = warp_band_comb<D>(cv0, cf0, cv1, cf1, len, k, e2c, c, xr, len >= k * k, sv2, si2, lane);
+        const int res = warp_band_comb<D>(cv0, cf0, cv1, cf1, len, k, e2c, c, len >= k * k, sv2, si2, lane);
+        if (MODE == FIN_BAND && res != BAND_DONE) {
+            if (lane == 0) qb[atomicAdd(a.queue + 1, 1)] = static_cast<int>(item);
+            __syncwarp();
+            continue;
+        }
         if (res == BAND_NEAR_TIE) {
-            if (lane == 0) stat_add(c.err, STAT_BAND_F64);
+            if (lane == 0) tstat(c, STAT_BAND_F64);
             warp_band64<D>(cv0, cf0, cv1, cf1, len, k, e2c, len >= k * k, true, c, 0, sv2, si2, lane);
         } else if (res == BAND_OUTSIDE) {
-            if (lane == 0) { stat_add(c.err, STAT_COMB_FULL); stat_add(c.err, STAT_SERIAL); }
+            if (lane == 0) { tstat(c, STAT_COMB_FULL); tstat(c, STAT_SERIAL); }
             __syncwarp();
             sv0[lane] = av[0]; si0[lane] = ai[0];            // A1
             sv1[lane] = bv[0]; si1[lane] = bi[0];            // A2
@@ -883,6 +1001,8 @@ __global__ void __launch_bounds__(FW_WARPS * 32, 4) k_addr_finalize(const AddrAr
     }
     __syncwarp();                                           // per-warp staging is reused
     }
+    __syncwarp();
+    if (lane > 0 && lane < STAT_COUNT && wstat[wq][lane] != 0u) stat_add(a.err, lane, wstat[wq][lane]);
 }
 // ------------------------------------------------------------------------------------------
 // Kernel B, wide lists (k > 32): insertion-based merge and candidate selection
@@ -907,6 +1027,8 @@ __global__ void __launch_bounds__(F_THREADS) k_addr_finalize_wide(const AddrArgs
     const int64_t b = u / a.T, t = u - b * a.T;
     TokenCtx c;
     c.err = a.err;
+    c.stat = nullptr;
+    c.count_band = true;
     c.P = a.P[side];
     c.X = a.X[side];
     c.xoff = ((b * a.H + h) * a.T + t) * a.dk;
@@ -1068,6 +1190,14 @@ AddrPlan addr_plan(int dtype, int direct, int B, int H, int T, int dk, int S, in
     return p;
 }
 
+// Queues of the three-pass warp finalize (0 when the item ids would not fit in int32: a
+// single full pass is used then).
+size_t addr_queue_bytes(int B, int H, int T) {
+    const int64_t items = static_cast<int64_t>(2) * H * B * T;
+    if (2 * items >= (static_cast<int64_t>(1) << 31) - 2) return 0;
+    return static_cast<size_t>(2 + 2 * items) * sizeof(int);       // two counts, queues A and B
+}
+
 size_t addr_partial_bytes(const AddrPlan& plan, int B, int H, int T) {
     return static_cast<size_t>(2) * H * (2 * plan.ncc) * plan.L * static_cast<size_t>(B) * T * (sizeof(float) + sizeof(int));
 }
@@ -1081,11 +1211,19 @@ static cudaError_t launch_finalize(const AddrArgs& a, cudaStream_t stream) {
         int dev = 0, sms = 0, per_sm = 0;
         e = cudaGetDevice(&dev);
         if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_addr_finalize<D, L>, FW_WARPS * 32, 0);
+        if (e == cudaSuccess)
+            e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_addr_finalize<D, L, FIN_FAST>, FW_WARPS * 32, 0);
         if (e != cudaSuccess) return e;
         const int64_t need = (2 * a.H * BT + FW_WARPS - 1) / FW_WARPS;
         const int64_t full = static_cast<int64_t>(sms) * (per_sm > 0 ? per_sm : 1);
-        k_addr_finalize<D, L><<<static_cast<unsigned>(need < full ? need : full), FW_WARPS * 32, 0, stream>>>(a);
+        const unsigned grid = static_cast<unsigned>(need < full ? need : full);
+        if (a.queue != nullptr) {
+            e = cudaMemsetAsync(a.queue, 0, 2 * sizeof(int), stream);
+            if (e != cudaSuccess) return e;
+            k_addr_finalize<D, L, FIN_FAST><<<grid, FW_WARPS * 32, 0, stream>>>(a);
+            k_addr_finalize<D, L, FIN_BAND><<<grid, FW_WARPS * 32, 0, stream>>>(a);
+        }
+        k_addr_finalize<D, L, FIN_FULL><<<grid, FW_WARPS * 32, 0, stream>>>(a);
     } else {
         const size_t smB = static_cast<size_t>(6) * L * F_THREADS * sizeof(float);
         e = cudaFuncSetAttribute(k_addr_finalize_wide<D, L>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smB));

@@ -116,7 +116,7 @@ sdm_status check_shape(const sdm_shape* s, bool need_pkm, int64_t* S_out) {
 }
 
 struct Layout {
-    size_t idx_w, w_w, idx_r, w_r, pnorm, part_v, part_i, hz, total;
+    size_t idx_w, w_w, idx_r, w_r, pnorm, part_v, part_i, queue, hz, total;
     sdm::AddrPlan plan;
 };
 
@@ -134,6 +134,7 @@ Layout layout_for(const sdm_shape* s, int64_t S) {
     const size_t part = sdm::addr_partial_bytes(L.plan, s->B, s->H, s->T) / 2;
     L.part_v = off; off = align256(off + part);
     L.part_i = off; off = align256(off + part);
+    L.queue = off;  off = align256(off + sdm::addr_queue_bytes(s->B, s->H, s->T));
     L.hz = off;     off = align256(off + sdm::rec_workspace_bytes(s->B, s->H, s->T, s->k_write, s->k_read));
     L.total = off;
     return L;
@@ -161,6 +162,7 @@ sdm_status run_address(const sdm_shape* s, int64_t S, const Layout& L, const voi
     a.part_v = reinterpret_cast<float*>(ws + L.part_v);
     a.part_i = reinterpret_cast<int*>(ws + L.part_i);
     a.pnorm = reinterpret_cast<float*>(ws + L.pnorm);
+    a.queue = sdm::addr_queue_bytes(s->B, s->H, s->T) ? reinterpret_cast<int*>(ws + L.queue) : nullptr;
     a.err = err;
     cudaError_t e = sdm::launch_address(s->dtype, L.plan, a, stream);
     if (e != cudaSuccess) return cuda_fail(e, "addressing launch");
@@ -376,7 +378,8 @@ sdm_status sdm_device_status(int32_t* code, sdm_stream_t stream) {
     *code = host;
     if (host != 0)
         return fail(SDM_ERR_DEVICE, "device status word = 0x%x (bit 0: slot index outside [0, N) skipped; "
-                    "bit 1: slot list not strictly ascending)", host);
+                    "bit 1: slot list not strictly ascending; bit 2: bounded wait timed out; "
+                    "bit 3: selection invariant failed)", host);
     return ok();
 }
 

@@ -75,10 +75,12 @@ enum : int {
     STAT_COMB_MERGE = 6,     // the outer-sum band reached the L-th candidate: merge extended to 64
     STAT_BAND_F64 = 7,       // a band near-tie was decided by float64 rescoring
     STAT_SERIAL = 8,         // the serial float64 fallback ran (heavy ties)
-    STAT_COUNT = 9
+    STAT_HALF_BAND_ENTRIES = 9,   // sum over half bands of the entries rescored
+    STAT_COMB_BAND_ENTRIES = 10,  // sum over outer-sum bands of the entries rescored
+    STAT_COUNT = 11
 };
-__device__ __forceinline__ void stat_add(int* err, int which) {
-    if (err) atomicAdd(reinterpret_cast<unsigned*>(err) + which, 1u);
+__device__ __forceinline__ void stat_add(int* err, int which, unsigned n = 1u) {
+    if (err) atomicAdd(reinterpret_cast<unsigned*>(err) + which, n);
 }
 
 }  // namespace sdm

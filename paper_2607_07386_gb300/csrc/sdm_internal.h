@@ -27,6 +27,8 @@ struct AddrArgs {
     float* part_v;         // workspace [2H][2 ncc][L][B*T]: per-chunk top-L scores
     int* part_i;           //   ... and their column index within the half
     float* pnorm;          // workspace [2H]: max row norm of P per side and head
+    int* queue;            // workspace [2 + 2 (2 H B T)]: counts of queues A and B, then their
+                           // token-side ids (nullptr: one pass does everything)
     int* err;              // device status word
 };
 
@@ -41,6 +43,7 @@ AddrPlan addr_plan(int dtype, int direct, int B, int H, int T, int dk, int S, in
 bool mma_path_supported(int dtype, int direct, int dk, int S, int kmax);
 cudaError_t launch_address_mma(const AddrPlan& plan, const AddrArgs& a, cudaStream_t stream);
 size_t addr_partial_bytes(const AddrPlan& plan, int B, int H, int T);
+size_t addr_queue_bytes(int B, int H, int T);
 cudaError_t launch_address(int dtype, const AddrPlan& plan, const AddrArgs& a, cudaStream_t stream);
 
 // ---------------------------------------------------------------- K-REC
