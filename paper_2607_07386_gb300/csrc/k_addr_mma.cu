@@ -7,8 +7,9 @@
 // accumulation in TMEM), and each of the 128 threads then owns one token's TMEM row.
 //
 // Per-token top-L selection of the chunk (L = k + 4; the finalize kernel certifies it), all
-// branch-free so a warp's 32 tokens run in lockstep:
-//   1. the two largest scores of each group of GS consecutive columns (<= 32 groups);
+// branch-free so a warp's 32 tokens run in lockstep; the passes over TMEM are loops over
+// 32-column blocks (compact code: the kernel is instruction-fetch bound when unrolled):
+//   1. the two largest scores of each of the 32 column classes mod 32;
 //   2. theta0 = L-th largest of those 64 values (bitonic network) -- a provable lower bound
 //      on the L-th largest score, since >= L distinct columns are >= it;
 //   3. survivors (score >= theta0) compacted into a per-thread shared-memory buffer with
@@ -27,12 +28,19 @@ namespace sdm {
 namespace {
 
 constexpr int MM_THREADS = 128;      // = tokens per CTA = TMEM lanes
-constexpr int MM_COLS = 512;         // TMEM columns (fp32 accumulators) = max chunk width
 constexpr int MM_NB = 256;           // columns per MMA instruction
 constexpr int MM_BUF = 64;           // survivor slots per thread
 constexpr long long MM_WAIT_CYCLES = 4000000000LL;   // ~2 s at 2 GHz: bounded waits
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) { return static_cast<uint32_t>(__cvta_generic_to_shared(p)); }
+
+// Bytes of the region that holds the chunk's rows of P and, once the MMA has completed,
+// the survivor buffers (values and indices, MM_BUF slots per thread).
+__host__ __device__ constexpr uint32_t mma_region_bytes(int atoms, int cols) {
+    return static_cast<uint32_t>(atoms) * cols * 128 > 2u * MM_BUF * MM_THREADS * 4
+               ? static_cast<uint32_t>(atoms) * cols * 128
+               : 2u * MM_BUF * MM_THREADS * 4;
+}
 
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" ::"r"(bar), "r"(count) : "memory");
@@ -151,7 +159,9 @@ struct MmaLaunch {
     int* err;
 };
 
-template <int GS>
+// COLS: TMEM columns (fp32 accumulators) = maximum chunk width (512: one CTA per SM;
+// 256: two CTAs per SM).
+template <int COLS>
 __global__ void __launch_bounds__(MM_THREADS, 1) k_addr_mma(const __grid_constant__ CUtensorMap tx_q,
                                                             const __grid_constant__ CUtensorMap tx_k,
                                                             const __grid_constant__ CUtensorMap tp_q,
@@ -162,8 +172,8 @@ __global__ void __launch_bounds__(MM_THREADS, 1) k_addr_mma(const __grid_constan
     const uint32_t base = (raw + 1023u) & ~1023u;
     unsigned char* sm = sm_raw + (base - raw);
     const uint32_t sA = base;                                   // [atoms][128 rows][128 B]
-    const uint32_t sB = sA + a.atoms * 128 * 128;                // [atoms][512 rows][128 B]; survivors later
-    const uint32_t sBar = sB + a.atoms * MM_COLS * 128;          // 3 mbarriers + TMEM address
+    const uint32_t sB = sA + a.atoms * 128 * 128;                // [atoms][COLS rows][128 B]; survivors later
+    const uint32_t sBar = sB + mma_region_bytes(a.atoms, COLS);  // 3 mbarriers + TMEM address
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(sm + (sBar - base) + 32);
     float* buf_v = reinterpret_cast<float*>(sm + (sB - base));                       // [MM_BUF][128]
     int* buf_i = reinterpret_cast<int*>(sm + (sB - base) + MM_BUF * MM_THREADS * 4);  // [MM_BUF][128]
@@ -182,7 +192,7 @@ __global__ void __launch_bounds__(MM_THREADS, 1) k_addr_mma(const __grid_constan
     const uint32_t bar_x = sBar, bar_p = sBar + 8, bar_mma = sBar + 16;
 
     if (warp == 0) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(smem_u32(tmem_slot)), "r"(MM_COLS) : "memory");
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;\n" ::"r"(smem_u32(tmem_slot)), "r"(COLS) : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;\n" ::: "memory");
     }
     if (tid == 0) {
@@ -206,7 +216,7 @@ __global__ void __launch_bounds__(MM_THREADS, 1) k_addr_mma(const __grid_constan
         mbar_expect_tx(bar_p, a.atoms * nblk * a.pb * 128);
         for (int at = 0; at < a.atoms; ++at)
             for (int nb = 0; nb < nblk; ++nb)
-                tma_load_3d(sB + at * MM_COLS * 128 + nb * MM_NB * 128, tp, at * 64, hf * a.S + c0 + nb * MM_NB, h, bar_p);
+                tma_load_3d(sB + at * COLS * 128 + nb * MM_NB * 128, tp, at * 64, hf * a.S + c0 + nb * MM_NB, h, bar_p);
         ok = mbar_wait(bar_x, 0) && mbar_wait(bar_p, 0);
         if (ok) {
             asm volatile("tcgen05.fence::after_thread_sync;\n" ::: "memory");
@@ -215,7 +225,7 @@ __global__ void __launch_bounds__(MM_THREADS, 1) k_addr_mma(const __grid_constan
                 const uint32_t idesc = mma_idesc(n);
                 for (int ks = 0; ks < a.atoms * 4; ++ks) {
                     const uint32_t aoff = (ks >> 2) * 128 * 128 + (ks & 3) * 32;
-                    const uint32_t boff = (ks >> 2) * MM_COLS * 128 + nb * MM_NB * 128 + (ks & 3) * 32;
+                    const uint32_t boff = (ks >> 2) * COLS * 128 + nb * MM_NB * 128 + (ks & 3) * 32;
                     mma_bf16(tmem + nb * MM_NB, sw128_desc(sA + aoff), sw128_desc(sB + boff), idesc, ks > 0 ? 1u : 0u);
                 }
             }
@@ -232,31 +242,27 @@ __global__ void __launch_bounds__(MM_THREADS, 1) k_addr_mma(const __grid_constan
     const int b = b0 + tid / a.bt, t = t0 + tid % a.bt;
     const bool valid = ok && b < a.B && t < a.T;
     const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-    constexpr int CB = GS;                          // 32-column blocks covered by 32 groups of GS columns
-    const int ng = npad / GS;                       // groups with columns (<= 32)
+    const int nblk32 = npad / 32 + ((npad & 31) ? 1 : 0);   // 32-column blocks with columns
 
-    // 1-2. top-2 of each group of GS columns, threshold = L-th largest of those (>= L columns reach it)
+    // 1-2. top-2 of each column class mod 32; threshold = L-th largest of those 64 values
+    // (>= L distinct columns reach it, so it is a lower bound on the L-th largest score)
     float theta = -INFINITY;
     if (ok) {
         float m1[32], m2[32];
 #pragma unroll
         for (int i = 0; i < 32; ++i) { m1[i] = -INFINITY; m2[i] = -INFINITY; }
+#pragma unroll 1
+        for (int cb = 0; cb < nblk32; ++cb) {
+            float v[32];
+            tmem_ld32(trow + cb * 32, v);
 #pragma unroll
-        for (int cb = 0; cb < CB; ++cb) {
-            if (cb * 32 < npad) {           // warp-uniform
-                float v[32];
-                tmem_ld32(trow + cb * 32, v);
-#pragma unroll
-                for (int j = 0; j < 32; ++j) {
-                    const int col = cb * 32 + j;
-                    const float x = col < np ? v[j] : -INFINITY;
-                    const int gi = (cb * 32 + j) / GS;
-                    m2[gi] = fmaxf(m2[gi], fminf(m1[gi], x));
-                    m1[gi] = fmaxf(m1[gi], x);
-                }
+            for (int j = 0; j < 32; ++j) {
+                const float x = cb * 32 + j < np ? v[j] : -INFINITY;
+                m2[j] = fmaxf(m2[j], fminf(m1[j], x));
+                m1[j] = fmaxf(m1[j], x);
             }
         }
-        if (2 * ng >= L) {
+        if (np >= L) {
             float g64[64];
 #pragma unroll
             for (int i = 0; i < 32; ++i) { g64[i] = m1[i]; g64[32 + i] = m2[i]; }
@@ -276,21 +282,19 @@ __global__ void __launch_bounds__(MM_THREADS, 1) k_addr_mma(const __grid_constan
     for (int round = 0; round < 3; ++round) {
         int cnt = 0;
         if (ok) {
+#pragma unroll 1
+            for (int cb = 0; cb < nblk32; ++cb) {
+                float v[32];
+                tmem_ld32(trow + cb * 32, v);
 #pragma unroll
-            for (int cb = 0; cb < MM_COLS / 32; ++cb) {
-                if (cb * 32 < npad) {
-                    float v[32];
-                    tmem_ld32(trow + cb * 32, v);
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) {
-                        const int col = cb * 32 + j;
-                        const bool keep = col < np && v[j] >= theta;
-                        if (keep && cnt < MM_BUF) {
-                            buf_v[cnt * MM_THREADS + tid] = v[j];
-                            buf_i[cnt * MM_THREADS + tid] = c0 + col;
-                        }
-                        cnt += keep ? 1 : 0;
+                for (int j = 0; j < 32; ++j) {
+                    const int col = cb * 32 + j;
+                    const bool keep = col < np && v[j] >= theta;
+                    if (keep && cnt < MM_BUF) {
+                        buf_v[cnt * MM_THREADS + tid] = v[j];
+                        buf_i[cnt * MM_THREADS + tid] = c0 + col;
                     }
+                    cnt += keep ? 1 : 0;
                 }
             }
         }
@@ -348,7 +352,7 @@ __global__ void __launch_bounds__(MM_THREADS, 1) k_addr_mma(const __grid_constan
 
     asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
     __syncthreads();
-    if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem), "r"(MM_COLS) : "memory");
+    if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem), "r"(COLS) : "memory");
 }
 
 // ------------------------------------------------------------------------------------------
@@ -374,9 +378,13 @@ bool mma_path_supported(int dtype, int direct, int dk, int S, int kmax) {
     return dtype == 1 && !direct && (dk == 64 || dk == 128) && kmax <= 32 && S >= 16;
 }
 
-size_t mma_smem_bytes(int dk) {
+// A CTA allocates `cols` TMEM columns of the SM's 512: a 512-column CTA asks for enough
+// shared memory that no second CTA is resident beside it.
+size_t mma_smem_bytes(int dk, int cols) {
     const int atoms = (dk + 63) / 64;
-    return 1024 + static_cast<size_t>(atoms) * (128 * 128 + MM_COLS * 128) + 64;
+    const size_t need = 1024 + static_cast<size_t>(atoms) * 128 * 128 + mma_region_bytes(atoms, cols) + 64;
+    const size_t one_per_sm = 120 * 1024;
+    return cols >= 512 && need < one_per_sm ? one_per_sm : need;
 }
 
 cudaError_t launch_address_mma(const AddrPlan& plan, const AddrArgs& aa, cudaStream_t stream) {
@@ -422,26 +430,18 @@ cudaError_t launch_address_mma(const AddrPlan& plan, const AddrArgs& aa, cudaStr
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
     }
-    const size_t smem = mma_smem_bytes(aa.dk);
-    const int cwp = (plan.cw + 15) & ~15;
-    int gs = 1;
-    while (cwp / gs > 32) gs *= 2;          // at most 32 groups (top-2 of each: 64 values)
     dim3 grid(static_cast<unsigned>(a.ntt * nbt), 2 * plan.ncc, 2 * aa.H);
     cudaError_t e = cudaSuccess;
-    switch (gs) {
-#define SDM_MMA_CASE(G)                                                                                                       \
-    case G:                                                                                                                   \
-        e = cudaFuncSetAttribute(k_addr_mma<G>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));       \
-        if (e != cudaSuccess) return e;                                                                                       \
-        k_addr_mma<G><<<grid, MM_THREADS, smem, stream>>>(maps[0], maps[1], maps[2], maps[3], a);                             \
-        break;
-        SDM_MMA_CASE(1)
-        SDM_MMA_CASE(2)
-        SDM_MMA_CASE(4)
-        SDM_MMA_CASE(8)
-        SDM_MMA_CASE(16)
-#undef SDM_MMA_CASE
-        default: return cudaErrorInvalidValue;
+    if (plan.cw <= 256) {
+        const size_t smem = mma_smem_bytes(aa.dk, 256);
+        e = cudaFuncSetAttribute(k_addr_mma<256>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+        if (e != cudaSuccess) return e;
+        k_addr_mma<256><<<grid, MM_THREADS, smem, stream>>>(maps[0], maps[1], maps[2], maps[3], a);
+    } else {
+        const size_t smem = mma_smem_bytes(aa.dk, 512);
+        e = cudaFuncSetAttribute(k_addr_mma<512>, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+        if (e != cudaSuccess) return e;
+        k_addr_mma<512><<<grid, MM_THREADS, smem, stream>>>(maps[0], maps[1], maps[2], maps[3], a);
     }
     return cudaGetLastError();
 }
