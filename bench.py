@@ -36,6 +36,12 @@ METRIC = "SDM recurrence tokens/s per layer (1 GB300) and achieved HBM GB/s vs ~
 UNIT = "tokens/s"
 
 
+# DRAM bytes per token-head moved by the recurrence phase (hazard pass + recurrence), from an
+# ncu capture of dram__bytes_read.sum + dram__bytes_write.sum at the layer geometry with B=1
+# (profiles/recurrence_layer_1p4b_b1_dram_traffic.txt): 1,507,923,456 B / 65,536 token-heads.
+RECUR_DRAM_BYTES_PER_TOKEN_HEAD = 1507923456 / 65536
+
+
 def _peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -298,7 +304,9 @@ def run_ours(args, cfg):
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": kernels_per_step * args.steps,
         "roofline": {"bound": "hbm", "kernel": "k_recur", "achieved": achieved, "peak": peaks["hbm_gbs"],
-                     "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "traffic": None,
+                     "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
+                     "traffic": RECUR_DRAM_BYTES_PER_TOKEN_HEAD * B * H * T if cfg.name == "layer_1p4b" else None,
+                     "traffic_source": "ncu dram bytes of the hazard pass + recurrence at B=1, scaled to B*H*T",
                      "peak_source": peaks["source"], "bytes_per_launch": rec_bytes, "ms_per_launch": rec_ms},
         "phase_ms": ph,
         "step_hbm": {"algorithmic_bytes": step_bytes, "gbs": step_bytes / (ms_step * 1e-3) / 1e9,
