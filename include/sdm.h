@@ -118,6 +118,19 @@ sdm_status sdm_forward(const sdm_shape* shape, const void* P_q, const void* P_k,
                        int32_t* idx_w, float* w_w, int32_t* idx_r, float* w_r,
                        void* workspace, size_t workspace_bytes, sdm_stream_t stream);
 
+/* sdm_init_memory followed by sdm_forward in one call: every sequence's memory starts as
+ * a copy of M0 [H, N, d_v] (Sec. 3.1 "Learned initial state"), then the whole hot path
+ * runs over the T tokens.  Same results as the two calls.  The broadcast runs on a
+ * library-owned side stream of the current device, ordered after the work already on
+ * `stream` and joined back into `stream` before the recurrence, so it overlaps the
+ * addressing.  M0 must not overlap mem.  Calls from several host threads on one device
+ * are ordered by a lock while they enqueue. */
+sdm_status sdm_forward_m0(const sdm_shape* shape, const void* M0, const void* P_q, const void* P_k,
+                          const void* q, const void* k, const void* v,
+                          const void* alpha, const void* beta, void* mem, void* y,
+                          int32_t* idx_w, float* w_w, int32_t* idx_r, float* w_r,
+                          void* workspace, size_t workspace_bytes, sdm_stream_t stream);
+
 /* One decode step for B independent sequences: sdm_forward with shape->T == 1 and
  * the per-token tensors shaped [B, H, d] / [B, H]. */
 sdm_status sdm_decode_step(const sdm_shape* shape, const void* P_q, const void* P_k,

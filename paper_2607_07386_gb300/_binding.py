@@ -65,6 +65,8 @@ def lib():
             L.sdm_init_memory.argtypes = [_SHP, _VP, _VP, _VP]
             fwd = [_SHP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _I32P, _VP, _I32P, _VP, _VP, _SZ, _VP]
             L.sdm_forward.argtypes = fwd
+            L.sdm_forward_m0.argtypes = [fwd[0], _VP] + fwd[1:]
+            L.sdm_forward_m0.restype = ctypes.c_int
             L.sdm_decode_step.argtypes = fwd
             L.sdm_address.argtypes = [_SHP, _VP, _VP, _VP, _VP, _I32P, _VP, _I32P, _VP, _VP, _SZ, _VP]
             L.sdm_recur.argtypes = [_SHP, _I32P, _VP, _I32P, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP]
@@ -144,6 +146,15 @@ def forward(shape: SdmShape, P_q, P_k, q, k, v, alpha, beta, mem, y, workspace, 
     _check(lib().sdm_forward(ctypes.byref(shape), _ptr(P_q), _ptr(P_k), _ptr(q), _ptr(k), _ptr(v), _ptr(alpha),
                              _ptr(beta), _ptr(mem), _ptr(y), _ptr(idx_w), _ptr(w_w), _ptr(idx_r), _ptr(w_r),
                              _ptr(workspace), nb, _stream(stream)))
+
+
+def forward_m0(shape: SdmShape, M0, P_q, P_k, q, k, v, alpha, beta, mem, y, workspace, idx_w=None, w_w=None,
+               idx_r=None, w_r=None, stream=None, workspace_nbytes=None):
+    """sdm_forward_m0: mem = M0 broadcast (overlapping the addressing), then the forward pass."""
+    nb = workspace_nbytes if workspace_nbytes is not None else (_nbytes(workspace) or 0)
+    _check(lib().sdm_forward_m0(ctypes.byref(shape), _ptr(M0), _ptr(P_q), _ptr(P_k), _ptr(q), _ptr(k), _ptr(v),
+                                _ptr(alpha), _ptr(beta), _ptr(mem), _ptr(y), _ptr(idx_w), _ptr(w_w), _ptr(idx_r),
+                                _ptr(w_r), _ptr(workspace), nb, _stream(stream)))
 
 
 def decode_step(shape: SdmShape, P_q, P_k, q, k, v, alpha, beta, mem, y, workspace, idx_w=None, w_w=None,

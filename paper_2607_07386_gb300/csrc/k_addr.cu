@@ -1217,6 +1217,11 @@ static cudaError_t launch_finalize(const AddrArgs& a, cudaStream_t stream) {
         const int64_t need = (2 * a.H * BT + FW_WARPS - 1) / FW_WARPS;
         const int64_t full = static_cast<int64_t>(sms) * (per_sm > 0 ? per_sm : 1);
         const unsigned grid = static_cast<unsigned>(need < full ? need : full);
+        // same carveout as the tensor-core kernel and the M0 copy: they share SMs
+        for (auto fn : {k_addr_finalize<D, L, FIN_FAST>, k_addr_finalize<D, L, FIN_BAND>, k_addr_finalize<D, L, FIN_FULL>}) {
+            e = cudaFuncSetAttribute(fn, cudaFuncAttributePreferredSharedMemoryCarveout, cudaSharedmemCarveoutMaxShared);
+            if (e != cudaSuccess) return e;
+        }
         if (a.queue != nullptr) {
             e = cudaMemsetAsync(a.queue, 0, 2 * sizeof(int), stream);
             if (e != cudaSuccess) return e;

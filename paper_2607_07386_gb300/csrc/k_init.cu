@@ -28,14 +28,21 @@ __global__ void __launch_bounds__(INIT_THREADS) k_init_memory(const uint4* __res
     }
 }
 
-cudaError_t launch_init_memory(const void* M0, void* mem, int64_t bytes_per_seq, int B, cudaStream_t stream) {
+cudaError_t launch_init_memory(const void* M0, void* mem, int64_t bytes_per_seq, int B, cudaStream_t stream,
+                               int ctas_per_sm) {
     const int64_t nvec = bytes_per_seq / 16;
     int dev = 0, sms = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     int64_t want = (nvec + INIT_THREADS * INIT_UNROLL - 1) / (INIT_THREADS * INIT_UNROLL);
-    const int64_t cap = static_cast<int64_t>(sms) * 8;   // 8 x 256 threads = a full SM
+    const int64_t cap = static_cast<int64_t>(sms) * ctas_per_sm;   // 8 x 256 threads = a full SM
     const int grid = static_cast<int>(want < cap ? (want > 0 ? want : 1) : cap);
+    // The copy needs no shared memory; asking for the shared-memory-heavy carveout anyway
+    // lets an SM hold it beside the addressing kernels (an SM changes its carveout only
+    // when idle, so kernels with different carveouts cannot share it).
+    cudaError_t e = cudaFuncSetAttribute(k_init_memory, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                         cudaSharedmemCarveoutMaxShared);
+    if (e != cudaSuccess) return e;
     k_init_memory<<<grid, INIT_THREADS, 0, stream>>>(reinterpret_cast<const uint4*>(M0), reinterpret_cast<uint4*>(mem),
                                                      nvec, B);
     return cudaGetLastError();

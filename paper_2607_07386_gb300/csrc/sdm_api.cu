@@ -9,6 +9,7 @@
 #include <string.h>
 
 #include <atomic>
+#include <mutex>
 #include <string>
 
 static_assert(sizeof(sdm_shape) == 48, "sdm_shape layout is part of the ABI");
@@ -55,6 +56,37 @@ sdm_status status_word(int** out) {
         g_status_addr[dev].store(p, std::memory_order_release);
     }
     *out = p;
+    return SDM_OK;
+}
+
+// Per-device side stream and fork/join events for the M0 broadcast that overlaps the
+// addressing in sdm_forward_m0 (created on first use; the mutex orders the host-side
+// enqueue of fork/join sequences from concurrent callers).
+struct SideStream {
+    cudaStream_t stream = nullptr;
+    cudaEvent_t fork = nullptr, join = nullptr;
+};
+SideStream g_side[kMaxDevices];
+constexpr int kCopyCtasPerSm = 2;     // M0 copy CTAs per SM beside the addressing
+std::mutex g_side_mutex[kMaxDevices];
+
+sdm_status side_stream(int* dev_out, SideStream** out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev < 0 || dev >= kMaxDevices) return fail(SDM_ERR_UNSUPPORTED, "device ordinal %d >= %d", dev, kMaxDevices);
+    SideStream& ss = g_side[dev];
+    if (ss.stream == nullptr) {
+        e = cudaStreamCreateWithFlags(&ss.stream, cudaStreamNonBlocking);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ss.fork, cudaEventDisableTiming);
+        if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ss.join, cudaEventDisableTiming);
+        if (e != cudaSuccess) {
+            ss = SideStream{};
+            return cuda_fail(e, "side stream creation");
+        }
+    }
+    *dev_out = dev;
+    *out = &ss;
     return SDM_OK;
 }
 
@@ -184,7 +216,7 @@ sdm_status check_vec(const void* p, const char* name, size_t align) {
 sdm_status forward_impl(const char* who, const sdm_shape* s, const void* P_q, const void* P_k, const void* q,
                         const void* k, const void* v, const void* alpha, const void* beta, void* mem, void* y,
                         int32_t* idx_w, float* w_w, int32_t* idx_r, float* w_r, void* workspace,
-                        size_t workspace_bytes, cudaStream_t stream, bool run_recurrence) {
+                        size_t workspace_bytes, cudaStream_t stream, bool run_recurrence, const void* M0 = nullptr) {
     int64_t S = 0;
     SDM_TRY(check_shape(s, true, &S));
     const size_t es = elem_bytes(s->dtype);
@@ -229,6 +261,11 @@ sdm_status forward_impl(const char* who, const sdm_shape* s, const void* P_q, co
         const Range ry{y, bht * rowb, "y"};
         for (int i = 0; i < 7; ++i)
             if (overlaps(ry, others[i])) return fail(SDM_ERR_INVALID_ARG, "%s: y overlaps %s", who, others[i].name);
+        if (M0 != nullptr) {
+            SDM_TRY(check_vec(M0, "M0", 16));
+            if (overlaps(rm, Range{M0, static_cast<size_t>(s->H) * static_cast<size_t>(s->N) * rowb, "M0"}))
+                return fail(SDM_ERR_INVALID_ARG, "%s: mem overlaps M0", who);
+        }
     }
     char* ws = static_cast<char*>(workspace);
     int32_t* iw = idx_w ? idx_w : reinterpret_cast<int32_t*>(ws + L.idx_w);
@@ -237,7 +274,29 @@ sdm_status forward_impl(const char* who, const sdm_shape* s, const void* P_q, co
     float* wr = w_r ? w_r : reinterpret_cast<float*>(ws + L.w_r);
     int* err = nullptr;
     SDM_TRY(status_word(&err));
-    SDM_TRY(run_address(s, S, L, P_q, P_k, q, k, iw, ww, ir, wr, ws, err, stream));
+    if (run_recurrence && M0 != nullptr) {
+        // mem = M0 broadcast on the side stream, running beside the addressing (independent
+        // data) and joined back before the recurrence.  Two CTAs per SM leave room for the
+        // addressing kernels.  (Started after the score kernel instead, beside the finalize
+        // passes, it measured slower: the copy's traffic slows whichever kernel it shares
+        // the SMs with, and the finalize more than the tensor-core kernel.)
+        int dev = 0;
+        SideStream* ss = nullptr;
+        SDM_TRY(side_stream(&dev, &ss));
+        std::lock_guard<std::mutex> lock(g_side_mutex[dev]);
+        cudaError_t e = cudaEventRecord(ss->fork, stream);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(ss->stream, ss->fork, 0);
+        if (e == cudaSuccess)
+            e = sdm::launch_init_memory(M0, mem, static_cast<int64_t>(static_cast<size_t>(s->H) * s->N * rowb), s->B,
+                                        ss->stream, kCopyCtasPerSm);
+        if (e == cudaSuccess) e = cudaEventRecord(ss->join, ss->stream);
+        if (e != cudaSuccess) return cuda_fail(e, "M0 broadcast on the side stream");
+        SDM_TRY(run_address(s, S, L, P_q, P_k, q, k, iw, ww, ir, wr, ws, err, stream));
+        e = cudaStreamWaitEvent(stream, ss->join, 0);
+        if (e != cudaSuccess) return cuda_fail(e, "join of the M0 broadcast");
+    } else {
+        SDM_TRY(run_address(s, S, L, P_q, P_k, q, k, iw, ww, ir, wr, ws, err, stream));
+    }
     if (run_recurrence) {
         sdm::RecArgs r{};
         r.idx_w = iw; r.w_w = ww; r.idx_r = ir; r.w_r = wr;
@@ -291,6 +350,16 @@ sdm_status sdm_forward(const sdm_shape* s, const void* P_q, const void* P_k, con
                        sdm_stream_t stream) {
     return forward_impl("sdm_forward", s, P_q, P_k, q, k, v, alpha, beta, mem, y, idx_w, w_w, idx_r, w_r, workspace,
                         workspace_bytes, reinterpret_cast<cudaStream_t>(stream), true);
+}
+
+sdm_status sdm_forward_m0(const sdm_shape* s, const void* M0, const void* P_q, const void* P_k, const void* q,
+                          const void* k, const void* v, const void* alpha, const void* beta, void* mem, void* y,
+                          int32_t* idx_w, float* w_w, int32_t* idx_r, float* w_r, void* workspace,
+                          size_t workspace_bytes, sdm_stream_t stream) {
+    if (s != nullptr && s->B > 0 && s->H > 0 && s->T > 0 && M0 == nullptr)
+        return fail(SDM_ERR_INVALID_ARG, "sdm_forward_m0: M0 is NULL");
+    return forward_impl("sdm_forward_m0", s, P_q, P_k, q, k, v, alpha, beta, mem, y, idx_w, w_w, idx_r, w_r, workspace,
+                        workspace_bytes, reinterpret_cast<cudaStream_t>(stream), true, M0);
 }
 
 sdm_status sdm_decode_step(const sdm_shape* s, const void* P_q, const void* P_k, const void* q, const void* k,

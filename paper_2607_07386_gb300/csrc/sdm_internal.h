@@ -10,7 +10,9 @@
 namespace sdm {
 
 // ---------------------------------------------------------------- K-INIT
-cudaError_t launch_init_memory(const void* M0, void* mem, int64_t bytes_per_seq, int B, cudaStream_t stream);
+// ctas_per_sm: 8 fills the SMs (the copy alone); fewer leave room for kernels running beside it.
+cudaError_t launch_init_memory(const void* M0, void* mem, int64_t bytes_per_seq, int B, cudaStream_t stream,
+                               int ctas_per_sm = 8);
 
 // ---------------------------------------------------------------- K-ADDR
 // "which" 0 = read side (q with P_q -> idx_r, w_r), 1 = write side (k with P_k -> idx_w, w_w).

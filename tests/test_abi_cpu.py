@@ -35,7 +35,7 @@ def test_header_declares_the_boundary():
     names = declared_functions()
     for required in ("sdm_abi_version", "sdm_last_error", "sdm_workspace_bytes", "sdm_init_memory",
                      "sdm_forward", "sdm_decode_step", "sdm_recur", "sdm_address", "sdm_device_status",
-                     "sdm_recur_workspace_bytes", "sdm_device_stats"):
+                     "sdm_recur_workspace_bytes", "sdm_device_stats", "sdm_forward_m0"):
         assert required in names
 
 

@@ -392,6 +392,25 @@ def test_batch_slices_are_independent(sdm):
     assert torch.equal(out1["y"][0], outB["y"][2]) and torch.equal(out1["mem"][0], outB["mem"][2])
 
 
+@pytest.mark.parametrize("name", ["tiny_fp32", "small_bf16"])
+def test_forward_m0_equals_init_then_forward(sdm, name):
+    """sdm_forward_m0 (broadcast overlapping the addressing) gives, bit for bit, what
+    sdm_init_memory followed by sdm_forward gives."""
+    cfg = synth.CONFIGS[name]
+    dev = G.device_inputs(cfg)
+    ref = G.run_forward(cfg, dev)
+    shape = G.shape_of(cfg)
+    out = G.alloc_outputs(cfg, cfg.T)
+    mem = torch.full_like(ref["mem"], 7.0)          # stale contents must be overwritten
+    sdm.forward_m0(shape, dev["M0"], dev.get("P_q"), dev.get("P_k"), dev["q"], dev["k"], dev["v"], dev["alpha"],
+                   dev["beta"], mem, out["y"], G.workspace(shape), idx_w=out["idx_w"], w_w=out["w_w"],
+                   idx_r=out["idx_r"], w_r=out["w_r"])
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    assert torch.equal(out["idx_w"], ref["idx_w"]) and torch.equal(out["idx_r"], ref["idx_r"])
+    assert torch.equal(out["y"], ref["y"]) and torch.equal(mem, ref["mem"])
+
+
 # ------------------------------------------------------------------ full-size workloads
 
 @pytest.mark.fullsize
