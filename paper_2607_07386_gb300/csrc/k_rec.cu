@@ -19,7 +19,7 @@ RecPlan rec_plan(int dtype, int B, int H, int T, int dv, int kw, int kr) {
     // widest d-range per warp (<= 128 B) that still gives a few hundred warps
     int dch = 1;
     while (dch < 8 && nch % (dch * 2) == 0) dch *= 2;
-    while (dch > 2 && chains * (nch / dch) < 384) dch /= 2;      // keep >= 32-byte pieces
+    while (dch > 2 && chains * (nch / dch) < 1024) dch /= 2;     // many warps; keep >= 32-byte pieces
     int spt = (kmax + (32 / dch) - 1) / (32 / dch);
     while (spt > 8 && dch > 1) { dch /= 2; spt = (kmax + (32 / dch) - 1) / (32 / dch); }   // k = 64 with wide ranges
     p.dch = dch;

@@ -80,6 +80,7 @@ template <class D, int DCH, int SPT, int LA>
 __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const int32_t* __restrict__ hz, int kmax,
                                               int vec_lists) {
     constexpr int E = D::E;
+    constexpr int E2 = E / 2;
     constexpr int G = 32 / DCH;
     constexpr int KS = G * SPT;
     constexpr int KP = rec_ks_pad(KS);
@@ -215,11 +216,14 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
         lds_vec<SPT>(m + 3 * KP + g * SPT, *reinterpret_cast<int(*)[SPT]>(wr));
         lds_vec<SPT>(m + 4 * KP + g * SPT, hzv);
 
-        // ---- gathers (stale rows replaced from the written ring), decay, partial sums
-        float r[SPT][E];
-        float pp[E], yp[E];
+        // ---- gathers (stale rows replaced from the written ring), decay, partial sums.
+        // Element math in fp32 pairs on the packed fp32x2 units (each lane of a pair rounds
+        // like the scalar operation).
+        float2 r[SPT][E2];
+        float2 pp[E2], yp[E2];
 #pragma unroll
-        for (int e = 0; e < E; ++e) { pp[e] = 0.f; yp[e] = 0.f; }
+        for (int e = 0; e < E2; ++e) { pp[e] = make_float2(0.f, 0.f); yp[e] = make_float2(0.f, 0.f); }
+        const float2 alpha2 = make_float2(alpha, alpha);
         bool fix = false;
         bool okw[SPT];
 #pragma unroll
@@ -239,42 +243,49 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
             fix |= rfix && okr;
             const uint4 mw = lds128(aw);
             const uint4 mr = lds128(ar);
-            float f[E], h[E];
-            unpack16<D>(mw, f);
-            unpack16<D>(mr, h);
+            float2 f[E2], h[E2];
+            unpack16x2<D>(mw, f);
+            unpack16x2<D>(mr, h);
             const float wj = okw[j] ? ww[j] : 0.f;
             const float rho = (okr && !rfix) ? wr[j] : 0.f;
+            const float2 wj2 = make_float2(wj, wj), rho2 = make_float2(rho, rho);
 #pragma unroll
-            for (int e = 0; e < E; ++e) {
-                r[j][e] = alpha * f[e];
-                pp[e] = fmaf(wj, r[j][e], pp[e]);
-                yp[e] = fmaf(rho, h[e], yp[e]);
+            for (int e = 0; e < E2; ++e) {
+                r[j][e] = __fmul2_rn(alpha2, f[e]);
+                pp[e] = __ffma2_rn(wj2, r[j][e], pp[e]);
+                yp[e] = __ffma2_rn(rho2, h[e], yp[e]);
             }
         }
 #pragma unroll
         for (int off = DCH; off < 32; off <<= 1) {
 #pragma unroll
-            for (int e = 0; e < E; ++e) {
-                pp[e] += __shfl_xor_sync(0xffffffffu, pp[e], off);
-                yp[e] += __shfl_xor_sync(0xffffffffu, yp[e], off);
+            for (int e = 0; e < E2; ++e) {
+                const float2 qp = make_float2(__shfl_xor_sync(0xffffffffu, pp[e].x, off), __shfl_xor_sync(0xffffffffu, pp[e].y, off));
+                const float2 qy = make_float2(__shfl_xor_sync(0xffffffffu, yp[e].x, off), __shfl_xor_sync(0xffffffffu, yp[e].y, off));
+                pp[e] = __fadd2_rn(pp[e], qp);
+                yp[e] = __fadd2_rn(yp[e], qy);
             }
         }
         // ---- delta = v - v~ and the write
-        float delta[E];
-        unpack16<D>(lds128(mslot + 5 * KP * 4 + c * 16), delta);
+        float2 d2[E2];
+        unpack16x2<D>(lds128(mslot + 5 * KP * 4 + c * 16), d2);
 #pragma unroll
-        for (int e = 0; e < E; ++e) delta[e] -= pp[e];
+        for (int e = 0; e < E2; ++e) d2[e] = __fadd2_rn(d2[e], make_float2(-pp[e].x, -pp[e].y));
         const uint32_t wslot = my_wring + ws * KS * SLOTB;
 #pragma unroll
         for (int j = 0; j < SPT; ++j) {
             const float bw = beta * ww[j];
-            float o[E];
+            const float2 bw2 = make_float2(bw, bw);
+            float2 o[E2];
 #pragma unroll
-            for (int e = 0; e < E; ++e) o[e] = fmaf(bw, delta[e], r[j][e]);
-            const uint4 packed = pack16<D>(o);
+            for (int e = 0; e < E2; ++e) o[e] = __ffma2_rn(bw2, d2[e], r[j][e]);
+            const uint4 packed = pack16x2<D>(o);
             if (okw[j]) *reinterpret_cast<uint4*>(Mw + static_cast<uint64_t>(iw[j]) * rowbytes) = packed;
             sts128(wslot + j * SLOTB, packed, okw[j]);
         }
+        float delta[E];
+#pragma unroll
+        for (int e = 0; e < E2; ++e) { delta[2 * e] = d2[e].x; delta[2 * e + 1] = d2[e].y; }
         // ---- reads of slots this token wrote (rare): recompute the writer's value
         if (__any_sync(0xffffffffu, fix)) {
             float yc[E];
@@ -309,9 +320,9 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
                 for (int e = 0; e < E; ++e) yc[e] += __shfl_xor_sync(0xffffffffu, yc[e], off);
             }
 #pragma unroll
-            for (int e = 0; e < E; ++e) yp[e] += yc[e];
+            for (int e = 0; e < E2; ++e) yp[e] = __fadd2_rn(yp[e], make_float2(yc[2 * e], yc[2 * e + 1]));
         }
-        if (g == 0) *reinterpret_cast<uint4*>(yb + static_cast<int64_t>(t) * rowbytes) = pack16<D>(yp);
+        if (g == 0) *reinterpret_cast<uint4*>(yb + static_cast<int64_t>(t) * rowbytes) = pack16x2<D>(yp);
         // ---- prefetch: rows of token t+LA (rows slot of token t), lists of token t+2LA (slot of t-1)
         {
             int mfut = ms + LA; mfut -= mfut >= MR ? MR : 0;

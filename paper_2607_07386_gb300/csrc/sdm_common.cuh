@@ -48,6 +48,31 @@ template <> __device__ __forceinline__ uint4 pack16<BF16>(const float* f) {
     return make_uint4(w[0], w[1], w[2], w[3]);
 }
 
+// The same, as fp32 pairs (element 2q in .x, 2q + 1 in .y) for the packed fp32x2 units.
+template <class D> __device__ __forceinline__ void unpack16x2(const uint4& u, float2* f);
+template <> __device__ __forceinline__ void unpack16x2<F32>(const uint4& u, float2* f) {
+    f[0] = make_float2(__uint_as_float(u.x), __uint_as_float(u.y));
+    f[1] = make_float2(__uint_as_float(u.z), __uint_as_float(u.w));
+}
+template <> __device__ __forceinline__ void unpack16x2<BF16>(const uint4& u, float2* f) {
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int q = 0; q < 4; ++q) f[q] = make_float2(__uint_as_float(w[q] << 16), __uint_as_float(w[q] & 0xffff0000u));
+}
+template <class D> __device__ __forceinline__ uint4 pack16x2(const float2* f);
+template <> __device__ __forceinline__ uint4 pack16x2<F32>(const float2* f) {
+    return make_uint4(__float_as_uint(f[0].x), __float_as_uint(f[0].y), __float_as_uint(f[1].x), __float_as_uint(f[1].y));
+}
+template <> __device__ __forceinline__ uint4 pack16x2<BF16>(const float2* f) {
+    uint32_t w[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        __nv_bfloat162 h = __floats2bfloat162_rn(f[q].x, f[q].y);
+        w[q] = *reinterpret_cast<uint32_t*>(&h);
+    }
+    return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
 // One storage element -> fp32 (exact).
 template <class D> __device__ __forceinline__ float load_elem(const void* base, int64_t i);
 template <> __device__ __forceinline__ float load_elem<F32>(const void* base, int64_t i) {
