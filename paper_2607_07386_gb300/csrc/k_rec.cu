@@ -27,6 +27,10 @@ RecPlan rec_plan(int dtype, int B, int H, int T, int dv, int kw, int kr) {
     p.spt = spt <= 1 ? 1 : spt <= 2 ? 2 : spt <= 4 ? 4 : 8;
     p.threads = 32;
     p.la = T <= 1 ? 1 : 4;
+    // writer/reader warp pairs: measured faster only with short slot lists (k <= 16) and
+    // few units (256 at B=4 H=8 k=16: 1.34 -> 1.12 ms); with k = 32 the hand-over costs more
+    // than it saves (1024 units: 4.33 -> 5.69 ms; 256 units, T = 65536: 51.8 -> 55.2 ms)
+    p.split = p.la > 1 && kmax <= 16 && chains * p.nsplit < 768;
     p.smem = rec_smem_bytes(p.la, (32 / dch) * p.spt, dch);
     return p;
 }

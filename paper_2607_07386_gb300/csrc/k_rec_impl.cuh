@@ -352,9 +352,13 @@ cudaError_t launch_rec_kernel(const RecPlan& p, const RecArgs& a, const int32_t*
     return cudaGetLastError();
 }
 
+template <class D, int DCH, int SPT, int LA>
+cudaError_t launch_rec_split(const RecPlan& p, const RecArgs& a, const int32_t* hz, int vec_lists, cudaStream_t s);
+
 template <class D, int DCH, int SPT>
 cudaError_t launch_rec_la(const RecPlan& p, const RecArgs& a, const int32_t* hz, int vl, cudaStream_t s) {
-    return p.la == 1 ? launch_rec_kernel<D, DCH, SPT, 1>(p, a, hz, vl, s) : launch_rec_kernel<D, DCH, SPT, 4>(p, a, hz, vl, s);
+    if (p.la == 1) return launch_rec_kernel<D, DCH, SPT, 1>(p, a, hz, vl, s);
+    return p.split ? launch_rec_split<D, DCH, SPT, 4>(p, a, hz, vl, s) : launch_rec_kernel<D, DCH, SPT, 4>(p, a, hz, vl, s);
 }
 
 template <class D, int DCH>
@@ -377,6 +381,327 @@ cudaError_t launch_rec_dtype(const RecPlan& p, const RecArgs& a, const int32_t* 
         case 8: return launch_rec_spt<D, 8>(p, a, hz, vl, s);
         default: return cudaErrorInvalidValue;
     }
+}
+
+}  // namespace sdm
+
+namespace sdm {
+
+// ------------------------------------------------------------------------------------------
+// K-REC, writer/reader split.  One CTA of two warps per (chain, d-range): warp 0 does the
+// decay, prediction and delta write of token t (Eqs. sdm-decay, sdm-write) while warp 1
+// does the read of token t-1 (Eq. sdm-read), so each warp's per-token instruction chain is
+// about half of the fused one.  They meet in the ring of rows written by the last LA+1
+// tokens (read-gathers of slots written in the hazard window, including by the token itself,
+// take the writer's row from there) and hand over through two mbarriers:
+//   written[t] (writer -> reader): token t's rows are in memory and in the ring;
+//   read[t]    (reader -> writer): token t is read, so ring entry t - LA is free again.
+// The writer of token t waits for read[t-1] only before its stores; the reader of token t
+// waits for written[t].  Neither can run two phases ahead of the other, so the waits on
+// phase parity are unambiguous.  Every wait is bounded; on timeout both warps leave the
+// token loop and the device status gets its timeout bit.
+// ------------------------------------------------------------------------------------------
+constexpr long long REC_WAIT_CYCLES = 4000000000LL;    // ~2 s at 2 GHz
+
+__host__ __device__ inline size_t rec_split_smem_bytes(int la, int ks, int dch) {
+    return static_cast<size_t>(2) * la * ks * dch * 16                // prefetched rows: write, read
+         + static_cast<size_t>(la + 1) * ks * dch * 16                // rows written lately
+         + static_cast<size_t>(2) * (2 * la + 1) * rec_meta_stride(ks, dch)   // lists, per warp
+         + 32;                                                        // two mbarriers + abort flag
+}
+
+__device__ __forceinline__ void rec_mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(bar) : "memory");
+}
+// Bounded wait for the completion of the phase with parity `par`; false on timeout or abort.
+__device__ __forceinline__ bool rec_mbar_wait(uint32_t bar, uint32_t par, volatile int* abort_flag) {
+    const long long t0 = clock64();
+    while (true) {
+        uint32_t ok;
+        asm volatile("{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+                     : "=r"(ok) : "r"(bar), "r"(par) : "memory");
+        if (ok) return true;
+        if (*abort_flag || clock64() - t0 > REC_WAIT_CYCLES) return false;
+    }
+}
+
+template <class D, int DCH, int SPT, int LA>
+__global__ void __launch_bounds__(64) k_recur_split(const RecArgs a, int nsplit, const int32_t* __restrict__ hz,
+                                                    int kmax, int vec_lists) {
+    static_assert(LA >= 1, "look-ahead");
+    constexpr int E = D::E;
+    constexpr int E2 = E / 2;
+    constexpr int G = 32 / DCH;
+    constexpr int KS = G * SPT;
+    constexpr int KP = rec_ks_pad(KS);
+    constexpr int MR = 2 * LA + 1;
+    constexpr int RING = LA + 1;
+    constexpr uint32_t SLOTB = DCH * 16;
+    extern __shared__ __align__(16) unsigned char smS[];
+    const int warp = threadIdx.x >> 5;                       // 0: writer, 1: reader
+    const int lane = threadIdx.x & 31;
+    const int meta_stride = static_cast<int>(rec_meta_stride(KS, DCH));
+    const uint32_t sm0 = static_cast<uint32_t>(__cvta_generic_to_shared(smS));
+    const uint32_t rows0 = sm0 + warp * (LA * KS * SLOTB);                   // own [LA][KS][DCH] x 16 B
+    const uint32_t wring0 = sm0 + 2 * LA * KS * SLOTB;                      // shared [RING][KS][DCH] x 16 B
+    const uint32_t metab = wring0 + RING * KS * SLOTB;
+    const uint32_t meta0 = metab + warp * MR * meta_stride;                 // own [MR][stride]
+    unsigned char* meta_gen = smS + (meta0 - sm0);
+    const uint32_t bar_written = metab + 2 * MR * meta_stride;
+    const uint32_t bar_read = bar_written + 8;
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smS + (bar_written - sm0) + 16);
+    if (threadIdx.x == 0) {
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;\n" ::"r"(bar_written) : "memory");
+        asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;\n" ::"r"(bar_read) : "memory");
+        *abort_flag = 0;
+    }
+    __syncthreads();
+
+    const int c = lane % DCH;
+    const int g = lane / DCH;
+    const int kw = a.kw, kr = a.kr;
+    const int kmine = warp == 0 ? kw : kr;                   // list this warp gathers
+    const int64_t chain = blockIdx.x / nsplit;
+    const int split = blockIdx.x - static_cast<int>(chain) * nsplit;
+    const uint32_t rowbytes = static_cast<uint32_t>(a.dv) * D::BYTES;
+    const int64_t dbyte = static_cast<int64_t>(split * DCH) * 16;
+    const char* Mc = static_cast<const char*>(a.mem) + chain * a.N * static_cast<int64_t>(rowbytes) + dbyte + c * 16;
+    char* Mw = const_cast<char*>(Mc);
+    const char* vrange = static_cast<const char*>(a.v) + chain * a.T * static_cast<int64_t>(rowbytes) + dbyte;
+    char* yb = static_cast<char*>(a.y) + chain * a.T * static_cast<int64_t>(rowbytes) + dbyte + c * 16;
+    const int T = a.T;
+    const int64_t tok0 = chain * T;
+    const uint32_t N = static_cast<uint32_t>(a.N);
+    const uint32_t my_rows = rows0 + (g * SPT * DCH + c) * 16;
+    const uint32_t my_wring = wring0 + (g * SPT * DCH + c) * 16;
+    const uint32_t wring_c = wring0 + c * 16;
+    bool mine[SPT];
+#pragma unroll
+    for (int j = 0; j < SPT; ++j) mine[j] = g * SPT + j < kmine;
+
+    // lists of token t (16-byte pieces when vec_lists; same layout as the fused kernel)
+    const int qw = kw / 4, qr = kr / 4;
+    const int npieces = 2 * qw + 2 * qr + kmax / 4;
+    const char* psrc[3];
+    uint32_t pstride[3], poff[3];
+    bool pvalid[3];
+#pragma unroll
+    for (int q = 0; q < 3; ++q) {
+        const int p = lane + 32 * q;
+        pvalid[q] = vec_lists && p < npieces;
+        const char* src = reinterpret_cast<const char*>(a.idx_w);
+        uint32_t stride = kw * 4, off = 0, sub = 0;
+        if (p < qw) { src = reinterpret_cast<const char*>(a.idx_w); stride = kw * 4; off = 0; sub = p; }
+        else if (p < 2 * qw) { src = reinterpret_cast<const char*>(a.w_w); stride = kw * 4; off = KP * 4; sub = p - qw; }
+        else if (p < 2 * qw + qr) { src = reinterpret_cast<const char*>(a.idx_r); stride = kr * 4; off = 2 * KP * 4; sub = p - 2 * qw; }
+        else if (p < 2 * qw + 2 * qr) { src = reinterpret_cast<const char*>(a.w_r); stride = kr * 4; off = 3 * KP * 4; sub = p - 2 * qw - qr; }
+        else { src = reinterpret_cast<const char*>(hz); stride = kmax * 4; off = 4 * KP * 4; sub = p - 2 * qw - 2 * qr; }
+        psrc[q] = src + tok0 * stride + sub * 16;
+        pstride[q] = stride;
+        poff[q] = off + sub * 16;
+    }
+    auto copy_meta = [&](int t, uint32_t slot_addr) {
+        if (t >= T) return;
+        if (vec_lists) {
+#pragma unroll
+            for (int q = 0; q < 3; ++q)
+                if (pvalid[q]) cp_async16z(slot_addr + poff[q], psrc[q] + static_cast<int64_t>(t) * pstride[q], 16);
+        } else {
+            int* dst = reinterpret_cast<int*>(meta_gen + (slot_addr - meta0));
+            const int64_t tok = tok0 + t;
+            for (int p = lane; p < 2 * kw + 2 * kr + kmax; p += 32) {
+                const void* src;
+                int* d;
+                if (p < kw) { src = a.idx_w + tok * kw + p; d = dst + p; }
+                else if (p < 2 * kw) { src = a.w_w + tok * kw + (p - kw); d = dst + KP + (p - kw); }
+                else if (p < 2 * kw + kr) { src = a.idx_r + tok * kr + (p - 2 * kw); d = dst + 2 * KP + (p - 2 * kw); }
+                else if (p < 2 * kw + 2 * kr) { src = a.w_r + tok * kr + (p - 2 * kw - kr); d = dst + 3 * KP + (p - 2 * kw - kr); }
+                else { src = hz + tok * kmax + (p - 2 * kw - 2 * kr); d = dst + 4 * KP + (p - 2 * kw - 2 * kr); }
+                cp_async4(d, src);
+            }
+        }
+        if (warp == 0 && lane < DCH)
+            cp_async16z(slot_addr + 5 * KP * 4 + lane * 16, vrange + static_cast<int64_t>(t) * rowbytes + lane * 16, 16);
+    };
+    // rows token t gathers from this warp's list (writer: write slots; reader: read slots)
+    const int list_off = warp == 0 ? 0 : 2 * KP;
+    auto copy_rows = [&](int t, uint32_t meta_addr, uint32_t rows_slot) {
+        if (t >= T) return;
+        const int* m = reinterpret_cast<const int*>(meta_gen + (meta_addr - meta0));
+        int ix[SPT];
+        lds_vec<SPT>(m + list_off + g * SPT, ix);
+#pragma unroll
+        for (int j = 0; j < SPT; ++j) {
+            const bool ok = mine[j] && static_cast<uint32_t>(ix[j]) < N;
+            cp_async16z(rows_slot + j * SLOTB, Mc + static_cast<uint64_t>(ok ? ix[j] : 0) * rowbytes, ok ? 16 : 0);
+        }
+    };
+
+    // prologue: lists of tokens [0, LA); then rows of [0, LA) with lists of [LA, 2LA)
+    for (int u = 0; u < LA; ++u) copy_meta(u, meta0 + u * meta_stride);
+    cp_async_commit();
+    cp_async_wait<0>();
+    __syncwarp();
+    for (int u = 0; u < LA; ++u) {
+        copy_rows(u, meta0 + u * meta_stride, my_rows + u * KS * SLOTB);
+        copy_meta(u + LA, meta0 + (u + LA) * meta_stride);
+        cp_async_commit();
+    }
+    auto prefetch = [&](int t, int ms, int rs) {     // rows of t+LA into the slot of t; lists of t+2LA
+        int mfut = ms + LA; mfut -= mfut >= MR ? MR : 0;
+        copy_rows(t + LA, meta0 + mfut * meta_stride, my_rows + rs * KS * SLOTB);
+        int mnew = ms + 2 * LA; mnew -= mnew >= MR ? MR : 0;
+        copy_meta(t + 2 * LA, meta0 + mnew * meta_stride);
+        cp_async_commit();
+    };
+
+    bool bad = false, timed_out = false;
+    if (warp == 0) {
+        // ------------------------------------------------------------------ writer
+        float a_cur = 0.f, b_cur = 0.f, a_nxt = 0.f, b_nxt = 0.f;
+        if (lane < T) { a_nxt = load_elem<D>(a.alpha, tok0 + lane); b_nxt = load_elem<D>(a.beta, tok0 + lane); }
+        int ms = 0, rs = 0, ws = 0;
+        for (int t = 0; t < T; ++t) {
+            if ((t & 31) == 0) {
+                a_cur = a_nxt; b_cur = b_nxt;
+                const int tn = t + 32 + lane;
+                if (tn < T) { a_nxt = load_elem<D>(a.alpha, tok0 + tn); b_nxt = load_elem<D>(a.beta, tok0 + tn); }
+            }
+            const float alpha = __shfl_sync(0xffffffffu, a_cur, t & 31);
+            const float beta = __shfl_sync(0xffffffffu, b_cur, t & 31);
+            cp_async_wait<LA - 1>();
+            __syncwarp();
+            const int* m = reinterpret_cast<const int*>(meta_gen + ms * meta_stride);
+            const uint32_t rslot = my_rows + rs * KS * SLOTB;
+            int iw[SPT], hzv[SPT];
+            float ww[SPT];
+            lds_vec<SPT>(m + g * SPT, iw);
+            lds_vec<SPT>(m + KP + g * SPT, *reinterpret_cast<int(*)[SPT]>(ww));
+            lds_vec<SPT>(m + 4 * KP + g * SPT, hzv);
+            float2 r[SPT][E2];
+            float2 pp[E2];
+#pragma unroll
+            for (int e = 0; e < E2; ++e) pp[e] = make_float2(0.f, 0.f);
+            const float2 alpha2 = make_float2(alpha, alpha);
+            bool okw[SPT];
+#pragma unroll
+            for (int j = 0; j < SPT; ++j) {
+                okw[j] = mine[j] && static_cast<uint32_t>(iw[j]) < N;
+                bad |= mine[j] && !okw[j];
+                const int hw = okw[j] ? (hzv[j] & 0xffff) : 0;      // never decode unused slots
+                int rw = ws - ((hw - 1) >> 6); rw += rw < 0 ? RING : 0;
+                const uint32_t aw = hw ? wring_c + (rw * KS + ((hw - 1) & 63)) * SLOTB : rslot + j * SLOTB;
+                float2 f[E2];
+                unpack16x2<D>(lds128(aw), f);
+                const float wj = okw[j] ? ww[j] : 0.f;
+                const float2 wj2 = make_float2(wj, wj);
+#pragma unroll
+                for (int e = 0; e < E2; ++e) {
+                    r[j][e] = __fmul2_rn(alpha2, f[e]);
+                    pp[e] = __ffma2_rn(wj2, r[j][e], pp[e]);
+                }
+            }
+#pragma unroll
+            for (int off = DCH; off < 32; off <<= 1) {
+#pragma unroll
+                for (int e = 0; e < E2; ++e)
+                    pp[e] = __fadd2_rn(pp[e], make_float2(__shfl_xor_sync(0xffffffffu, pp[e].x, off),
+                                                          __shfl_xor_sync(0xffffffffu, pp[e].y, off)));
+            }
+            float2 d2[E2];
+            unpack16x2<D>(lds128(meta0 + ms * meta_stride + 5 * KP * 4 + c * 16), d2);
+#pragma unroll
+            for (int e = 0; e < E2; ++e) d2[e] = __fadd2_rn(d2[e], make_float2(-pp[e].x, -pp[e].y));
+            uint4 packed[SPT];
+#pragma unroll
+            for (int j = 0; j < SPT; ++j) {
+                const float bw = beta * ww[j];
+                const float2 bw2 = make_float2(bw, bw);
+                float2 o[E2];
+#pragma unroll
+                for (int e = 0; e < E2; ++e) o[e] = __ffma2_rn(bw2, d2[e], r[j][e]);
+                packed[j] = pack16x2<D>(o);
+            }
+            // ring entry of token t - LA - 1 is free once the reader is done with token t - 1
+            if (t > 0 && !rec_mbar_wait(bar_read, static_cast<uint32_t>((t - 1) & 1), abort_flag)) { timed_out = true; break; }
+            const uint32_t wslot = my_wring + ws * KS * SLOTB;
+#pragma unroll
+            for (int j = 0; j < SPT; ++j) {
+                if (okw[j]) *reinterpret_cast<uint4*>(Mw + static_cast<uint64_t>(iw[j]) * rowbytes) = packed[j];
+                sts128(wslot + j * SLOTB, packed[j], okw[j]);
+            }
+            __syncwarp();
+            if (lane == 0) rec_mbar_arrive(bar_written);
+            prefetch(t, ms, rs);
+            ms = ms + 1 == MR ? 0 : ms + 1;
+            rs = rs + 1 == LA ? 0 : rs + 1;
+            ws = ws + 1 == RING ? 0 : ws + 1;
+        }
+    } else {
+        // ------------------------------------------------------------------ reader
+        int ms = 0, rs = 0, ws = 0;
+        for (int t = 0; t < T; ++t) {
+            cp_async_wait<LA - 1>();
+            __syncwarp();
+            const int* m = reinterpret_cast<const int*>(meta_gen + ms * meta_stride);
+            const uint32_t rslot = my_rows + rs * KS * SLOTB;
+            int ir[SPT], hzv[SPT];
+            float wr[SPT];
+            lds_vec<SPT>(m + 2 * KP + g * SPT, ir);
+            lds_vec<SPT>(m + 3 * KP + g * SPT, *reinterpret_cast<int(*)[SPT]>(wr));
+            lds_vec<SPT>(m + 4 * KP + g * SPT, hzv);
+            if (!rec_mbar_wait(bar_written, static_cast<uint32_t>(t & 1), abort_flag)) { timed_out = true; break; }
+            float2 yp[E2];
+#pragma unroll
+            for (int e = 0; e < E2; ++e) yp[e] = make_float2(0.f, 0.f);
+#pragma unroll
+            for (int j = 0; j < SPT; ++j) {
+                const bool okr = mine[j] && static_cast<uint32_t>(ir[j]) < N;
+                bad |= mine[j] && !okr;
+                const int hr = okr ? ((hzv[j] >> 16) & 0xffff) : 0;
+                int rr = ws - ((hr - 1) >> 6); rr += rr < 0 ? RING : 0;
+                const uint32_t ar = hr ? wring_c + (rr * KS + ((hr - 1) & 63)) * SLOTB : rslot + j * SLOTB;
+                float2 h[E2];
+                unpack16x2<D>(lds128(ar), h);
+                const float rho = okr ? wr[j] : 0.f;
+                const float2 rho2 = make_float2(rho, rho);
+#pragma unroll
+                for (int e = 0; e < E2; ++e) yp[e] = __ffma2_rn(rho2, h[e], yp[e]);
+            }
+            __syncwarp();
+            if (lane == 0) rec_mbar_arrive(bar_read);          // ring reads of token t done
+#pragma unroll
+            for (int off = DCH; off < 32; off <<= 1) {
+#pragma unroll
+                for (int e = 0; e < E2; ++e)
+                    yp[e] = __fadd2_rn(yp[e], make_float2(__shfl_xor_sync(0xffffffffu, yp[e].x, off),
+                                                          __shfl_xor_sync(0xffffffffu, yp[e].y, off)));
+            }
+            if (g == 0) *reinterpret_cast<uint4*>(yb + static_cast<int64_t>(t) * rowbytes) = pack16x2<D>(yp);
+            prefetch(t, ms, rs);
+            ms = ms + 1 == MR ? 0 : ms + 1;
+            rs = rs + 1 == LA ? 0 : rs + 1;
+            ws = ws + 1 == RING ? 0 : ws + 1;
+        }
+    }
+    if (timed_out) *abort_flag = 1;
+    cp_async_wait<0>();
+    if (__any_sync(0xffffffffu, bad) && lane == 0) flag_error(a.err, ERR_BAD_INDEX);
+    if (__any_sync(0xffffffffu, timed_out) && lane == 0) flag_error(a.err, ERR_TIMEOUT);
+}
+
+template <class D, int DCH, int SPT, int LA>
+cudaError_t launch_rec_split(const RecPlan& p, const RecArgs& a, const int32_t* hz, int vec_lists, cudaStream_t s) {
+    const size_t smem = rec_split_smem_bytes(LA, (32 / DCH) * SPT, DCH);
+    if (smem > 48 * 1024) {
+        cudaError_t e = cudaFuncSetAttribute(k_recur_split<D, DCH, SPT, LA>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             static_cast<int>(smem));
+        if (e != cudaSuccess) return e;
+    }
+    const int64_t chains = static_cast<int64_t>(a.B) * a.H;
+    k_recur_split<D, DCH, SPT, LA><<<static_cast<unsigned>(chains * p.nsplit), 64, smem, s>>>(a, p.nsplit, hz, p.kmax,
+                                                                                                vec_lists);
+    return cudaGetLastError();
 }
 
 }  // namespace sdm

@@ -68,6 +68,7 @@ struct RecPlan {
     int spt;      // slots per thread per token
     int la;       // lookahead depth (tokens whose gathers are in flight)
     int kmax;     // max(k_write, k_read)
+    int split;    // writer and reader warps per (chain, d-range) (look-ahead > 1 only)
     size_t smem;  // dynamic shared memory per CTA
 };
 RecPlan rec_plan(int dtype, int B, int H, int T, int dv, int kw, int kr);
