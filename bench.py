@@ -37,9 +37,10 @@ UNIT = "tokens/s"
 
 
 # DRAM bytes per token-head moved by the recurrence phase (hazard pass + recurrence), from an
-# ncu capture of dram__bytes_read.sum + dram__bytes_write.sum at the layer geometry with B=1
-# (profiles/recurrence_layer_1p4b_b1_dram_traffic.txt): 1,507,923,456 B / 65,536 token-heads.
-RECUR_DRAM_BYTES_PER_TOKEN_HEAD = 1507923456 / 65536
+# ncu capture of dram__bytes_read.sum + dram__bytes_write.sum at the layer geometry with B=2,
+# the same kernels as at B=8 (profiles/recurrence_layer_1p4b_dram_traffic.txt):
+# 3,205,865,728 B / 131,072 token-heads.
+RECUR_DRAM_BYTES_PER_TOKEN_HEAD = 3205865728 / 131072
 
 
 def _peaks():
@@ -305,7 +306,7 @@ def run_ours(args, cfg):
         "roofline": {"bound": "hbm", "kernel": "k_recur", "achieved": achieved, "peak": peaks["hbm_gbs"],
                      "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
                      "traffic": RECUR_DRAM_BYTES_PER_TOKEN_HEAD * B * H * T if cfg.name == "layer_1p4b" else None,
-                     "traffic_source": "ncu dram bytes of the hazard pass + recurrence at B=1, scaled to B*H*T",
+                     "traffic_source": "ncu dram bytes of the hazard pass + recurrence at B=2, scaled to B*H*T",
                      "peak_source": peaks["source"], "bytes_per_launch": rec_bytes, "ms_per_launch": rec_ms},
         "phase_ms": ph,
         "step_hbm": {"algorithmic_bytes": step_bytes, "gbs": step_bytes / (ms_step * 1e-3) / 1e9,
