@@ -1202,6 +1202,175 @@ size_t addr_partial_bytes(const AddrPlan& plan, int B, int H, int T) {
     return static_cast<size_t>(2) * H * (2 * plan.ncc) * plan.L * static_cast<size_t>(B) * T * (sizeof(float) + sizeof(int));
 }
 
+// ------------------------------------------------------------------------------------------
+// Certified pass, one thread per token-side (one column chunk per half, k <= 32).  Same
+// decisions as the warp pass (MODE 0), with the outer-sum candidates taken from a binary
+// max-heap of the k row heads A1[i] + A2[j_i] in shared memory (the rows start sorted, so the
+// array of first heads already is a heap): k + 1 pops give the k-th and (k+1)-th values.
+// Exact tie order is irrelevant here: a certified boundary has a positive gap, so equal
+// values never straddle it.  Token-sides with an uncertified boundary go to queue A.
+// ------------------------------------------------------------------------------------------
+constexpr int FT_THREADS = 64;
+
+__host__ __device__ constexpr int ft_words(int km) { return 8 * km + 4; }   // shared words per thread
+
+template <class D, int L>
+__global__ void __launch_bounds__(FT_THREADS) k_addr_finalize_thread(const AddrArgs a) {
+    constexpr int KM = L - 4;                     // largest k served
+    constexpr int LOG = KM <= 8 ? 3 : KM <= 16 ? 4 : 5;
+    extern __shared__ float fts[];
+    const int tid = threadIdx.x;
+    // per-thread columns [word][FT_THREADS]: conflict-free for any word index
+    float* const A1v = fts + tid;                 // [KM + 1]
+    int* const A1i = reinterpret_cast<int*>(fts) + (KM + 1) * FT_THREADS + tid;   // [KM]
+    float* const A2v = fts + (2 * KM + 1) * FT_THREADS + tid;                     // [KM + 1]
+    int* const A2i = reinterpret_cast<int*>(fts) + (3 * KM + 2) * FT_THREADS + tid;   // [KM]
+    float* const hv = fts + (4 * KM + 2) * FT_THREADS + tid;                      // [KM] heap values
+    int* const hp = reinterpret_cast<int*>(fts) + (5 * KM + 2) * FT_THREADS + tid; // [KM] row | col << 8
+    float* const ov = fts + (6 * KM + 2) * FT_THREADS + tid;                      // [KM + 1] popped values
+    int* const os = reinterpret_cast<int*>(fts) + (7 * KM + 3) * FT_THREADS + tid; // [KM + 1] popped slots
+    constexpr int W = FT_THREADS;
+
+    const uint32_t BT = static_cast<uint32_t>(a.B) * static_cast<uint32_t>(a.T);
+    const uint32_t items = 2u * static_cast<uint32_t>(a.H) * BT;      // < 2^31 (a queue exists)
+    const uint32_t item = blockIdx.x * FT_THREADS + tid;
+    if (item >= items) return;                    // no barrier in this kernel
+    const uint32_t z = item / BT, u = item - z * BT;
+    const int side = static_cast<int>(z) / a.H, h = static_cast<int>(z) % a.H;
+    const int k = a.kk[side];
+    const int S = a.S;
+    const uint32_t b = u / static_cast<uint32_t>(a.T), t = u - b * static_cast<uint32_t>(a.T);
+    const void* X = a.X[side];
+    const int64_t xoff = ((static_cast<int64_t>(b) * a.H + h) * a.T + t) * a.dk;
+
+    float e2 = 0.f;
+    if (a.P[side] != nullptr) {
+        float ss = 0.f;
+        const char* xr = static_cast<const char*>(X) + xoff * D::BYTES;
+        if ((reinterpret_cast<uintptr_t>(xr) & 15) == 0 && (a.dk * D::BYTES) % 16 == 0) {
+            for (int q = 0; q < a.dk * D::BYTES / 16; ++q) {
+                float f[D::E];
+                unpack16<D>(__ldg(reinterpret_cast<const uint4*>(xr) + q), f);
+#pragma unroll
+                for (int e = 0; e < D::E; ++e) ss = fmaf(f[e], f[e], ss);
+            }
+        } else {
+            for (int d = 0; d < a.dk; ++d) {
+                const float xv = load_elem<D>(X, xoff + d);
+                ss = fmaf(xv, xv, ss);
+            }
+        }
+        // (1 + 2^-12) covers the roundings of ||x||^2, its square root and the products
+        e2 = __fmul_ru(__fmul_ru(__fmul_ru(2.f * a.cbound, a.pnorm[side * a.H + h]), sqrtf(ss)), 1.f + 0x1p-12f);
+    }
+    auto defer = [&]() { a.queue[2 + atomicAdd(a.queue, 1)] = static_cast<int>(item); };
+
+    // the two half lists (chunk 0 of each half), first k + 1 entries
+    float amax[2];
+#pragma unroll
+    for (int hf = 0; hf < 2; ++hf) {
+        const int64_t base = part_at(static_cast<int>(z), 1, hf, BT, u, L, 0);
+        const float4* pv = reinterpret_cast<const float4*>(a.part_v + base);
+        const int4* pi = reinterpret_cast<const int4*>(a.part_i + base);
+        float* Av = hf ? A2v : A1v;
+        int* Ai = hf ? A2i : A1i;
+#pragma unroll
+        for (int q = 0; q < L / 4; ++q) {
+            if (4 * q <= k) {
+                const float4 v4 = __ldg(pv + q);
+                const int4 i4 = __ldg(pi + q);
+                const float vv[4] = {v4.x, v4.y, v4.z, v4.w};
+                const int ii[4] = {i4.x, i4.y, i4.z, i4.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const int p = 4 * q + e;
+                    if (p <= k && p <= KM) Av[p * W] = vv[e];
+                    if (p < k && p < KM) Ai[p * W] = ii[e];
+                }
+            }
+        }
+        const float vk = Av[(k - 1) * W], vk1 = Av[k * W];
+        if (!(S <= k || __fsub_rd(vk, vk1) > e2)) { defer(); return; }
+        amax[hf] = fmaxf(fabsf(Av[0]), fabsf(vk));
+    }
+    const float e2c = __fadd_ru(__fmul_ru(2.f, e2), __fmul_ru(0x1p-21f, __fadd_ru(amax[0], amax[1])));
+
+    // k-way merge of the rows i (head A1[i] + A2[j_i]) through a max-heap of size k
+    const float a20 = A2v[0];
+    for (int i = 0; i < k; ++i) { hv[i * W] = A1v[i * W] + a20; hp[i * W] = i; }
+    for (int r = 0; r <= k; ++r) {
+        const float v = hv[0];
+        const int pk = hp[0];
+        const int i = pk & 255, j = pk >> 8;
+        ov[r * W] = v;
+        os[r * W] = A1i[i * W] * S + A2i[j * W];
+        const int j1 = j + 1;
+        const float nv = j1 < k ? A1v[i * W] + A2v[j1 * W] : -INFINITY;
+        const int np = i | (j1 << 8);
+        int pos = 0;
+        bool done = false;
+#pragma unroll
+        for (int lvl = 0; lvl < LOG; ++lvl) {
+            const int c = 2 * pos + 1;
+            const float v1 = c < k ? hv[c * W] : -INFINITY;
+            const float v2 = c + 1 < k ? hv[(c + 1) * W] : -INFINITY;
+            const int cm = v2 > v1 ? c + 1 : c;
+            const float vm = fmaxf(v1, v2);
+            if (!done && vm > nv) {
+                hv[pos * W] = vm;
+                hp[pos * W] = hp[cm * W];
+                pos = cm;
+            } else {
+                done = true;
+            }
+        }
+        hv[pos * W] = nv;
+        hp[pos * W] = np;
+    }
+    if (!(__fsub_rd(ov[(k - 1) * W], ov[k * W]) > e2c)) { defer(); return; }
+
+    // softmax over the k selected scores, then ascending slot order (bitonic network)
+    const float vmax = ov[0];
+    float ew[KM];
+    int sl[KM];
+    float zsum = 0.f;
+#pragma unroll
+    for (int r = 0; r < KM; ++r) {
+        if (r < k) {
+            ew[r] = expf(ov[r * W] - vmax);
+            sl[r] = os[r * W];
+            zsum += ew[r];
+        } else {
+            ew[r] = 0.f;
+            sl[r] = INT_MAX;
+        }
+    }
+#pragma unroll
+    for (int size = 2; size <= KM; size <<= 1)
+#pragma unroll
+        for (int stride = size >> 1; stride > 0; stride >>= 1)
+#pragma unroll
+            for (int i = 0; i < KM; ++i) {
+                const int jx = i ^ stride;
+                if (jx > i) {
+                    const bool up = (i & size) == 0;
+                    const bool sw = up ? (sl[i] > sl[jx]) : (sl[i] < sl[jx]);
+                    const int si = sl[i];
+                    const float ei = ew[i];
+                    sl[i] = sw ? sl[jx] : si;  ew[i] = sw ? ew[jx] : ei;
+                    sl[jx] = sw ? si : sl[jx]; ew[jx] = sw ? ei : ew[jx];
+                }
+            }
+    const float inv = 1.f / zsum;
+    const int64_t tokoff = ((static_cast<int64_t>(b) * a.H + h) * a.T + t) * k;
+    int32_t* oi = a.idx[side] + tokoff;
+    float* ow = a.w[side] + tokoff;
+#pragma unroll
+    for (int r = 0; r < KM; ++r)
+        if (r < k) { oi[r] = sl[r]; ow[r] = ew[r] / zsum; }
+    (void)inv;
+}
+
 template <class D, int L>
 static cudaError_t launch_finalize(const AddrArgs& a, cudaStream_t stream) {
     const int64_t BT = static_cast<int64_t>(a.B) * a.T;
@@ -1225,7 +1394,17 @@ static cudaError_t launch_finalize(const AddrArgs& a, cudaStream_t stream) {
         if (a.queue != nullptr) {
             e = cudaMemsetAsync(a.queue, 0, 2 * sizeof(int), stream);
             if (e != cudaSuccess) return e;
-            k_addr_finalize<D, L, FIN_FAST><<<grid, FW_WARPS * 32, 0, stream>>>(a);
+            if (a.ncc == 1) {                    // certified pass, one thread per token-side
+                const size_t smt = static_cast<size_t>(ft_words(L - 4)) * FT_THREADS * sizeof(float);
+                e = cudaFuncSetAttribute(k_addr_finalize_thread<D, L>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smt));
+                if (e != cudaSuccess) return e;
+                const int64_t items = 2 * a.H * BT;
+                k_addr_finalize_thread<D, L><<<static_cast<unsigned>((items + FT_THREADS - 1) / FT_THREADS), FT_THREADS,
+                                               smt, stream>>>(a);
+            } else {
+                k_addr_finalize<D, L, FIN_FAST><<<grid, FW_WARPS * 32, 0, stream>>>(a);
+            }
             k_addr_finalize<D, L, FIN_BAND><<<grid, FW_WARPS * 32, 0, stream>>>(a);
         }
         k_addr_finalize<D, L, FIN_FULL><<<grid, FW_WARPS * 32, 0, stream>>>(a);
