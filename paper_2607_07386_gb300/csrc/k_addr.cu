@@ -1371,6 +1371,296 @@ __global__ void __launch_bounds__(FT_THREADS) k_addr_finalize_thread(const AddrA
     (void)inv;
 }
 
+// ------------------------------------------------------------------------------------------
+// Band pass, one thread per token-side of queue A (one column chunk per half, k <= 32): the
+// band of an uncertified boundary (entries within twice the error bound of it) is re-ranked
+// by compensated scores, one thread computing each score sequentially.  A band that leaves
+// the kept candidates, holds more than 32 entries, or has two entries closer than their
+// compensated bounds goes to queue B (float64 and whole-half paths).
+// ------------------------------------------------------------------------------------------
+constexpr int BT_THREADS = 32;
+__host__ __device__ constexpr int bt_words(int L) { return 4 * L + 2 * (L - 4) + 2 * 64 + 4 * 32; }
+
+// Compensated score of column j of half hf by one thread (16-byte loads when aligned); the
+// same error-free splitting and the same 2^-28 sum|P x| bound as ff_score_warp.
+template <class D>
+__device__ FF ff_score_thread(const void* P, const void* X, int64_t xoff, int64_t prow0, int dk, int S, int hf, int j) {
+    if (P == nullptr) return FF{load_elem<D>(X, xoff + static_cast<int64_t>(hf) * S + j), 0.f, 0.f};
+    const int64_t prow = (prow0 + static_cast<int64_t>(hf) * S + j) * dk;
+    float sum = 0.f, err = 0.f, mag = 0.f;
+    auto term = [&](float pv, float xv) {
+        const float p = __fmul_rn(pv, xv);
+        const float pe = __fmaf_rn(pv, xv, -p);
+        float t, e2;
+        two_sum(sum, p, t, e2);
+        sum = t;
+        err = __fadd_rn(err, __fadd_rn(e2, pe));
+        mag = __fadd_rn(mag, fabsf(p));
+    };
+    const char* pr = static_cast<const char*>(P) + prow * D::BYTES;
+    const char* xr = static_cast<const char*>(X) + xoff * D::BYTES;
+    if (((reinterpret_cast<uintptr_t>(pr) | reinterpret_cast<uintptr_t>(xr)) & 15) == 0 && (dk * D::BYTES) % 16 == 0) {
+        for (int q = 0; q < dk * D::BYTES / 16; ++q) {
+            float fp[D::E], fx[D::E];
+            unpack16<D>(__ldg(reinterpret_cast<const uint4*>(pr) + q), fp);
+            unpack16<D>(__ldg(reinterpret_cast<const uint4*>(xr) + q), fx);
+#pragma unroll
+            for (int e = 0; e < D::E; ++e) term(fp[e], fx[e]);
+        }
+    } else {
+        for (int d = 0; d < dk; ++d) term(load_elem<D>(P, prow + d), load_elem<D>(X, xoff + d));
+    }
+    FF r;
+    r.h = __fadd_rn(sum, err);
+    r.l = __fsub_rn(err, __fsub_rn(r.h, sum));
+    r.b = __fmul_ru(0x1p-28f, mag);
+    return r;
+}
+
+// f versus e (compensated values): +1 if f is certainly larger, -1 if certainly smaller, 0 if
+// equal with zero bounds (exact values: the caller breaks the tie); sets unsure when the two
+// are closer than their bounds.
+__device__ __forceinline__ int ff_cmp(const FF& f, const FF& e, bool& unsure) {
+    float t, r;
+    two_sum(f.h, -e.h, t, r);
+    const float w = __fadd_rn(__fsub_rn(f.l, e.l), r);
+    const float diff = __fadd_rn(t, w);
+    const float slack = __fmul_ru(0x1p-21f, __fadd_ru(__fadd_ru(fabsf(t), fabsf(r)), __fadd_ru(fabsf(f.l), fabsf(e.l))));
+    const float tol = __fadd_ru(__fadd_ru(f.b, e.b), slack);
+    if (tol > 0.f && fabsf(diff) <= tol) { unsure = true; return 0; }
+    return diff > 0.f ? 1 : diff < 0.f ? -1 : 0;
+}
+
+template <class D, int L>
+__global__ void __launch_bounds__(BT_THREADS) k_addr_band_thread(const AddrArgs a) {
+    constexpr int KM = L - 4;
+    constexpr int LOG = KM <= 8 ? 3 : KM <= 16 ? 4 : 5;
+    constexpr int W = BT_THREADS;
+    extern __shared__ float bts[];
+    const int tid = threadIdx.x;
+    float* const A1v = bts + tid;                                              // [L]
+    int* const A1i = reinterpret_cast<int*>(bts) + L * W + tid;                // [L]
+    float* const A2v = bts + 2 * L * W + tid;                                  // [L]
+    int* const A2i = reinterpret_cast<int*>(bts) + 3 * L * W + tid;            // [L]
+    float* const hv = bts + 4 * L * W + tid;                                   // [KM]
+    int* const hp = reinterpret_cast<int*>(bts) + (4 * L + KM) * W + tid;      // [KM]
+    float* const ov = bts + (4 * L + 2 * KM) * W + tid;                        // [64] candidates
+    int* const os = reinterpret_cast<int*>(bts) + (4 * L + 2 * KM + 64) * W + tid;   // [64]
+    float* const bh = bts + (4 * L + 2 * KM + 128) * W + tid;                  // [32] band: h
+    float* const bl = bts + (4 * L + 2 * KM + 160) * W + tid;                  // [32]       l
+    float* const bb = bts + (4 * L + 2 * KM + 192) * W + tid;                  // [32]       bound
+    int* const bc = reinterpret_cast<int*>(bts) + (4 * L + 2 * KM + 224) * W + tid;  // [32] chosen flag
+
+    const uint32_t BT = static_cast<uint32_t>(a.B) * static_cast<uint32_t>(a.T);
+    const uint32_t nq = static_cast<uint32_t>(*reinterpret_cast<volatile int*>(a.queue));
+    const uint32_t q = blockIdx.x * BT_THREADS + tid;
+    if (q >= nq) return;
+    const uint32_t all = 2u * static_cast<uint32_t>(a.H) * BT;
+    const uint32_t item = static_cast<uint32_t>(a.queue[2 + q]);
+    int* const qb = a.queue + 2 + all;
+    auto defer = [&]() { qb[atomicAdd(a.queue + 1, 1)] = static_cast<int>(item); };
+    const uint32_t z = item / BT, u = item - z * BT;
+    const int side = static_cast<int>(z) / a.H, h = static_cast<int>(z) % a.H;
+    const int k = a.kk[side];
+    const int S = a.S;
+    const uint32_t b = u / static_cast<uint32_t>(a.T), t = u - b * static_cast<uint32_t>(a.T);
+    const void* X = a.X[side];
+    const void* P = a.P[side];
+    const int64_t xoff = ((static_cast<int64_t>(b) * a.H + h) * a.T + t) * a.dk;
+    const int64_t prow0 = static_cast<int64_t>(h) * 2 * S;
+
+    float e2 = 0.f;
+    if (P != nullptr) {
+        float ss = 0.f;
+        for (int d = 0; d < a.dk; ++d) {
+            const float xv = load_elem<D>(X, xoff + d);
+            ss = fmaf(xv, xv, ss);
+        }
+        e2 = __fmul_ru(__fmul_ru(__fmul_ru(2.f * a.cbound, a.pnorm[side * a.H + h]), sqrtf(ss)), 1.f + 0x1p-12f);
+    }
+    uint32_t stat_hb = 0, stat_he = 0, stat_cb = 0, stat_ce = 0, stat_cm = 0;
+
+    float amax[2];
+    for (int hf = 0; hf < 2; ++hf) {
+        const int64_t base = part_at(static_cast<int>(z), 1, hf, BT, u, L, 0);
+        float* Av = hf ? A2v : A1v;
+        int* Ai = hf ? A2i : A1i;
+        for (int p = 0; p < L; ++p) { Av[p * W] = __ldg(a.part_v + base + p); Ai[p * W] = __ldg(a.part_i + base + p); }
+        const float vk = Av[(k - 1) * W], vk1 = Av[k * W];
+        if (!(S <= k || __fsub_rd(vk, vk1) > e2)) {
+            // band of the half boundary
+            ++stat_hb;
+            const float lo = __fsub_rd(vk, e2), hi = __fadd_ru(vk1, e2);
+            if (S > L && Av[(L - 1) * W] >= lo) { defer(); goto done; }
+            int cin = 0, m = 0;
+            for (int p = 0; p < L; ++p) {        // (-inf padding never enters a band)
+                const float v = Av[p * W];
+                cin += v > hi ? 1 : 0;
+                m += (v >= lo && v <= hi && v != -INFINITY) ? 1 : 0;
+            }
+            if (m > 32) { defer(); goto done; }
+            stat_he += m;
+            for (int e = 0; e < m; ++e) {
+                const FF f = ff_score_thread<D>(P, X, xoff, prow0, a.dk, S, hf, Ai[(cin + e) * W]);
+                bh[e * W] = f.h; bl[e * W] = f.l; bb[e * W] = f.b;
+            }
+            bool unsure = false;
+            for (int e = 0; e < m; ++e) {
+                const FF fe{bh[e * W], bl[e * W], bb[e * W]};
+                const int ie = Ai[(cin + e) * W];
+                int rank = 0;
+                for (int f = 0; f < m; ++f) {
+                    if (f == e) continue;
+                    const FF ff{bh[f * W], bl[f * W], bb[f * W]};
+                    const int c = ff_cmp(ff, fe, unsure);
+                    rank += (c > 0 || (c == 0 && Ai[(cin + f) * W] < ie)) ? 1 : 0;
+                }
+                bc[e * W] = rank < k - cin ? 1 : 0;
+            }
+            if (unsure) { defer(); goto done; }
+            // chosen band entries, in list order, after the certain prefix
+            int q2 = cin;
+            for (int e = 0; e < m; ++e) {
+                if (bc[e * W]) {
+                    const float v = Av[(cin + e) * W];
+                    const int ix = Ai[(cin + e) * W];
+                    Av[q2 * W] = v; Ai[q2 * W] = ix;       // q2 <= cin + e: in-place compaction
+                    ++q2;
+                }
+            }
+        }
+        amax[hf] = fmaxf(fabsf(Av[0]), fabsf(Av[(k - 1) * W]));
+    }
+    {
+        const float e2c = __fadd_ru(__fmul_ru(2.f, e2), __fmul_ru(0x1p-21f, __fadd_ru(amax[0], amax[1])));
+        // outer-sum candidates by a max-heap of the row heads (k+4 of them, 64 if the band needs)
+        const float a20 = A2v[0];
+        for (int i = 0; i < k; ++i) { hv[i * W] = A1v[i * W] + a20; hp[i * W] = i; }
+        const int kk2 = k * k;
+        int npop = 0;
+        auto pops = [&](int upto) {
+            for (; npop < upto; ++npop) {
+                const float v = hv[0];
+                const int pk = hp[0];
+                const int i = pk & 255, j = pk >> 8;
+                ov[npop * W] = v;
+                os[npop * W] = (j < k) ? A1i[i * W] * S + A2i[j * W] : INT_MAX;
+                const int j1 = j + 1;
+                const float nv = j1 < k ? A1v[i * W] + A2v[j1 * W] : -INFINITY;
+                const int np = i | (j1 << 8);
+                int pos = 0;
+                bool stop = false;
+#pragma unroll
+                for (int lvl = 0; lvl < LOG; ++lvl) {
+                    const int c = 2 * pos + 1;
+                    const float v1 = c < k ? hv[c * W] : -INFINITY;
+                    const float v2 = c + 1 < k ? hv[(c + 1) * W] : -INFINITY;
+                    const int cm = v2 > v1 ? c + 1 : c;
+                    const float vm = fmaxf(v1, v2);
+                    if (!stop && vm > nv) { hv[pos * W] = vm; hp[pos * W] = hp[cm * W]; pos = cm; }
+                    else stop = true;
+                }
+                hv[pos * W] = nv;
+                hp[pos * W] = np;
+            }
+        };
+        const int len0 = kk2 < L ? kk2 : L;
+        pops(len0 > k + 1 ? len0 : k + 1);
+        int len = npop;
+        const float ck = ov[(k - 1) * W], ck1 = k < npop ? ov[k * W] : -INFINITY;
+        int nsel = k;                              // selected: candidates [0, k) unless a band is resolved
+        if (!(ck1 == -INFINITY || __fsub_rd(ck, ck1) > e2c)) {
+            ++stat_cb;
+            const float lo = __fsub_rd(ck, e2c), hi = __fadd_ru(ck1, e2c);
+            if (kk2 > len && ov[(len - 1) * W] != -INFINITY && ov[(len - 1) * W] >= lo) {
+                ++stat_cm;
+                pops(kk2 < 64 ? kk2 : 64);
+                len = npop;
+            }
+            const bool all_cands = len >= kk2;
+            if (!all_cands && ov[(len - 1) * W] != -INFINITY && ov[(len - 1) * W] >= lo) { defer(); goto done; }
+            int cin = 0, m = 0;
+            for (int p = 0; p < len; ++p) {      // (exhausted rows, -inf, never enter a band)
+                const float v = ov[p * W];
+                cin += v > hi ? 1 : 0;
+                m += (v >= lo && v <= hi && v != -INFINITY) ? 1 : 0;
+            }
+            if (m > 32) { defer(); goto done; }
+            stat_ce += m;
+            for (int e = 0; e < m; ++e) {
+                const int f = os[(cin + e) * W];
+                const FF s1 = ff_score_thread<D>(P, X, xoff, prow0, a.dk, S, 0, f / S);
+                const FF s2 = ff_score_thread<D>(P, X, xoff, prow0, a.dk, S, 1, f % S);
+                const FF sm = ff_add(s1, s2, P == nullptr);
+                bh[e * W] = sm.h; bl[e * W] = sm.l; bb[e * W] = sm.b;
+            }
+            bool unsure = false;
+            for (int e = 0; e < m; ++e) {
+                const FF fe{bh[e * W], bl[e * W], bb[e * W]};
+                const int ie = os[(cin + e) * W];
+                int rank = 0;
+                for (int f = 0; f < m; ++f) {
+                    if (f == e) continue;
+                    const FF ff{bh[f * W], bl[f * W], bb[f * W]};
+                    const int c = ff_cmp(ff, fe, unsure);
+                    rank += (c > 0 || (c == 0 && os[(cin + f) * W] < ie)) ? 1 : 0;
+                }
+                bc[e * W] = rank < k - cin ? 1 : 0;
+            }
+            if (unsure) { defer(); goto done; }
+            int q2 = cin;
+            for (int e = 0; e < m; ++e) {
+                if (bc[e * W]) {
+                    const float v = ov[(cin + e) * W];
+                    const int f = os[(cin + e) * W];
+                    ov[q2 * W] = v; os[q2 * W] = f;
+                    ++q2;
+                }
+            }
+            nsel = q2;                             // = k
+        }
+        // softmax over the k selected scores, then ascending slot order
+        float vmax = -INFINITY;
+        for (int r = 0; r < nsel; ++r) vmax = fmaxf(vmax, ov[r * W]);
+        float ew[KM];
+        int sl[KM];
+        float zsum = 0.f;
+#pragma unroll
+        for (int r = 0; r < KM; ++r) {
+            if (r < k) { ew[r] = expf(ov[r * W] - vmax); sl[r] = os[r * W]; zsum += ew[r]; }
+            else { ew[r] = 0.f; sl[r] = INT_MAX; }
+        }
+#pragma unroll
+        for (int size = 2; size <= KM; size <<= 1)
+#pragma unroll
+            for (int stride = size >> 1; stride > 0; stride >>= 1)
+#pragma unroll
+                for (int i = 0; i < KM; ++i) {
+                    const int jx = i ^ stride;
+                    if (jx > i) {
+                        const bool up = (i & size) == 0;
+                        const bool sw = up ? (sl[i] > sl[jx]) : (sl[i] < sl[jx]);
+                        const int si = sl[i];
+                        const float ei = ew[i];
+                        sl[i] = sw ? sl[jx] : si;  ew[i] = sw ? ew[jx] : ei;
+                        sl[jx] = sw ? si : sl[jx]; ew[jx] = sw ? ei : ew[jx];
+                    }
+                }
+        const int64_t tokoff = ((static_cast<int64_t>(b) * a.H + h) * a.T + t) * k;
+        int32_t* oi = a.idx[side] + tokoff;
+        float* ow = a.w[side] + tokoff;
+#pragma unroll
+        for (int r = 0; r < KM; ++r)
+            if (r < k) { oi[r] = sl[r]; ow[r] = ew[r] / zsum; }
+    }
+done:
+    if (stat_hb) stat_add(a.err, STAT_HALF_BAND, stat_hb);
+    if (stat_he) stat_add(a.err, STAT_HALF_BAND_ENTRIES, stat_he);
+    if (stat_cb) stat_add(a.err, STAT_COMB_BAND, stat_cb);
+    if (stat_ce) stat_add(a.err, STAT_COMB_BAND_ENTRIES, stat_ce);
+    if (stat_cm) stat_add(a.err, STAT_COMB_MERGE, stat_cm);
+}
+
 template <class D, int L>
 static cudaError_t launch_finalize(const AddrArgs& a, cudaStream_t stream) {
     const int64_t BT = static_cast<int64_t>(a.B) * a.T;
@@ -1405,7 +1695,17 @@ static cudaError_t launch_finalize(const AddrArgs& a, cudaStream_t stream) {
             } else {
                 k_addr_finalize<D, L, FIN_FAST><<<grid, FW_WARPS * 32, 0, stream>>>(a);
             }
-            k_addr_finalize<D, L, FIN_BAND><<<grid, FW_WARPS * 32, 0, stream>>>(a);
+            if (a.ncc == 1) {                    // band pass, one thread per queued token-side
+                const size_t smb = static_cast<size_t>(bt_words(L)) * BT_THREADS * sizeof(float);
+                e = cudaFuncSetAttribute(k_addr_band_thread<D, L>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         static_cast<int>(smb));
+                if (e != cudaSuccess) return e;
+                const int64_t items = 2 * a.H * BT;       // upper bound of the queue length
+                k_addr_band_thread<D, L><<<static_cast<unsigned>((items + BT_THREADS - 1) / BT_THREADS), BT_THREADS,
+                                           smb, stream>>>(a);
+            } else {
+                k_addr_finalize<D, L, FIN_BAND><<<grid, FW_WARPS * 32, 0, stream>>>(a);
+            }
         }
         k_addr_finalize<D, L, FIN_FULL><<<grid, FW_WARPS * 32, 0, stream>>>(a);
     } else {
