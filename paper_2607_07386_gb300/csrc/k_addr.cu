@@ -939,7 +939,7 @@ __global__ void __launch_bounds__(FW_WARPS * 32, 4) k_addr_finalize(const AddrAr
         const float vl = lane_get(cv0, cv1, L - 1);
         if (k * k > L && vl != -INFINITY &&
             vl >= __fsub_rd(lane_get(cv0, cv1, k - 1), e2c)) {
-            if (lane == 0 && c.count_band) tstat(c, STAT_COMB_MERGE);
+            if (lane == 0) tstat(c, STAT_COMB_MERGE);
             len = min(64, k * k);
             merge_steps(L, len);
         }
@@ -1379,7 +1379,8 @@ __global__ void __launch_bounds__(FT_THREADS) k_addr_finalize_thread(const AddrA
 // compensated bounds goes to queue B (float64 and whole-half paths).
 // ------------------------------------------------------------------------------------------
 constexpr int BT_THREADS = 32;
-__host__ __device__ constexpr int bt_words(int L) { return 4 * L + 2 * (L - 4) + 2 * 64 + 4 * 32; }
+constexpr int BT_BAND = 8;        // band entries re-ranked here; wider bands go to queue B
+__host__ __device__ constexpr int bt_words(int L) { return 4 * L + 2 * (L - 4) + 2 * L + 4 * BT_BAND; }
 
 // Compensated score of column j of half hf by one thread (16-byte loads when aligned); the
 // same error-free splitting and the same 2^-28 sum|P x| bound as ff_score_warp.
@@ -1444,12 +1445,12 @@ __global__ void __launch_bounds__(BT_THREADS) k_addr_band_thread(const AddrArgs 
     int* const A2i = reinterpret_cast<int*>(bts) + 3 * L * W + tid;            // [L]
     float* const hv = bts + 4 * L * W + tid;                                   // [KM]
     int* const hp = reinterpret_cast<int*>(bts) + (4 * L + KM) * W + tid;      // [KM]
-    float* const ov = bts + (4 * L + 2 * KM) * W + tid;                        // [64] candidates
-    int* const os = reinterpret_cast<int*>(bts) + (4 * L + 2 * KM + 64) * W + tid;   // [64]
-    float* const bh = bts + (4 * L + 2 * KM + 128) * W + tid;                  // [32] band: h
-    float* const bl = bts + (4 * L + 2 * KM + 160) * W + tid;                  // [32]       l
-    float* const bb = bts + (4 * L + 2 * KM + 192) * W + tid;                  // [32]       bound
-    int* const bc = reinterpret_cast<int*>(bts) + (4 * L + 2 * KM + 224) * W + tid;  // [32] chosen flag
+    float* const ov = bts + (4 * L + 2 * KM) * W + tid;                        // [L] candidates
+    int* const os = reinterpret_cast<int*>(bts) + (5 * L + 2 * KM) * W + tid;  // [L]
+    float* const bh = bts + (6 * L + 2 * KM) * W + tid;                        // [BT_BAND] band: h
+    float* const bl = bts + (6 * L + 2 * KM + BT_BAND) * W + tid;              //                 l
+    float* const bb = bts + (6 * L + 2 * KM + 2 * BT_BAND) * W + tid;          //                 bound
+    int* const bc = reinterpret_cast<int*>(bts) + (6 * L + 2 * KM + 3 * BT_BAND) * W + tid;   // chosen
 
     const uint32_t BT = static_cast<uint32_t>(a.B) * static_cast<uint32_t>(a.T);
     const uint32_t nq = static_cast<uint32_t>(*reinterpret_cast<volatile int*>(a.queue));
@@ -1478,7 +1479,7 @@ __global__ void __launch_bounds__(BT_THREADS) k_addr_band_thread(const AddrArgs 
         }
         e2 = __fmul_ru(__fmul_ru(__fmul_ru(2.f * a.cbound, a.pnorm[side * a.H + h]), sqrtf(ss)), 1.f + 0x1p-12f);
     }
-    uint32_t stat_hb = 0, stat_he = 0, stat_cb = 0, stat_ce = 0, stat_cm = 0;
+    uint32_t stat_hb = 0, stat_he = 0, stat_cb = 0, stat_ce = 0;
 
     float amax[2];
     for (int hf = 0; hf < 2; ++hf) {
@@ -1498,7 +1499,7 @@ __global__ void __launch_bounds__(BT_THREADS) k_addr_band_thread(const AddrArgs 
                 cin += v > hi ? 1 : 0;
                 m += (v >= lo && v <= hi && v != -INFINITY) ? 1 : 0;
             }
-            if (m > 32) { defer(); goto done; }
+            if (m > BT_BAND) { defer(); goto done; }
             stat_he += m;
             for (int e = 0; e < m; ++e) {
                 const FF f = ff_score_thread<D>(P, X, xoff, prow0, a.dk, S, hf, Ai[(cin + e) * W]);
@@ -1572,11 +1573,7 @@ __global__ void __launch_bounds__(BT_THREADS) k_addr_band_thread(const AddrArgs 
         if (!(ck1 == -INFINITY || __fsub_rd(ck, ck1) > e2c)) {
             ++stat_cb;
             const float lo = __fsub_rd(ck, e2c), hi = __fadd_ru(ck1, e2c);
-            if (kk2 > len && ov[(len - 1) * W] != -INFINITY && ov[(len - 1) * W] >= lo) {
-                ++stat_cm;
-                pops(kk2 < 64 ? kk2 : 64);
-                len = npop;
-            }
+            // a band reaching the last kept candidate (merge to be extended): queue B
             const bool all_cands = len >= kk2;
             if (!all_cands && ov[(len - 1) * W] != -INFINITY && ov[(len - 1) * W] >= lo) { defer(); goto done; }
             int cin = 0, m = 0;
@@ -1585,7 +1582,7 @@ __global__ void __launch_bounds__(BT_THREADS) k_addr_band_thread(const AddrArgs 
                 cin += v > hi ? 1 : 0;
                 m += (v >= lo && v <= hi && v != -INFINITY) ? 1 : 0;
             }
-            if (m > 32) { defer(); goto done; }
+            if (m > BT_BAND) { defer(); goto done; }
             stat_ce += m;
             for (int e = 0; e < m; ++e) {
                 const int f = os[(cin + e) * W];
@@ -1658,7 +1655,6 @@ done:
     if (stat_he) stat_add(a.err, STAT_HALF_BAND_ENTRIES, stat_he);
     if (stat_cb) stat_add(a.err, STAT_COMB_BAND, stat_cb);
     if (stat_ce) stat_add(a.err, STAT_COMB_BAND_ENTRIES, stat_ce);
-    if (stat_cm) stat_add(a.err, STAT_COMB_MERGE, stat_cm);
 }
 
 template <class D, int L>
