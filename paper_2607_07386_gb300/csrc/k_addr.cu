@@ -589,16 +589,14 @@ __device__ __forceinline__ void warp_sort64_desc(float& a, float& b, int lane) {
     }
 }
 
-// Compensated score of column j of half hf by one lane (sequential d; same splitting and
-// the same 2^-28 sum|P x| bound as ff_score_warp).
+// Compensated score of column j of half hf by one thread (16-byte loads when aligned); the
+// same error-free splitting and the same 2^-28 sum|P x| bound as ff_score_warp.
 template <class D>
-__device__ FF ff_score_lane(const TokenCtx& c, int hf, int j) {
-    if (c.P == nullptr) return FF{load_elem<D>(c.X, c.xoff + static_cast<int64_t>(hf) * c.S + j), 0.f, 0.f};
-    const int64_t prow = (c.prow0 + static_cast<int64_t>(hf) * c.S + j) * c.dk;
+__device__ FF ff_score_thread(const void* P, const void* X, int64_t xoff, int64_t prow0, int dk, int S, int hf, int j) {
+    if (P == nullptr) return FF{load_elem<D>(X, xoff + static_cast<int64_t>(hf) * S + j), 0.f, 0.f};
+    const int64_t prow = (prow0 + static_cast<int64_t>(hf) * S + j) * dk;
     float sum = 0.f, err = 0.f, mag = 0.f;
-#pragma unroll 4
-    for (int d = 0; d < c.dk; ++d) {
-        const float pv = load_elem<D>(c.P, prow + d), xv = load_elem<D>(c.X, c.xoff + d);
+    auto term = [&](float pv, float xv) {
         const float p = __fmul_rn(pv, xv);
         const float pe = __fmaf_rn(pv, xv, -p);
         float t, e2;
@@ -606,6 +604,19 @@ __device__ FF ff_score_lane(const TokenCtx& c, int hf, int j) {
         sum = t;
         err = __fadd_rn(err, __fadd_rn(e2, pe));
         mag = __fadd_rn(mag, fabsf(p));
+    };
+    const char* pr = static_cast<const char*>(P) + prow * D::BYTES;
+    const char* xr = static_cast<const char*>(X) + xoff * D::BYTES;
+    if (((reinterpret_cast<uintptr_t>(pr) | reinterpret_cast<uintptr_t>(xr)) & 15) == 0 && (dk * D::BYTES) % 16 == 0) {
+        for (int q = 0; q < dk * D::BYTES / 16; ++q) {
+            float fp[D::E], fx[D::E];
+            unpack16<D>(__ldg(reinterpret_cast<const uint4*>(pr) + q), fp);
+            unpack16<D>(__ldg(reinterpret_cast<const uint4*>(xr) + q), fx);
+#pragma unroll
+            for (int e = 0; e < D::E; ++e) term(fp[e], fx[e]);
+        }
+    } else {
+        for (int d = 0; d < dk; ++d) term(load_elem<D>(P, prow + d), load_elem<D>(X, xoff + d));
     }
     FF r;
     r.h = __fadd_rn(sum, err);
@@ -626,11 +637,24 @@ template <class D>
 __device__ __noinline__ bool warp_full_half(int k, float e2, const TokenCtx& c, int hf, float* ov, int* oi,
                                             int* scratch, int lane) {
     const int S = c.S;
-    auto fp32_score = [&](int j) -> float {
+    const char* xr = static_cast<const char*>(c.X) + c.xoff * D::BYTES;
+    const bool vec = ((reinterpret_cast<uintptr_t>(c.P) | reinterpret_cast<uintptr_t>(xr)) & 15) == 0 &&
+                     (c.dk * D::BYTES) % 16 == 0;
+    auto fp32_score = [&](int j) -> float {             // sequential FMA over d (error <= eps)
         const int64_t prow = (c.prow0 + static_cast<int64_t>(hf) * S + j) * c.dk;
         float acc = 0.f;
-#pragma unroll 8
-        for (int d = 0; d < c.dk; ++d) acc = fmaf(load_elem<D>(c.P, prow + d), load_elem<D>(c.X, c.xoff + d), acc);
+        if (vec) {
+            const uint4* pr = reinterpret_cast<const uint4*>(static_cast<const char*>(c.P) + prow * D::BYTES);
+            for (int q = 0; q < c.dk * D::BYTES / 16; ++q) {
+                float fp[D::E], fx[D::E];
+                unpack16<D>(__ldg(pr + q), fp);
+                unpack16<D>(__ldg(reinterpret_cast<const uint4*>(xr) + q), fx);
+#pragma unroll
+                for (int e = 0; e < D::E; ++e) acc = fmaf(fp[e], fx[e], acc);
+            }
+        } else {
+            for (int d = 0; d < c.dk; ++d) acc = fmaf(load_elem<D>(c.P, prow + d), load_elem<D>(c.X, c.xoff + d), acc);
+        }
         return acc;
     };
     float t1 = -INFINITY, t2 = -INFINITY;
@@ -658,8 +682,8 @@ __device__ __noinline__ bool warp_full_half(int k, float e2, const TokenCtx& c, 
     const int j1 = lane + 32 < m ? scratch[lane + 32] : 0;
     __syncwarp();
     FF f0{0.f, 0.f, 0.f}, f1{0.f, 0.f, 0.f};
-    if (lane < m) f0 = ff_score_lane<D>(c, hf, j0);
-    if (lane + 32 < m) f1 = ff_score_lane<D>(c, hf, j1);
+    if (lane < m) f0 = ff_score_thread<D>(c.P, c.X, c.xoff, c.prow0, c.dk, S, hf, j0);
+    if (lane + 32 < m) f1 = ff_score_thread<D>(c.P, c.X, c.xoff, c.prow0, c.dk, S, hf, j1);
     // rank both own entries against all m (pairs closer than their bounds: give up)
     int r0 = 0, r1 = 0;
     bool unsure = false;
@@ -1381,42 +1405,6 @@ __global__ void __launch_bounds__(FT_THREADS) k_addr_finalize_thread(const AddrA
 constexpr int BT_THREADS = 32;
 constexpr int BT_BAND = 8;        // band entries re-ranked here; wider bands go to queue B
 __host__ __device__ constexpr int bt_words(int L) { return 4 * L + 2 * (L - 4) + 2 * L + 4 * BT_BAND; }
-
-// Compensated score of column j of half hf by one thread (16-byte loads when aligned); the
-// same error-free splitting and the same 2^-28 sum|P x| bound as ff_score_warp.
-template <class D>
-__device__ FF ff_score_thread(const void* P, const void* X, int64_t xoff, int64_t prow0, int dk, int S, int hf, int j) {
-    if (P == nullptr) return FF{load_elem<D>(X, xoff + static_cast<int64_t>(hf) * S + j), 0.f, 0.f};
-    const int64_t prow = (prow0 + static_cast<int64_t>(hf) * S + j) * dk;
-    float sum = 0.f, err = 0.f, mag = 0.f;
-    auto term = [&](float pv, float xv) {
-        const float p = __fmul_rn(pv, xv);
-        const float pe = __fmaf_rn(pv, xv, -p);
-        float t, e2;
-        two_sum(sum, p, t, e2);
-        sum = t;
-        err = __fadd_rn(err, __fadd_rn(e2, pe));
-        mag = __fadd_rn(mag, fabsf(p));
-    };
-    const char* pr = static_cast<const char*>(P) + prow * D::BYTES;
-    const char* xr = static_cast<const char*>(X) + xoff * D::BYTES;
-    if (((reinterpret_cast<uintptr_t>(pr) | reinterpret_cast<uintptr_t>(xr)) & 15) == 0 && (dk * D::BYTES) % 16 == 0) {
-        for (int q = 0; q < dk * D::BYTES / 16; ++q) {
-            float fp[D::E], fx[D::E];
-            unpack16<D>(__ldg(reinterpret_cast<const uint4*>(pr) + q), fp);
-            unpack16<D>(__ldg(reinterpret_cast<const uint4*>(xr) + q), fx);
-#pragma unroll
-            for (int e = 0; e < D::E; ++e) term(fp[e], fx[e]);
-        }
-    } else {
-        for (int d = 0; d < dk; ++d) term(load_elem<D>(P, prow + d), load_elem<D>(X, xoff + d));
-    }
-    FF r;
-    r.h = __fadd_rn(sum, err);
-    r.l = __fsub_rn(err, __fsub_rn(r.h, sum));
-    r.b = __fmul_ru(0x1p-28f, mag);
-    return r;
-}
 
 // f versus e (compensated values): +1 if f is certainly larger, -1 if certainly smaller, 0 if
 // equal with zero bounds (exact values: the caller breaks the tie); sets unsure when the two
