@@ -1236,7 +1236,9 @@ size_t addr_partial_bytes(const AddrPlan& plan, int B, int H, int T) {
 // ------------------------------------------------------------------------------------------
 constexpr int FT_THREADS = 64;
 
-__host__ __device__ constexpr int ft_words(int km) { return 8 * km + 4; }   // shared words per thread
+// Shared bytes per thread: values and popped candidates as 32-bit words, list indices and
+// heap positions as 16-bit (one column chunk per half: indices < 512).
+__host__ __device__ constexpr int ft_bytes(int km) { return 4 * (km + 1) * 4 + 4 * km + 2 * km * 3; }
 
 template <class D, int L>
 __global__ void __launch_bounds__(FT_THREADS) k_addr_finalize_thread(const AddrArgs a) {
@@ -1244,16 +1246,17 @@ __global__ void __launch_bounds__(FT_THREADS) k_addr_finalize_thread(const AddrA
     constexpr int LOG = KM <= 8 ? 3 : KM <= 16 ? 4 : 5;
     extern __shared__ float fts[];
     const int tid = threadIdx.x;
-    // per-thread columns [word][FT_THREADS]: conflict-free for any word index
-    float* const A1v = fts + tid;                 // [KM + 1]
-    int* const A1i = reinterpret_cast<int*>(fts) + (KM + 1) * FT_THREADS + tid;   // [KM]
-    float* const A2v = fts + (2 * KM + 1) * FT_THREADS + tid;                     // [KM + 1]
-    int* const A2i = reinterpret_cast<int*>(fts) + (3 * KM + 2) * FT_THREADS + tid;   // [KM]
-    float* const hv = fts + (4 * KM + 2) * FT_THREADS + tid;                      // [KM] heap values
-    int* const hp = reinterpret_cast<int*>(fts) + (5 * KM + 2) * FT_THREADS + tid; // [KM] row | col << 8
-    float* const ov = fts + (6 * KM + 2) * FT_THREADS + tid;                      // [KM + 1] popped values
-    int* const os = reinterpret_cast<int*>(fts) + (7 * KM + 3) * FT_THREADS + tid; // [KM + 1] popped slots
     constexpr int W = FT_THREADS;
+    // per-thread columns [element][FT_THREADS]: conflict-free for any element index
+    float* const A1v = fts + tid;                                             // [KM + 1]
+    float* const A2v = fts + (KM + 1) * W + tid;                              // [KM + 1]
+    float* const ov = fts + 2 * (KM + 1) * W + tid;                           // [KM + 1] popped values
+    int* const os = reinterpret_cast<int*>(fts) + 3 * (KM + 1) * W + tid;     // [KM + 1] popped slots
+    float* const hv = fts + 4 * (KM + 1) * W + tid;                           // [KM] heap values
+    unsigned short* const h16 = reinterpret_cast<unsigned short*>(fts + (4 * (KM + 1) + KM) * W);
+    unsigned short* const A1i = h16 + tid;                                    // [KM]
+    unsigned short* const A2i = h16 + KM * W + tid;                           // [KM]
+    unsigned short* const hp = h16 + 2 * KM * W + tid;                        // [KM] row | col << 8
 
     const uint32_t BT = static_cast<uint32_t>(a.B) * static_cast<uint32_t>(a.T);
     const uint32_t items = 2u * static_cast<uint32_t>(a.H) * BT;      // < 2^31 (a queue exists)
@@ -1297,7 +1300,7 @@ __global__ void __launch_bounds__(FT_THREADS) k_addr_finalize_thread(const AddrA
         const float4* pv = reinterpret_cast<const float4*>(a.part_v + base);
         const int4* pi = reinterpret_cast<const int4*>(a.part_i + base);
         float* Av = hf ? A2v : A1v;
-        int* Ai = hf ? A2i : A1i;
+        unsigned short* Ai = hf ? A2i : A1i;
 #pragma unroll
         for (int q = 0; q < L / 4; ++q) {
             if (4 * q <= k) {
@@ -1309,7 +1312,7 @@ __global__ void __launch_bounds__(FT_THREADS) k_addr_finalize_thread(const AddrA
                 for (int e = 0; e < 4; ++e) {
                     const int p = 4 * q + e;
                     if (p <= k && p <= KM) Av[p * W] = vv[e];
-                    if (p < k && p < KM) Ai[p * W] = ii[e];
+                    if (p < k && p < KM) Ai[p * W] = static_cast<unsigned short>(ii[e]);
                 }
             }
         }
@@ -1321,16 +1324,16 @@ __global__ void __launch_bounds__(FT_THREADS) k_addr_finalize_thread(const AddrA
 
     // k-way merge of the rows i (head A1[i] + A2[j_i]) through a max-heap of size k
     const float a20 = A2v[0];
-    for (int i = 0; i < k; ++i) { hv[i * W] = A1v[i * W] + a20; hp[i * W] = i; }
+    for (int i = 0; i < k; ++i) { hv[i * W] = A1v[i * W] + a20; hp[i * W] = static_cast<unsigned short>(i); }
     for (int r = 0; r <= k; ++r) {
         const float v = hv[0];
         const int pk = hp[0];
         const int i = pk & 255, j = pk >> 8;
         ov[r * W] = v;
-        os[r * W] = A1i[i * W] * S + A2i[j * W];
+        os[r * W] = static_cast<int>(A1i[i * W]) * S + static_cast<int>(A2i[(j < k ? j : 0) * W]);
         const int j1 = j + 1;
         const float nv = j1 < k ? A1v[i * W] + A2v[j1 * W] : -INFINITY;
-        const int np = i | (j1 << 8);
+        const unsigned short np = static_cast<unsigned short>(i | (j1 << 8));
         int pos = 0;
         bool done = false;
 #pragma unroll
@@ -1669,7 +1672,7 @@ static cudaError_t launch_finalize(const AddrArgs& a, cudaStream_t stream) {
             e = cudaMemsetAsync(a.queue, 0, 2 * sizeof(int), stream);
             if (e != cudaSuccess) return e;
             if (a.ncc == 1) {                    // certified pass, one thread per token-side
-                const size_t smt = static_cast<size_t>(ft_words(L - 4)) * FT_THREADS * sizeof(float);
+                const size_t smt = static_cast<size_t>(ft_bytes(L - 4)) * FT_THREADS;
                 e = cudaFuncSetAttribute(k_addr_finalize_thread<D, L>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smt));
                 if (e != cudaSuccess) return e;
