@@ -608,12 +608,24 @@ __device__ FF ff_score_thread(const void* P, const void* X, int64_t xoff, int64_
     const char* pr = static_cast<const char*>(P) + prow * D::BYTES;
     const char* xr = static_cast<const char*>(X) + xoff * D::BYTES;
     if (((reinterpret_cast<uintptr_t>(pr) | reinterpret_cast<uintptr_t>(xr)) & 15) == 0 && (dk * D::BYTES) % 16 == 0) {
-        for (int q = 0; q < dk * D::BYTES / 16; ++q) {
-            float fp[D::E], fx[D::E];
-            unpack16<D>(__ldg(reinterpret_cast<const uint4*>(pr) + q), fp);
-            unpack16<D>(__ldg(reinterpret_cast<const uint4*>(xr) + q), fx);
+        const int nq = dk * D::BYTES / 16;
+        for (int q0 = 0; q0 < nq; q0 += 4) {            // four 16-byte loads in flight per operand
+            uint4 pq[4], xq[4];
 #pragma unroll
-            for (int e = 0; e < D::E; ++e) term(fp[e], fx[e]);
+            for (int u = 0; u < 4; ++u)
+                if (q0 + u < nq) {
+                    pq[u] = __ldg(reinterpret_cast<const uint4*>(pr) + q0 + u);
+                    xq[u] = __ldg(reinterpret_cast<const uint4*>(xr) + q0 + u);
+                }
+#pragma unroll
+            for (int u = 0; u < 4; ++u)
+                if (q0 + u < nq) {
+                    float fp[D::E], fx[D::E];
+                    unpack16<D>(pq[u], fp);
+                    unpack16<D>(xq[u], fx);
+#pragma unroll
+                    for (int e = 0; e < D::E; ++e) term(fp[e], fx[e]);
+                }
         }
     } else {
         for (int d = 0; d < dk; ++d) term(load_elem<D>(P, prow + d), load_elem<D>(X, xoff + d));
@@ -1175,26 +1187,38 @@ __global__ void __launch_bounds__(F_THREADS) k_addr_finalize_wide(const AddrArgs
 // ------------------------------------------------------------------------------------------
 template <class D>
 __global__ void __launch_bounds__(256) k_pnorm(const AddrArgs a) {
-    const int side = blockIdx.x / a.H, h = blockIdx.x % a.H;
-    const void* P = a.P[side];
-    __shared__ float red[256];
+    // one warp per row of P (lanes split d), four consecutive rows per warp; the row norms are
+    // folded into pnorm[side * H + h] (zeroed before) by an integer atomicMax, which orders
+    // non-negative floats correctly.  (1 + 2^-12) covers the roundings of the norm.
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int rows = 2 * a.S;
+    const int64_t total = static_cast<int64_t>(2) * a.H * rows;
+    const int64_t r0 = (static_cast<int64_t>(blockIdx.x) * 8 + warp) * 4;
+    int zcur = -1;
     float mx = 0.f;
-    for (int j = threadIdx.x; j < 2 * a.S; j += 256) {
-        const int64_t row = (static_cast<int64_t>(h) * 2 * a.S + j) * a.dk;
+    for (int q = 0; q < 4; ++q) {
+        const int64_t r = r0 + q;
+        if (r >= total) break;                       // warp-uniform
+        const int zs = static_cast<int>(r / rows);
+        const int64_t jrow = r - static_cast<int64_t>(zs) * rows;
+        const int side = zs / a.H, h = zs % a.H;
+        const int64_t row = (static_cast<int64_t>(h) * rows + jrow) * a.dk;
         float ss = 0.f;
-        for (int d = 0; d < a.dk; ++d) {
-            const float p = load_elem<D>(P, row + d);
+        for (int d = lane; d < a.dk; d += 32) {
+            const float p = load_elem<D>(a.P[side], row + d);
             ss = fmaf(p, p, ss);
         }
-        mx = fmaxf(mx, sqrtf(ss));
+#pragma unroll
+        for (int off = 16; off > 0; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
+        const float nrm = sqrtf(ss) * (1.f + 0x1p-12f);
+        if (zs != zcur) {
+            if (zcur >= 0 && lane == 0) atomicMax(reinterpret_cast<int*>(a.pnorm) + zcur, __float_as_int(mx));
+            zcur = zs;
+            mx = 0.f;
+        }
+        mx = fmaxf(mx, nrm);
     }
-    red[threadIdx.x] = mx;
-    __syncthreads();
-    for (int s = 128; s > 0; s >>= 1) {
-        if (threadIdx.x < s) red[threadIdx.x] = fmaxf(red[threadIdx.x], red[threadIdx.x + s]);
-        __syncthreads();
-    }
-    if (threadIdx.x == 0) a.pnorm[blockIdx.x] = red[0] * (1.f + 0x1p-12f);
+    if (zcur >= 0 && lane == 0) atomicMax(reinterpret_cast<int*>(a.pnorm) + zcur, __float_as_int(mx));
 }
 
 // ------------------------------------------------------------------------------------------
@@ -1208,7 +1232,10 @@ AddrPlan addr_plan(int dtype, int direct, int B, int H, int T, int dk, int S, in
     const int64_t base = 2LL * H * tiles * 2;   // sides x heads x token tiles x halves
     int ncc = 1;
     while ((S + ncc - 1) / ncc > 512) ncc *= 2;                      // chunks of <= 512 columns
-    while (base * ncc < 512 && (S / (2 * ncc)) >= 64) ncc *= 2;      // enough CTAs, chunks >= 64 columns
+    // FFMA path: more chunks when the token tiles alone give too few CTAs.  The tensor-core
+    // path keeps one chunk per half (512 TMEM columns), so the one-thread passes finish it.
+    if (!p.mma)
+        while (base * ncc < 512 && (S / (2 * ncc)) >= 64) ncc *= 2;  // enough CTAs, chunks >= 64 columns
     p.ncc = ncc;
     p.cw = (S + ncc - 1) / ncc;
     return p;
@@ -1275,11 +1302,20 @@ __global__ void __launch_bounds__(FT_THREADS) k_addr_finalize_thread(const AddrA
         float ss = 0.f;
         const char* xr = static_cast<const char*>(X) + xoff * D::BYTES;
         if ((reinterpret_cast<uintptr_t>(xr) & 15) == 0 && (a.dk * D::BYTES) % 16 == 0) {
-            for (int q = 0; q < a.dk * D::BYTES / 16; ++q) {
-                float f[D::E];
-                unpack16<D>(__ldg(reinterpret_cast<const uint4*>(xr) + q), f);
+            const int nq = a.dk * D::BYTES / 16;
+            for (int q0 = 0; q0 < nq; q0 += 4) {
+                uint4 xq[4];
 #pragma unroll
-                for (int e = 0; e < D::E; ++e) ss = fmaf(f[e], f[e], ss);
+                for (int u = 0; u < 4; ++u)
+                    if (q0 + u < nq) xq[u] = __ldg(reinterpret_cast<const uint4*>(xr) + q0 + u);
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    if (q0 + u < nq) {
+                        float f[D::E];
+                        unpack16<D>(xq[u], f);
+#pragma unroll
+                        for (int e = 0; e < D::E; ++e) ss = fmaf(f[e], f[e], ss);
+                    }
             }
         } else {
             for (int d = 0; d < a.dk; ++d) {
@@ -1464,9 +1500,28 @@ __global__ void __launch_bounds__(BT_THREADS) k_addr_band_thread(const AddrArgs 
     float e2 = 0.f;
     if (P != nullptr) {
         float ss = 0.f;
-        for (int d = 0; d < a.dk; ++d) {
-            const float xv = load_elem<D>(X, xoff + d);
-            ss = fmaf(xv, xv, ss);
+        const char* xr = static_cast<const char*>(X) + xoff * D::BYTES;
+        if ((reinterpret_cast<uintptr_t>(xr) & 15) == 0 && (a.dk * D::BYTES) % 16 == 0) {
+            const int nq = a.dk * D::BYTES / 16;
+            for (int q0 = 0; q0 < nq; q0 += 4) {
+                uint4 xq[4];
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    if (q0 + u < nq) xq[u] = __ldg(reinterpret_cast<const uint4*>(xr) + q0 + u);
+#pragma unroll
+                for (int u = 0; u < 4; ++u)
+                    if (q0 + u < nq) {
+                        float f[D::E];
+                        unpack16<D>(xq[u], f);
+#pragma unroll
+                        for (int e = 0; e < D::E; ++e) ss = fmaf(f[e], f[e], ss);
+                    }
+            }
+        } else {
+            for (int d = 0; d < a.dk; ++d) {
+                const float xv = load_elem<D>(X, xoff + d);
+                ss = fmaf(xv, xv, ss);
+            }
         }
         e2 = __fmul_ru(__fmul_ru(__fmul_ru(2.f * a.cbound, a.pnorm[side * a.H + h]), sqrtf(ss)), 1.f + 0x1p-12f);
     }
@@ -1477,7 +1532,15 @@ __global__ void __launch_bounds__(BT_THREADS) k_addr_band_thread(const AddrArgs 
         const int64_t base = part_at(static_cast<int>(z), 1, hf, BT, u, L, 0);
         float* Av = hf ? A2v : A1v;
         int* Ai = hf ? A2i : A1i;
-        for (int p = 0; p < L; ++p) { Av[p * W] = __ldg(a.part_v + base + p); Ai[p * W] = __ldg(a.part_i + base + p); }
+        const float4* pv = reinterpret_cast<const float4*>(a.part_v + base);   // L % 4 == 0, 16-byte aligned
+        const int4* pi = reinterpret_cast<const int4*>(a.part_i + base);
+#pragma unroll
+        for (int q4 = 0; q4 < L / 4; ++q4) {
+            const float4 v4 = __ldg(pv + q4);
+            const int4 i4 = __ldg(pi + q4);
+            Av[(4 * q4) * W] = v4.x; Av[(4 * q4 + 1) * W] = v4.y; Av[(4 * q4 + 2) * W] = v4.z; Av[(4 * q4 + 3) * W] = v4.w;
+            Ai[(4 * q4) * W] = i4.x; Ai[(4 * q4 + 1) * W] = i4.y; Ai[(4 * q4 + 2) * W] = i4.z; Ai[(4 * q4 + 3) * W] = i4.w;
+        }
         const float vk = Av[(k - 1) * W], vk1 = Av[k * W];
         if (!(S <= k || __fsub_rd(vk, vk1) > e2)) {
             // band of the half boundary
@@ -1708,7 +1771,10 @@ template <class D, int L>
 static cudaError_t launch_typed(const AddrPlan& plan, const AddrArgs& a, cudaStream_t stream) {
     const int64_t BT = static_cast<int64_t>(a.B) * a.T;
     if (a.P[0] != nullptr) {
-        k_pnorm<D><<<2 * a.H, 256, 0, stream>>>(a);
+        cudaError_t e = cudaMemsetAsync(a.pnorm, 0, static_cast<size_t>(2) * a.H * sizeof(float), stream);
+        if (e != cudaSuccess) return e;
+        const int64_t rows = static_cast<int64_t>(2) * a.H * 2 * a.S;
+        k_pnorm<D><<<static_cast<unsigned>((rows + 31) / 32), 256, 0, stream>>>(a);
     }
     if (plan.mma) {
         cudaError_t e = launch_address_mma(plan, a, stream);
