@@ -33,9 +33,18 @@ intermediates stay in float64.
 Tie-breaking (the paper is silent): per half by (score desc, index asc); over
 the outer sum by (score desc, slot asc).
 
+5. Lazy (copy-on-write) seeding of M0 (Sec. 3.1 "Learned Initial State"): the
+   memory of a sequence is an overlay of the rows written so far over the
+   read-only M0 of its head; a gather of a slot nobody has written returns the
+   M0 row.  The results equal those of the copied memory of item 2.
+6. Access diagnostics (App. "Memory Utilization and Access"): the normalised
+   effective number of keys exp(H(p)) / k, the cumulative mass curve C(m) of
+   the descending-sorted weights, and the fraction of unique slots accessed.
+
 Parity pins: see ``tests/test_oracle_pins.py`` (GDN reduction, dense masked
 form, beta = 0 closed form, single-slot recall, brute-force top-k including
-forced ties, invariants, the paper's state-size tables).
+forced ties, invariants, the paper's state-size tables, lazy overlay against
+the copied memory, diagnostics closed forms).
 """
 from __future__ import annotations
 
@@ -46,6 +55,7 @@ import numpy as np
 __all__ = [
     "to_f64", "round_storage", "half_scores", "topk_half", "pkm_select", "address",
     "recur", "forward_slice", "state_elements_per_layer", "n_global_layers",
+    "touched_mask", "recur_lazy", "materialize", "eff_keys_fraction", "cumulative_mass", "unique_fraction",
 ]
 
 
@@ -189,6 +199,66 @@ def forward_slice(M0_h: np.ndarray, P_q, P_k, q, k, v, alpha, beta, N: int, k_wr
         M = np.array(M0_h, dtype=np.float64, copy=True)
     y64, y = recur(M, idx_w, w_w, idx_r, w_r, v, alpha, beta, store)
     return {"y": y, "y64": y64, "M": M, "idx_w": idx_w, "w_w": w_w, "idx_r": idx_r, "w_r": w_r}
+
+
+# --------------------------------------------------------------------------------------
+# lazy (copy-on-write) initial state (Sec. 3.1 "Learned Initial State M0")
+# --------------------------------------------------------------------------------------
+
+def touched_mask(idx_w: np.ndarray, N: int, prior: np.ndarray | None = None) -> np.ndarray:
+    """Boolean [N]: slots written by any token of idx_w ([T, k_write]), or already marked in prior."""
+    m = np.zeros(N, dtype=bool) if prior is None else np.array(prior, dtype=bool, copy=True)
+    m[np.asarray(idx_w, dtype=np.int64).ravel()] = True
+    return m
+
+
+def recur_lazy(M0_h: np.ndarray, overlay: dict, idx_w, w_w, idx_r, w_r, v, alpha, beta, store: str):
+    """The recurrence of ``recur`` on a copy-on-write memory: ``overlay`` maps slot -> row
+    (float64) for the slots written so far and is updated in place; every other slot reads
+    M0_h (never modified).  Returns (y64, R(y)) like ``recur``."""
+    def row(s):
+        return overlay[s] if s in overlay else M0_h[s]
+    T = v.shape[0]
+    y = np.empty((T, M0_h.shape[1]), dtype=np.float64)
+    for t in range(T):
+        iw = [int(s) for s in idx_w[t]]
+        decayed = [alpha[t] * row(s) for s in iw]                       # Eq. sdm-decay
+        pred = sum(w_w[t][n] * decayed[n] for n in range(len(iw)))      # v~_t
+        delta = v[t] - pred
+        for n, s in enumerate(iw):                                      # Eq. sdm-write
+            overlay[s] = round_storage(decayed[n] + beta[t] * w_w[t][n] * delta, store)
+        y[t] = sum(w_r[t][n] * row(int(s)) for n, s in enumerate(idx_r[t]))   # Eq. sdm-read
+    return y, round_storage(y, store)
+
+
+def materialize(M0_h: np.ndarray, overlay: dict) -> np.ndarray:
+    """Dense memory of a copy-on-write state: M0_h with the overlay's rows in place."""
+    M = np.array(M0_h, dtype=np.float64, copy=True)
+    for s, r in overlay.items():
+        M[s] = r
+    return M
+
+
+# --------------------------------------------------------------------------------------
+# access diagnostics (App. "Memory Utilization and Access")
+# --------------------------------------------------------------------------------------
+
+def eff_keys_fraction(p: np.ndarray) -> np.ndarray:
+    """u(p) = exp(H(p)) / k per token, H(p) = -sum_i p_i log p_i (0 log 0 = 0); p: [..., k]."""
+    p = np.asarray(p, dtype=np.float64)
+    plogp = np.where(p > 0, p * np.log(np.where(p > 0, p, 1.0)), 0.0)
+    return np.exp(-plogp.sum(axis=-1)) / p.shape[-1]
+
+
+def cumulative_mass(p: np.ndarray) -> np.ndarray:
+    """C(m) = sum of the m largest weights, m = 1..k, per token; p: [..., k] -> [..., k]."""
+    p = np.asarray(p, dtype=np.float64)
+    return np.cumsum(-np.sort(-p, axis=-1), axis=-1)
+
+
+def unique_fraction(idx: np.ndarray, N: int) -> float:
+    """Fraction of the N slots that appear in idx (any shape)."""
+    return np.unique(np.asarray(idx, dtype=np.int64)).size / N
 
 
 # --------------------------------------------------------------------------------------

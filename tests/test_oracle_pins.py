@@ -255,6 +255,99 @@ def test_forward_slice_is_address_then_recur():
     assert np.array_equal(M0, O.forward_slice(M0, Pq, Pk, q, kk, v, a, b, N, k, k, "f64")["M"]) is False
 
 
+# ------------------------------------------------------------------ lazy M0 (copy-on-write)
+
+def test_lazy_overlay_equals_dense_masked_form():
+    """The copy-on-write memory (overlay of written rows over a read-only M0) gives the
+    dense update's y and final memory; its keys are exactly the slots ever written."""
+    rng = np.random.default_rng(21)
+    M0, idx_w, w_w, idx_r, w_r, V, alpha, beta = _random_sparse_case(rng, N=60, T=70)
+    M0_ro = M0.copy()
+    M0_ro.setflags(write=False)
+    overlay = {}
+    y64, _ = O.recur_lazy(M0_ro, overlay, idx_w, w_w, idx_r, w_r, V, alpha, beta, "f64")
+    M_ref, y_ref = _dense_masked_sdm(M0, idx_w, w_w, idx_r, w_r, V, alpha, beta)
+    np.testing.assert_allclose(y64, y_ref, rtol=1e-12, atol=1e-12)
+    np.testing.assert_allclose(O.materialize(M0_ro, overlay), M_ref, rtol=1e-12, atol=1e-12)
+    written = set(int(s) for s in idx_w.ravel())
+    assert set(overlay) == written
+    mask = O.touched_mask(idx_w, M0.shape[0])
+    assert np.array_equal(np.flatnonzero(mask), np.array(sorted(written)))
+    # slots never written keep M0 exactly
+    assert np.array_equal(O.materialize(M0_ro, overlay)[~mask], M0[~mask])
+
+
+def test_lazy_continuation_and_prior_mask():
+    """A sequence split over two calls carries the overlay (and the touched mask with it)."""
+    rng = np.random.default_rng(22)
+    M0, idx_w, w_w, idx_r, w_r, V, alpha, beta = _random_sparse_case(rng, N=50, T=64)
+    M0 = O.round_storage(M0 * 0.02, "bf16")
+    V = O.round_storage(V, "bf16")
+    ov_a = {}
+    _, ya = O.recur_lazy(M0, ov_a, idx_w, w_w, idx_r, w_r, V, alpha, beta, "bf16")
+    ov_b = {}
+    c = 29
+    _, yb1 = O.recur_lazy(M0, ov_b, idx_w[:c], w_w[:c], idx_r[:c], w_r[:c], V[:c], alpha[:c], beta[:c], "bf16")
+    m1 = O.touched_mask(idx_w[:c], 50)
+    _, yb2 = O.recur_lazy(M0, ov_b, idx_w[c:], w_w[c:], idx_r[c:], w_r[c:], V[c:], alpha[c:], beta[c:], "bf16")
+    assert np.array_equal(ya, np.concatenate([yb1, yb2]))
+    assert set(ov_a) == set(ov_b) and all(np.array_equal(ov_a[s], ov_b[s]) for s in ov_a)
+    assert np.array_equal(O.touched_mask(idx_w[c:], 50, prior=m1), O.touched_mask(idx_w, 50))
+    Md = M0.copy()
+    _, yd = O.recur(Md, idx_w, w_w, idx_r, w_r, V, alpha, beta, "bf16")
+    assert np.array_equal(yd, ya) and np.array_equal(O.materialize(M0, ov_a), Md)
+
+
+# ------------------------------------------------------------------ access diagnostics
+
+@pytest.mark.parametrize("k", [1, 4, 32, 64])
+def test_eff_keys_and_cumulative_mass_closed_forms(k):
+    uniform = np.full((3, k), 1.0 / k)
+    np.testing.assert_allclose(O.eff_keys_fraction(uniform), 1.0, rtol=1e-14)
+    np.testing.assert_allclose(O.cumulative_mass(uniform), np.tile(np.arange(1, k + 1) / k, (3, 1)), rtol=1e-14)
+    onehot = np.zeros((2, k))
+    onehot[0, k - 1] = 1.0
+    onehot[1, 0] = 1.0
+    np.testing.assert_allclose(O.eff_keys_fraction(onehot), 1.0 / k, rtol=1e-14)
+    np.testing.assert_allclose(O.cumulative_mass(onehot), 1.0, rtol=1e-14)
+    if k >= 2:
+        # mass split evenly over two keys: exp(H) = 2, C = [1/2, 1, 1, ...]
+        two = np.zeros(k)
+        two[[0, k - 1]] = 0.5
+        np.testing.assert_allclose(O.eff_keys_fraction(two), 2.0 / k, rtol=1e-14)
+        np.testing.assert_allclose(O.cumulative_mass(two), np.r_[0.5, np.ones(k - 1)], rtol=1e-14)
+        # geometric weights p_i = (1-r) r^i / (1 - r^k): H in closed form
+        r = 0.7
+        i = np.arange(k)
+        p = (1 - r) * r ** i / (1 - r ** k)
+        H = -np.sum(p * (np.log((1 - r) / (1 - r ** k)) + i * np.log(r)))
+        rng = np.random.default_rng(23)
+        pp = rng.permutation(p)
+        np.testing.assert_allclose(O.eff_keys_fraction(pp), np.exp(H) / k, rtol=1e-12)
+        np.testing.assert_allclose(O.cumulative_mass(pp), (1 - r ** (i + 1)) / (1 - r ** k), rtol=1e-12)
+
+
+def test_cumulative_mass_invariants_on_softmax_weights():
+    rng = np.random.default_rng(24)
+    z = rng.standard_normal((50, 16)) * 2
+    p = np.exp(z) / np.exp(z).sum(axis=1, keepdims=True)
+    C = O.cumulative_mass(p)
+    np.testing.assert_allclose(C[:, -1], 1.0, rtol=1e-13)
+    assert np.all(np.diff(C, axis=1) >= 0) and np.all(np.diff(C, n=2, axis=1) <= 1e-15)   # nondecreasing, concave
+    np.testing.assert_allclose(C[:, 0], p.max(axis=1), rtol=1e-15)
+    u = O.eff_keys_fraction(p)
+    assert np.all(u > 1.0 / 16 - 1e-15) and np.all(u <= 1.0 + 1e-15)
+
+
+def test_unique_fraction_counts():
+    N = 64
+    assert O.unique_fraction(np.arange(N).reshape(8, 8), N) == 1.0
+    assert O.unique_fraction(np.full((5, 3), 7), N) == 1.0 / N
+    rng = np.random.default_rng(25)
+    idx = rng.integers(0, N, (40, 4))
+    assert O.unique_fraction(idx, N) == len(set(idx.ravel().tolist())) / N
+
+
 # ------------------------------------------------------------------ geometry (printed numbers)
 
 def test_table1_sdm_state_sizes():
@@ -337,3 +430,21 @@ def test_pins_reject_planted_mistakes():
     s1, s2 = rng.standard_normal(8), rng.standard_normal(8)
     idx, _, _ = O.pkm_select(s2[None], s1[None], 4)
     assert not np.array_equal(idx[0], _brute_topk(s1, s2, 4))
+    # a copy-on-write memory whose reads ignore the overlay (always M0) fails the dense pin
+    M0c, iw, ww, ir, wr, Vc, al, be = _random_sparse_case(rng)
+    _, y_ref = _dense_masked_sdm(M0c, iw, ww, ir, wr, Vc, al, be)
+    ys = []
+    ov = {}
+    for t in range(Vc.shape[0]):
+        d = [al[t] * (ov[s] if s in ov else M0c[s]) for s in iw[t]]
+        pred = sum(ww[t][n] * d[n] for n in range(len(d)))
+        for n, s in enumerate(iw[t]):
+            ov[s] = d[n] + be[t] * ww[t][n] * (Vc[t] - pred)
+        ys.append(sum(wr[t][n] * M0c[s] for n, s in enumerate(ir[t])))
+    assert not np.allclose(np.array(ys), y_ref, atol=1e-6)
+    # effective keys without the exponential (entropy / k) fails the two-key closed form
+    two = np.array([0.5, 0.0, 0.0, 0.5])
+    assert not np.isclose(-np.sum(np.where(two > 0, two * np.log(np.where(two > 0, two, 1)), 0)) / 4, 2.0 / 4)
+    # cumulative mass of the weights in slot order (unsorted) fails the geometric closed form
+    p = np.array([0.1, 0.6, 0.3])
+    assert not np.allclose(np.cumsum(p), O.cumulative_mass(p))
