@@ -189,6 +189,10 @@ def run_reference(args, cfg):
 
 # ----------------------------------------------------------------------------- GPU arm
 
+def tokens_step_of(B: int, T: int, world: int) -> int:
+    return B * T * world
+
+
 def run_ours(args, cfg):
     import torch
     import paper_2607_07386_gb300 as sdm
@@ -284,6 +288,35 @@ def run_ours(args, cfg):
         ph["address"] += e[1].elapsed_time(e[2]) / args.steps
         ph["recurrence"] += e[2].elapsed_time(e[3]) / args.steps
 
+    # ---- the same step on the copy-on-write memory (sdm_forward_lazy, no broadcast): every
+    # step is a fresh sequence, so its touched bitmaps are cleared first
+    lazy = None
+    if T > 1:
+        ws_l = torch.empty(sdm.lazy_workspace_bytes(shape), dtype=torch.uint8, device="cuda")
+        touched = torch.empty((B, H, sdm.touched_words(shape)), dtype=torch.int32, device="cuda")
+
+        def lazy_step():
+            touched.zero_()
+            sdm.forward_lazy(shape, dev["M0"], touched, dev["P_q"], dev["P_k"], dev["q"], dev["k"], dev["v"],
+                             dev["alpha"], dev["beta"], mem, y, ws_l, stream=stream)
+
+        for _ in range(args.warmup):
+            lazy_step()
+        barrier()
+        ev0.record(stream)
+        for _ in range(args.steps):
+            lazy_step()
+        ev1.record(stream)
+        barrier()
+        ms_lazy = max_over_ranks(ev0.elapsed_time(ev1)) / args.steps
+        if sdm.device_status(stream) != 0:
+            raise RuntimeError("device status word set during the lazy-M0 benchmark")
+        lazy = {"value": tokens_step_of(B, T, world) / (ms_lazy * 1e-3), "unit": UNIT, "ms_per_step": ms_lazy,
+                "step": "bitmap clear + sdm_forward_lazy: addressing + first-writer table + recurrence gathering "
+                        "unwritten rows from M0 (no broadcast; same y and memory state as the broadcast step)",
+                "gpu_launches": 10 * args.steps}
+        del ws_l, touched
+
     # ---- end to end through the public API with host buffers (pinned), copies inside the region
     h2d = sum(t.numel() * t.element_size() for t in host_pinned.values())
     y_host = torch.empty(y.shape, dtype=dt, pin_memory=True)
@@ -366,6 +399,7 @@ def run_ours(args, cfg):
                      "traffic_source": "ncu dram bytes of the hazard pass + recurrence at B=2, scaled to B*H*T",
                      "peak_source": peaks["source"], "bytes_per_launch": rec_bytes, "ms_per_launch": rec_ms},
         "phase_ms": ph,
+        "lazy_m0": lazy,
         "step_hbm": {"algorithmic_bytes": step_bytes, "gbs": step_bytes / (ms_step * 1e-3) / 1e9,
                      "frac_of_measured": step_bytes / (ms_step * 1e-3) / 1e9 / peaks["hbm_gbs"],
                      "frac_of_8tbs": step_bytes / (ms_step * 1e-3) / 1e9 / 8000.0},

@@ -131,6 +131,35 @@ sdm_status sdm_forward_m0(const sdm_shape* shape, const void* M0, const void* P_
                           int32_t* idx_w, float* w_w, int32_t* idx_r, float* w_r,
                           void* workspace, size_t workspace_bytes, sdm_stream_t stream);
 
+/* Bytes of workspace sdm_forward_lazy needs for `shape`: sdm_workspace_bytes plus a
+ * first-writer table of B*H*N int32.  Returns 0 for an invalid shape. */
+size_t sdm_lazy_workspace_bytes(const sdm_shape* shape);
+
+/* sdm_forward on a copy-on-write memory seeded lazily from M0 (Sec. 3.1 "Learned initial
+ * state"), in place of the B-fold broadcast of sdm_forward_m0.
+ * touched: [B, H, ceil(N/32)] uint32 bitmaps, read and updated: bit (s % 32) of word
+ * s / 32 of chain (b, h) is set once slot s has been written.  A clear bit means the
+ * slot's value is M0[h, s] and mem[b, h, s] is neither read nor written; a set bit
+ * means mem[b, h, s] holds the slot.  Start a sequence with all bits clear (mem may hold
+ * anything); pass the same mem and touched to continue it.
+ * After the call, the memory described by (M0, touched, mem) equals the memory of
+ * sdm_forward_m0 (or of sdm_init_memory + sdm_forward calls), and y and the slot lists
+ * are the same, bit for bit; sdm_materialize turns it into the dense memory.
+ * M0: [H, N, d_v]; other arguments as in sdm_forward_m0; workspace: at least
+ * sdm_lazy_workspace_bytes(shape), 256-byte aligned.  touched must not overlap any
+ * other buffer; M0 must not overlap mem. */
+sdm_status sdm_forward_lazy(const sdm_shape* shape, const void* M0, uint32_t* touched,
+                            const void* P_q, const void* P_k, const void* q, const void* k,
+                            const void* v, const void* alpha, const void* beta, void* mem, void* y,
+                            int32_t* idx_w, float* w_w, int32_t* idx_r, float* w_r,
+                            void* workspace, size_t workspace_bytes, sdm_stream_t stream);
+
+/* Dense memory of a copy-on-write state: mem[b, h, s] = M0[h, s] for every slot whose
+ * bit in touched ([B, H, ceil(N/32)] uint32, as sdm_forward_lazy leaves it) is clear;
+ * other rows are left as they are.  M0: [H, N, d_v]; mem: [B, H, N, d_v]. */
+sdm_status sdm_materialize(const sdm_shape* shape, const void* M0, const uint32_t* touched, void* mem,
+                           sdm_stream_t stream);
+
 /* One decode step for B independent sequences: sdm_forward with shape->T == 1 and
  * the per-token tensors shaped [B, H, d] / [B, H]. */
 sdm_status sdm_decode_step(const sdm_shape* shape, const void* P_q, const void* P_k,

@@ -68,6 +68,12 @@ def lib():
             L.sdm_forward_m0.argtypes = [fwd[0], _VP] + fwd[1:]
             L.sdm_forward_m0.restype = ctypes.c_int
             L.sdm_decode_step.argtypes = fwd
+            L.sdm_forward_lazy.argtypes = [fwd[0], _VP, _VP] + fwd[1:]
+            L.sdm_forward_lazy.restype = ctypes.c_int
+            L.sdm_lazy_workspace_bytes.restype = ctypes.c_size_t
+            L.sdm_lazy_workspace_bytes.argtypes = [_SHP]
+            L.sdm_materialize.argtypes = [_SHP, _VP, _VP, _VP, _VP]
+            L.sdm_materialize.restype = ctypes.c_int
             L.sdm_address.argtypes = [_SHP, _VP, _VP, _VP, _VP, _I32P, _VP, _I32P, _VP, _VP, _SZ, _VP]
             L.sdm_recur.argtypes = [_SHP, _I32P, _VP, _I32P, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP]
             L.sdm_recur_workspace_bytes.restype = ctypes.c_size_t
@@ -155,6 +161,33 @@ def forward_m0(shape: SdmShape, M0, P_q, P_k, q, k, v, alpha, beta, mem, y, work
     _check(lib().sdm_forward_m0(ctypes.byref(shape), _ptr(M0), _ptr(P_q), _ptr(P_k), _ptr(q), _ptr(k), _ptr(v),
                                 _ptr(alpha), _ptr(beta), _ptr(mem), _ptr(y), _ptr(idx_w), _ptr(w_w), _ptr(idx_r),
                                 _ptr(w_r), _ptr(workspace), nb, _stream(stream)))
+
+
+def lazy_workspace_bytes(shape: SdmShape) -> int:
+    n = lib().sdm_lazy_workspace_bytes(ctypes.byref(shape))
+    if n == 0:
+        raise SdmError(1, last_error())
+    return n
+
+
+def touched_words(shape: SdmShape) -> int:
+    """uint32 words of one chain's touched bitmap (ceil(N / 32))."""
+    return (shape.N + 31) // 32
+
+
+def forward_lazy(shape: SdmShape, M0, touched, P_q, P_k, q, k, v, alpha, beta, mem, y, workspace, idx_w=None,
+                 w_w=None, idx_r=None, w_r=None, stream=None, workspace_nbytes=None):
+    """sdm_forward_lazy: the forward pass on a copy-on-write memory seeded from M0; touched is
+    the [B, H, ceil(N/32)] uint32 (int32 tensors work too) bitmap of written slots."""
+    nb = workspace_nbytes if workspace_nbytes is not None else (_nbytes(workspace) or 0)
+    _check(lib().sdm_forward_lazy(ctypes.byref(shape), _ptr(M0), _ptr(touched), _ptr(P_q), _ptr(P_k), _ptr(q), _ptr(k),
+                                  _ptr(v), _ptr(alpha), _ptr(beta), _ptr(mem), _ptr(y), _ptr(idx_w), _ptr(w_w),
+                                  _ptr(idx_r), _ptr(w_r), _ptr(workspace), nb, _stream(stream)))
+
+
+def materialize(shape: SdmShape, M0, touched, mem, stream=None):
+    """sdm_materialize: write M0's rows into the untouched slots of mem."""
+    _check(lib().sdm_materialize(ctypes.byref(shape), _ptr(M0), _ptr(touched), _ptr(mem), _stream(stream)))
 
 
 def decode_step(shape: SdmShape, P_q, P_k, q, k, v, alpha, beta, mem, y, workspace, idx_w=None, w_w=None,

@@ -11,7 +11,9 @@ namespace sdm {
 // ------------------------------------------------------------------------------------------
 // Hazard pass.  hz[(chain*T + t)*kmax + n] = write code (low 16 bits) | read code << 16;
 // code 0 = no hazard, else 1 + delta*64 + n' (writer t - delta, position n' of its list),
-// delta in [1, LA] for the write-gather and [0, LA] for the read-gather.
+// delta in [1, LA] for the write-gather and [0, LA] for the read-gather.  Codes stay below
+// 2^15; bit 15 of each half marks a fresh slot (lazy initial memory: no token wrote it
+// before t, so the gather reads M0's row), set only when firstw is given.
 // Slot lists must be ascending within each token (as the addressing produces them).
 // ------------------------------------------------------------------------------------------
 // One warp per token: lane n holds slot n (and n + 32) of the token's lists; the write list
@@ -35,7 +37,8 @@ __device__ __forceinline__ int warp_find(int lo_val, int hi_val, int k, int s) {
     return (pos < k && v == s) ? pos : -1;
 }
 
-__global__ void __launch_bounds__(256) k_hazard(const RecArgs a, int LA, int kmax, int32_t* hz) {
+__global__ void __launch_bounds__(256) k_hazard(const RecArgs a, int LA, int kmax, int32_t* hz,
+                                                const int32_t* __restrict__ firstw) {
     const int64_t BT = static_cast<int64_t>(a.B) * a.H * a.T;
     const int64_t tok = static_cast<int64_t>(blockIdx.x) * 8 + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
@@ -67,15 +70,23 @@ __global__ void __launch_bounds__(256) k_hazard(const RecArgs a, int LA, int kma
             if (cr[q] == 0 && sr[q] >= 0 && pr_pos >= 0) cr[q] = 1 + d * 64 + pr_pos;
         }
     }
+    if (firstw) {
+        const int32_t* fw = firstw + chain * a.N;
+        const uint32_t N = static_cast<uint32_t>(a.N);
+        for (int q = 0; q < nq; ++q) {
+            if (static_cast<uint32_t>(sw[q]) < N && __ldg(fw + sw[q]) >= t) cw[q] |= 0x8000;
+            if (static_cast<uint32_t>(sr[q]) < N && __ldg(fw + sr[q]) >= t) cr[q] |= 0x8000;
+        }
+    }
     for (int q = 0; q < nq; ++q) {
         const int n = lane + 32 * q;
         if (n < kmax) hz[tok * kmax + n] = cw[q] | (cr[q] << 16);
     }
 }
 
-cudaError_t launch_hazard(const RecArgs& a, int la, int kmax, int32_t* hz, cudaStream_t stream) {
+cudaError_t launch_hazard(const RecArgs& a, int la, int kmax, int32_t* hz, cudaStream_t stream, const int32_t* firstw) {
     const int64_t BT = static_cast<int64_t>(a.B) * a.H * a.T;
-    k_hazard<<<static_cast<unsigned>((BT + 7) / 8), 256, 0, stream>>>(a, la, kmax, hz);
+    k_hazard<<<static_cast<unsigned>((BT + 7) / 8), 256, 0, stream>>>(a, la, kmax, hz, firstw);
     return cudaGetLastError();
 }
 

@@ -7,7 +7,7 @@ namespace sdm {
 
 cudaError_t launch_recur_bf16(const RecPlan& p, const RecArgs& a, const int32_t* hz, int vec_lists, cudaStream_t s);
 cudaError_t launch_recur_f32(const RecPlan& p, const RecArgs& a, const int32_t* hz, int vec_lists, cudaStream_t s);
-cudaError_t launch_hazard(const RecArgs& a, int la, int kmax, int32_t* hz, cudaStream_t stream);
+cudaError_t launch_hazard(const RecArgs& a, int la, int kmax, int32_t* hz, cudaStream_t stream, const int32_t* firstw);
 
 RecPlan rec_plan(int dtype, int B, int H, int T, int dv, int kw, int kr) {
     RecPlan p{};
@@ -40,9 +40,9 @@ size_t rec_workspace_bytes(int B, int H, int T, int kw, int kr) {
     return static_cast<size_t>(B) * H * T * kmax * sizeof(int32_t);
 }
 
-cudaError_t launch_recur(int dtype, const RecArgs& a, int32_t* hz_ws, cudaStream_t stream) {
+cudaError_t launch_recur(int dtype, const RecArgs& a, int32_t* hz_ws, cudaStream_t stream, const int32_t* firstw) {
     const RecPlan p = rec_plan(dtype, a.B, a.H, a.T, a.dv, a.kw, a.kr);
-    cudaError_t e = launch_hazard(a, p.la, p.kmax, hz_ws, stream);
+    cudaError_t e = launch_hazard(a, p.la, p.kmax, hz_ws, stream, a.M0 ? firstw : nullptr);
     if (e != cudaSuccess) return e;
     auto al16 = [](const void* q) { return (reinterpret_cast<uintptr_t>(q) & 15) == 0; };
     const int vec_lists = (a.kw % 4 == 0) && (a.kr % 4 == 0) && (p.kmax % 4 == 0) && al16(a.idx_w) && al16(a.w_w) &&

@@ -105,6 +105,9 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
     const int64_t dbyte = static_cast<int64_t>(split * DCH) * 16;
     const char* Mc = static_cast<const char*>(a.mem) + chain * a.N * static_cast<int64_t>(rowbytes) + dbyte + c * 16;
     char* Mw = const_cast<char*>(Mc);
+    // fresh slots (lazy initial memory: bit 15 of a hazard code) gather M0's row of the head
+    const char* M0c = a.M0 ? static_cast<const char*>(a.M0) + (chain % a.H) * a.N * static_cast<int64_t>(rowbytes) + dbyte + c * 16
+                           : Mc;
     const char* vrange = static_cast<const char*>(a.v) + chain * a.T * static_cast<int64_t>(rowbytes) + dbyte;
     char* yb = static_cast<char*>(a.y) + chain * a.T * static_cast<int64_t>(rowbytes) + dbyte + c * 16;
     const int T = a.T;
@@ -166,15 +169,18 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
     auto copy_rows = [&](int t, uint32_t meta_addr, uint32_t rows_slot) {
         if (t >= T) return;
         const int* m = reinterpret_cast<const int*>(meta_gen + (meta_addr - meta0));
-        int iw[SPT], ir[SPT];
+        int iw[SPT], ir[SPT], hc[SPT];
         lds_vec<SPT>(m + g * SPT, iw);
         lds_vec<SPT>(m + 2 * KP + g * SPT, ir);
+        lds_vec<SPT>(m + 4 * KP + g * SPT, hc);
 #pragma unroll
         for (int j = 0; j < SPT; ++j) {
             const bool ow = my_w[j] && static_cast<uint32_t>(iw[j]) < N;
             const bool orr = my_r[j] && static_cast<uint32_t>(ir[j]) < N;
-            cp_async16z(rows_slot + j * SLOTB, Mc + static_cast<uint64_t>(ow ? iw[j] : 0) * rowbytes, ow ? 16 : 0);
-            cp_async16z(rows_slot + KS * SLOTB + j * SLOTB, Mc + static_cast<uint64_t>(orr ? ir[j] : 0) * rowbytes, orr ? 16 : 0);
+            const char* bw = (hc[j] & 0x8000) ? M0c : Mc;
+            const char* br = hc[j] < 0 ? M0c : Mc;             // bit 31: fresh read slot
+            cp_async16z(rows_slot + j * SLOTB, bw + static_cast<uint64_t>(ow ? iw[j] : 0) * rowbytes, ow ? 16 : 0);
+            cp_async16z(rows_slot + KS * SLOTB + j * SLOTB, br + static_cast<uint64_t>(orr ? ir[j] : 0) * rowbytes, orr ? 16 : 0);
         }
     };
 
@@ -232,8 +238,8 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
             const bool okr = my_r[j] && static_cast<uint32_t>(ir[j]) < N;
             bad |= (my_w[j] && !okw[j]) || (my_r[j] && !okr);
             // hazard codes of unused or invalid slots are garbage: never decode them
-            const int hw = okw[j] ? (hzv[j] & 0xffff) : 0;
-            const int hr = okr ? ((hzv[j] >> 16) & 0xffff) : 0;
+            const int hw = okw[j] ? (hzv[j] & 0x7fff) : 0;
+            const int hr = okr ? ((hzv[j] >> 16) & 0x7fff) : 0;
             const int dw = (hw - 1) >> 6, dr = (hr - 1) >> 6;
             int rw = ws - dw; rw += rw < 0 ? RING : 0;
             int rr = ws - dr; rr += rr < 0 ? RING : 0;
@@ -293,11 +299,11 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
             for (int e = 0; e < E; ++e) yc[e] = 0.f;
 #pragma unroll
             for (int j = 0; j < SPT; ++j) {
-                const int hr = (hzv[j] >> 16) & 0xffff;
+                const int hr = (hzv[j] >> 16) & 0x7fff;
                 const bool okr = my_r[j] && static_cast<uint32_t>(ir[j]) < N;
                 if (okr && hr && ((hr - 1) >> 6) == 0) {
                     const int np = (hr - 1) & 63;
-                    const int hwn = m[4 * KP + np] & 0xffff;        // the writer's own hazard code
+                    const int hwn = m[4 * KP + np] & 0x7fff;        // the writer's own hazard code
                     uint32_t ab = rslot + (KS + j) * SLOTB;       // same prefetch as the writer's
                     if (hwn) {
                         int rw = ws - ((hwn - 1) >> 6); rw += rw < 0 ? RING : 0;
@@ -467,6 +473,9 @@ __global__ void __launch_bounds__(64) k_recur_split(const RecArgs a, int nsplit,
     const int64_t dbyte = static_cast<int64_t>(split * DCH) * 16;
     const char* Mc = static_cast<const char*>(a.mem) + chain * a.N * static_cast<int64_t>(rowbytes) + dbyte + c * 16;
     char* Mw = const_cast<char*>(Mc);
+    // fresh slots (lazy initial memory: bit 15 of a hazard code) gather M0's row of the head
+    const char* M0c = a.M0 ? static_cast<const char*>(a.M0) + (chain % a.H) * a.N * static_cast<int64_t>(rowbytes) + dbyte + c * 16
+                           : Mc;
     const char* vrange = static_cast<const char*>(a.v) + chain * a.T * static_cast<int64_t>(rowbytes) + dbyte;
     char* yb = static_cast<char*>(a.y) + chain * a.T * static_cast<int64_t>(rowbytes) + dbyte + c * 16;
     const int T = a.T;
@@ -528,12 +537,15 @@ __global__ void __launch_bounds__(64) k_recur_split(const RecArgs a, int nsplit,
     auto copy_rows = [&](int t, uint32_t meta_addr, uint32_t rows_slot) {
         if (t >= T) return;
         const int* m = reinterpret_cast<const int*>(meta_gen + (meta_addr - meta0));
-        int ix[SPT];
+        int ix[SPT], hc[SPT];
         lds_vec<SPT>(m + list_off + g * SPT, ix);
+        lds_vec<SPT>(m + 4 * KP + g * SPT, hc);
+        const int fresh_bit = warp == 0 ? 0x8000 : static_cast<int>(0x80000000u);   // write / read half
 #pragma unroll
         for (int j = 0; j < SPT; ++j) {
             const bool ok = mine[j] && static_cast<uint32_t>(ix[j]) < N;
-            cp_async16z(rows_slot + j * SLOTB, Mc + static_cast<uint64_t>(ok ? ix[j] : 0) * rowbytes, ok ? 16 : 0);
+            const char* src = (hc[j] & fresh_bit) ? M0c : Mc;
+            cp_async16z(rows_slot + j * SLOTB, src + static_cast<uint64_t>(ok ? ix[j] : 0) * rowbytes, ok ? 16 : 0);
         }
     };
 
@@ -588,7 +600,7 @@ __global__ void __launch_bounds__(64) k_recur_split(const RecArgs a, int nsplit,
             for (int j = 0; j < SPT; ++j) {
                 okw[j] = mine[j] && static_cast<uint32_t>(iw[j]) < N;
                 bad |= mine[j] && !okw[j];
-                const int hw = okw[j] ? (hzv[j] & 0xffff) : 0;      // never decode unused slots
+                const int hw = okw[j] ? (hzv[j] & 0x7fff) : 0;      // never decode unused slots
                 int rw = ws - ((hw - 1) >> 6); rw += rw < 0 ? RING : 0;
                 const uint32_t aw = hw ? wring_c + (rw * KS + ((hw - 1) & 63)) * SLOTB : rslot + j * SLOTB;
                 float2 f[E2];
@@ -658,7 +670,7 @@ __global__ void __launch_bounds__(64) k_recur_split(const RecArgs a, int nsplit,
             for (int j = 0; j < SPT; ++j) {
                 const bool okr = mine[j] && static_cast<uint32_t>(ir[j]) < N;
                 bad |= mine[j] && !okr;
-                const int hr = okr ? ((hzv[j] >> 16) & 0xffff) : 0;
+                const int hr = okr ? ((hzv[j] >> 16) & 0x7fff) : 0;
                 int rr = ws - ((hr - 1) >> 6); rr += rr < 0 ? RING : 0;
                 const uint32_t ar = hr ? wring_c + (rr * KS + ((hr - 1) & 63)) * SLOTB : rslot + j * SLOTB;
                 float2 h[E2];

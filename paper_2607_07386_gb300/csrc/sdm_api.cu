@@ -148,11 +148,12 @@ sdm_status check_shape(const sdm_shape* s, bool need_pkm, int64_t* S_out) {
 }
 
 struct Layout {
-    size_t idx_w, w_w, idx_r, w_r, pnorm, part_v, part_i, queue, hz, total;
+    size_t idx_w, w_w, idx_r, w_r, pnorm, part_v, part_i, queue, hz, firstw, total;
     sdm::AddrPlan plan;
 };
 
-Layout layout_for(const sdm_shape* s, int64_t S) {
+// lazy: also the first-writer table of the copy-on-write initial memory ([B*H, N] int32).
+Layout layout_for(const sdm_shape* s, int64_t S, bool lazy = false) {
     Layout L{};
     const size_t bht = static_cast<size_t>(s->B) * s->H * s->T;
     const int kmax = s->k_write > s->k_read ? s->k_write : s->k_read;
@@ -168,6 +169,8 @@ Layout layout_for(const sdm_shape* s, int64_t S) {
     L.part_i = off; off = align256(off + part);
     L.queue = off;  off = align256(off + sdm::addr_queue_bytes(s->B, s->H, s->T));
     L.hz = off;     off = align256(off + sdm::rec_workspace_bytes(s->B, s->H, s->T, s->k_write, s->k_read));
+    L.firstw = off;
+    if (lazy) off = align256(off + static_cast<size_t>(s->B) * s->H * static_cast<size_t>(s->N) * 4);
     L.total = off;
     return L;
 }
@@ -213,10 +216,17 @@ sdm_status check_vec(const void* p, const char* name, size_t align) {
         if (_st != SDM_OK) return _st; \
     } while (0)
 
+// Copy-on-write initial memory (sdm_forward_lazy): M0 and the chains' touched bitmaps.
+struct LazyIn {
+    const void* M0;
+    uint32_t* touched;
+};
+
 sdm_status forward_impl(const char* who, const sdm_shape* s, const void* P_q, const void* P_k, const void* q,
                         const void* k, const void* v, const void* alpha, const void* beta, void* mem, void* y,
                         int32_t* idx_w, float* w_w, int32_t* idx_r, float* w_r, void* workspace,
-                        size_t workspace_bytes, cudaStream_t stream, bool run_recurrence, const void* M0 = nullptr) {
+                        size_t workspace_bytes, cudaStream_t stream, bool run_recurrence, const void* M0 = nullptr,
+                        const LazyIn* lazy = nullptr) {
     int64_t S = 0;
     SDM_TRY(check_shape(s, true, &S));
     const size_t es = elem_bytes(s->dtype);
@@ -240,7 +250,7 @@ sdm_status forward_impl(const char* who, const sdm_shape* s, const void* P_q, co
         SDM_TRY(check_vec(idx_r, "idx_r", 4));
         SDM_TRY(check_vec(w_r, "w_r", 4));
     }
-    const Layout L = layout_for(s, S);
+    const Layout L = layout_for(s, S, lazy != nullptr);
     if (!workspace) return fail(SDM_ERR_INVALID_ARG, "%s: workspace is NULL (need %zu bytes)", who, L.total);
     if (!aligned(workspace, 256)) return fail(SDM_ERR_INVALID_ARG, "%s: workspace must be 256-byte aligned", who);
     if (workspace_bytes < L.total)
@@ -265,6 +275,18 @@ sdm_status forward_impl(const char* who, const sdm_shape* s, const void* P_q, co
             SDM_TRY(check_vec(M0, "M0", 16));
             if (overlaps(rm, Range{M0, static_cast<size_t>(s->H) * static_cast<size_t>(s->N) * rowb, "M0"}))
                 return fail(SDM_ERR_INVALID_ARG, "%s: mem overlaps M0", who);
+        }
+        if (lazy != nullptr) {
+            SDM_TRY(check_vec(lazy->M0, "M0", 16));
+            SDM_TRY(check_vec(lazy->touched, "touched", 4));
+            const Range r0{lazy->M0, static_cast<size_t>(s->H) * static_cast<size_t>(s->N) * rowb, "M0"};
+            const Range rt{lazy->touched, static_cast<size_t>(s->B) * s->H * static_cast<size_t>((s->N + 31) / 32) * 4,
+                           "touched"};
+            if (overlaps(rm, r0)) return fail(SDM_ERR_INVALID_ARG, "%s: mem overlaps M0", who);
+            if (overlaps(rm, rt)) return fail(SDM_ERR_INVALID_ARG, "%s: mem overlaps touched", who);
+            for (const Range& r : others)
+                if (overlaps(rt, r)) return fail(SDM_ERR_INVALID_ARG, "%s: touched overlaps %s", who, r.name);
+            if (overlaps(rt, r0)) return fail(SDM_ERR_INVALID_ARG, "%s: touched overlaps M0", who);
         }
     }
     char* ws = static_cast<char*>(workspace);
@@ -304,7 +326,18 @@ sdm_status forward_impl(const char* who, const sdm_shape* s, const void* P_q, co
         r.B = s->B; r.H = s->H; r.T = s->T; r.dv = s->d_v; r.kw = s->k_write; r.kr = s->k_read;
         r.N = s->N;
         r.err = err;
-        cudaError_t e = sdm::launch_recur(s->dtype, r, reinterpret_cast<int32_t*>(ws + L.hz), stream);
+        int32_t* firstw = nullptr;
+        if (lazy != nullptr) {
+            // first writer of every slot in this call, then the chains' bitmaps for the next
+            // call; the recurrence gathers rows nobody has written from M0
+            firstw = reinterpret_cast<int32_t*>(ws + L.firstw);
+            const int64_t chains = static_cast<int64_t>(s->B) * s->H;
+            cudaError_t e = sdm::launch_lazy_prepare(lazy->touched, firstw, iw, chains, s->T, s->k_write, s->N, stream);
+            if (e == cudaSuccess) e = sdm::launch_lazy_bitmap(firstw, lazy->touched, chains, s->N, stream);
+            if (e != cudaSuccess) return cuda_fail(e, "lazy initial memory launch");
+            r.M0 = lazy->M0;
+        }
+        cudaError_t e = sdm::launch_recur(s->dtype, r, reinterpret_cast<int32_t*>(ws + L.hz), stream, firstw);
         if (e != cudaSuccess) return cuda_fail(e, "recurrence launch");
     }
     return ok();
@@ -360,6 +393,39 @@ sdm_status sdm_forward_m0(const sdm_shape* s, const void* M0, const void* P_q, c
         return fail(SDM_ERR_INVALID_ARG, "sdm_forward_m0: M0 is NULL");
     return forward_impl("sdm_forward_m0", s, P_q, P_k, q, k, v, alpha, beta, mem, y, idx_w, w_w, idx_r, w_r, workspace,
                         workspace_bytes, reinterpret_cast<cudaStream_t>(stream), true, M0);
+}
+
+size_t sdm_lazy_workspace_bytes(const sdm_shape* shape) {
+    int64_t S = 0;
+    if (check_shape(shape, true, &S) != SDM_OK) return 0;
+    return layout_for(shape, S, true).total;
+}
+
+sdm_status sdm_forward_lazy(const sdm_shape* s, const void* M0, uint32_t* touched, const void* P_q, const void* P_k,
+                            const void* q, const void* k, const void* v, const void* alpha, const void* beta, void* mem,
+                            void* y, int32_t* idx_w, float* w_w, int32_t* idx_r, float* w_r, void* workspace,
+                            size_t workspace_bytes, sdm_stream_t stream) {
+    const LazyIn lz{M0, touched};
+    return forward_impl("sdm_forward_lazy", s, P_q, P_k, q, k, v, alpha, beta, mem, y, idx_w, w_w, idx_r, w_r,
+                        workspace, workspace_bytes, reinterpret_cast<cudaStream_t>(stream), true, nullptr, &lz);
+}
+
+sdm_status sdm_materialize(const sdm_shape* s, const void* M0, const uint32_t* touched, void* mem, sdm_stream_t stream) {
+    SDM_TRY(check_shape(s, false, nullptr));
+    const size_t rowb = static_cast<size_t>(s->d_v) * elem_bytes(s->dtype);
+    const size_t per_seq = static_cast<size_t>(s->H) * static_cast<size_t>(s->N) * rowb;
+    if (per_seq == 0 || s->B == 0) return ok();
+    SDM_TRY(check_vec(M0, "M0", 16));
+    SDM_TRY(check_vec(touched, "touched", 4));
+    SDM_TRY(check_vec(mem, "mem", 16));
+    const Range rm{mem, per_seq * s->B, "mem"};
+    const Range rt{touched, static_cast<size_t>(s->B) * s->H * static_cast<size_t>((s->N + 31) / 32) * 4, "touched"};
+    if (overlaps(rm, Range{M0, per_seq, "M0"})) return fail(SDM_ERR_INVALID_ARG, "sdm_materialize: M0 overlaps mem");
+    if (overlaps(rm, rt)) return fail(SDM_ERR_INVALID_ARG, "sdm_materialize: touched overlaps mem");
+    cudaError_t e = sdm::launch_materialize(M0, touched, mem, static_cast<int64_t>(s->B) * s->H, s->H, s->N,
+                                            static_cast<int64_t>(rowb), reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "materialize launch");
+    return ok();
 }
 
 sdm_status sdm_decode_step(const sdm_shape* s, const void* P_q, const void* P_k, const void* q, const void* k,

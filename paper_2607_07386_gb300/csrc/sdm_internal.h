@@ -55,6 +55,8 @@ struct RecArgs {
     const void* v;                            // [B, H, T, dv]
     const void* alpha; const void* beta;      // [B, H, T]
     void* mem;                                // [B, H, N, dv]
+    const void* M0;                           // [H, N, dv]: source of fresh rows (lazy initial
+                                              // memory), or nullptr
     void* y;                                  // [B, H, T, dv]
     int B, H, T, dv, kw, kr;
     int64_t N;
@@ -75,7 +77,20 @@ RecPlan rec_plan(int dtype, int B, int H, int T, int dv, int kw, int kr);
 // Scratch of the recurrence: the hazard table [B, H, T, max(kw, kr)] int32.
 size_t rec_workspace_bytes(int B, int H, int T, int kw, int kr);
 // Runs the hazard pass, then the recurrence.  hz_ws: rec_workspace_bytes() of scratch.
-cudaError_t launch_recur(int dtype, const RecArgs& a, int32_t* hz_ws, cudaStream_t stream);
+// firstw (lazy initial memory, with a.M0 set): [B*H, N] first writer of each slot in this
+// call (-1: written by an earlier call; INT_MAX: not written), see k_lazy.cu.
+cudaError_t launch_recur(int dtype, const RecArgs& a, int32_t* hz_ws, cudaStream_t stream,
+                         const int32_t* firstw = nullptr);
+
+// ---------------------------------------------------------------- K-LAZY (k_lazy.cu)
+// firstw from the touched bitmap [chains, ceil(N/32)], then the first writer of every slot.
+cudaError_t launch_lazy_prepare(const uint32_t* touched, int32_t* firstw, const int32_t* idx_w, int64_t chains, int T,
+                                int kw, int64_t N, cudaStream_t stream);
+// touched bitmap from firstw (after launch_lazy_prepare).
+cudaError_t launch_lazy_bitmap(const int32_t* firstw, uint32_t* touched, int64_t chains, int64_t N, cudaStream_t stream);
+// mem rows of untouched slots = M0 rows (rowbytes a multiple of 16).
+cudaError_t launch_materialize(const void* M0, const uint32_t* touched, void* mem, int64_t chains, int H, int64_t N,
+                               int64_t rowbytes, cudaStream_t stream);
 
 // Error reporting and the checks of sdm_recur (minus its workspace), for entry points
 // in other translation units (sdm_api.cu).

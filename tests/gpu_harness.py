@@ -57,5 +57,34 @@ def run_forward(cfg: synth.SdmConfig, dev: dict, T0: int = 0, T1: int | None = N
     return out
 
 
+def run_forward_lazy(cfg: synth.SdmConfig, dev: dict, T0: int = 0, T1: int | None = None, mem=None, touched=None):
+    """sdm_forward_lazy over tokens [T0, T1); a fresh sequence (all touched bits clear, mem
+    filled with a value no slot holds) unless `mem` and `touched` continue one."""
+    import torch
+    import paper_2607_07386_gb300 as sdm
+    T1 = cfg.tokens_per_seq if T1 is None else T1
+    T = T1 - T0
+    shape = shape_of(cfg, T)
+    if mem is None:
+        mem = torch.full((cfg.B, cfg.H, cfg.N, cfg.d_v), 7.0, dtype=torch_dtype(cfg.dtype), device="cuda")
+        touched = torch.zeros((cfg.B, cfg.H, sdm.touched_words(shape)), dtype=torch.int32, device="cuda")
+    sl = lambda name: dev[name][:, :, T0:T1].contiguous()
+    out = alloc_outputs(cfg, T)
+    ws = torch.empty(sdm.lazy_workspace_bytes(shape), dtype=torch.uint8, device="cuda")
+    sdm.forward_lazy(shape, dev["M0"], touched, dev.get("P_q"), dev.get("P_k"), sl("q"), sl("k"), sl("v"),
+                     sl("alpha"), sl("beta"), mem, out["y"], ws, idx_w=out["idx_w"], w_w=out["w_w"],
+                     idx_r=out["idx_r"], w_r=out["w_r"])
+    out["mem"] = mem
+    out["touched"] = touched
+    return out
+
+
+def touched_bits(touched, N: int) -> np.ndarray:
+    """[B, H, ceil(N/32)] int32 bitmaps -> bool [B, H, N] (bit s % 32 of word s // 32)."""
+    w = touched.cpu().numpy().astype(np.int64) & 0xFFFFFFFF
+    bits = (w[..., :, None] >> np.arange(32)) & 1
+    return bits.reshape(w.shape[0], w.shape[1], -1)[..., :N].astype(bool)
+
+
 def host(t, dtype: str) -> np.ndarray:
     return from_torch(t, dtype)

@@ -106,6 +106,33 @@ def test_forward_rejects_null_misaligned_small_workspace_and_aliasing(sdm):
     assert sdm.lib().sdm_forward(None, *([None] * 14), 0, None) == 1
 
 
+def test_lazy_workspace_covers_first_writer_table(sdm):
+    s = sdm.SdmShape.make(8, 16, 4096, 128, 128, 262144, 32, 32, "bf16")
+    assert sdm.lazy_workspace_bytes(s) >= sdm.workspace_bytes(s) + 8 * 16 * 262144 * 4
+    assert sdm.touched_words(s) == 8192
+
+
+def test_forward_lazy_and_materialize_reject_bad_bitmaps(sdm):
+    s = _shape(sdm)
+    L = sdm.lib()
+    need = sdm.lazy_workspace_bytes(s)
+    mem = FAKE + 0x10000000
+
+    def lazy(touched, M0=FAKE + 0x800000):
+        return L.sdm_forward_lazy(ctypes.byref(s), M0, touched, FAKE, FAKE + 0x100000, FAKE + 0x200000,
+                                  FAKE + 0x300000, FAKE + 0x400000, FAKE + 0x500000, FAKE + 0x600000, mem,
+                                  FAKE + 0x700000, None, None, None, None, FAKE + 0x40000000, need, None)
+    assert lazy(None) == 1 and "touched is NULL" in sdm.last_error()
+    assert lazy(FAKE + 0x900002) == 1 and "touched is not 4-byte aligned" in sdm.last_error()
+    assert lazy(mem + 4096) == 1 and "mem overlaps touched" in sdm.last_error()
+    assert lazy(FAKE + 0x700000) == 1 and "touched overlaps y" in sdm.last_error()
+    assert lazy(FAKE + 0x900000, M0=None) == 1 and "M0 is NULL" in sdm.last_error()
+    assert L.sdm_forward_lazy(ctypes.byref(s), FAKE + 0x800000, FAKE + 0x900000, *([FAKE] * 9), None, None, None,
+                              None, FAKE + 0x40000000, 16, None) == 1 and "too small" in sdm.last_error()
+    assert L.sdm_materialize(ctypes.byref(s), FAKE, mem + 64, mem, None) == 1 and "overlaps" in sdm.last_error()
+    assert L.sdm_materialize(ctypes.byref(s), None, FAKE, mem, None) == 1 and "M0 is NULL" in sdm.last_error()
+
+
 def test_decode_step_requires_T_equal_1(sdm):
     s = _shape(sdm, T=2)
     L = sdm.lib()

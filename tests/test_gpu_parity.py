@@ -411,6 +411,52 @@ def test_forward_m0_equals_init_then_forward(sdm, name):
     assert torch.equal(out["y"], ref["y"]) and torch.equal(mem, ref["mem"])
 
 
+# ------------------------------------------------------------------ lazy (copy-on-write) M0
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("name", ["tiny_fp32", "small_bf16"])
+def test_forward_lazy_equals_broadcast_and_touched_set_is_the_oracle_write_set(sdm, name):
+    """sdm_forward_lazy never reads or writes mem rows of slots nobody wrote, gives y and the
+    slot lists of init + forward bit for bit, and after sdm_materialize the same memory;
+    its touched bitmap is the set of slots the oracle's own selection writes."""
+    cfg = synth.CONFIGS[name]
+    dev = G.device_inputs(cfg)
+    ref = G.run_forward(cfg, dev)
+    out = G.run_forward_lazy(cfg, dev)
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    for key in ("idx_w", "w_w", "idx_r", "w_r", "y"):
+        assert torch.equal(out[key], ref[key]), key
+    bits = G.touched_bits(out["touched"], cfg.N)
+    mask = torch.from_numpy(bits).to("cuda")
+    assert torch.all(out["mem"][~mask] == 7.0)                 # untouched rows: never written
+    assert torch.equal(out["mem"][mask], ref["mem"][mask])
+    sdm.materialize(G.shape_of(cfg), dev["M0"], out["touched"], out["mem"])
+    torch.cuda.synchronize()
+    assert torch.equal(out["mem"], ref["mem"])
+    slices = [(0, 0), (cfg.B - 1, cfg.H - 1)]
+    for (b, h), r in oracle_slices(cfg, slices, workers=1).items():
+        assert np.array_equal(np.flatnonzero(bits[b, h]), r["touched"]), (b, h)
+
+
+@pytest.mark.gpu
+def test_forward_lazy_continues_a_sequence_across_calls(sdm):
+    """Two lazy calls over tokens [0, T1) and [T1, T) with the same mem and touched give what
+    one call over [0, T) gives (bitmaps included)."""
+    cfg = synth.SMALL_BF16
+    dev = G.device_inputs(cfg)
+    one = G.run_forward_lazy(cfg, dev)
+    T1 = 777
+    a = G.run_forward_lazy(cfg, dev, 0, T1)
+    b = G.run_forward_lazy(cfg, dev, T1, cfg.T, mem=a["mem"], touched=a["touched"])
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    assert torch.equal(torch.cat([a["y"], b["y"]], dim=2), one["y"])
+    assert torch.equal(b["touched"], one["touched"])
+    mask = torch.from_numpy(G.touched_bits(one["touched"], cfg.N)).to("cuda")
+    assert torch.equal(b["mem"][mask], one["mem"][mask])
+
+
 # ------------------------------------------------------------------ full-size workloads
 
 @pytest.mark.fullsize
