@@ -160,6 +160,24 @@ sdm_status sdm_forward_lazy(const sdm_shape* shape, const void* M0, uint32_t* to
 sdm_status sdm_materialize(const sdm_shape* shape, const void* M0, const uint32_t* touched, void* mem,
                            sdm_stream_t stream);
 
+/* Bytes of workspace sdm_access_stats needs (two slot bitmaps per chain); 0 if invalid. */
+size_t sdm_access_stats_workspace_bytes(const sdm_shape* shape);
+
+/* Access diagnostics of a selection (App. "Memory Utilization and Access"), as float64
+ * sums over all B*H*T tokens, written to the device array out (4 + k_write + k_read):
+ *   out[0], out[1]: sum of u(p) = exp(H(p)) / k, H(p) = -sum p_i log p_i, over the write
+ *                   weights w_w and over the read weights w_r (normalised effective keys);
+ *   out[2], out[3]: distinct slots written (idx_w) and read (idx_r), summed over chains;
+ *   out[4 + m - 1]            (m = 1..k_write): sum of C(m) of the write weights,
+ *   out[4 + k_write + m - 1]  (m = 1..k_read):  sum of C(m) of the read weights,
+ *                   C(m) = the sum of the m largest weights of the token.
+ * Divide by B*H*T (or by N * B*H for the slot counts) for means and fractions.  Inputs as
+ * sdm_address produces them ([B, H, T, k] each, k <= 64); indices outside [0, N) are not
+ * counted.  workspace: >= sdm_access_stats_workspace_bytes(shape), 256-byte aligned. */
+sdm_status sdm_access_stats(const sdm_shape* shape, const int32_t* idx_w, const float* w_w,
+                            const int32_t* idx_r, const float* w_r, double* out,
+                            void* workspace, size_t workspace_bytes, sdm_stream_t stream);
+
 /* One decode step for B independent sequences: sdm_forward with shape->T == 1 and
  * the per-token tensors shaped [B, H, d] / [B, H]. */
 sdm_status sdm_decode_step(const sdm_shape* shape, const void* P_q, const void* P_k,

@@ -74,6 +74,10 @@ def lib():
             L.sdm_lazy_workspace_bytes.argtypes = [_SHP]
             L.sdm_materialize.argtypes = [_SHP, _VP, _VP, _VP, _VP]
             L.sdm_materialize.restype = ctypes.c_int
+            L.sdm_access_stats_workspace_bytes.restype = ctypes.c_size_t
+            L.sdm_access_stats_workspace_bytes.argtypes = [_SHP]
+            L.sdm_access_stats.argtypes = [_SHP, _I32P, _VP, _I32P, _VP, _VP, _VP, _SZ, _VP]
+            L.sdm_access_stats.restype = ctypes.c_int
             L.sdm_address.argtypes = [_SHP, _VP, _VP, _VP, _VP, _I32P, _VP, _I32P, _VP, _VP, _SZ, _VP]
             L.sdm_recur.argtypes = [_SHP, _I32P, _VP, _I32P, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP]
             L.sdm_recur_workspace_bytes.restype = ctypes.c_size_t
@@ -188,6 +192,21 @@ def forward_lazy(shape: SdmShape, M0, touched, P_q, P_k, q, k, v, alpha, beta, m
 def materialize(shape: SdmShape, M0, touched, mem, stream=None):
     """sdm_materialize: write M0's rows into the untouched slots of mem."""
     _check(lib().sdm_materialize(ctypes.byref(shape), _ptr(M0), _ptr(touched), _ptr(mem), _stream(stream)))
+
+
+def access_stats_workspace_bytes(shape: SdmShape) -> int:
+    n = lib().sdm_access_stats_workspace_bytes(ctypes.byref(shape))
+    if n == 0:
+        raise SdmError(1, last_error())
+    return n
+
+
+def access_stats(shape: SdmShape, idx_w, w_w, idx_r, w_r, out, workspace, stream=None, workspace_nbytes=None):
+    """sdm_access_stats: float64 sums of the access diagnostics into the device tensor out
+    (4 + k_write + k_read entries)."""
+    nb = workspace_nbytes if workspace_nbytes is not None else (_nbytes(workspace) or 0)
+    _check(lib().sdm_access_stats(ctypes.byref(shape), _ptr(idx_w), _ptr(w_w), _ptr(idx_r), _ptr(w_r), _ptr(out),
+                                  _ptr(workspace), nb, _stream(stream)))
 
 
 def decode_step(shape: SdmShape, P_q, P_k, q, k, v, alpha, beta, mem, y, workspace, idx_w=None, w_w=None,

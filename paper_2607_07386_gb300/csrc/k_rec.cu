@@ -32,6 +32,12 @@ RecPlan rec_plan(int dtype, int B, int H, int T, int dv, int kw, int kr) {
     // than it saves (1024 units: 4.33 -> 5.69 ms; 256 units, T = 65536: 51.8 -> 55.2 ms)
     p.split = p.la > 1 && kmax <= 16 && chains * p.nsplit < 768;
     p.smem = rec_smem_bytes(p.la, (32 / dch) * p.spt, dch);
+    // four consecutive d-ranges of a chain per CTA: an SM then serves the rows of fewer chains,
+    // whose gathers hit fewer memory pages (layer_1p4b: 9.83 -> 9.67 ms per broadcast step,
+    // 9.41 -> 8.71 ms per lazy step, where the gathers span both mem and M0; 8 per CTA: 9.94
+    // and 8.98 ms)
+    // (only with enough warps to fill the SMs: long_ctx's 256 warps run 1% slower in 64 CTAs)
+    p.wpc = p.la > 1 && p.nsplit % 4 == 0 && chains * p.nsplit >= 512 ? 4 : 1;
     return p;
 }
 

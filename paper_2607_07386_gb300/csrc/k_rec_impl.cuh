@@ -76,9 +76,16 @@ __device__ __forceinline__ void cp_async16z(uint32_t dst, const void* src, int s
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
 }
 
+// Shared memory of one warp of k_recur, rounded so that consecutive warps' regions stay aligned.
+__host__ __device__ inline size_t rec_warp_smem_bytes(int la, int ks, int dch) {
+    return (rec_smem_bytes(la, ks, dch) + 127) / 128 * 128;
+}
+
+// One warp per (chain, d-range); a CTA holds blockDim.x / 32 consecutive warps (the d-ranges
+// of one chain when it holds nsplit of them), each with its own shared-memory region.
 template <class D, int DCH, int SPT, int LA>
-__global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const int32_t* __restrict__ hz, int kmax,
-                                              int vec_lists) {
+__global__ void __launch_bounds__(256) k_recur(const RecArgs a, int nsplit, const int32_t* __restrict__ hz, int kmax,
+                                               int vec_lists) {
     constexpr int E = D::E;
     constexpr int E2 = E / 2;
     constexpr int G = 32 / DCH;
@@ -87,20 +94,24 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
     constexpr int MR = 2 * LA + 1;
     constexpr int RING = LA + 1;
     constexpr uint32_t SLOTB = DCH * 16;                 // bytes of one slot's d-range in a ring
-    extern __shared__ __align__(16) unsigned char smR[];
-    const uint32_t sm0 = static_cast<uint32_t>(__cvta_generic_to_shared(smR));
+    extern __shared__ __align__(128) unsigned char smR[];
+    const int lane = threadIdx.x & 31;
+    const int wib = threadIdx.x >> 5;                                        // warp in the CTA
+    const int64_t gw = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + wib;
+    if (gw >= static_cast<int64_t>(a.B) * a.H * nsplit) return;              // whole warps
+    const uint32_t smbase = static_cast<uint32_t>(__cvta_generic_to_shared(smR));
+    const uint32_t sm0 = smbase + wib * static_cast<uint32_t>(rec_warp_smem_bytes(LA, KS, DCH));
     const uint32_t rows0 = sm0;                                              // [LA][2][KS][DCH] x 16 B
     const uint32_t wring0 = rows0 + LA * 2 * KS * SLOTB;                     // [RING][KS][DCH] x 16 B
     const uint32_t meta0 = wring0 + RING * KS * SLOTB;                       // [MR][stride]
-    unsigned char* meta_gen = smR + (meta0 - sm0);
+    unsigned char* meta_gen = smR + (meta0 - smbase);
     const int meta_stride = static_cast<int>(rec_meta_stride(KS, DCH));
 
-    const int lane = threadIdx.x;
     const int c = lane % DCH;
     const int g = lane / DCH;
     const int kw = a.kw, kr = a.kr;
-    const int64_t chain = blockIdx.x / nsplit;
-    const int split = blockIdx.x - static_cast<int>(chain) * nsplit;
+    const int64_t chain = gw / nsplit;
+    const int split = static_cast<int>(gw - chain * nsplit);
     const uint32_t rowbytes = static_cast<uint32_t>(a.dv) * D::BYTES;
     const int64_t dbyte = static_cast<int64_t>(split * DCH) * 16;
     const char* Mc = static_cast<const char*>(a.mem) + chain * a.N * static_cast<int64_t>(rowbytes) + dbyte + c * 16;
@@ -108,6 +119,7 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
     // fresh slots (lazy initial memory: bit 15 of a hazard code) gather M0's row of the head
     const char* M0c = a.M0 ? static_cast<const char*>(a.M0) + (chain % a.H) * a.N * static_cast<int64_t>(rowbytes) + dbyte + c * 16
                            : Mc;
+    const bool lazy = a.M0 != nullptr;
     const char* vrange = static_cast<const char*>(a.v) + chain * a.T * static_cast<int64_t>(rowbytes) + dbyte;
     char* yb = static_cast<char*>(a.y) + chain * a.T * static_cast<int64_t>(rowbytes) + dbyte + c * 16;
     const int T = a.T;
@@ -172,9 +184,10 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
         int iw[SPT], ir[SPT], hc[SPT];
         lds_vec<SPT>(m + g * SPT, iw);
         lds_vec<SPT>(m + 2 * KP + g * SPT, ir);
-        lds_vec<SPT>(m + 4 * KP + g * SPT, hc);
+        if (lazy) lds_vec<SPT>(m + 4 * KP + g * SPT, hc);
 #pragma unroll
         for (int j = 0; j < SPT; ++j) {
+            if (!lazy) hc[j] = 0;
             const bool ow = my_w[j] && static_cast<uint32_t>(iw[j]) < N;
             const bool orr = my_r[j] && static_cast<uint32_t>(ir[j]) < N;
             const char* bw = (hc[j] & 0x8000) ? M0c : Mc;
@@ -347,14 +360,16 @@ __global__ void __launch_bounds__(32) k_recur(const RecArgs a, int nsplit, const
 
 template <class D, int DCH, int SPT, int LA>
 cudaError_t launch_rec_kernel(const RecPlan& p, const RecArgs& a, const int32_t* hz, int vec_lists, cudaStream_t s) {
-    const size_t smem = rec_smem_bytes(LA, (32 / DCH) * SPT, DCH);
+    const int wpc = p.wpc > 0 ? p.wpc : 1;
+    const size_t smem = wpc * rec_warp_smem_bytes(LA, (32 / DCH) * SPT, DCH);
     if (smem > 48 * 1024) {
         cudaError_t e = cudaFuncSetAttribute(k_recur<D, DCH, SPT, LA>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              static_cast<int>(smem));
         if (e != cudaSuccess) return e;
     }
-    const int64_t chains = static_cast<int64_t>(a.B) * a.H;
-    k_recur<D, DCH, SPT, LA><<<static_cast<unsigned>(chains * p.nsplit), 32, smem, s>>>(a, p.nsplit, hz, p.kmax, vec_lists);
+    const int64_t warps = static_cast<int64_t>(a.B) * a.H * p.nsplit;
+    k_recur<D, DCH, SPT, LA><<<static_cast<unsigned>((warps + wpc - 1) / wpc), 32 * wpc, smem, s>>>(a, p.nsplit, hz,
+                                                                                                 p.kmax, vec_lists);
     return cudaGetLastError();
 }
 
@@ -476,6 +491,7 @@ __global__ void __launch_bounds__(64) k_recur_split(const RecArgs a, int nsplit,
     // fresh slots (lazy initial memory: bit 15 of a hazard code) gather M0's row of the head
     const char* M0c = a.M0 ? static_cast<const char*>(a.M0) + (chain % a.H) * a.N * static_cast<int64_t>(rowbytes) + dbyte + c * 16
                            : Mc;
+    const bool lazy = a.M0 != nullptr;
     const char* vrange = static_cast<const char*>(a.v) + chain * a.T * static_cast<int64_t>(rowbytes) + dbyte;
     char* yb = static_cast<char*>(a.y) + chain * a.T * static_cast<int64_t>(rowbytes) + dbyte + c * 16;
     const int T = a.T;
@@ -539,7 +555,10 @@ __global__ void __launch_bounds__(64) k_recur_split(const RecArgs a, int nsplit,
         const int* m = reinterpret_cast<const int*>(meta_gen + (meta_addr - meta0));
         int ix[SPT], hc[SPT];
         lds_vec<SPT>(m + list_off + g * SPT, ix);
-        lds_vec<SPT>(m + 4 * KP + g * SPT, hc);
+        if (lazy) lds_vec<SPT>(m + 4 * KP + g * SPT, hc);
+#pragma unroll
+        for (int j = 0; j < SPT; ++j)
+            if (!lazy) hc[j] = 0;
         const int fresh_bit = warp == 0 ? 0x8000 : static_cast<int>(0x80000000u);   // write / read half
 #pragma unroll
         for (int j = 0; j < SPT; ++j) {

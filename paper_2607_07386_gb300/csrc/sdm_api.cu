@@ -428,6 +428,41 @@ sdm_status sdm_materialize(const sdm_shape* s, const void* M0, const uint32_t* t
     return ok();
 }
 
+size_t sdm_access_stats_workspace_bytes(const sdm_shape* s) {
+    if (check_shape(s, false, nullptr) != SDM_OK) return 0;
+    return align256(static_cast<size_t>(2) * s->B * s->H * static_cast<size_t>((s->N + 31) / 32) * 4) + 256;
+}
+
+sdm_status sdm_access_stats(const sdm_shape* s, const int32_t* idx_w, const float* w_w, const int32_t* idx_r,
+                            const float* w_r, double* out, void* workspace, size_t workspace_bytes,
+                            sdm_stream_t stream) {
+    SDM_TRY(check_shape(s, false, nullptr));
+    SDM_TRY(check_vec(out, "out", 8));
+    const size_t bht = static_cast<size_t>(s->B) * s->H * s->T;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (bht == 0) {
+        cudaError_t e = cudaMemsetAsync(out, 0, static_cast<size_t>(4 + s->k_write + s->k_read) * sizeof(double), st);
+        if (e != cudaSuccess) return cuda_fail(e, "sdm_access_stats");
+        return ok();
+    }
+    SDM_TRY(check_vec(idx_w, "idx_w", 4));
+    SDM_TRY(check_vec(w_w, "w_w", 4));
+    SDM_TRY(check_vec(idx_r, "idx_r", 4));
+    SDM_TRY(check_vec(w_r, "w_r", 4));
+    const size_t need = align256(static_cast<size_t>(2) * s->B * s->H * static_cast<size_t>((s->N + 31) / 32) * 4);
+    if (!workspace) return fail(SDM_ERR_INVALID_ARG, "sdm_access_stats: workspace is NULL (need %zu bytes)", need);
+    if (!aligned(workspace, 256)) return fail(SDM_ERR_INVALID_ARG, "sdm_access_stats: workspace must be 256-byte aligned");
+    if (workspace_bytes < need)
+        return fail(SDM_ERR_INVALID_ARG, "sdm_access_stats: workspace too small (%zu < %zu bytes)", workspace_bytes, need);
+    const Range ro{out, static_cast<size_t>(4 + s->k_write + s->k_read) * sizeof(double), "out"};
+    if (overlaps(ro, Range{workspace, need, "workspace"}))
+        return fail(SDM_ERR_INVALID_ARG, "sdm_access_stats: out overlaps workspace");
+    cudaError_t e = sdm::launch_access_stats(idx_w, w_w, idx_r, w_r, static_cast<int64_t>(s->B) * s->H, s->T,
+                                             s->k_write, s->k_read, s->N, static_cast<uint32_t*>(workspace), out, st);
+    if (e != cudaSuccess) return cuda_fail(e, "access stats launch");
+    return ok();
+}
+
 sdm_status sdm_decode_step(const sdm_shape* s, const void* P_q, const void* P_k, const void* q, const void* k,
                            const void* v, const void* alpha, const void* beta, void* mem, void* y, int32_t* idx_w,
                            float* w_w, int32_t* idx_r, float* w_r, void* workspace, size_t workspace_bytes,

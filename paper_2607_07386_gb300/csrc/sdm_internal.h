@@ -71,6 +71,7 @@ struct RecPlan {
     int la;       // lookahead depth (tokens whose gathers are in flight)
     int kmax;     // max(k_write, k_read)
     int split;    // writer and reader warps per (chain, d-range) (look-ahead > 1 only)
+    int wpc;      // warps per CTA of the fused kernel (consecutive d-ranges of a chain)
     size_t smem;  // dynamic shared memory per CTA
 };
 RecPlan rec_plan(int dtype, int B, int H, int T, int dv, int kw, int kr);
@@ -88,6 +89,11 @@ cudaError_t launch_lazy_prepare(const uint32_t* touched, int32_t* firstw, const 
                                 int kw, int64_t N, cudaStream_t stream);
 // touched bitmap from firstw (after launch_lazy_prepare).
 cudaError_t launch_lazy_bitmap(const int32_t* firstw, uint32_t* touched, int64_t chains, int64_t N, cudaStream_t stream);
+// Access diagnostics (k_stats.cu): bits = 2 * chains * ceil(N/32) words of scratch; out =
+// 4 + kw + kr float64 sums (see sdm_access_stats).
+cudaError_t launch_access_stats(const int32_t* idx_w, const float* w_w, const int32_t* idx_r, const float* w_r,
+                                int64_t chains, int T, int kw, int kr, int64_t N, uint32_t* bits, double* out,
+                                cudaStream_t stream);
 // mem rows of untouched slots = M0 rows (rowbytes a multiple of 16).
 cudaError_t launch_materialize(const void* M0, const uint32_t* touched, void* mem, int64_t chains, int H, int64_t N,
                                int64_t rowbytes, cudaStream_t stream);

@@ -133,6 +133,22 @@ def test_forward_lazy_and_materialize_reject_bad_bitmaps(sdm):
     assert L.sdm_materialize(ctypes.byref(s), None, FAKE, mem, None) == 1 and "M0 is NULL" in sdm.last_error()
 
 
+def test_access_stats_rejects_bad_arguments(sdm):
+    s = _shape(sdm)
+    L = sdm.lib()
+    need = sdm.access_stats_workspace_bytes(s)
+    assert need >= 2 * 2 * 2 * (1024 // 32) * 4
+    args = [FAKE, FAKE + 0x100000, FAKE + 0x200000, FAKE + 0x300000]
+    assert L.sdm_access_stats(ctypes.byref(s), *args, None, FAKE + 0x400000, need, None) == 1
+    assert "out is NULL" in sdm.last_error()
+    assert L.sdm_access_stats(ctypes.byref(s), *args, FAKE + 0x500004, FAKE + 0x400000, need, None) == 1
+    assert "8-byte aligned" in sdm.last_error()
+    assert L.sdm_access_stats(ctypes.byref(s), *args, FAKE + 0x500000, FAKE + 0x400000, 16, None) == 1
+    assert "too small" in sdm.last_error()
+    assert L.sdm_access_stats(ctypes.byref(s), *args, FAKE + 0x400000, FAKE + 0x400000, need, None) == 1
+    assert "out overlaps workspace" in sdm.last_error()
+
+
 def test_decode_step_requires_T_equal_1(sdm):
     s = _shape(sdm, T=2)
     L = sdm.lib()

@@ -457,6 +457,46 @@ def test_forward_lazy_continues_a_sequence_across_calls(sdm):
     assert torch.equal(b["mem"][mask], one["mem"][mask])
 
 
+# ------------------------------------------------------------------ access diagnostics
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("name", ["tiny_fp32", "small_bf16"])
+def test_access_stats_match_the_oracle_diagnostics(sdm, name):
+    """sdm_access_stats on the library's own selection equals the oracle's diagnostics of the
+    oracle's selection: unique slot counts exactly (the index sets are identical), the sums of
+    u(p) and C(m) to float32 rounding of the weights."""
+    from oracle.reference_run import slice_f64
+    cfg = synth.CONFIGS[name]
+    dev = G.device_inputs(cfg)
+    shape = G.shape_of(cfg)
+    out = G.alloc_outputs(cfg, cfg.T)
+    sdm.address(shape, dev.get("P_q"), dev.get("P_k"), dev["q"], dev["k"], out["idx_w"], out["w_w"], out["idx_r"],
+                out["w_r"], G.workspace(shape))
+    stats = torch.empty(4 + cfg.k_write + cfg.k_read, dtype=torch.float64, device="cuda")
+    ws = torch.empty(sdm.access_stats_workspace_bytes(shape), dtype=torch.uint8, device="cuda")
+    sdm.access_stats(shape, out["idx_w"], out["w_w"], out["idx_r"], out["w_r"], stats, ws)
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    got = stats.cpu().numpy()
+    exp = np.zeros_like(got)
+    for b in range(cfg.B):
+        for h in range(cfg.H):
+            x = slice_f64(cfg, b, h)
+            iw, _, ww = O.address(x["P_k"], x["k"], cfg.N, cfg.k_write)
+            ir, _, wr = O.address(x["P_q"], x["q"], cfg.N, cfg.k_read)
+            exp[0] += O.eff_keys_fraction(ww).sum()
+            exp[1] += O.eff_keys_fraction(wr).sum()
+            exp[2] += O.unique_fraction(iw, cfg.N) * cfg.N
+            exp[3] += O.unique_fraction(ir, cfg.N) * cfg.N
+            exp[4:4 + cfg.k_write] += O.cumulative_mass(ww).sum(axis=0)
+            exp[4 + cfg.k_write:] += O.cumulative_mass(wr).sum(axis=0)
+    assert got[2] == exp[2] and got[3] == exp[3]
+    np.testing.assert_allclose(got[[0, 1]], exp[[0, 1]], rtol=2e-5)
+    np.testing.assert_allclose(got[4:], exp[4:], rtol=2e-5)
+    tokens = cfg.B * cfg.H * cfg.T
+    np.testing.assert_allclose(got[4 + cfg.k_write - 1], tokens, rtol=1e-5)    # C(k) = 1 per token
+
+
 # ------------------------------------------------------------------ full-size workloads
 
 @pytest.mark.fullsize
