@@ -37,7 +37,11 @@ the outer sum by (score desc, slot asc).
    memory of a sequence is an overlay of the rows written so far over the
    read-only M0 of its head; a gather of a slot nobody has written returns the
    M0 row.  The results equal those of the copied memory of item 2.
-6. Access diagnostics (App. "Memory Utilization and Access"): the normalised
+6. Gate preparation and output epilogue around the path (Sec. 3.1, item 2 and
+   "Norm, Gating, and Head Mixing"): alpha_t = exp(-A softplus(W_a x_t + b_dt)),
+   beta_t = sigmoid(W_b x_t) per head; z = g (.) RMSNorm(y) per head, the heads
+   concatenated per token and mixed by W_o.
+7. Access diagnostics (App. "Memory Utilization and Access"): the normalised
    effective number of keys exp(H(p)) / k, the cumulative mass curve C(m) of
    the descending-sorted weights, and the fraction of unique slots accessed.
 
@@ -56,6 +60,7 @@ __all__ = [
     "to_f64", "round_storage", "half_scores", "topk_half", "pkm_select", "address",
     "recur", "forward_slice", "state_elements_per_layer", "n_global_layers",
     "touched_mask", "recur_lazy", "materialize", "eff_keys_fraction", "cumulative_mass", "unique_fraction",
+    "softplus", "gates", "norm_gate", "head_mix",
 ]
 
 
@@ -259,6 +264,45 @@ def cumulative_mass(p: np.ndarray) -> np.ndarray:
 def unique_fraction(idx: np.ndarray, N: int) -> float:
     """Fraction of the N slots that appear in idx (any shape)."""
     return np.unique(np.asarray(idx, dtype=np.int64)).size / N
+
+
+# --------------------------------------------------------------------------------------
+# gate preparation and output epilogue (Sec. 3.1)
+# --------------------------------------------------------------------------------------
+
+def softplus(z: np.ndarray) -> np.ndarray:
+    """softplus(z) = log(1 + e^z), evaluated as logaddexp(0, z) (no overflow)."""
+    return np.logaddexp(0.0, np.asarray(z, dtype=np.float64))
+
+
+def gates(x: np.ndarray, W_a: np.ndarray, b_dt: np.ndarray, A: np.ndarray, W_b: np.ndarray):
+    """Per-head forget and input gates of every token (Sec. 3.1, after Eq. sdm-write):
+    alpha_t = exp(-A softplus(W_a x_t + b_dt)), beta_t = sigmoid(W_b x_t).
+
+    x: [T, d]; W_a, W_b: [H, d]; b_dt, A: [H].  Returns (alpha, beta), each [H, T] float64.
+    """
+    x = np.asarray(x, dtype=np.float64)
+    za = x @ np.asarray(W_a, dtype=np.float64).T + np.asarray(b_dt, dtype=np.float64)[None, :]
+    zb = x @ np.asarray(W_b, dtype=np.float64).T
+    alpha = np.exp(-np.asarray(A, dtype=np.float64)[None, :] * softplus(za))
+    beta = 1.0 / (1.0 + np.exp(-zb))
+    return alpha.T, beta.T
+
+
+def norm_gate(y: np.ndarray, g: np.ndarray, gamma: np.ndarray, eps: float) -> np.ndarray:
+    """g (.) RMSNorm(y) for one head (Sec. 3.1 "Norm, Gating, and Head Mixing"):
+    y, g: [T, d_v]; gamma: [d_v] RMSNorm scale; returns g * gamma * y / sqrt(mean(y^2) + eps)."""
+    y = np.asarray(y, dtype=np.float64)
+    rms = np.sqrt(np.mean(y * y, axis=-1, keepdims=True) + eps)
+    return np.asarray(g, dtype=np.float64) * np.asarray(gamma, dtype=np.float64)[None, :] * y / rms
+
+
+def head_mix(z: np.ndarray, W_o: np.ndarray) -> np.ndarray:
+    """Output projection mixing the heads: z [H, T, d_v] -> o [T, d] = concat_h(z_h) W_o^T,
+    W_o: [d, H * d_v] (head h owns columns h*d_v .. (h+1)*d_v - 1)."""
+    H, T, dv = z.shape
+    zt = np.transpose(np.asarray(z, dtype=np.float64), (1, 0, 2)).reshape(T, H * dv)
+    return zt @ np.asarray(W_o, dtype=np.float64).T
 
 
 # --------------------------------------------------------------------------------------

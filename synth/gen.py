@@ -6,6 +6,9 @@ to the storage dtype, so any (b, h) slice or head can be regenerated alone:
 
 * per head h:        M0 [N, d_v], P_q / P_k [2 sqrt(N), d_k]
 * per slice (b, h):  q, k [T_seq, d_k], v [T_seq, d_v], alpha, beta [T_seq]
+* layer side (the gate preparation and output epilogue around the path), with
+  d_model = H * d_v:  x [B, T, d_model]; W_a, W_b [H, d_model]; b_dt, A [H]; g
+  [B, H, T, d_v]; gamma [d_v]
 
 For the decode workload T_seq = prefill + timed steps and step s uses token s
 of every slice.  Storage format: ``np.float32`` for "f32"; ``np.uint16``
@@ -29,6 +32,13 @@ class TensorId(enum.IntEnum):
     V = 6
     ALPHA = 7
     BETA = 8
+    X = 9
+    W_A = 10
+    W_B = 11
+    B_DT = 12
+    A_LOG = 13
+    G = 14
+    GAMMA = 15
 
 
 def _rng(seed: int, tid: TensorId, *coords: int) -> np.random.Generator:
@@ -118,3 +128,30 @@ def full_inputs(cfg: SdmConfig, b0: int = 0) -> dict:
 def decode_step_inputs(full: dict, s: int) -> dict:
     """Inputs of decode step s for every (b, h) (token s of each sequence), from ``full_inputs``."""
     return {name: np.ascontiguousarray(full[name][:, :, s]) for name in ("q", "k", "v", "alpha", "beta")}
+
+
+def layer_inputs(cfg: SdmConfig) -> dict:
+    """Inputs of the steps around the path for the whole workload, with d_model = H * d_v:
+
+    * x [B, T, d_model] ~ N(0, 1), the layer input;
+    * W_a, W_b [H, d_model] ~ N(0, 1 / d_model), the gate projections;
+    * A [H] ~ U(0, 16) and b_dt [H] = inv_softplus(U(0.001, 0.1)), the initialisation the
+      paper states (Sec. 4, "SDM Configuration");
+    * g [B, H, T, d_v] = sigmoid(N(0, 1)), the output gate;
+    * gamma [d_v] ~ 1 + 0.1 N(0, 1), the RMSNorm scale.
+
+    x, W_a, W_b and g are rounded to the storage dtype; A, b_dt and gamma stay float32.
+    """
+    d = cfg.H * cfg.d_v
+    T = cfg.tokens_per_seq
+    r = lambda a: round_f64_to_storage(a, cfg.dtype)
+    x = _rng(cfg.seed, TensorId.X).standard_normal((cfg.B, T, d))
+    wa = _rng(cfg.seed, TensorId.W_A).standard_normal((cfg.H, d)) / np.sqrt(d)
+    wb = _rng(cfg.seed, TensorId.W_B).standard_normal((cfg.H, d)) / np.sqrt(d)
+    A = _rng(cfg.seed, TensorId.A_LOG).uniform(0.0, 16.0, cfg.H)
+    u = _rng(cfg.seed, TensorId.B_DT).uniform(0.001, 0.1, cfg.H)
+    b_dt = np.log(np.expm1(u))                      # inv_softplus(u)
+    g = _sigmoid(_rng(cfg.seed, TensorId.G).standard_normal((cfg.B, cfg.H, T, cfg.d_v)))
+    gamma = 1.0 + 0.1 * _rng(cfg.seed, TensorId.GAMMA).standard_normal(cfg.d_v)
+    return {"x": r(x), "W_a": r(wa), "W_b": r(wb), "A": A.astype(np.float32), "b_dt": b_dt.astype(np.float32),
+            "g": r(g), "gamma": gamma.astype(np.float32)}

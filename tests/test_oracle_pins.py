@@ -348,6 +348,67 @@ def test_unique_fraction_counts():
     assert O.unique_fraction(idx, N) == len(set(idx.ravel().tolist())) / N
 
 
+# ------------------------------------------------------------------ gates and output epilogue
+
+def test_softplus_known_values_and_asymptotes():
+    np.testing.assert_allclose(O.softplus(np.array([0.0])), [math.log(2.0)], rtol=1e-15)
+    z = np.array([-800.0, -30.0, 30.0, 800.0])
+    np.testing.assert_allclose(O.softplus(z), [0.0, math.exp(-30.0), 30.0 + math.exp(-30.0), 800.0], rtol=1e-12)
+    zz = np.linspace(-5, 5, 41)
+    np.testing.assert_allclose(O.softplus(zz) - O.softplus(-zz), zz, atol=1e-14)   # softplus(z) - softplus(-z) = z
+
+
+def test_gates_closed_forms():
+    """W = 0: alpha = exp(-A c) when b_dt = inv_softplus(c), beta = 1/2; A = 0: alpha = 1;
+    beta(-z) = 1 - beta(z); the paper's initialisation keeps softplus(b_dt) in [0.001, 0.1]."""
+    rng = np.random.default_rng(31)
+    T, d, H = 7, 12, 5
+    x = rng.standard_normal((T, d))
+    c = rng.uniform(0.001, 0.1, H)
+    b_dt = np.log(np.expm1(c))
+    A = rng.uniform(0, 16, H)
+    alpha, beta = O.gates(x, np.zeros((H, d)), b_dt, A, np.zeros((H, d)))
+    np.testing.assert_allclose(alpha, np.tile(np.exp(-A * c)[:, None], (1, T)), rtol=1e-13)
+    np.testing.assert_allclose(beta, 0.5, rtol=1e-15)
+    W = rng.standard_normal((H, d))
+    a1, b1 = O.gates(x, W, b_dt, np.zeros(H), W)
+    a2, b2 = O.gates(-x, W, b_dt, np.zeros(H), W)
+    np.testing.assert_allclose(a1, 1.0, rtol=1e-15)
+    np.testing.assert_allclose(b1 + b2, 1.0, rtol=1e-14)
+    # one explicit token and head, summed by hand
+    za = sum(W[2, i] * x[3, i] for i in range(d)) + b_dt[2]
+    al, _ = O.gates(x, W, b_dt, A, W)
+    np.testing.assert_allclose(al[2, 3], math.exp(-A[2] * math.log1p(math.exp(za))), rtol=1e-13)
+
+
+def test_norm_gate_closed_forms_and_invariance():
+    rng = np.random.default_rng(32)
+    T, dv = 6, 16
+    g = rng.uniform(0, 1, (T, dv))
+    gamma = 1 + 0.1 * rng.standard_normal(dv)
+    c = rng.uniform(0.5, 3, T) * rng.choice([-1, 1], T)
+    y = np.tile(c[:, None], (1, dv))                     # constant rows: RMSNorm(y) = sign(c)
+    np.testing.assert_allclose(O.norm_gate(y, g, gamma, 0.0), g * gamma[None, :] * np.sign(c)[:, None], rtol=1e-14)
+    y = rng.standard_normal((T, dv))
+    s = rng.uniform(0.1, 10, T)[:, None]
+    np.testing.assert_allclose(O.norm_gate(s * y, g, gamma, 0.0), O.norm_gate(y, g, gamma, 0.0), rtol=1e-13)
+    z = O.norm_gate(y, np.ones((T, dv)), np.ones(dv), 0.0)
+    np.testing.assert_allclose(np.mean(z * z, axis=1), 1.0, rtol=1e-13)   # unit mean square
+    # eps: rows of zeros stay zero, and eps > 0 shrinks the norm
+    assert np.all(O.norm_gate(np.zeros((2, dv)), g[:2], gamma, 1e-6) == 0)
+    assert np.all(np.abs(O.norm_gate(y, g, gamma, 1e-2)) < np.abs(O.norm_gate(y, g, gamma, 0.0)))
+
+
+def test_head_mix_is_a_sum_over_heads():
+    rng = np.random.default_rng(33)
+    H, T, dv, d = 3, 4, 5, 7
+    z = rng.standard_normal((H, T, dv))
+    W = rng.standard_normal((d, H * dv))
+    o = O.head_mix(z, W)
+    ref = sum(z[h] @ W[:, h * dv:(h + 1) * dv].T for h in range(H))
+    np.testing.assert_allclose(o, ref, rtol=1e-13, atol=1e-13)
+
+
 # ------------------------------------------------------------------ geometry (printed numbers)
 
 def test_table1_sdm_state_sizes():
@@ -448,3 +509,12 @@ def test_pins_reject_planted_mistakes():
     # cumulative mass of the weights in slot order (unsorted) fails the geometric closed form
     p = np.array([0.1, 0.6, 0.3])
     assert not np.allclose(np.cumsum(p), O.cumulative_mass(p))
+    # RMSNorm without the square root (y / mean(y^2)) fails the scale invariance
+    y = rng.standard_normal((3, 8))
+    bad = lambda yy: yy / np.mean(yy * yy, axis=-1, keepdims=True)
+    assert not np.allclose(bad(4.0 * y), bad(y))
+    # softplus replaced by max(z, 0) fails softplus(0) = log 2
+    assert not np.isclose(max(0.0, 0.0), math.log(2.0))
+    # a gate without the bias fails the W = 0 closed form
+    c = np.array([0.05])
+    assert not np.isclose(np.exp(-3.0 * O.softplus(0.0)), np.exp(-3.0 * c[0]))
