@@ -160,6 +160,26 @@ sdm_status sdm_forward_lazy(const sdm_shape* shape, const void* M0, uint32_t* to
 sdm_status sdm_materialize(const sdm_shape* shape, const void* M0, const uint32_t* touched, void* mem,
                            sdm_stream_t stream);
 
+/* Gates of every token and head from the layer input (Sec. 3.1, after Eq. sdm-write):
+ *   alpha[b, h, t] = exp(-A[h] * softplus(W_a[h] . x[b, t] + b_dt[h])),
+ *   beta[b, h, t]  = sigmoid(W_b[h] . x[b, t]).
+ * x: [B, T, d_model], W_a, W_b: [H, d_model] (storage dtype, 16-byte aligned;
+ * d_model * element size a multiple of 16 bytes); b_dt, A: [H] float32; alpha, beta:
+ * [B, H, T] storage dtype (the layout sdm_forward takes).  H <= 32.  Uses shape B, H, T
+ * and dtype only.  fp32 arithmetic; outputs rounded to nearest. */
+sdm_status sdm_gates(const sdm_shape* shape, int32_t d_model, const void* x, const void* W_a,
+                     const void* W_b, const float* b_dt, const float* A, void* alpha, void* beta,
+                     sdm_stream_t stream);
+
+/* Output gate of every head (Sec. 3.1, "Norm, Gating, and Head Mixing"):
+ *   z[b, t, h, :] = g[b, h, t, :] * gamma * y[b, h, t, :] / sqrt(mean(y[b, h, t, :]^2) + eps).
+ * y, g: [B, H, T, d_v] storage dtype; gamma: [d_v] float32 RMSNorm scale; eps >= 0;
+ * z: [B, T, H, d_v] storage dtype, i.e. [B*T, H*d_v] row-major, the operand of the
+ * head-mixing projection o = z W_o^T (a plain GEMM the caller runs).  d_v * element size
+ * <= 1024 bytes.  16-byte aligned buffers; z must not overlap y, g or gamma. */
+sdm_status sdm_norm_gate(const sdm_shape* shape, const void* y, const void* g, const float* gamma,
+                         float eps, void* z, sdm_stream_t stream);
+
 /* Bytes of workspace sdm_access_stats needs (two slot bitmaps per chain); 0 if invalid. */
 size_t sdm_access_stats_workspace_bytes(const sdm_shape* shape);
 

@@ -9,5 +9,5 @@ from ._binding import (  # noqa: F401
     ADDR_DIRECT, ADDR_PROJECTED, DTYPE_BF16, DTYPE_F32, SdmError, SdmShape, abi_version, address,
     decode_step, device_stats, device_status, forward, forward_m0, init_memory, last_error, lib, lib_path, recur, recur_noalloc,
     recur_workspace_bytes, workspace_bytes, RECUR_NOALLOC_SCRATCH_BYTES, forward_lazy, lazy_workspace_bytes,
-    materialize, touched_words, access_stats, access_stats_workspace_bytes,
+    materialize, touched_words, access_stats, access_stats_workspace_bytes, gates, norm_gate,
 )

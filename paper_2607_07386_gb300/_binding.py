@@ -74,6 +74,10 @@ def lib():
             L.sdm_lazy_workspace_bytes.argtypes = [_SHP]
             L.sdm_materialize.argtypes = [_SHP, _VP, _VP, _VP, _VP]
             L.sdm_materialize.restype = ctypes.c_int
+            L.sdm_gates.argtypes = [_SHP, ctypes.c_int32, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP]
+            L.sdm_gates.restype = ctypes.c_int
+            L.sdm_norm_gate.argtypes = [_SHP, _VP, _VP, _VP, ctypes.c_float, _VP, _VP]
+            L.sdm_norm_gate.restype = ctypes.c_int
             L.sdm_access_stats_workspace_bytes.restype = ctypes.c_size_t
             L.sdm_access_stats_workspace_bytes.argtypes = [_SHP]
             L.sdm_access_stats.argtypes = [_SHP, _I32P, _VP, _I32P, _VP, _VP, _VP, _SZ, _VP]
@@ -192,6 +196,17 @@ def forward_lazy(shape: SdmShape, M0, touched, P_q, P_k, q, k, v, alpha, beta, m
 def materialize(shape: SdmShape, M0, touched, mem, stream=None):
     """sdm_materialize: write M0's rows into the untouched slots of mem."""
     _check(lib().sdm_materialize(ctypes.byref(shape), _ptr(M0), _ptr(touched), _ptr(mem), _stream(stream)))
+
+
+def gates(shape: SdmShape, d_model: int, x, W_a, W_b, b_dt, A, alpha, beta, stream=None):
+    """sdm_gates: alpha, beta [B, H, T] from the layer input x [B, T, d_model]."""
+    _check(lib().sdm_gates(ctypes.byref(shape), int(d_model), _ptr(x), _ptr(W_a), _ptr(W_b), _ptr(b_dt), _ptr(A),
+                           _ptr(alpha), _ptr(beta), _stream(stream)))
+
+
+def norm_gate(shape: SdmShape, y, g, gamma, eps: float, z, stream=None):
+    """sdm_norm_gate: z [B, T, H, d_v] = g * gamma * RMSNorm(y) per head."""
+    _check(lib().sdm_norm_gate(ctypes.byref(shape), _ptr(y), _ptr(g), _ptr(gamma), float(eps), _ptr(z), _stream(stream)))
 
 
 def access_stats_workspace_bytes(shape: SdmShape) -> int:

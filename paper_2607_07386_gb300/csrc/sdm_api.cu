@@ -428,6 +428,61 @@ sdm_status sdm_materialize(const sdm_shape* s, const void* M0, const uint32_t* t
     return ok();
 }
 
+sdm_status sdm_gates(const sdm_shape* s, int32_t d_model, const void* x, const void* W_a, const void* W_b,
+                     const float* b_dt, const float* A, void* alpha, void* beta, sdm_stream_t stream) {
+    SDM_TRY(check_shape(s, false, nullptr));
+    const size_t es = elem_bytes(s->dtype);
+    if (s->H > 32) return fail(SDM_ERR_UNSUPPORTED, "sdm_gates: H > 32 is not supported (H=%d)", s->H);
+    if (d_model < 1 || (static_cast<size_t>(d_model) * es) % 16 != 0)
+        return fail(SDM_ERR_UNSUPPORTED, "sdm_gates: d_model * element size must be a positive multiple of 16 bytes (d_model=%d)",
+                    d_model);
+    const size_t bt = static_cast<size_t>(s->B) * s->T;
+    if (bt == 0 || s->H == 0) return ok();
+    SDM_TRY(check_vec(x, "x", 16));
+    SDM_TRY(check_vec(W_a, "W_a", 16));
+    SDM_TRY(check_vec(W_b, "W_b", 16));
+    SDM_TRY(check_vec(b_dt, "b_dt", 4));
+    SDM_TRY(check_vec(A, "A", 4));
+    SDM_TRY(check_vec(alpha, "alpha", es));
+    SDM_TRY(check_vec(beta, "beta", es));
+    const size_t gbytes = bt * s->H * es;
+    const Range ra{alpha, gbytes, "alpha"}, rb{beta, gbytes, "beta"};
+    const Range ins[] = {{x, bt * d_model * es, "x"}, {W_a, static_cast<size_t>(s->H) * d_model * es, "W_a"},
+                         {W_b, static_cast<size_t>(s->H) * d_model * es, "W_b"}, {b_dt, s->H * 4u, "b_dt"},
+                         {A, s->H * 4u, "A"}};
+    for (const Range& r : ins)
+        if (overlaps(ra, r) || overlaps(rb, r)) return fail(SDM_ERR_INVALID_ARG, "sdm_gates: a gate output overlaps %s", r.name);
+    if (overlaps(ra, rb)) return fail(SDM_ERR_INVALID_ARG, "sdm_gates: alpha overlaps beta");
+    cudaError_t e = sdm::launch_gates(s->dtype, x, W_a, W_b, b_dt, A, alpha, beta, s->B, s->T, s->H, d_model,
+                                      reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "gates launch");
+    return ok();
+}
+
+sdm_status sdm_norm_gate(const sdm_shape* s, const void* y, const void* g, const float* gamma, float eps, void* z,
+                         sdm_stream_t stream) {
+    SDM_TRY(check_shape(s, false, nullptr));
+    const size_t es = elem_bytes(s->dtype);
+    if (static_cast<size_t>(s->d_v) * es > 1024)
+        return fail(SDM_ERR_UNSUPPORTED, "sdm_norm_gate: d_v * element size must be <= 1024 bytes (d_v=%d)", s->d_v);
+    if (!(eps >= 0.f)) return fail(SDM_ERR_INVALID_ARG, "sdm_norm_gate: eps must be >= 0");
+    const size_t rows = static_cast<size_t>(s->B) * s->H * s->T;
+    if (rows == 0) return ok();
+    SDM_TRY(check_vec(y, "y", 16));
+    SDM_TRY(check_vec(g, "g", 16));
+    SDM_TRY(check_vec(gamma, "gamma", 4));
+    SDM_TRY(check_vec(z, "z", 16));
+    const size_t bytes = rows * s->d_v * es;
+    const Range rz{z, bytes, "z"};
+    const Range ins[] = {{y, bytes, "y"}, {g, bytes, "g"}, {gamma, s->d_v * 4u, "gamma"}};
+    for (const Range& r : ins)
+        if (overlaps(rz, r)) return fail(SDM_ERR_INVALID_ARG, "sdm_norm_gate: z overlaps %s", r.name);
+    cudaError_t e = sdm::launch_norm_gate(s->dtype, y, g, gamma, eps, z, s->B, s->H, s->T, s->d_v,
+                                          reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "norm_gate launch");
+    return ok();
+}
+
 size_t sdm_access_stats_workspace_bytes(const sdm_shape* s) {
     if (check_shape(s, false, nullptr) != SDM_OK) return 0;
     return align256(static_cast<size_t>(2) * s->B * s->H * static_cast<size_t>((s->N + 31) / 32) * 4) + 256;

@@ -89,6 +89,11 @@ cudaError_t launch_lazy_prepare(const uint32_t* touched, int32_t* firstw, const 
                                 int kw, int64_t N, cudaStream_t stream);
 // touched bitmap from firstw (after launch_lazy_prepare).
 cudaError_t launch_lazy_bitmap(const int32_t* firstw, uint32_t* touched, int64_t chains, int64_t N, cudaStream_t stream);
+// Gate preparation and output epilogue (k_gates.cu).  dtype 0 = fp32, 1 = bf16 storage.
+cudaError_t launch_gates(int dtype, const void* x, const void* W_a, const void* W_b, const float* b_dt, const float* A,
+                         void* alpha, void* beta, int B, int T, int H, int d, cudaStream_t stream);
+cudaError_t launch_norm_gate(int dtype, const void* y, const void* g, const float* gamma, float eps, void* z, int B, int H,
+                             int T, int dv, cudaStream_t stream);
 // Access diagnostics (k_stats.cu): bits = 2 * chains * ceil(N/32) words of scratch; out =
 // 4 + kw + kr float64 sums (see sdm_access_stats).
 cudaError_t launch_access_stats(const int32_t* idx_w, const float* w_w, const int32_t* idx_r, const float* w_r,

@@ -149,6 +149,28 @@ def test_access_stats_rejects_bad_arguments(sdm):
     assert "out overlaps workspace" in sdm.last_error()
 
 
+def test_gates_and_norm_gate_reject_bad_arguments(sdm):
+    s = _shape(sdm)
+    L = sdm.lib()
+    gate_args = lambda **o: [o.get(k, v) for k, v in (("x", FAKE), ("W_a", FAKE + 0x100000), ("W_b", FAKE + 0x200000),
+                                                       ("b_dt", FAKE + 0x300000), ("A", FAKE + 0x400000),
+                                                       ("alpha", FAKE + 0x500000), ("beta", FAKE + 0x600000))]
+    assert L.sdm_gates(ctypes.byref(s), 12, *gate_args(), None) == 2 and "multiple of 16" in sdm.last_error()
+    assert L.sdm_gates(ctypes.byref(s), 64, *gate_args(x=None), None) == 1 and "x is NULL" in sdm.last_error()
+    assert L.sdm_gates(ctypes.byref(s), 64, *gate_args(alpha=FAKE + 8), None) == 1 and "overlaps x" in sdm.last_error()
+    assert L.sdm_gates(ctypes.byref(s), 64, *gate_args(beta=FAKE + 0x500000), None) == 1
+    assert "alpha overlaps beta" in sdm.last_error()
+    big = _shape(sdm, H=33, N=4096, k_write=8, k_read=8)
+    assert L.sdm_gates(ctypes.byref(big), 64, *gate_args(), None) == 2 and "H > 32" in sdm.last_error()
+    ng = lambda **o: L.sdm_norm_gate(ctypes.byref(o.pop("shape", s)), o.get("y", FAKE), o.get("g", FAKE + 0x100000),
+                                     o.get("gamma", FAKE + 0x200000), ctypes.c_float(o.get("eps", 1e-6)),
+                                     o.get("z", FAKE + 0x300000), None)
+    assert ng(z=None) == 1 and "z is NULL" in sdm.last_error()
+    assert ng(z=FAKE + 0x100000 + 64) == 1 and "z overlaps g" in sdm.last_error()
+    assert ng(eps=-1.0) == 1 and "eps" in sdm.last_error()
+    assert ng(shape=_shape(sdm, d_v=1024)) == 2 and "1024 bytes" in sdm.last_error()
+
+
 def test_decode_step_requires_T_equal_1(sdm):
     s = _shape(sdm, T=2)
     L = sdm.lib()

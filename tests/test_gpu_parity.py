@@ -18,6 +18,7 @@ pytestmark = [pytest.mark.gpu,
               pytest.mark.skipif(not torch.cuda.is_available(), reason="needs a CUDA GPU")]
 
 from tests import gpu_harness as G  # noqa: E402
+from synth.torch_io import to_torch  # noqa: E402
 
 TOL = {"bf16": 2e-3, "f32": 1e-5}
 
@@ -455,6 +456,84 @@ def test_forward_lazy_continues_a_sequence_across_calls(sdm):
     assert torch.equal(b["touched"], one["touched"])
     mask = torch.from_numpy(G.touched_bits(one["touched"], cfg.N)).to("cuda")
     assert torch.equal(b["mem"][mask], one["mem"][mask])
+
+
+# ------------------------------------------------------------------ gates and output epilogue
+
+def _storage_ulp(ref: np.ndarray, dtype: str) -> np.ndarray:
+    """Spacing of the storage dtype at |ref| (one rounding step)."""
+    bits = 8 if dtype == "bf16" else 24
+    _, e = np.frexp(np.abs(ref))
+    return np.ldexp(1.0, e - bits)
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("name", ["tiny_fp32", "small_bf16"])
+def test_gates_match_the_oracle(sdm, name):
+    """sdm_gates against the oracle's gates of the same inputs.  Tolerance from the arithmetic:
+    the fp32 dot products are within (d+2) 2^-24 sum|W x| of the exact ones (gamma_d bound);
+    alpha moves by at most alpha A sigmoid(z) |dz|, beta by beta (1 - beta) |dz|; expf and
+    log1pf add a few ulps; storage rounding may flip one ulp."""
+    from synth.gen import layer_inputs
+    cfg = synth.CONFIGS[name]
+    li = layer_inputs(cfg)
+    d = cfg.H * cfg.d_v
+    to = lambda a: to_torch(a, cfg.dtype)
+    x, Wa, Wb, g = to(li["x"]), to(li["W_a"]), to(li["W_b"]), to(li["g"])
+    b_dt = torch.from_numpy(li["b_dt"]).cuda()
+    A = torch.from_numpy(li["A"]).cuda()
+    dt = G.torch_dtype(cfg.dtype)
+    alpha = torch.empty((cfg.B, cfg.H, cfg.T), dtype=dt, device="cuda")
+    beta = torch.empty_like(alpha)
+    sdm.gates(G.shape_of(cfg), d, x, Wa, Wb, b_dt, A, alpha, beta)
+    torch.cuda.synchronize()
+    ga, gb = G.host(alpha, cfg.dtype), G.host(beta, cfg.dtype)
+    f = lambda a: O.to_f64(a, cfg.dtype)
+    X, WA, WB = f(li["x"]), f(li["W_a"]), f(li["W_b"])
+    Af, bf = li["A"].astype(np.float64), li["b_dt"].astype(np.float64)
+    for b in range(cfg.B):
+        ra, rb = O.gates(X[b], WA, bf, Af, WB)                      # [H, T]
+        za = X[b] @ WA.T + bf[None, :]
+        zb = X[b] @ WB.T
+        dza = ((d + 2) * 2.0 ** -24 * (np.abs(X[b]) @ np.abs(WA).T) + 2.0 ** -24 * np.abs(za)).T
+        dzb = ((d + 2) * 2.0 ** -24 * (np.abs(X[b]) @ np.abs(WB).T)).T
+        sig = lambda z: 1 / (1 + np.exp(-z))
+        tol_a = ra * Af[:, None] * sig(za.T) * dza + 8 * 2.0 ** -24 * (1 + Af[:, None]) * ra + _storage_ulp(ra, cfg.dtype)
+        tol_b = rb * (1 - rb) * dzb + 8 * 2.0 ** -24 * rb + _storage_ulp(rb, cfg.dtype)
+        ea = np.abs(f(ga[b]) - O.round_storage(ra, cfg.dtype))
+        eb = np.abs(f(gb[b]) - O.round_storage(rb, cfg.dtype))
+        assert np.all(ea <= tol_a), (b, float(ea.max()))
+        assert np.all(eb <= tol_b), (b, float(eb.max()))
+        if cfg.dtype == "bf16":       # a flipped bf16 rounding needs an fp32 error near a tie: rare
+            assert np.mean(ea == 0) > 0.95 and np.mean(eb == 0) > 0.95
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("name", ["tiny_fp32", "small_bf16"])
+def test_norm_gate_matches_the_oracle(sdm, name):
+    """sdm_norm_gate against the oracle (y stands in as the seeded v tensor).  fp32 relative
+    error of g * gamma * y / sqrt(mean(y^2) + eps) is below (d_v / 2 + 6) 2^-24; storage
+    rounding may flip one ulp.  z comes back token-major [B, T, H, d_v]."""
+    from synth.gen import layer_inputs
+    cfg = synth.CONFIGS[name]
+    li = layer_inputs(cfg)
+    dev = G.device_inputs(cfg)
+    y = dev["v"]
+    g = to_torch(li["g"], cfg.dtype)
+    gamma = torch.from_numpy(li["gamma"]).cuda()
+    eps = 1e-6
+    z = torch.empty((cfg.B, cfg.T, cfg.H, cfg.d_v), dtype=y.dtype, device="cuda")
+    sdm.norm_gate(G.shape_of(cfg), y, g, gamma, eps, z)
+    torch.cuda.synchronize()
+    got = O.to_f64(G.host(z, cfg.dtype), cfg.dtype)
+    Y = O.to_f64(G.host(y, cfg.dtype), cfg.dtype)
+    Gf = O.to_f64(li["g"], cfg.dtype)
+    for b in range(cfg.B):
+        for h in range(cfg.H):
+            ref = O.norm_gate(Y[b, h], Gf[b, h], li["gamma"].astype(np.float64), eps)
+            tol = (cfg.d_v / 2 + 6) * 2.0 ** -24 * np.abs(ref) + _storage_ulp(ref, cfg.dtype)
+            err = np.abs(got[b, :, h] - O.round_storage(ref, cfg.dtype))
+            assert np.all(err <= tol), (b, h, float(err.max()))
 
 
 # ------------------------------------------------------------------ access diagnostics
