@@ -15,7 +15,8 @@
 
 namespace sdm {
 
-constexpr int GT_THREADS = 256;
+constexpr int GT_THREADS = 256;        // k_norm_gate
+constexpr int GG_THREADS = 512;        // k_gates: 16 warps share one copy of W_a, W_b per SM
 constexpr size_t GT_SMEM_MAX = 200 * 1024;
 
 template <class D> __device__ __forceinline__ void store_elem(void* base, int64_t i, float v);
@@ -47,7 +48,7 @@ template <> struct Chunk8<BF16> {
 
 // NH >= 2H accumulators per lane.
 template <class D, int NH>
-__global__ void __launch_bounds__(GT_THREADS) k_gates(const void* __restrict__ x, const void* __restrict__ W_a,
+__global__ void __launch_bounds__(GG_THREADS) k_gates(const void* __restrict__ x, const void* __restrict__ W_a,
                                                       const void* __restrict__ W_b, const float* __restrict__ b_dt,
                                                       const float* __restrict__ A, void* __restrict__ alpha,
                                                       void* __restrict__ beta, int64_t tokens, int T, int H, int d,
@@ -59,15 +60,15 @@ __global__ void __launch_bounds__(GT_THREADS) k_gates(const void* __restrict__ x
     const uint4* Wg_b = static_cast<const uint4*>(W_b);
     uint4* Ws = reinterpret_cast<uint4*>(smG);              // [2H][nq]: W_a rows, then W_b rows
     if (use_smem) {
-        for (int i = threadIdx.x; i < rows * nq; i += GT_THREADS) {
+        for (int i = threadIdx.x; i < rows * nq; i += GG_THREADS) {
             const int r = i / nq, q = i - r * nq;
             Ws[i] = r < H ? __ldg(Wg_a + static_cast<int64_t>(r) * nq + q) : __ldg(Wg_b + static_cast<int64_t>(r - H) * nq + q);
         }
         __syncthreads();
     }
     const int lane = threadIdx.x & 31;
-    const int64_t wstride = static_cast<int64_t>(gridDim.x) * (GT_THREADS / 32);
-    for (int64_t u = static_cast<int64_t>(blockIdx.x) * (GT_THREADS / 32) + (threadIdx.x >> 5); u < tokens; u += wstride) {
+    const int64_t wstride = static_cast<int64_t>(gridDim.x) * (GG_THREADS / 32);
+    for (int64_t u = static_cast<int64_t>(blockIdx.x) * (GG_THREADS / 32) + (threadIdx.x >> 5); u < tokens; u += wstride) {
         const uint4* xr = static_cast<const uint4*>(x) + u * nq;
         float acc[NH];
 #pragma unroll
@@ -124,11 +125,13 @@ __global__ void __launch_bounds__(GT_THREADS) k_norm_gate(const void* __restrict
         const uint2* yr = static_cast<const uint2*>(y) + u * nc;
         const uint2* gr = static_cast<const uint2*>(g) + u * nc;
         float fy[MC][C::E];
+        uint2 gv[MC];
         float ss = 0.f;
 #pragma unroll
-        for (int m = 0; m < MC; ++m) {
+        for (int m = 0; m < MC; ++m) {                       // y and g of the row in flight together
             const int c = lane + 32 * m;
             if (c < nc) {
+                gv[m] = __ldg(gr + c);
                 C::unpack(__ldg(yr + c), fy[m]);
 #pragma unroll
                 for (int e = 0; e < C::E; ++e) ss = fmaf(fy[m][e], fy[m][e], ss);
@@ -146,7 +149,7 @@ __global__ void __launch_bounds__(GT_THREADS) k_norm_gate(const void* __restrict
             const int c = lane + 32 * m;
             if (c < nc) {
                 float fg[C::E], o[C::E];
-                C::unpack(__ldg(gr + c), fg);
+                C::unpack(gv[m], fg);
 #pragma unroll
                 for (int e = 0; e < C::E; ++e) o[e] = fg[e] * __ldg(gamma + c * C::E + e) * (fy[m][e] * inv);
                 zr[c] = C::pack(o);
@@ -156,12 +159,12 @@ __global__ void __launch_bounds__(GT_THREADS) k_norm_gate(const void* __restrict
 }
 
 namespace {
-unsigned persistent_grid(int64_t warps_wanted) {
+unsigned persistent_grid(int64_t warps_wanted, int threads = GT_THREADS) {
     int dev = 0, sms = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    int64_t grid = (warps_wanted + GT_THREADS / 32 - 1) / (GT_THREADS / 32);
-    const int64_t cap = static_cast<int64_t>(sms > 0 ? sms : 1) * 8;
+    int64_t grid = (warps_wanted + threads / 32 - 1) / (threads / 32);
+    const int64_t cap = static_cast<int64_t>(sms > 0 ? sms : 1) * (2048 / threads);   // a full SM of threads
     return static_cast<unsigned>(grid < 1 ? 1 : (grid < cap ? grid : cap));
 }
 
@@ -176,7 +179,7 @@ cudaError_t gates_nh(const void* x, const void* W_a, const void* W_b, const floa
         if (e != cudaSuccess) return e;
     }
     const int64_t tokens = static_cast<int64_t>(B) * T;
-    k_gates<D, NH><<<persistent_grid(tokens), GT_THREADS, smem, s>>>(x, W_a, W_b, b_dt, A, alpha, beta, tokens, T, H, d,
+    k_gates<D, NH><<<persistent_grid(tokens, GG_THREADS), GG_THREADS, smem, s>>>(x, W_a, W_b, b_dt, A, alpha, beta, tokens, T, H, d,
                                                                     use_smem);
     return cudaGetLastError();
 }
