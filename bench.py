@@ -193,6 +193,27 @@ def tokens_step_of(B: int, T: int, world: int) -> int:
     return B * T * world
 
 
+def shard_b0(rank: int, B: int) -> int:
+    """First global sequence of a rank's shard: each rank owns B whole sequences (their (b, h)
+    chains are independent), so per-rank work is fixed as ranks are added (weak scaling)."""
+    return rank * B
+
+
+def reduce_max(x: float, dist=None, device="cpu") -> float:
+    """Max of x over all ranks (x itself on one rank): the job's time is its slowest rank's."""
+    if dist is None or not dist.is_initialized() or dist.get_world_size() == 1:
+        return x
+    import torch
+    t = torch.tensor([x], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def weak_scaling_value(B: int, T: int, world: int, ms_max: float) -> float:
+    """Whole-job tokens/s: every rank's B*T tokens over the slowest rank's step time."""
+    return tokens_step_of(B, T, world) / (ms_max * 1e-3)
+
+
 def run_ours(args, cfg):
     import torch
     import paper_2607_07386_gb300 as sdm
@@ -213,7 +234,7 @@ def run_ours(args, cfg):
     build()   # no-op when up to date; loads in every rank
 
     # ---- inputs (rank r owns sequences [r*B, (r+1)*B) of the global batch), resident in HBM
-    full = synth.full_inputs(cfg, b0=rank * cfg.B)
+    full = synth.full_inputs(cfg, b0=shard_b0(rank, cfg.B))
     dt = torch_dtype(cfg.dtype)
     dev = {n: to_torch(a, cfg.dtype) for n, a in full.items()}
     host_pinned = {n: torch.from_numpy(np.ascontiguousarray(full[n]).view(np.int16 if cfg.dtype == "bf16" else np.float32))
@@ -240,11 +261,7 @@ def run_ours(args, cfg):
         torch.cuda.synchronize()
 
     def max_over_ranks(x: float) -> float:
-        if world == 1:
-            return x
-        t = torch.tensor([x], device="cuda", dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
+        return reduce_max(x, dist if world > 1 else None, device="cuda")
 
     for _ in range(args.warmup):
         step()
@@ -426,7 +443,7 @@ def run_ours(args, cfg):
     step_bytes = cfg.algorithmic_bytes_per_token_head() * B * H * T + (1 + B) * H * N * dv * cfg.elem_bytes
     kernels_per_step = 8   # init, P row norms, scores, finalize (3 passes), hazard pass, recurrence
     line = {
-        "metric": METRIC, "value": tokens_step / (ms_step * 1e-3), "unit": UNIT, "n_gpus": world,
+        "metric": METRIC, "value": weak_scaling_value(B, T, world, ms_step), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": cfg.dtype, "data": "synthetic",
         "config": {"workload": _workload_desc(cfg), "global_batch": B * world, "seq_len": T,
