@@ -458,6 +458,29 @@ def test_forward_lazy_continues_a_sequence_across_calls(sdm):
     assert torch.equal(b["mem"][mask], one["mem"][mask])
 
 
+@pytest.mark.gpu
+def test_forward_lazy_one_token_per_call_equals_one_call(sdm):
+    """The lazy memory carried over T single-token calls (the decode shape: look-ahead 1) gives
+    the y, bitmap and written rows of one T-token call and of the broadcast forward."""
+    cfg = synth.SdmConfig("lazy_steps", B=3, H=2, T=64, d_k=64, d_v=64, N=4096, k_write=8, k_read=8,
+                          dtype="bf16", seed=53, alpha_mu=3.0)
+    dev = G.device_inputs(cfg)
+    whole = G.run_forward(cfg, dev)
+    one = G.run_forward_lazy(cfg, dev)
+    step = G.run_forward_lazy(cfg, dev, 0, 1)
+    ys = [step["y"]]
+    for t in range(1, cfg.T):
+        step = G.run_forward_lazy(cfg, dev, t, t + 1, mem=step["mem"], touched=step["touched"])
+        ys.append(step["y"])
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    assert torch.equal(torch.cat(ys, dim=2), one["y"]) and torch.equal(one["y"], whole["y"])
+    assert torch.equal(step["touched"], one["touched"])
+    sdm.materialize(G.shape_of(cfg), dev["M0"], step["touched"], step["mem"])
+    torch.cuda.synchronize()
+    assert torch.equal(step["mem"], whole["mem"])
+
+
 # ------------------------------------------------------------------ gates and output epilogue
 
 def _storage_ulp(ref: np.ndarray, dtype: str) -> np.ndarray:
@@ -467,15 +490,27 @@ def _storage_ulp(ref: np.ndarray, dtype: str) -> np.ndarray:
     return np.ldexp(1.0, e - bits)
 
 
+_GATE_CFGS = {
+    "tiny_fp32": synth.TINY_FP32,
+    "small_bf16": synth.SMALL_BF16,
+    "h32_bf16": synth.SdmConfig("h32", B=2, H=32, T=96, d_k=32, d_v=32, N=1024, k_write=8, k_read=8, dtype="bf16",
+                                seed=54, alpha_mu=3.0),
+    "dv256_bf16": synth.SdmConfig("dv256", B=2, H=2, T=80, d_k=32, d_v=256, N=1024, k_write=8, k_read=8,
+                                  dtype="bf16", seed=55, alpha_mu=3.0),
+    "dv256_f32": synth.SdmConfig("dv256f", B=1, H=3, T=50, d_k=32, d_v=256, N=1024, k_write=8, k_read=8,
+                                 dtype="f32", seed=56, alpha_mu=3.0),
+}
+
+
 @pytest.mark.gpu
-@pytest.mark.parametrize("name", ["tiny_fp32", "small_bf16"])
+@pytest.mark.parametrize("name", ["tiny_fp32", "small_bf16", "h32_bf16"])
 def test_gates_match_the_oracle(sdm, name):
     """sdm_gates against the oracle's gates of the same inputs.  Tolerance from the arithmetic:
     the fp32 dot products are within (d+2) 2^-24 sum|W x| of the exact ones (gamma_d bound);
     alpha moves by at most alpha A sigmoid(z) |dz|, beta by beta (1 - beta) |dz|; expf and
     log1pf add a few ulps; storage rounding may flip one ulp."""
     from synth.gen import layer_inputs
-    cfg = synth.CONFIGS[name]
+    cfg = _GATE_CFGS[name]
     li = layer_inputs(cfg)
     d = cfg.H * cfg.d_v
     to = lambda a: to_torch(a, cfg.dtype)
@@ -509,13 +544,13 @@ def test_gates_match_the_oracle(sdm, name):
 
 
 @pytest.mark.gpu
-@pytest.mark.parametrize("name", ["tiny_fp32", "small_bf16"])
+@pytest.mark.parametrize("name", ["tiny_fp32", "small_bf16", "dv256_bf16", "dv256_f32"])
 def test_norm_gate_matches_the_oracle(sdm, name):
     """sdm_norm_gate against the oracle (y stands in as the seeded v tensor).  fp32 relative
     error of g * gamma * y / sqrt(mean(y^2) + eps) is below (d_v / 2 + 6) 2^-24; storage
     rounding may flip one ulp.  z comes back token-major [B, T, H, d_v]."""
     from synth.gen import layer_inputs
-    cfg = synth.CONFIGS[name]
+    cfg = _GATE_CFGS[name]
     li = layer_inputs(cfg)
     dev = G.device_inputs(cfg)
     y = dev["v"]
@@ -574,6 +609,32 @@ def test_access_stats_match_the_oracle_diagnostics(sdm, name):
     np.testing.assert_allclose(got[4:], exp[4:], rtol=2e-5)
     tokens = cfg.B * cfg.H * cfg.T
     np.testing.assert_allclose(got[4 + cfg.k_write - 1], tokens, rtol=1e-5)    # C(k) = 1 per token
+
+
+@pytest.mark.gpu
+def test_access_stats_wide_lists_match_the_oracle(sdm):
+    """sdm_access_stats on seeded explicit lists with k_write = 64 (two weights per lane) and
+    k_read = 20, against the oracle's diagnostics of the same lists."""
+    B, H, T, N, kw, kr = 2, 3, 70, 4096, 64, 20
+    rng = np.random.default_rng(57)
+    iw = np.sort(np.stack([rng.choice(N, kw, replace=False) for _ in range(B * H * T)]), axis=1).astype(np.int32)
+    ir = np.sort(np.stack([rng.choice(N, kr, replace=False) for _ in range(B * H * T)]), axis=1).astype(np.int32)
+    ww = rng.dirichlet(np.full(kw, 0.3), B * H * T).astype(np.float32)
+    wr = rng.dirichlet(np.full(kr, 2.0), B * H * T).astype(np.float32)
+    shape = sdm.SdmShape.make(B, H, T, 64, 64, N, kw, kr, "f32")
+    dv = lambda a, k: torch.from_numpy(a.reshape(B, H, T, k)).cuda()
+    stats = torch.empty(4 + kw + kr, dtype=torch.float64, device="cuda")
+    ws = torch.empty(sdm.access_stats_workspace_bytes(shape), dtype=torch.uint8, device="cuda")
+    sdm.access_stats(shape, dv(iw, kw), dv(ww, kw), dv(ir, kr), dv(wr, kr), stats, ws)
+    torch.cuda.synchronize()
+    got = stats.cpu().numpy()
+    w64, r64 = ww.astype(np.float64), wr.astype(np.float64)
+    uniq = lambda idx: sum(np.unique(idx.reshape(B * H, T * idx.shape[1])[c]).size for c in range(B * H))
+    assert got[2] == uniq(iw) and got[3] == uniq(ir)
+    np.testing.assert_allclose(got[0], O.eff_keys_fraction(w64).sum(), rtol=2e-5)
+    np.testing.assert_allclose(got[1], O.eff_keys_fraction(r64).sum(), rtol=2e-5)
+    np.testing.assert_allclose(got[4:4 + kw], O.cumulative_mass(w64).sum(axis=0), rtol=2e-5)
+    np.testing.assert_allclose(got[4 + kw:], O.cumulative_mass(r64).sum(axis=0), rtol=2e-5)
 
 
 # ------------------------------------------------------------------ full-size workloads
