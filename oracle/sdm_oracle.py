@@ -41,7 +41,13 @@ the outer sum by (score desc, slot asc).
    "Norm, Gating, and Head Mixing"): alpha_t = exp(-A softplus(W_a x_t + b_dt)),
    beta_t = sigmoid(W_b x_t) per head; z = g (.) RMSNorm(y) per head, the heads
    concatenated per token and mixed by W_o.
-7. Access diagnostics (App. "Memory Utilization and Access"): the normalised
+7. The chunkwise (WY) form of the same recurrence (App. A.1-A.2): per chunk of C
+   tokens, segmented cumulative log-decays, the gated sparse inner products A
+   (write-write) and QK (read-write) by a two-pointer merge of sorted slot lists,
+   a unit lower-triangular solve, then gather, correct, scatter and output against
+   the chunk-initial memory.  Equal to item 3-4 up to rounding when the storage
+   is exact; storage rounding is applied at chunk boundaries only.
+8. Access diagnostics (App. "Memory Utilization and Access"): the normalised
    effective number of keys exp(H(p)) / k, the cumulative mass curve C(m) of
    the descending-sorted weights, and the fraction of unique slots accessed.
 
@@ -60,7 +66,7 @@ __all__ = [
     "to_f64", "round_storage", "half_scores", "topk_half", "pkm_select", "address",
     "recur", "forward_slice", "state_elements_per_layer", "n_global_layers",
     "touched_mask", "recur_lazy", "materialize", "eff_keys_fraction", "cumulative_mass", "unique_fraction",
-    "softplus", "gates", "norm_gate", "head_mix",
+    "softplus", "gates", "norm_gate", "head_mix", "sparse_ip", "recur_chunkwise",
 ]
 
 
@@ -204,6 +210,91 @@ def forward_slice(M0_h: np.ndarray, P_q, P_k, q, k, v, alpha, beta, N: int, k_wr
         M = np.array(M0_h, dtype=np.float64, copy=True)
     y64, y = recur(M, idx_w, w_w, idx_r, w_r, v, alpha, beta, store)
     return {"y": y, "y64": y64, "M": M, "idx_w": idx_w, "w_w": w_w, "idx_r": idx_r, "w_r": w_r}
+
+
+# --------------------------------------------------------------------------------------
+# chunkwise (WY) form (App. A.1 "Intra-Chunk Parallel vs. Chunkwise Recurrent", A.2)
+# --------------------------------------------------------------------------------------
+
+def sparse_ip(idx_a, val_a, lam_a, idx_b, val_b, lam_b) -> float:
+    """Gated sparse inner product of two tokens (App. A.2, Eq. sparse-ip):
+    sum over matching slots idx_a[n] == idx_b[m] of val_a[n] val_b[m] exp(lam_a[n] - lam_b[m]).
+    Both index lists must be strictly ascending; they are walked together (two pointers)."""
+    total = 0.0
+    a = b = 0
+    while a < len(idx_a) and b < len(idx_b):
+        ia, ib = idx_a[a], idx_b[b]
+        if ia == ib:
+            total += val_a[a] * val_b[b] * math.exp(lam_a[a] - lam_b[b])
+            a += 1
+            b += 1
+        elif ia < ib:
+            a += 1
+        else:
+            b += 1
+    return total
+
+
+def recur_chunkwise(M: np.ndarray, idx_w, w_w, idx_r, w_r, v, alpha, beta, C: int, store: str):
+    """The recurrence of ``recur`` in chunkwise form (App. A.1-A.2), chunks of C tokens.
+
+    Phase 1 (per chunk, independent of the memory): lam_w[t, n], the cumulative log-decay of
+    slot idx_w[t, n] over the chunk's writers of that slot up to and including t; lam_r[t, n]
+    the same for read slot idx_r[t, n] after token t's own write; the lower-triangular
+    A[t, s] = sparse_ip(write t, write s) for s < t and QK[t, s] = sparse_ip(read t, write s)
+    for s <= t; M_sys = I + diag(beta) A; dV_const = M_sys^-1 diag(beta) V and
+    B = M_sys^-1 diag(-beta).
+    Phase 2 (sequential over chunks): retrieved[t] = sum_n w e^lam_w M[idx_w[t, n]] and
+    inter[t] = sum_n rho e^lam_r M[idx_r[t, n]] from the chunk-initial memory; the written
+    deltas u = dV_const + B retrieved (u_t = beta_t (v_t - v~_t)); y = inter + QK u; then
+    every written slot i becomes e^(lam_i) M[i] + sum_t e^(lam_i - lam_(t,i)) w_(t,i) u_t with
+    lam_i its decay over the whole chunk, rounded to the storage dtype.
+
+    M: [N, d_v] float64, updated in place.  Returns (y [T, d_v] float64, R(y)).
+    """
+    from scipy.linalg import solve_triangular
+    T = v.shape[0]
+    y = np.empty((T, M.shape[1]), dtype=np.float64)
+    for c0 in range(0, T, C):
+        c1 = min(T, c0 + C)
+        n = c1 - c0
+        # ---- phase 1: segmented cumulative log-decay, interaction matrices, triangular solve
+        acc = {}
+        lam_w = np.zeros(idx_w[c0:c1].shape)
+        lam_r = np.zeros(idx_r[c0:c1].shape)
+        for t in range(n):
+            la = math.log(alpha[c0 + t])
+            for m, i in enumerate(idx_w[c0 + t]):
+                acc[int(i)] = acc.get(int(i), 0.0) + la
+                lam_w[t, m] = acc[int(i)]
+            for m, j in enumerate(idx_r[c0 + t]):
+                lam_r[t, m] = acc.get(int(j), 0.0)
+        A = np.zeros((n, n))
+        QK = np.zeros((n, n))
+        for t in range(n):
+            for s_ in range(n):
+                if s_ < t:
+                    A[t, s_] = sparse_ip(idx_w[c0 + t], w_w[c0 + t], lam_w[t], idx_w[c0 + s_], w_w[c0 + s_], lam_w[s_])
+                if s_ <= t:
+                    QK[t, s_] = sparse_ip(idx_r[c0 + t], w_r[c0 + t], lam_r[t], idx_w[c0 + s_], w_w[c0 + s_], lam_w[s_])
+        bet = np.asarray(beta[c0:c1], dtype=np.float64)
+        M_sys = np.eye(n) + bet[:, None] * A
+        dV_const = solve_triangular(M_sys, bet[:, None] * v[c0:c1], lower=True, unit_diagonal=True)
+        Bm = solve_triangular(M_sys, np.diag(-bet), lower=True, unit_diagonal=True)
+        # ---- phase 2: gather, correct, output, scatter
+        retrieved = np.stack([(w_w[c0 + t] * np.exp(lam_w[t])) @ M[idx_w[c0 + t]] for t in range(n)])
+        inter = np.stack([(w_r[c0 + t] * np.exp(lam_r[t])) @ M[idx_r[c0 + t]] for t in range(n)])
+        u = dV_const + Bm @ retrieved
+        y[c0:c1] = inter + QK @ u
+        touched = sorted(acc)
+        new = {i: math.exp(acc[i]) * M[i] for i in touched}
+        for t in range(n):
+            for m, i in enumerate(idx_w[c0 + t]):
+                i = int(i)
+                new[i] = new[i] + math.exp(acc[i] - lam_w[t, m]) * w_w[c0 + t][m] * u[t]
+        for i in touched:
+            M[i] = round_storage(new[i], store)
+    return y, round_storage(y, store)
 
 
 # --------------------------------------------------------------------------------------

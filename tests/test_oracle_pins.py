@@ -255,6 +255,79 @@ def test_forward_slice_is_address_then_recur():
     assert np.array_equal(M0, O.forward_slice(M0, Pq, Pk, q, kk, v, a, b, N, k, k, "f64")["M"]) is False
 
 
+# ------------------------------------------------------------------ chunkwise (WY) form
+
+def _brute_sparse_ip(ia, va, la, ib, vb, lb):
+    return sum(va[n] * vb[m] * math.exp(la[n] - lb[m]) for n in range(len(ia)) for m in range(len(ib)) if ia[n] == ib[m])
+
+
+def test_sparse_ip_two_pointer_equals_brute_force():
+    rng = np.random.default_rng(41)
+    for _ in range(200):
+        ka, kb = rng.integers(1, 9, 2)
+        ia = np.sort(rng.choice(20, ka, replace=False))
+        ib = np.sort(rng.choice(20, kb, replace=False))
+        va, vb = rng.standard_normal(ka), rng.standard_normal(kb)
+        la, lb = -rng.uniform(0, 3, ka), -rng.uniform(0, 3, kb)
+        assert abs(O.sparse_ip(ia, va, la, ib, vb, lb) - _brute_sparse_ip(ia, va, la, ib, vb, lb)) < 1e-13
+
+
+@pytest.mark.parametrize("C", [1, 3, 8, 60])
+@pytest.mark.parametrize("N", [40, 9])          # N = 9 with 5 writes per token: slots collide constantly
+def test_chunkwise_equals_dense_masked_form(C, N):
+    rng = np.random.default_rng(42 + N)
+    M0, idx_w, w_w, idx_r, w_r, V, alpha, beta = _random_sparse_case(rng, N=N, T=60)
+    M = M0.copy()
+    y64, _ = O.recur_chunkwise(M, idx_w, w_w, idx_r, w_r, V, alpha, beta, C, "f64")
+    M_ref, y_ref = _dense_masked_sdm(M0, idx_w, w_w, idx_r, w_r, V, alpha, beta)
+    np.testing.assert_allclose(y64, y_ref, rtol=1e-11, atol=1e-11)
+    np.testing.assert_allclose(M, M_ref, rtol=1e-11, atol=1e-11)
+
+
+def test_chunkwise_gdn_special_case():
+    """All slots selected with dense key weights (Sec. 3.1 "Connection to GDN"): the chunkwise form
+    is the chunkwise GDN, and equals the textbook GDN update token by token."""
+    rng = np.random.default_rng(43)
+    dqk, dv, T = 6, 5, 24
+    M0 = rng.standard_normal((dqk, dv))
+    K = rng.standard_normal((T, dqk)) / np.sqrt(dqk)
+    Q = rng.standard_normal((T, dqk))
+    V = rng.standard_normal((T, dv))
+    a = rng.uniform(0.7, 1.0, T)
+    b = rng.uniform(0.1, 0.9, T)
+    alls = np.tile(np.arange(dqk), (T, 1))
+    M = M0.copy()
+    y64, _ = O.recur_chunkwise(M, alls, K, alls, Q, V, a, b, 8, "f64")
+    M_ref, y_ref = _gdn_textbook(M0, K, V, Q, a, b)
+    np.testing.assert_allclose(y64, y_ref, rtol=1e-11, atol=1e-11)
+    np.testing.assert_allclose(M, M_ref, rtol=1e-11, atol=1e-11)
+
+
+def test_chunkwise_rounding_only_at_chunk_boundaries():
+    """With bf16 storage the chunkwise form rounds the memory at chunk boundaries only, and its reads
+    within a chunk see the unrounded intra-chunk writes (the token-serial form reads rows rounded
+    after each token).  So the two forms differ by bf16 rounding alone, for any C."""
+    rng = np.random.default_rng(44)
+    M0, idx_w, w_w, idx_r, w_r, V, alpha, beta = _random_sparse_case(rng, N=50, T=48)
+    M0 = O.round_storage(M0 * 0.02, "bf16")
+    V = O.round_storage(V, "bf16")
+    Ms = M0.copy()
+    _, ys = O.recur(Ms, idx_w, w_w, idx_r, w_r, V, alpha, beta, "bf16")
+    Me = M0.copy()
+    ye, _ = O.recur(Me, idx_w, w_w, idx_r, w_r, V, alpha, beta, "f64")    # exact storage
+    rel = lambda a, b: np.linalg.norm(a - b) / np.linalg.norm(b)
+    # a read row has gone through at most max_writes roundings (2^-9 relative each) plus its own
+    bound = (1 + np.bincount(idx_w.ravel()).max()) * 2.0 ** -9
+    assert rel(ys, ye) < bound
+    for C in (1, 8, 48):
+        Mc = M0.copy()
+        _, yc = O.recur_chunkwise(Mc, idx_w, w_w, idx_r, w_r, V, alpha, beta, C, "bf16")
+        assert rel(yc, ye) < bound, C
+        assert np.array_equal(O.round_storage(Mc, "bf16"), Mc)              # stored rows are bf16 values
+        touched = np.unique(idx_w)
+        assert rel(Mc[touched], Me[touched]) < bound, C
+
+
 # ------------------------------------------------------------------ lazy M0 (copy-on-write)
 
 def test_lazy_overlay_equals_dense_masked_form():
@@ -509,6 +582,33 @@ def test_pins_reject_planted_mistakes():
     # cumulative mass of the weights in slot order (unsorted) fails the geometric closed form
     p = np.array([0.1, 0.6, 0.3])
     assert not np.allclose(np.cumsum(p), O.cumulative_mass(p))
+    # chunkwise form without the decay factor in A, or with beta of the column token in M_sys,
+    # fails the dense pin
+    M0w, iw, ww, ir, wr, Vw, al, be = _random_sparse_case(rng, N=9, T=20)
+    _, y_ref = _dense_masked_sdm(M0w, iw, ww, ir, wr, Vw, al, be)
+    def chunk_variant(no_decay_in_A=False, beta_col=False):
+        n = Vw.shape[0]
+        acc, lw, lr = {}, np.zeros(iw.shape), np.zeros(ir.shape)
+        for t in range(n):
+            for m, i in enumerate(iw[t]):
+                acc[int(i)] = acc.get(int(i), 0.0) + math.log(al[t])
+                lw[t, m] = acc[int(i)]
+            for m, j in enumerate(ir[t]):
+                lr[t, m] = acc.get(int(j), 0.0)
+        z = lambda x: np.zeros_like(x) if no_decay_in_A else x
+        A = np.array([[O.sparse_ip(iw[t], ww[t], z(lw[t]), iw[s_], ww[s_], z(lw[s_])) if s_ < t else 0.0
+                       for s_ in range(n)] for t in range(n)])
+        QK = np.array([[O.sparse_ip(ir[t], wr[t], lr[t], iw[s_], ww[s_], lw[s_]) if s_ <= t else 0.0
+                        for s_ in range(n)] for t in range(n)])
+        Msys = np.eye(n) + (A * be[None, :] if beta_col else be[:, None] * A)
+        Minv = np.linalg.inv(Msys)
+        ret = np.stack([(ww[t] * np.exp(lw[t])) @ M0w[iw[t]] for t in range(n)])
+        inter = np.stack([(wr[t] * np.exp(lr[t])) @ M0w[ir[t]] for t in range(n)])
+        u = Minv @ (be[:, None] * Vw) - Minv @ (be[:, None] * ret)
+        return inter + QK @ u
+    assert np.allclose(chunk_variant(), y_ref, atol=1e-10)             # the variant machinery is right
+    assert not np.allclose(chunk_variant(no_decay_in_A=True), y_ref, atol=1e-6)
+    assert not np.allclose(chunk_variant(beta_col=True), y_ref, atol=1e-6)
     # RMSNorm without the square root (y / mean(y^2)) fails the scale invariance
     y = rng.standard_normal((3, 8))
     bad = lambda yy: yy / np.mean(yy * yy, axis=-1, keepdims=True)
