@@ -47,7 +47,13 @@ the outer sum by (score desc, slot asc).
    a unit lower-triangular solve, then gather, correct, scatter and output against
    the chunk-initial memory.  Equal to item 3-4 up to rounding when the storage
    is exact; storage rounding is applied at chunk boundaries only.
-8. Access diagnostics (App. "Memory Utilization and Access"): the normalised
+8. The backward of the recurrence with in-place undo (App. A.3): the forward
+   updates the memory in place and keeps, per token, the rows its write
+   overwrote (O(T W d_v) beside the O(N d_v) memory); the backward walks the
+   tokens in reverse, restores each token's pre-write rows from that log, and
+   carries the adjoint of the memory for the touched rows only.  Gradients are
+   those of the exact recurrence (storage rounding is not differentiated).
+9. Access diagnostics (App. "Memory Utilization and Access"): the normalised
    effective number of keys exp(H(p)) / k, the cumulative mass curve C(m) of
    the descending-sorted weights, and the fraction of unique slots accessed.
 
@@ -67,6 +73,7 @@ __all__ = [
     "recur", "forward_slice", "state_elements_per_layer", "n_global_layers",
     "touched_mask", "recur_lazy", "materialize", "eff_keys_fraction", "cumulative_mass", "unique_fraction",
     "softplus", "gates", "norm_gate", "head_mix", "sparse_ip", "recur_chunkwise",
+    "recur_forward_undo", "recur_backward",
 ]
 
 
@@ -295,6 +302,73 @@ def recur_chunkwise(M: np.ndarray, idx_w, w_w, idx_r, w_r, v, alpha, beta, C: in
         for i in touched:
             M[i] = round_storage(new[i], store)
     return y, round_storage(y, store)
+
+
+# --------------------------------------------------------------------------------------
+# backward with in-place undo (App. A.3 "Memory-Efficient Backward")
+# --------------------------------------------------------------------------------------
+
+def recur_forward_undo(M: np.ndarray, idx_w, w_w, idx_r, w_r, v, alpha, beta):
+    """``recur`` with exact storage that also returns the undo log: for every token, the rows
+    M_{t-1}[I^w_t] its write overwrote.  M is updated in place to M_T.
+    Returns (y [T, d_v], undo [T, k_w, d_v])."""
+    T = v.shape[0]
+    y = np.empty((T, M.shape[1]))
+    undo = np.empty((T, idx_w.shape[1], M.shape[1]))
+    for t in range(T):
+        iw = idx_w[t]
+        undo[t] = M[iw]
+        decayed = alpha[t] * M[iw]
+        delta = v[t] - w_w[t] @ decayed
+        M[iw] = decayed + beta[t] * w_w[t][:, None] * delta[None, :]
+        y[t] = w_r[t] @ M[idx_r[t]]
+    return y, undo
+
+
+def recur_backward(M: np.ndarray, undo, idx_w, w_w, idx_r, w_r, v, alpha, beta, dy):
+    """Reverse-mode gradients of sum_t <dy_t, y_t> through the recurrence, from the final memory
+    M (= M_T, restored in place to M_0 on return) and the undo log of ``recur_forward_undo``.
+
+    Token t, in reverse: the read y_t = sum_n rho_n M_t[r_n] gives d rho_n = <dy_t, M_t[r_n]> and
+    adds rho_n dy_t to the memory adjoint G at r_n.  The write M_t[i] = r_i + beta w_i delta with
+    r_i = alpha M_{t-1}[i] and delta = v_t - sum_m w_m r_m gives, with G_i the adjoint of M_t[i]:
+    d delta = beta sum_i w_i G_i, d beta = sum_i w_i <G_i, delta>, d w_i = beta <G_i, delta> -
+    <r_i, d delta>, d v_t = d delta, d r_i = G_i - w_i d delta, d alpha = sum_i <d r_i, M_{t-1}[i]>,
+    and the adjoint of M_{t-1}[i] becomes alpha d r_i.  M_{t-1}[I^w_t] comes back from the log.
+
+    Returns dict: dv [T, d_v], dalpha [T], dbeta [T], dw_w [T, k_w], dw_r [T, k_r], dM0 [N, d_v].
+    """
+    T, dvdim = v.shape
+    G = {}
+    out = {"dv": np.zeros_like(v), "dalpha": np.zeros(T), "dbeta": np.zeros(T),
+           "dw_w": np.zeros(w_w.shape), "dw_r": np.zeros(w_r.shape)}
+    zero = np.zeros(dvdim)
+    for t in range(T - 1, -1, -1):
+        # read of the post-write memory M_t
+        for n, j in enumerate(idx_r[t]):
+            j = int(j)
+            out["dw_r"][t, n] = dy[t] @ M[j]
+            G[j] = G.get(j, zero) + w_r[t][n] * dy[t]
+        # write: recover M_{t-1} on the written rows, then the chain rule through the update
+        iw = [int(i) for i in idx_w[t]]
+        prev = undo[t]
+        r = alpha[t] * prev
+        delta = v[t] - w_w[t] @ r
+        Gi = np.stack([G.get(i, zero) for i in iw])
+        d_delta = beta[t] * (w_w[t] @ Gi)
+        out["dbeta"][t] = np.sum(w_w[t] * (Gi @ delta))
+        out["dw_w"][t] = beta[t] * (Gi @ delta) - r @ d_delta
+        out["dv"][t] = d_delta
+        d_r = Gi - w_w[t][:, None] * d_delta[None, :]
+        out["dalpha"][t] = np.sum(d_r * prev)
+        for m, i in enumerate(iw):
+            G[i] = alpha[t] * d_r[m]
+            M[i] = prev[m]                           # undo: M_t[i] -> M_{t-1}[i]
+    dM0 = np.zeros_like(M)
+    for i, g in G.items():
+        dM0[i] = g
+    out["dM0"] = dM0
+    return out
 
 
 # --------------------------------------------------------------------------------------

@@ -328,6 +328,67 @@ def test_chunkwise_rounding_only_at_chunk_boundaries():
         assert rel(Mc[touched], Me[touched]) < bound, C
 
 
+# ------------------------------------------------------------------ backward with in-place undo
+
+def _torch_dense_loss(M0, idx_w, w_w, idx_r, w_r, V, alpha, beta, dy):
+    """sum_t <dy_t, y_t> of the dense masked update written in torch (autograd does the rest)."""
+    import torch
+    N = M0.shape[0]
+    M = M0
+    loss = 0.0
+    for t in range(V.shape[0]):
+        mask = torch.zeros(N, dtype=torch.float64).index_put((torch.as_tensor(idx_w[t]),), torch.ones(len(idx_w[t]), dtype=torch.float64))
+        kappa = torch.zeros(N, dtype=torch.float64).index_put((torch.as_tensor(idx_w[t]),), w_w[t])
+        rho = torch.zeros(N, dtype=torch.float64).index_put((torch.as_tensor(idx_r[t]),), w_r[t])
+        Mt = (1.0 + (alpha[t] - 1.0) * mask)[:, None] * M
+        M = Mt + beta[t] * torch.outer(kappa, V[t] - Mt.T @ kappa)
+        loss = loss + dy[t] @ (M.T @ rho)
+    return loss
+
+
+@pytest.mark.parametrize("N", [30, 7])
+def test_backward_with_undo_equals_autograd_of_the_dense_form(N):
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(61 + N)
+    M0, idx_w, w_w, idx_r, w_r, V, alpha, beta = _random_sparse_case(rng, N=N, T=25, kw=4, kr=3)
+    dy = rng.standard_normal(V.shape)
+    M = M0.copy()
+    y, undo = O.recur_forward_undo(M, idx_w, w_w, idx_r, w_r, V, alpha, beta)
+    M_ref, y_ref = _dense_masked_sdm(M0, idx_w, w_w, idx_r, w_r, V, alpha, beta)
+    np.testing.assert_allclose(y, y_ref, rtol=1e-12, atol=1e-12)
+    g = O.recur_backward(M, undo, idx_w, w_w, idx_r, w_r, V, alpha, beta, dy)
+    assert np.array_equal(M, M0)                                   # the undo restored M_0 exactly
+    leaf = lambda a: torch.tensor(a, dtype=torch.float64, requires_grad=True)
+    tM0, tww, twr, tV, ta, tb = map(leaf, (M0, w_w, w_r, V, alpha, beta))
+    loss = _torch_dense_loss(tM0, idx_w, tww, idx_r, twr, tV, ta, tb, torch.tensor(dy))
+    loss.backward()
+    for name, t in (("dM0", tM0), ("dw_w", tww), ("dw_r", twr), ("dv", tV), ("dalpha", ta), ("dbeta", tb)):
+        np.testing.assert_allclose(g[name], t.grad.numpy(), rtol=1e-10, atol=1e-11, err_msg=name)
+
+
+def test_backward_finite_differences():
+    rng = np.random.default_rng(63)
+    M0, idx_w, w_w, idx_r, w_r, V, alpha, beta = _random_sparse_case(rng, N=12, T=10, kw=3, kr=3)
+    dy = rng.standard_normal(V.shape)
+    def loss(a=alpha, b=beta, vv=V, m0=M0):
+        M = m0.copy()
+        y, _ = O.recur_forward_undo(M, idx_w, w_w, idx_r, w_r, vv, a, b)
+        return float(np.sum(dy * y))
+    M = M0.copy()
+    _, undo = O.recur_forward_undo(M, idx_w, w_w, idx_r, w_r, V, alpha, beta)
+    g = O.recur_backward(M, undo, idx_w, w_w, idx_r, w_r, V, alpha, beta, dy)
+    h = 1e-6
+    for t in (0, 4, 9):
+        e = np.zeros_like(alpha)
+        e[t] = h
+        assert abs((loss(a=alpha + e) - loss(a=alpha - e)) / (2 * h) - g["dalpha"][t]) < 1e-7
+        assert abs((loss(b=beta + e) - loss(b=beta - e)) / (2 * h) - g["dbeta"][t]) < 1e-7
+    i = int(idx_w[2, 1])
+    E = np.zeros_like(M0)
+    E[i, 0] = h
+    assert abs((loss(m0=M0 + E) - loss(m0=M0 - E)) / (2 * h) - g["dM0"][i, 0]) < 1e-7
+
+
 # ------------------------------------------------------------------ lazy M0 (copy-on-write)
 
 def test_lazy_overlay_equals_dense_masked_form():
@@ -609,6 +670,25 @@ def test_pins_reject_planted_mistakes():
     assert np.allclose(chunk_variant(), y_ref, atol=1e-10)             # the variant machinery is right
     assert not np.allclose(chunk_variant(no_decay_in_A=True), y_ref, atol=1e-6)
     assert not np.allclose(chunk_variant(beta_col=True), y_ref, atol=1e-6)
+    # a backward that reads the pre-write memory (the read-before-write mistake) fails autograd
+    torch_mod = pytest.importorskip("torch")
+    M0b, iwb, wwb, irb, wrb, Vb, alb, beb = _random_sparse_case(rng, N=7, T=12, kw=4, kr=3)
+    dyb = rng.standard_normal(Vb.shape)
+    Mb = M0b.copy()
+    _, und = O.recur_forward_undo(Mb, iwb, wwb, irb, wrb, Vb, alb, beb)
+    gb = O.recur_backward(Mb, und, iwb, wwb, irb, wrb, Vb, alb, beb, dyb)
+    lf = lambda a: torch_mod.tensor(a, dtype=torch_mod.float64, requires_grad=True)
+    tw = lf(wrb)
+    _torch_dense_loss(torch_mod.tensor(M0b), iwb, torch_mod.tensor(wwb), irb, tw, torch_mod.tensor(Vb),
+                      torch_mod.tensor(alb), torch_mod.tensor(beb), torch_mod.tensor(dyb)).backward()
+    np.testing.assert_allclose(gb["dw_r"], tw.grad.numpy(), rtol=1e-10, atol=1e-11)
+    Mw = M0b.copy()
+    wrong = np.zeros(wrb.shape)
+    for t in range(Vb.shape[0]):                                 # d rho from M_{t-1} instead of M_t
+        wrong[t] = Mw[irb[t]] @ dyb[t]
+        d_ = alb[t] * Mw[iwb[t]]
+        Mw[iwb[t]] = d_ + beb[t] * wwb[t][:, None] * (Vb[t] - wwb[t] @ d_)[None, :]
+    assert not np.allclose(wrong, tw.grad.numpy(), atol=1e-6)
     # RMSNorm without the square root (y / mean(y^2)) fails the scale invariance
     y = rng.standard_normal((3, 8))
     bad = lambda yy: yy / np.mean(yy * yy, axis=-1, keepdims=True)
