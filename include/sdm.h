@@ -222,6 +222,34 @@ sdm_status sdm_recur(const sdm_shape* shape, const int32_t* idx_w, const float* 
                      const void* alpha, const void* beta, void* mem, void* y,
                      void* workspace, size_t workspace_bytes, sdm_stream_t stream);
 
+/* Bytes of the undo log of sdm_recur_undo: B*H*T*k_write rows of d_v storage elements. */
+size_t sdm_undo_log_bytes(const sdm_shape* shape);
+
+/* sdm_recur that also writes the undo log of the backward (App. A.3): undo[b, h, t, n, :]
+ * = the row M_{t-1}[idx_w[b, h, t, n]] the write of token t overwrote, in storage bits
+ * ([B, H, T, k_write, d_v], sdm_undo_log_bytes(shape) bytes, 16-byte aligned, not
+ * overlapping any other buffer).  Entries of out-of-range slots are not written.  y and
+ * mem are those of sdm_recur, bit for bit. */
+sdm_status sdm_recur_undo(const sdm_shape* shape, const int32_t* idx_w, const float* w_w,
+                          const int32_t* idx_r, const float* w_r, const void* v,
+                          const void* alpha, const void* beta, void* mem, void* y, void* undo,
+                          void* workspace, size_t workspace_bytes, sdm_stream_t stream);
+
+/* Backward of the recurrence with in-place undo (App. A.3): reverse-mode gradients of
+ * L = sum_{b,h,t} <dy[b,h,t], y[b,h,t]> with the stored (rounded) rows treated as the
+ * forward's values.  mem: M_T as sdm_recur_undo left it, restored in place to M_0 (the
+ * state before that call) on return; undo: that call's log; dy: [B, H, T, d_v] storage
+ * dtype.  Outputs (float32, written): dv [B, H, T, d_v], dalpha, dbeta [B, H, T], dw_w
+ * [B, H, T, k_write], dw_r [B, H, T, k_read]; dM [B, H, N, d_v] float32 must be zero on
+ * entry and receives dL/dM_0 per sequence (sum over b for a shared M0).  Other arguments as
+ * in sdm_recur.  d_v must be a multiple of 32, at most 256.  Outputs must not overlap each
+ * other or the inputs. */
+sdm_status sdm_recur_backward(const sdm_shape* shape, const int32_t* idx_w, const float* w_w,
+                              const int32_t* idx_r, const float* w_r, const void* v,
+                              const void* alpha, const void* beta, void* mem, const void* undo,
+                              const void* dy, float* dv, float* dalpha, float* dbeta, float* dw_w,
+                              float* dw_r, float* dM, sdm_stream_t stream);
+
 /* Reads (host pointer `code`, synchronising on `stream`) and clears the device
  * status word of the current device: 0 = no fault; bit 0 = a slot index outside
  * [0, N) was skipped; bit 1 = a slot list given to the recurrence was not strictly

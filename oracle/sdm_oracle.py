@@ -308,10 +308,10 @@ def recur_chunkwise(M: np.ndarray, idx_w, w_w, idx_r, w_r, v, alpha, beta, C: in
 # backward with in-place undo (App. A.3 "Memory-Efficient Backward")
 # --------------------------------------------------------------------------------------
 
-def recur_forward_undo(M: np.ndarray, idx_w, w_w, idx_r, w_r, v, alpha, beta):
-    """``recur`` with exact storage that also returns the undo log: for every token, the rows
-    M_{t-1}[I^w_t] its write overwrote.  M is updated in place to M_T.
-    Returns (y [T, d_v], undo [T, k_w, d_v])."""
+def recur_forward_undo(M: np.ndarray, idx_w, w_w, idx_r, w_r, v, alpha, beta, store: str = "f64"):
+    """``recur`` that also returns the undo log: for every token, the rows M_{t-1}[I^w_t] its
+    write overwrote (stored values).  M is updated in place to M_T; written rows are rounded to
+    ``store``.  Returns (y [T, d_v] float64 from the stored rows, undo [T, k_w, d_v])."""
     T = v.shape[0]
     y = np.empty((T, M.shape[1]))
     undo = np.empty((T, idx_w.shape[1], M.shape[1]))
@@ -320,7 +320,7 @@ def recur_forward_undo(M: np.ndarray, idx_w, w_w, idx_r, w_r, v, alpha, beta):
         undo[t] = M[iw]
         decayed = alpha[t] * M[iw]
         delta = v[t] - w_w[t] @ decayed
-        M[iw] = decayed + beta[t] * w_w[t][:, None] * delta[None, :]
+        M[iw] = round_storage(decayed + beta[t] * w_w[t][:, None] * delta[None, :], store)
         y[t] = w_r[t] @ M[idx_r[t]]
     return y, undo
 

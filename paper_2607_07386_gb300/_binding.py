@@ -74,6 +74,13 @@ def lib():
             L.sdm_lazy_workspace_bytes.argtypes = [_SHP]
             L.sdm_materialize.argtypes = [_SHP, _VP, _VP, _VP, _VP]
             L.sdm_materialize.restype = ctypes.c_int
+            L.sdm_undo_log_bytes.restype = ctypes.c_size_t
+            L.sdm_undo_log_bytes.argtypes = [_SHP]
+            L.sdm_recur_undo.argtypes = [_SHP, _I32P, _VP, _I32P, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP]
+            L.sdm_recur_undo.restype = ctypes.c_int
+            L.sdm_recur_backward.argtypes = [_SHP, _I32P, _VP, _I32P, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP,
+                                             _VP, _VP, _VP, _VP, _VP]
+            L.sdm_recur_backward.restype = ctypes.c_int
             L.sdm_gates.argtypes = [_SHP, ctypes.c_int32, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP]
             L.sdm_gates.restype = ctypes.c_int
             L.sdm_norm_gate.argtypes = [_SHP, _VP, _VP, _VP, ctypes.c_float, _VP, _VP]
@@ -196,6 +203,30 @@ def forward_lazy(shape: SdmShape, M0, touched, P_q, P_k, q, k, v, alpha, beta, m
 def materialize(shape: SdmShape, M0, touched, mem, stream=None):
     """sdm_materialize: write M0's rows into the untouched slots of mem."""
     _check(lib().sdm_materialize(ctypes.byref(shape), _ptr(M0), _ptr(touched), _ptr(mem), _stream(stream)))
+
+
+def undo_log_bytes(shape: SdmShape) -> int:
+    n = lib().sdm_undo_log_bytes(ctypes.byref(shape))
+    if n == 0 and shape.B * shape.H * shape.T * shape.k_write > 0:
+        raise SdmError(1, last_error())
+    return n
+
+
+def recur_undo(shape: SdmShape, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem, y, undo, workspace, stream=None,
+               workspace_nbytes=None):
+    """sdm_recur_undo: sdm_recur plus the undo log [B, H, T, k_write, d_v] of the backward."""
+    nb = workspace_nbytes if workspace_nbytes is not None else (_nbytes(workspace) or 0)
+    _check(lib().sdm_recur_undo(ctypes.byref(shape), _ptr(idx_w), _ptr(w_w), _ptr(idx_r), _ptr(w_r), _ptr(v),
+                                _ptr(alpha), _ptr(beta), _ptr(mem), _ptr(y), _ptr(undo), _ptr(workspace), nb,
+                                _stream(stream)))
+
+
+def recur_backward(shape: SdmShape, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem, undo, dy, dv, dalpha, dbeta,
+                   dw_w, dw_r, dM, stream=None):
+    """sdm_recur_backward: gradients of sum <dy, y>; restores mem from M_T to M_0 with the undo log."""
+    _check(lib().sdm_recur_backward(ctypes.byref(shape), _ptr(idx_w), _ptr(w_w), _ptr(idx_r), _ptr(w_r), _ptr(v),
+                                    _ptr(alpha), _ptr(beta), _ptr(mem), _ptr(undo), _ptr(dy), _ptr(dv),
+                                    _ptr(dalpha), _ptr(dbeta), _ptr(dw_w), _ptr(dw_r), _ptr(dM), _stream(stream)))
 
 
 def gates(shape: SdmShape, d_model: int, x, W_a, W_b, b_dt, A, alpha, beta, stream=None):

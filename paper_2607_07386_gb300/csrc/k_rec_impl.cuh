@@ -120,6 +120,8 @@ __global__ void __launch_bounds__(256) k_recur(const RecArgs a, int nsplit, cons
     const char* M0c = a.M0 ? static_cast<const char*>(a.M0) + (chain % a.H) * a.N * static_cast<int64_t>(rowbytes) + dbyte + c * 16
                            : Mc;
     const bool lazy = a.M0 != nullptr;
+    // undo log of the backward: the pre-write chunk of every written row, in storage bits
+    char* undo_c = a.undo ? static_cast<char*>(a.undo) + dbyte + c * 16 : nullptr;
     const char* vrange = static_cast<const char*>(a.v) + chain * a.T * static_cast<int64_t>(rowbytes) + dbyte;
     char* yb = static_cast<char*>(a.y) + chain * a.T * static_cast<int64_t>(rowbytes) + dbyte + c * 16;
     const int T = a.T;
@@ -261,6 +263,8 @@ __global__ void __launch_bounds__(256) k_recur(const RecArgs a, int nsplit, cons
             const uint32_t ar = (hr && !rfix) ? wring_c + (rr * KS + ((hr - 1) & 63)) * SLOTB : rslot + (KS + j) * SLOTB;
             fix |= rfix && okr;
             const uint4 mw = lds128(aw);
+            if (undo_c && okw[j])
+                *reinterpret_cast<uint4*>(undo_c + ((tok0 + t) * kw + g * SPT + j) * static_cast<int64_t>(rowbytes)) = mw;
             const uint4 mr = lds128(ar);
             float2 f[E2], h[E2];
             unpack16x2<D>(mw, f);
@@ -492,6 +496,8 @@ __global__ void __launch_bounds__(64) k_recur_split(const RecArgs a, int nsplit,
     const char* M0c = a.M0 ? static_cast<const char*>(a.M0) + (chain % a.H) * a.N * static_cast<int64_t>(rowbytes) + dbyte + c * 16
                            : Mc;
     const bool lazy = a.M0 != nullptr;
+    // undo log of the backward: the pre-write chunk of every written row, in storage bits
+    char* undo_c = a.undo ? static_cast<char*>(a.undo) + dbyte + c * 16 : nullptr;
     const char* vrange = static_cast<const char*>(a.v) + chain * a.T * static_cast<int64_t>(rowbytes) + dbyte;
     char* yb = static_cast<char*>(a.y) + chain * a.T * static_cast<int64_t>(rowbytes) + dbyte + c * 16;
     const int T = a.T;
@@ -623,7 +629,10 @@ __global__ void __launch_bounds__(64) k_recur_split(const RecArgs a, int nsplit,
                 int rw = ws - ((hw - 1) >> 6); rw += rw < 0 ? RING : 0;
                 const uint32_t aw = hw ? wring_c + (rw * KS + ((hw - 1) & 63)) * SLOTB : rslot + j * SLOTB;
                 float2 f[E2];
-                unpack16x2<D>(lds128(aw), f);
+                const uint4 mw = lds128(aw);
+                if (undo_c && okw[j])
+                    *reinterpret_cast<uint4*>(undo_c + ((tok0 + t) * kw + g * SPT + j) * static_cast<int64_t>(rowbytes)) = mw;
+                unpack16x2<D>(mw, f);
                 const float wj = okw[j] ? ww[j] : 0.f;
                 const float2 wj2 = make_float2(wj, wj);
 #pragma unroll

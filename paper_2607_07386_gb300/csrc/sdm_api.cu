@@ -343,6 +343,11 @@ sdm_status forward_impl(const char* who, const sdm_shape* s, const void* P_q, co
     return ok();
 }
 
+// sdm_recur with an optional undo log (defined after the C entry points).
+sdm_status recur_impl(const char* who, const sdm_shape* s, const int32_t* idx_w, const float* w_w,
+                      const int32_t* idx_r, const float* w_r, const void* v, const void* alpha, const void* beta,
+                      void* mem, void* y, void* undo, void* workspace, size_t workspace_bytes, sdm_stream_t stream);
+
 }  // namespace
 
 extern "C" {
@@ -535,6 +540,88 @@ size_t sdm_recur_workspace_bytes(const sdm_shape* s) {
 sdm_status sdm_recur(const sdm_shape* s, const int32_t* idx_w, const float* w_w, const int32_t* idx_r,
                      const float* w_r, const void* v, const void* alpha, const void* beta, void* mem, void* y,
                      void* workspace, size_t workspace_bytes, sdm_stream_t stream) {
+    return recur_impl("sdm_recur", s, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem, y, nullptr, workspace,
+                      workspace_bytes, stream);
+}
+
+size_t sdm_undo_log_bytes(const sdm_shape* s) {
+    if (check_shape(s, false, nullptr) != SDM_OK) return 0;
+    return static_cast<size_t>(s->B) * s->H * s->T * s->k_write * s->d_v * elem_bytes(s->dtype);
+}
+
+sdm_status sdm_recur_undo(const sdm_shape* s, const int32_t* idx_w, const float* w_w, const int32_t* idx_r,
+                          const float* w_r, const void* v, const void* alpha, const void* beta, void* mem, void* y,
+                          void* undo, void* workspace, size_t workspace_bytes, sdm_stream_t stream) {
+    if (s != nullptr && static_cast<size_t>(s->B) * s->H * s->T > 0 && undo == nullptr)
+        return fail(SDM_ERR_INVALID_ARG, "sdm_recur_undo: undo is NULL");
+    return recur_impl("sdm_recur_undo", s, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem, y, undo, workspace,
+                      workspace_bytes, stream);
+}
+
+sdm_status sdm_recur_backward(const sdm_shape* s, const int32_t* idx_w, const float* w_w, const int32_t* idx_r,
+                              const float* w_r, const void* v, const void* alpha, const void* beta, void* mem,
+                              const void* undo, const void* dy, float* dv, float* dalpha, float* dbeta, float* dw_w,
+                              float* dw_r, float* dM, sdm_stream_t stream) {
+    SDM_TRY(check_shape(s, false, nullptr));
+    if (s->d_v % 32 != 0 || s->d_v > 256)
+        return fail(SDM_ERR_UNSUPPORTED, "sdm_recur_backward: d_v must be a multiple of 32, at most 256 (d_v=%d)", s->d_v);
+    const size_t es = elem_bytes(s->dtype);
+    const size_t bht = static_cast<size_t>(s->B) * s->H * s->T;
+    if (bht == 0) return ok();
+    SDM_TRY(check_vec(idx_w, "idx_w", 4));
+    SDM_TRY(check_vec(w_w, "w_w", 4));
+    SDM_TRY(check_vec(idx_r, "idx_r", 4));
+    SDM_TRY(check_vec(w_r, "w_r", 4));
+    SDM_TRY(check_vec(v, "v", es));
+    SDM_TRY(check_vec(alpha, "alpha", es));
+    SDM_TRY(check_vec(beta, "beta", es));
+    SDM_TRY(check_vec(mem, "mem", 16));
+    SDM_TRY(check_vec(undo, "undo", 16));
+    SDM_TRY(check_vec(dy, "dy", es));
+    SDM_TRY(check_vec(dv, "dv", 4));
+    SDM_TRY(check_vec(dalpha, "dalpha", 4));
+    SDM_TRY(check_vec(dbeta, "dbeta", 4));
+    SDM_TRY(check_vec(dw_w, "dw_w", 4));
+    SDM_TRY(check_vec(dw_r, "dw_r", 4));
+    SDM_TRY(check_vec(dM, "dM", 4));
+    const size_t rowb = static_cast<size_t>(s->d_v) * es;
+    const size_t memb = static_cast<size_t>(s->B) * s->H * static_cast<size_t>(s->N) * rowb;
+    const Range outs[] = {{mem, memb, "mem"}, {dv, bht * s->d_v * 4, "dv"}, {dalpha, bht * 4, "dalpha"},
+                          {dbeta, bht * 4, "dbeta"}, {dw_w, bht * s->k_write * 4, "dw_w"},
+                          {dw_r, bht * s->k_read * 4, "dw_r"},
+                          {dM, static_cast<size_t>(s->B) * s->H * static_cast<size_t>(s->N) * s->d_v * 4, "dM"}};
+    const Range ins[] = {{idx_w, bht * s->k_write * 4, "idx_w"}, {w_w, bht * s->k_write * 4, "w_w"},
+                         {idx_r, bht * s->k_read * 4, "idx_r"}, {w_r, bht * s->k_read * 4, "w_r"},
+                         {v, bht * rowb, "v"}, {alpha, bht * es, "alpha"}, {beta, bht * es, "beta"},
+                         {undo, bht * s->k_write * rowb, "undo"}, {dy, bht * rowb, "dy"}};
+    for (size_t i = 0; i < sizeof(outs) / sizeof(outs[0]); ++i) {
+        for (const Range& r : ins)
+            if (overlaps(outs[i], r)) return fail(SDM_ERR_INVALID_ARG, "sdm_recur_backward: %s overlaps %s", outs[i].name, r.name);
+        for (size_t j = i + 1; j < sizeof(outs) / sizeof(outs[0]); ++j)
+            if (overlaps(outs[i], outs[j]))
+                return fail(SDM_ERR_INVALID_ARG, "sdm_recur_backward: %s overlaps %s", outs[i].name, outs[j].name);
+    }
+    int* err = nullptr;
+    SDM_TRY(status_word(&err));
+    sdm::RecArgs r{};
+    r.idx_w = idx_w; r.w_w = w_w; r.idx_r = idx_r; r.w_r = w_r;
+    r.v = v; r.alpha = alpha; r.beta = beta; r.mem = mem;
+    r.B = s->B; r.H = s->H; r.T = s->T; r.dv = s->d_v; r.kw = s->k_write; r.kr = s->k_read;
+    r.N = s->N;
+    r.err = err;
+    cudaError_t e = sdm::launch_recur_backward(s->dtype, r, undo, dy, dv, dalpha, dbeta, dw_w, dw_r, dM,
+                                               reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "backward launch");
+    return ok();
+}
+
+}  // extern "C"
+
+namespace {
+
+sdm_status recur_impl(const char* who, const sdm_shape* s, const int32_t* idx_w, const float* w_w,
+                      const int32_t* idx_r, const float* w_r, const void* v, const void* alpha, const void* beta,
+                      void* mem, void* y, void* undo, void* workspace, size_t workspace_bytes, sdm_stream_t stream) {
     SDM_TRY(check_shape(s, false, nullptr));
     const size_t es = elem_bytes(s->dtype);
     const size_t bht = static_cast<size_t>(s->B) * s->H * s->T;
@@ -555,13 +642,21 @@ sdm_status sdm_recur(const sdm_shape* s, const int32_t* idx_w, const float* w_w,
                             {v, bht * rowb, "v"}, {alpha, bht * es, "alpha"}, {beta, bht * es, "beta"},
                             {y, bht * rowb, "y"}};
     for (const Range& r : others)
-        if (overlaps(rm, r)) return fail(SDM_ERR_INVALID_ARG, "sdm_recur: mem overlaps %s", r.name);
+        if (overlaps(rm, r)) return fail(SDM_ERR_INVALID_ARG, "%s: mem overlaps %s", who, r.name);
     const size_t need = align256(sdm::rec_workspace_bytes(s->B, s->H, s->T, s->k_write, s->k_read));
-    if (!workspace) return fail(SDM_ERR_INVALID_ARG, "sdm_recur: workspace is NULL (need %zu bytes)", need);
-    if (!aligned(workspace, 256)) return fail(SDM_ERR_INVALID_ARG, "sdm_recur: workspace must be 256-byte aligned");
+    if (!workspace) return fail(SDM_ERR_INVALID_ARG, "%s: workspace is NULL (need %zu bytes)", who, need);
+    if (!aligned(workspace, 256)) return fail(SDM_ERR_INVALID_ARG, "%s: workspace must be 256-byte aligned", who);
     if (workspace_bytes < need)
-        return fail(SDM_ERR_INVALID_ARG, "sdm_recur: workspace too small (%zu < %zu bytes)", workspace_bytes, need);
-    if (overlaps(rm, Range{workspace, need, "workspace"})) return fail(SDM_ERR_INVALID_ARG, "sdm_recur: mem overlaps workspace");
+        return fail(SDM_ERR_INVALID_ARG, "%s: workspace too small (%zu < %zu bytes)", who, workspace_bytes, need);
+    if (overlaps(rm, Range{workspace, need, "workspace"})) return fail(SDM_ERR_INVALID_ARG, "%s: mem overlaps workspace", who);
+    if (undo != nullptr) {
+        SDM_TRY(check_vec(undo, "undo", 16));
+        const Range ru{undo, bht * s->k_write * rowb, "undo"};
+        if (overlaps(ru, rm) || overlaps(ru, Range{workspace, need, "workspace"}))
+            return fail(SDM_ERR_INVALID_ARG, "%s: undo overlaps mem or the workspace", who);
+        for (const Range& r : others)
+            if (overlaps(ru, r)) return fail(SDM_ERR_INVALID_ARG, "%s: undo overlaps %s", who, r.name);
+    }
     int* err = nullptr;
     SDM_TRY(status_word(&err));
     sdm::RecArgs r{};
@@ -570,10 +665,15 @@ sdm_status sdm_recur(const sdm_shape* s, const int32_t* idx_w, const float* w_w,
     r.B = s->B; r.H = s->H; r.T = s->T; r.dv = s->d_v; r.kw = s->k_write; r.kr = s->k_read;
     r.N = s->N;
     r.err = err;
+    r.undo = undo;
     cudaError_t e = sdm::launch_recur(s->dtype, r, static_cast<int32_t*>(workspace), reinterpret_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "recurrence launch");
     return ok();
 }
+
+}  // namespace
+
+extern "C" {
 
 sdm_status sdm_device_stats(uint32_t* counts, int n, sdm_stream_t stream) {
     if (!counts || n < 0 || n > 15) return fail(SDM_ERR_INVALID_ARG, "counts must be non-NULL and n in [0, 15]");

@@ -57,6 +57,8 @@ struct RecArgs {
     void* mem;                                // [B, H, N, dv]
     const void* M0;                           // [H, N, dv]: source of fresh rows (lazy initial
                                               // memory), or nullptr
+    void* undo;                               // [B, H, T, kw, dv]: rows each write overwrote (the
+                                              // backward's undo log), or nullptr
     void* y;                                  // [B, H, T, dv]
     int B, H, T, dv, kw, kr;
     int64_t N;
@@ -82,6 +84,11 @@ size_t rec_workspace_bytes(int B, int H, int T, int kw, int kr);
 // call (-1: written by an earlier call; INT_MAX: not written), see k_lazy.cu.
 cudaError_t launch_recur(int dtype, const RecArgs& a, int32_t* hz_ws, cudaStream_t stream,
                          const int32_t* firstw = nullptr);
+
+// Backward of the recurrence with in-place undo (k_recur_bwd.cu).  a.mem holds M_T on entry and
+// M_0 on return; dM ([B, H, N, dv] fp32, zero on entry) receives dL/dM_0 per chain.
+cudaError_t launch_recur_backward(int dtype, const RecArgs& a, const void* undo, const void* dy, float* dv,
+                                  float* dalpha, float* dbeta, float* dw_w, float* dw_r, float* dM, cudaStream_t stream);
 
 // ---------------------------------------------------------------- K-LAZY (k_lazy.cu)
 // firstw from the touched bitmap [chains, ceil(N/32)], then the first writer of every slot.

@@ -171,6 +171,24 @@ def test_gates_and_norm_gate_reject_bad_arguments(sdm):
     assert ng(shape=_shape(sdm, d_v=1024)) == 2 and "1024 bytes" in sdm.last_error()
 
 
+def test_backward_entry_points_reject_bad_arguments(sdm):
+    s = _shape(sdm)
+    L = sdm.lib()
+    assert sdm.undo_log_bytes(s) == 2 * 2 * 16 * 8 * 32 * 2
+    base = [FAKE, FAKE + 0x100000, FAKE + 0x200000, FAKE + 0x300000, FAKE + 0x400000, FAKE + 0x500000,
+            FAKE + 0x600000, FAKE + 0x10000000, FAKE + 0x700000]
+    assert L.sdm_recur_undo(ctypes.byref(s), *base, None, FAKE + 0x40000000, 1 << 30, None) == 1
+    assert "undo is NULL" in sdm.last_error()
+    assert L.sdm_recur_undo(ctypes.byref(s), *base, FAKE + 0x10000000 + 256, FAKE + 0x40000000, 1 << 30, None) == 1
+    assert "undo overlaps" in sdm.last_error()
+    outs = [FAKE + 0x20000000 + i * 0x1000000 for i in range(6)]
+    bw = lambda shape, **o: L.sdm_recur_backward(ctypes.byref(shape), *base[:8], o.get("undo", FAKE + 0x800000),
+                                                 FAKE + 0x900000, *outs, None)
+    assert bw(_shape(sdm, d_v=48)) == 2 and "multiple of 32" in sdm.last_error()
+    assert bw(s, undo=None) == 1 and "undo is NULL" in sdm.last_error()
+    assert bw(s, undo=FAKE + 0x10000000) == 1 and "mem overlaps undo" in sdm.last_error()
+
+
 def test_decode_step_requires_T_equal_1(sdm):
     s = _shape(sdm, T=2)
     L = sdm.lib()

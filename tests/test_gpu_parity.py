@@ -481,6 +481,65 @@ def test_forward_lazy_one_token_per_call_equals_one_call(sdm):
     assert torch.equal(step["mem"], whole["mem"])
 
 
+# ------------------------------------------------------------------ backward with in-place undo
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_recur_backward_with_undo_matches_the_oracle(sdm, dtype):
+    """sdm_recur_undo gives sdm_recur's y and memory bit for bit plus an undo log;
+    sdm_recur_backward restores the memory to M_0 bit for bit and its gradients match the
+    oracle's backward through the same (stored-value) recurrence.  Tolerance: fp32 arithmetic
+    against float64 (1e-4), and for bf16 the rare rows whose rounding flips between the fp32
+    and float64 forwards (one ulp, 2^-8)."""
+    # k_read 12 runs the writer/reader kernel, 20 the fused one (both write the undo log)
+    B, H, N, T, kw, kr = 2, 1, 400, 90, 8, (12 if dtype == "f32" else 20)
+    dv = 64 if dtype == "f32" else 128
+    rng = np.random.default_rng(71)
+    M0 = O.round_storage(rng.standard_normal((B * H, N, dv)) * 0.3, dtype)
+    iw = np.stack([np.sort(rng.choice(N, kw, replace=False)) for _ in range(B * H * T)]).reshape(B, H, T, kw)
+    ir = np.stack([np.sort(rng.choice(N, kr, replace=False)) for _ in range(B * H * T)]).reshape(B, H, T, kr)
+    ww = rng.dirichlet(np.ones(kw), B * H * T).astype(np.float32).reshape(B, H, T, kw)
+    wr = rng.dirichlet(np.ones(kr), B * H * T).astype(np.float32).reshape(B, H, T, kr)
+    a = O.round_storage(1 / (1 + np.exp(-rng.standard_normal((B, H, T)) - 2)), dtype)
+    b = O.round_storage(1 / (1 + np.exp(-rng.standard_normal((B, H, T)))), dtype)
+    V = O.round_storage(rng.standard_normal((B, H, T, dv)), dtype)
+    dY = O.round_storage(rng.standard_normal((B, H, T, dv)), dtype)
+    st = lambda x: to_torch(O.to_bf16_bits(x) if dtype == "bf16" else x.astype(np.float32), dtype)
+    shape = sdm.SdmShape.make(B, H, T, 32, dv, N, kw, kr, dtype)
+    cu = lambda x: torch.from_numpy(np.ascontiguousarray(x)).cuda()
+    tiw, tir, tww, twr = cu(iw.astype(np.int32)), cu(ir.astype(np.int32)), cu(ww), cu(wr)
+    tv, ta, tb, tdy = st(V), st(a), st(b), st(dY)
+    mem = st(M0.reshape(B, H, N, dv))
+    mem_plain = mem.clone()
+    y = torch.empty((B, H, T, dv), dtype=mem.dtype, device="cuda")
+    y_plain = torch.empty_like(y)
+    undo = torch.empty(sdm.undo_log_bytes(shape), dtype=torch.uint8, device="cuda")
+    rws = torch.empty(sdm.recur_workspace_bytes(shape), dtype=torch.uint8, device="cuda")
+    sdm.recur_undo(shape, tiw, tww, tir, twr, tv, ta, tb, mem, y, undo, rws)
+    sdm.recur(shape, tiw, tww, tir, twr, tv, ta, tb, mem_plain, y_plain, rws)
+    torch.cuda.synchronize()
+    assert torch.equal(y, y_plain) and torch.equal(mem, mem_plain)
+    f32 = lambda *s_: torch.zeros(s_, dtype=torch.float32, device="cuda")
+    g_dv, g_da, g_db = f32(B, H, T, dv), f32(B, H, T), f32(B, H, T)
+    g_ww, g_wr, g_dM = f32(B, H, T, kw), f32(B, H, T, kr), f32(B, H, N, dv)
+    sdm.recur_backward(shape, tiw, tww, tir, twr, tv, ta, tb, mem, undo, tdy, g_dv, g_da, g_db, g_ww, g_wr, g_dM)
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    assert torch.equal(mem, st(M0.reshape(B, H, N, dv)))          # the undo restored M_0 exactly
+    tol = 1e-4 if dtype == "f32" else 5e-3
+    for c in range(B * H):
+        bb, hh = divmod(c, H)
+        Mo = M0[c].copy()
+        _, und = O.recur_forward_undo(Mo, iw[bb, hh], ww[bb, hh].astype(np.float64), ir[bb, hh],
+                                      wr[bb, hh].astype(np.float64), V[bb, hh], a[bb, hh], b[bb, hh], dtype)
+        g = O.recur_backward(Mo, und, iw[bb, hh], ww[bb, hh].astype(np.float64), ir[bb, hh],
+                             wr[bb, hh].astype(np.float64), V[bb, hh], a[bb, hh], b[bb, hh], dY[bb, hh])
+        for name, got in (("dv", g_dv), ("dalpha", g_da), ("dbeta", g_db), ("dw_w", g_ww), ("dw_r", g_wr),
+                          ("dM0", g_dM)):
+            e = rel_fro(got[bb, hh].cpu().numpy().astype(np.float64), g[name])
+            assert e <= tol, (dtype, c, name, e)
+
+
 # ------------------------------------------------------------------ gates and output epilogue
 
 def _storage_ulp(ref: np.ndarray, dtype: str) -> np.ndarray:
