@@ -222,6 +222,18 @@ sdm_status sdm_recur(const sdm_shape* shape, const int32_t* idx_w, const float* 
                      const void* alpha, const void* beta, void* mem, void* y,
                      void* workspace, size_t workspace_bytes, sdm_stream_t stream);
 
+/* The recurrence of sdm_recur in chunkwise (WY) form (App. A.1-A.2): per chunk of `chunk`
+ * tokens (1..32), segmented cumulative log-decays, gated sparse inner products by two-pointer
+ * merge, a unit lower-triangular solve, then gather, correct, output and scatter against the
+ * chunk-initial memory.  The memory is rounded to the storage dtype at chunk boundaries only
+ * and reads inside a chunk see its unrounded writes, so results differ from sdm_recur's by
+ * storage rounding alone (chunk = 1: reads of slots the same token writes).  Arguments and
+ * layouts as in sdm_recur (no workspace); d_v <= 256, k_write, k_read <= 64. */
+sdm_status sdm_recur_chunkwise(const sdm_shape* shape, const int32_t* idx_w, const float* w_w,
+                               const int32_t* idx_r, const float* w_r, const void* v,
+                               const void* alpha, const void* beta, void* mem, void* y,
+                               int32_t chunk, sdm_stream_t stream);
+
 /* Bytes of the undo log of sdm_recur_undo: B*H*T*k_write rows of d_v storage elements. */
 size_t sdm_undo_log_bytes(const sdm_shape* shape);
 

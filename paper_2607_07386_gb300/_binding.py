@@ -74,6 +74,8 @@ def lib():
             L.sdm_lazy_workspace_bytes.argtypes = [_SHP]
             L.sdm_materialize.argtypes = [_SHP, _VP, _VP, _VP, _VP]
             L.sdm_materialize.restype = ctypes.c_int
+            L.sdm_recur_chunkwise.argtypes = [_SHP, _I32P, _VP, _I32P, _VP, _VP, _VP, _VP, _VP, _VP, ctypes.c_int32, _VP]
+            L.sdm_recur_chunkwise.restype = ctypes.c_int
             L.sdm_undo_log_bytes.restype = ctypes.c_size_t
             L.sdm_undo_log_bytes.argtypes = [_SHP]
             L.sdm_recur_undo.argtypes = [_SHP, _I32P, _VP, _I32P, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP]
@@ -203,6 +205,12 @@ def forward_lazy(shape: SdmShape, M0, touched, P_q, P_k, q, k, v, alpha, beta, m
 def materialize(shape: SdmShape, M0, touched, mem, stream=None):
     """sdm_materialize: write M0's rows into the untouched slots of mem."""
     _check(lib().sdm_materialize(ctypes.byref(shape), _ptr(M0), _ptr(touched), _ptr(mem), _stream(stream)))
+
+
+def recur_chunkwise(shape: SdmShape, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem, y, chunk: int, stream=None):
+    """sdm_recur_chunkwise: the recurrence in chunkwise (WY) form, chunks of `chunk` <= 32 tokens."""
+    _check(lib().sdm_recur_chunkwise(ctypes.byref(shape), _ptr(idx_w), _ptr(w_w), _ptr(idx_r), _ptr(w_r), _ptr(v),
+                                     _ptr(alpha), _ptr(beta), _ptr(mem), _ptr(y), int(chunk), _stream(stream)))
 
 
 def undo_log_bytes(shape: SdmShape) -> int:

@@ -544,6 +544,21 @@ sdm_status sdm_recur(const sdm_shape* s, const int32_t* idx_w, const float* w_w,
                       workspace_bytes, stream);
 }
 
+sdm_status sdm_recur_chunkwise(const sdm_shape* s, const int32_t* idx_w, const float* w_w, const int32_t* idx_r,
+                               const float* w_r, const void* v, const void* alpha, const void* beta, void* mem,
+                               void* y, int32_t chunk, sdm_stream_t stream) {
+    if (chunk < 1 || chunk > 32) return fail(SDM_ERR_INVALID_ARG, "sdm_recur_chunkwise: chunk must be in [1, 32] (got %d)", chunk);
+    if (s != nullptr && s->d_v > 256)
+        return fail(SDM_ERR_UNSUPPORTED, "sdm_recur_chunkwise: d_v > 256 is not supported (d_v=%d)", s->d_v);
+    sdm::RecArgs r{};
+    bool empty = false;
+    SDM_TRY(sdm::recur_args("sdm_recur_chunkwise", s, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem, y, &r, &empty));
+    if (empty) return ok();
+    cudaError_t e = sdm::launch_recur_chunkwise(s->dtype, r, chunk, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "chunkwise recurrence launch");
+    return ok();
+}
+
 size_t sdm_undo_log_bytes(const sdm_shape* s) {
     if (check_shape(s, false, nullptr) != SDM_OK) return 0;
     return static_cast<size_t>(s->B) * s->H * s->T * s->k_write * s->d_v * elem_bytes(s->dtype);

@@ -90,6 +90,10 @@ cudaError_t launch_recur(int dtype, const RecArgs& a, int32_t* hz_ws, cudaStream
 cudaError_t launch_recur_backward(int dtype, const RecArgs& a, const void* undo, const void* dy, float* dv,
                                   float* dalpha, float* dbeta, float* dw_w, float* dw_r, float* dM, cudaStream_t stream);
 
+// Chunkwise (WY) form of the recurrence (k_chunk.cu), chunks of C <= 32 tokens; d_v <= 256.
+cudaError_t launch_recur_chunkwise(int dtype, const RecArgs& a, int C, cudaStream_t stream);
+size_t chunk_smem_bytes(int C, int kw, int kr, int dv);
+
 // ---------------------------------------------------------------- K-LAZY (k_lazy.cu)
 // firstw from the touched bitmap [chains, ceil(N/32)], then the first writer of every slot.
 cudaError_t launch_lazy_prepare(const uint32_t* touched, int32_t* firstw, const int32_t* idx_w, int64_t chains, int T,

@@ -481,6 +481,50 @@ def test_forward_lazy_one_token_per_call_equals_one_call(sdm):
     assert torch.equal(step["mem"], whole["mem"])
 
 
+# ------------------------------------------------------------------ chunkwise (WY) form
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("dtype,C", [("f32", 1), ("f32", 8), ("f32", 32), ("bf16", 16), ("bf16", 32)])
+def test_recur_chunkwise_matches_the_chunkwise_oracle(sdm, dtype, C):
+    """sdm_recur_chunkwise against the oracle's chunkwise form with the same chunk size (both round
+    the memory at chunk boundaries only); T = 75 leaves a ragged last chunk and N = 60 makes slots
+    collide within chunks.  Tolerance: fp32 forward substitution over C rows with fast
+    exponentials (C^2 2^-24 < 1e-4); bf16 storage rounding (2e-3)."""
+    B, H, N, T, kw, kr = 2, 2, 60, 75, 8, 6
+    dv = 64 if dtype == "f32" else 128
+    rng = np.random.default_rng(81 + C)
+    M0 = O.round_storage(rng.standard_normal((B * H, N, dv)) * 0.3, dtype)
+    iw = np.stack([np.sort(rng.choice(N, kw, replace=False)) for _ in range(B * H * T)]).reshape(B, H, T, kw)
+    ir = np.stack([np.sort(rng.choice(N, kr, replace=False)) for _ in range(B * H * T)]).reshape(B, H, T, kr)
+    ww = rng.dirichlet(np.ones(kw), B * H * T).astype(np.float32).reshape(B, H, T, kw)
+    wr = rng.dirichlet(np.ones(kr), B * H * T).astype(np.float32).reshape(B, H, T, kr)
+    a = O.round_storage(1 / (1 + np.exp(-rng.standard_normal((B, H, T)) - 2)), dtype)
+    b = O.round_storage(1 / (1 + np.exp(-rng.standard_normal((B, H, T)))), dtype)
+    V = O.round_storage(rng.standard_normal((B, H, T, dv)), dtype)
+    st = lambda x: to_torch(O.to_bf16_bits(x) if dtype == "bf16" else x.astype(np.float32), dtype)
+    cu = lambda x: torch.from_numpy(np.ascontiguousarray(x)).cuda()
+    shape = sdm.SdmShape.make(B, H, T, 32, dv, N, kw, kr, dtype)
+    mem = st(M0.reshape(B, H, N, dv))
+    y = torch.empty((B, H, T, dv), dtype=mem.dtype, device="cuda")
+    sdm.recur_chunkwise(shape, cu(iw.astype(np.int32)), cu(ww), cu(ir.astype(np.int32)), cu(wr), st(V), st(a), st(b),
+                        mem, y, C)
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    tol = 1e-4 if dtype == "f32" else TOL["bf16"]
+    gy = O.to_f64(G.host(y, dtype), dtype)
+    gm = O.to_f64(G.host(mem, dtype), dtype)
+    for c in range(B * H):
+        bb, hh = divmod(c, H)
+        Mo = M0[c].copy()
+        _, yo = O.recur_chunkwise(Mo, iw[bb, hh], ww[bb, hh].astype(np.float64), ir[bb, hh],
+                                  wr[bb, hh].astype(np.float64), V[bb, hh], a[bb, hh], b[bb, hh], C, dtype)
+        assert rel_fro(gy[bb, hh], yo) <= tol, (dtype, C, c, rel_fro(gy[bb, hh], yo))
+        assert rel_fro(gm[bb, hh], Mo) <= tol, (dtype, C, c)
+        untouched = np.setdiff1d(np.arange(N), iw[bb, hh].ravel())
+        assert np.array_equal(G.host(mem, dtype)[bb, hh][untouched],
+                              (O.to_bf16_bits(M0[c]) if dtype == "bf16" else M0[c].astype(np.float32))[untouched])
+
+
 # ------------------------------------------------------------------ backward with in-place undo
 
 @pytest.mark.gpu
