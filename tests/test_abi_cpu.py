@@ -189,6 +189,19 @@ def test_backward_entry_points_reject_bad_arguments(sdm):
     assert bw(s, undo=FAKE + 0x10000000) == 1 and "mem overlaps undo" in sdm.last_error()
 
 
+def test_chunkwise_rejects_bad_chunks_and_rows(sdm):
+    s = _shape(sdm)
+    L = sdm.lib()
+    args = [FAKE, FAKE + 0x100000, FAKE + 0x200000, FAKE + 0x300000, FAKE + 0x400000, FAKE + 0x500000,
+            FAKE + 0x600000, FAKE + 0x10000000, FAKE + 0x700000]
+    assert L.sdm_recur_chunkwise(ctypes.byref(s), *args, 0, None) == 1 and "[1, 32]" in sdm.last_error()
+    assert L.sdm_recur_chunkwise(ctypes.byref(s), *args, 33, None) == 1 and "[1, 32]" in sdm.last_error()
+    wide = _shape(sdm, d_v=512)
+    assert L.sdm_recur_chunkwise(ctypes.byref(wide), *args, 8, None) == 2 and "d_v > 256" in sdm.last_error()
+    assert L.sdm_recur_chunkwise(ctypes.byref(s), *args[:7], FAKE + 0x100000, FAKE + 0x700000, 8, None) == 1
+    assert "mem overlaps" in sdm.last_error()
+
+
 def test_decode_step_requires_T_equal_1(sdm):
     s = _shape(sdm, T=2)
     L = sdm.lib()
