@@ -73,7 +73,7 @@ __all__ = [
     "recur", "forward_slice", "state_elements_per_layer", "n_global_layers",
     "touched_mask", "recur_lazy", "materialize", "eff_keys_fraction", "cumulative_mass", "unique_fraction",
     "softplus", "gates", "norm_gate", "head_mix", "sparse_ip", "recur_chunkwise",
-    "recur_forward_undo", "recur_backward",
+    "recur_forward_undo", "recur_backward", "round_e4m3", "quantize_undo",
 ]
 
 
@@ -369,6 +369,31 @@ def recur_backward(M: np.ndarray, undo, idx_w, w_w, idx_r, w_r, v, alpha, beta, 
         dM0[i] = g
     out["dM0"] = dM0
     return out
+
+
+def round_e4m3(x: np.ndarray) -> np.ndarray:
+    """Nearest fp8 e4m3 value (ties to even) of x, |x| <= 448: 4 significant bits for
+    |x| >= 2^-6, a fixed step of 2^-9 below (subnormals)."""
+    x = np.asarray(x, dtype=np.float64)
+    _, e = np.frexp(x)
+    q = np.ldexp(1.0, np.maximum(e - 4, -9))
+    return np.rint(x / q) * q
+
+
+def quantize_undo(undo: np.ndarray, kind: str) -> np.ndarray:
+    """The undo log as a quantised snapshot would give it back (App. A.3: fp8 or int4 snapshots
+    for long sequences), one scale per logged row: "fp8" rounds row / s to e4m3 with
+    s = max|row| / 448; "int4" rounds row / s to the integers -7..7 with s = max|row| / 7;
+    "exact" returns the log unchanged."""
+    u = np.asarray(undo, dtype=np.float64)
+    if kind == "exact":
+        return u.copy()
+    top = {"fp8": 448.0, "int4": 7.0}[kind]
+    amax = np.max(np.abs(u), axis=-1, keepdims=True)
+    scale = np.where(amax > 0, amax / top, 1.0)
+    y = u / scale
+    q = round_e4m3(y) if kind == "fp8" else np.clip(np.rint(y), -7, 7)
+    return q * scale
 
 
 # --------------------------------------------------------------------------------------

@@ -389,6 +389,40 @@ def test_backward_finite_differences():
     assert abs((loss(m0=M0 + E) - loss(m0=M0 - E)) / (2 * h) - g["dM0"][i, 0]) < 1e-7
 
 
+def test_e4m3_rounding_equals_torch_float8():
+    torch = pytest.importorskip("torch")
+    if not hasattr(torch, "float8_e4m3fn"):
+        pytest.skip("torch without float8")
+    rng = np.random.default_rng(64)
+    x = np.concatenate([rng.standard_normal(4000) * 10.0 ** rng.integers(-4, 3, 4000),
+                        [0.0, 448.0, -448.0, 2.0 ** -6, 2.0 ** -9, 2.0 ** -10, 1.0625, 1.1875, 3 * 2.0 ** -10]])
+    x = np.clip(x, -448.0, 448.0).astype(np.float32).astype(np.float64)
+    ref = torch.from_numpy(x.astype(np.float32)).to(torch.float8_e4m3fn).to(torch.float64).numpy()
+    assert np.array_equal(O.round_e4m3(x), ref)
+
+
+def test_quantized_undo_log_bounds_and_effect_on_gradients():
+    """A quantised snapshot (App. A.3) restores each logged row within half a quantisation step
+    (fp8: 2^-4 relative to the row's largest entry at worst; int4: max|row| / 14); the backward
+    then restores an approximate M_0, and its gradients move further from the exact ones for the
+    coarser format."""
+    rng = np.random.default_rng(65)
+    M0, idx_w, w_w, idx_r, w_r, V, alpha, beta = _random_sparse_case(rng, N=30, T=40, kw=4, kr=3)
+    dy = rng.standard_normal(V.shape)
+    M = M0.copy()
+    _, undo = O.recur_forward_undo(M, idx_w, w_w, idx_r, w_r, V, alpha, beta)
+    amax = np.max(np.abs(undo), axis=-1, keepdims=True)
+    assert np.all(np.abs(O.quantize_undo(undo, "fp8") - undo) <= amax * 2.0 ** -4 + 1e-300)
+    assert np.all(np.abs(O.quantize_undo(undo, "int4") - undo) <= amax / 14 * (1 + 1e-12))
+    assert np.array_equal(O.quantize_undo(undo, "exact"), undo)
+    ref = O.recur_backward(M.copy(), undo, idx_w, w_w, idx_r, w_r, V, alpha, beta, dy)
+    err = {}
+    for kind in ("fp8", "int4"):
+        g = O.recur_backward(M.copy(), O.quantize_undo(undo, kind), idx_w, w_w, idx_r, w_r, V, alpha, beta, dy)
+        err[kind] = max(np.linalg.norm(g[n] - ref[n]) / np.linalg.norm(ref[n]) for n in ("dv", "dalpha", "dw_w", "dM0"))
+    assert 0 < err["fp8"] < err["int4"] and err["fp8"] < 0.1
+
+
 # ------------------------------------------------------------------ lazy M0 (copy-on-write)
 
 def test_lazy_overlay_equals_dense_masked_form():
