@@ -74,7 +74,8 @@ def _brute_topk(s1, s2, k):
 
 
 @pytest.mark.parametrize("S,k,integer", [(8, 3, False), (16, 8, False), (16, 8, True), (32, 16, True),
-                                         (8, 8, True), (64, 8, False), (5, 5, True)])
+                                         (8, 8, True), (64, 8, False), (5, 5, True), (1, 1, False),
+                                         (2, 2, True), (3, 1, True)])
 def test_pkm_two_stage_equals_brute_force(S, k, integer):
     rng = np.random.default_rng(S * 100 + k)
     T = 200
@@ -103,6 +104,12 @@ def test_address_projected_end_to_end_brute_force():
     s = X @ P.T
     for t in range(T):
         assert np.array_equal(idx[t], _brute_topk(s[t, :S], s[t, S:], k))
+
+
+def test_address_of_no_tokens_is_empty():
+    P = np.ones((8, 3))
+    idx, score, w = O.address(P, np.zeros((0, 3)), 16, 2)
+    assert idx.shape == (0, 2) and score.shape == (0, 2) and w.shape == (0, 2)
 
 
 def test_address_direct_mode_uses_x_halves():
