@@ -455,8 +455,12 @@ def run_ours(args, cfg):
         "gpu_launches": kernels_per_step * args.steps,
         "roofline": {"bound": "hbm", "kernel": "k_recur", "achieved": achieved, "peak": peaks["hbm_gbs"],
                      "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
-                     "traffic": RECUR_DRAM_BYTES_PER_TOKEN_HEAD * B * H * T if cfg.name == "layer_1p4b" else None,
-                     "traffic_source": "ncu dram bytes of the hazard pass + recurrence at B=2, scaled to B*H*T",
+                     # the DRAM counters were taken with one warp per CTA; the kernel now groups four
+                     # d-range warps of a chain per CTA, so the count is withheld until re-captured
+                     "traffic": None,
+                     "traffic_last_capture": RECUR_DRAM_BYTES_PER_TOKEN_HEAD * B * H * T if cfg.name == "layer_1p4b" else None,
+                     "traffic_source": "ncu dram bytes of the hazard pass + recurrence at B=2 (one warp per CTA), "
+                                       "scaled to B*H*T; not of the current launch shape",
                      "peak_source": peaks["source"], "bytes_per_launch": rec_bytes, "ms_per_launch": rec_ms},
         "phase_ms": ph,
         "lazy_m0": lazy,
