@@ -147,17 +147,31 @@ def _oracle_step(pool, cfg, slices, T):
     return max(pool.map(timed_worker, [(cfg, b, h, T) for b, h in slices]))
 
 
-def cpu_baseline(cfg, T=1024):
-    """Oracle throughput on a bounded sample: one (b, h) slice x T tokens per core; tokens/s
-    per layer = slice-tokens / H / time (slices are independent, so per-core work adds up)."""
+# The oracle sample, the same for the cpu_baseline key and the reference arm: each step runs
+# one (b, h) slice per host core over the slice's first ORACLE_T tokens.  Both legs measure
+# this one sample size, so they time the same work (the oracle's per-slice set-up, a float64
+# copy of the head's M0, is amortised over the same number of tokens).
+ORACLE_T = 512
+
+
+def _oracle_sample(cfg, pool, cores, steps, seed):
+    rng = np.random.default_rng(seed)
+    times = []
+    for _ in range(steps):
+        slices = [(int(rng.integers(cfg.B)), int(rng.integers(cfg.H))) for _ in range(cores)]
+        times.append(_oracle_step(pool, cfg, slices, ORACLE_T))
+    return cores * ORACLE_T / cfg.H * len(times) / sum(times), times
+
+
+def cpu_baseline(cfg):
+    """Oracle throughput on a bounded sample: one (b, h) slice x ORACLE_T tokens per core;
+    tokens/s per layer = slice-tokens / H / time (slices are independent, so per-core work adds up)."""
     cores = os.cpu_count() or 1
-    rng = np.random.default_rng(0)
-    slices = [(int(rng.integers(cfg.B)), int(rng.integers(cfg.H))) for _ in range(cores)]
     with _oracle_pool(cores) as pool:
-        dt = _oracle_step(pool, cfg, slices, T)
-    return {"value": cores * T / cfg.H / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
-            "sample": f"{cores} (b,h) slices x first {T} tokens of {cfg.name}, one float64 worker per core, "
-                      f"{dt:.1f} s (slowest worker, input generation excluded)"}
+        value, times = _oracle_sample(cfg, pool, cores, 1, 0)
+    return {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"{cores} (b,h) slices x first {ORACLE_T} tokens of {cfg.name}, one float64 worker per core, "
+                      f"{times[0]:.1f} s (slowest worker, input generation excluded)"}
 
 
 def run_reference(args, cfg):
@@ -165,16 +179,11 @@ def run_reference(args, cfg):
     if rank != 0:
         return
     cores = os.cpu_count() or 1
-    T = 256
-    rng = np.random.default_rng(1)
-    times = []
+    T = ORACLE_T
     with _oracle_pool(cores) as pool:
         for _ in range(args.warmup):
             _oracle_step(pool, cfg, [(0, 0)], 32)
-        for _ in range(args.steps):
-            slices = [(int(rng.integers(cfg.B)), int(rng.integers(cfg.H))) for _ in range(cores)]
-            times.append(_oracle_step(pool, cfg, slices, T))
-    value = cores * T / cfg.H * len(times) / sum(times)
+        value, times = _oracle_sample(cfg, pool, cores, args.steps, 1)
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * sum(times) / len(times),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",

@@ -45,7 +45,7 @@
 extern "C" {
 #endif
 
-#define SDM_ABI_VERSION 1
+#define SDM_ABI_VERSION 2
 
 /* Same type as cudaStream_t. */
 typedef struct CUstream_st* sdm_stream_t;
@@ -54,10 +54,10 @@ typedef enum {
     SDM_OK = 0,
     SDM_ERR_INVALID_ARG = 1,   /* bad shape, null pointer, misalignment, aliasing, small workspace */
     SDM_ERR_UNSUPPORTED = 2,   /* valid SDM shape this build has no kernel for (see sdm_last_error) */
-    SDM_ERR_OOM = 3,           /* reserved: the library itself never allocates */
+    /* 3 is not used: the library never allocates device memory, so it has no out-of-memory code */
     SDM_ERR_CUDA = 4,          /* a CUDA runtime call or launch failed (message has cudaGetErrorString) */
-    SDM_ERR_TIMEOUT = 5,       /* reserved for bounded device waits */
-    SDM_ERR_DEVICE = 6         /* device status word reported a bad slot index (sdm_device_status) */
+    SDM_ERR_TIMEOUT = 5,       /* sdm_device_status: a bounded device wait gave up (status bit 2) */
+    SDM_ERR_DEVICE = 6         /* sdm_device_status: any other device-side fault bit was set */
 } sdm_status;
 
 typedef enum { SDM_F32 = 0, SDM_BF16 = 1 } sdm_dtype;
@@ -228,7 +228,10 @@ sdm_status sdm_recur(const sdm_shape* shape, const int32_t* idx_w, const float* 
  * chunk-initial memory.  The memory is rounded to the storage dtype at chunk boundaries only
  * and reads inside a chunk see its unrounded writes, so results differ from sdm_recur's by
  * storage rounding alone (chunk = 1: reads of slots the same token writes).  Arguments and
- * layouts as in sdm_recur (no workspace); d_v <= 256, k_write, k_read <= 64. */
+ * layouts as in sdm_recur (no workspace); d_v <= 256, k_write, k_read <= 64.  Slot lists
+ * must be strictly ascending (the two-pointer merges rely on it); a violation sets bit 1
+ * of the device status word and leaves the results undefined.  A gate alpha of exactly 0
+ * decays by e^-80 (below fp32 precision of any stored value) instead of 0. */
 sdm_status sdm_recur_chunkwise(const sdm_shape* shape, const int32_t* idx_w, const float* w_w,
                                const int32_t* idx_r, const float* w_r, const void* v,
                                const void* alpha, const void* beta, void* mem, void* y,
@@ -255,7 +258,8 @@ sdm_status sdm_recur_undo(const sdm_shape* shape, const int32_t* idx_w, const fl
  * [B, H, T, k_write], dw_r [B, H, T, k_read]; dM [B, H, N, d_v] float32 must be zero on
  * entry and receives dL/dM_0 per sequence (sum over b for a shared M0).  Other arguments as
  * in sdm_recur.  d_v must be a multiple of 32, at most 256.  Outputs must not overlap each
- * other or the inputs. */
+ * other or the inputs.  Slot lists must be strictly ascending, as in sdm_recur; a violation
+ * sets bit 1 of the device status word. */
 sdm_status sdm_recur_backward(const sdm_shape* shape, const int32_t* idx_w, const float* w_w,
                               const int32_t* idx_r, const float* w_r, const void* v,
                               const void* alpha, const void* beta, void* mem, const void* undo,
@@ -264,11 +268,13 @@ sdm_status sdm_recur_backward(const sdm_shape* shape, const int32_t* idx_w, cons
 
 /* Reads (host pointer `code`, synchronising on `stream`) and clears the device
  * status word of the current device: 0 = no fault; bit 0 = a slot index outside
- * [0, N) was skipped; bit 1 = a slot list given to the recurrence was not strictly
- * ascending; bit 2 = a bounded wait of the tensor-core score kernel gave up (its
- * results are undefined); bit 3 = a selection invariant failed (a candidate list not
- * ordered by score; results undefined).  Returns SDM_ERR_DEVICE when the word was
- * non-zero. */
+ * [0, N) was skipped; bit 1 = a slot list given to the recurrence (forward, chunkwise
+ * or backward) was not strictly ascending; bit 2 = a bounded device wait gave up (the
+ * tensor-core score kernel's mbarrier waits, or the writer/reader hand-over of the
+ * recurrence): the kernel returned early and its results are undefined; bit 3 = a
+ * selection invariant failed (a candidate list not ordered by score; results
+ * undefined).  Returns SDM_ERR_TIMEOUT when bit 2 was set, else SDM_ERR_DEVICE when the
+ * word was non-zero, else SDM_OK; *code always receives the whole word. */
 sdm_status sdm_device_status(int32_t* code, sdm_stream_t stream);
 
 /* Size of the fixed device scratch behind sdm_recur_noalloc (its hazard table). */
@@ -278,11 +284,13 @@ sdm_status sdm_device_status(int32_t* code, sdm_stream_t stream);
  * SDM_RECUR_NOALLOC_SCRATCH_BYTES reserved by the library (the paper has no counterpart;
  * this serves callers that cannot provide device memory, e.g. a runtime whose own pool
  * owns the device, or a serving loop that must not call an allocator).  Same arguments,
- * layouts and results as sdm_recur.  Needs B*H*T*max(k_write,k_read)*4 bytes of that
- * scratch; larger shapes return SDM_ERR_UNSUPPORTED before launching anything.  Allocates
- * nothing.  The first call on a device looks the array's address up (host-side set-up;
- * make that first call before any stream capture).  One array per device: calls that
- * overlap on the GPU race on it and must be serialised by the caller. */
+ * layouts and results as sdm_recur, bit for bit.  Needs B*H*T*max(k_write,k_read)*4 bytes
+ * of that scratch; larger shapes return SDM_ERR_UNSUPPORTED before launching anything.
+ * Allocates nothing.  The first call on a device looks the array's address up (host-side
+ * set-up; make that first call before any stream capture); a device reset
+ * (cudaDeviceReset) afterwards is not supported, since the cached address would be stale.
+ * One array per device: calls that overlap on the GPU race on it and must be serialised
+ * by the caller. */
 sdm_status sdm_recur_noalloc(const sdm_shape* shape, const int32_t* idx_w, const float* w_w,
                              const int32_t* idx_r, const float* w_r, const void* v,
                              const void* alpha, const void* beta, void* mem, void* y,
@@ -303,6 +311,28 @@ sdm_status sdm_recur_noalloc(const sdm_shape* shape, const int32_t* idx_w, const
  *   [9] total entries of the outer-sum bands re-ranked ([2] bands)
  * Counters wrap modulo 2^32. */
 sdm_status sdm_device_stats(uint32_t* counts, int n, sdm_stream_t stream);
+
+/* Launch plan of the recurrence kernels for `shape` (the paper has no counterpart; for
+ * tests that must reach a given kernel variant, and for tuning).  Writes the first n
+ * (<= 6) of, in order: the 16-byte chunks of a memory row each warp owns (its d-range),
+ * the warps (d-ranges) per (b, h) chain, the slot positions each lane handles per token,
+ * the look-ahead in tokens of the row prefetch, 1 if the writer/reader kernel runs (else
+ * 0), and the warps per CTA of the fused kernel.  Host only: launches nothing. */
+sdm_status sdm_recur_plan(const sdm_shape* shape, int32_t* out, int n);
+
+/* Test hook for the bounded device waits (the paper has no counterpart).  Runs sdm_recur
+ * (same arguments and workspace) with every wait of the writer/reader recurrence kernel
+ * limited to wait_cycles SM clock cycles (1 .. 2^32) and with the writer warps withholding
+ * their first hand-over.  The readers' first wait therefore runs out; every CTA leaves its
+ * token loop and returns, and bit 2 of the device status word is set (sdm_device_status
+ * then returns SDM_ERR_TIMEOUT).  y and mem are left undefined.  Returns
+ * SDM_ERR_UNSUPPORTED when the writer/reader kernel does not serve `shape` (sdm_recur_plan
+ * field 4 is 0). */
+sdm_status sdm_test_recur_wait_timeout(const sdm_shape* shape, const int32_t* idx_w, const float* w_w,
+                                       const int32_t* idx_r, const float* w_r, const void* v,
+                                       const void* alpha, const void* beta, void* mem, void* y,
+                                       void* workspace, size_t workspace_bytes, int64_t wait_cycles,
+                                       sdm_stream_t stream);
 
 #ifdef __cplusplus
 }

@@ -11,8 +11,8 @@ _LIB_PATH = os.path.join(HERE, "lib", "libsdm.so")
 
 DTYPE_F32, DTYPE_BF16 = 0, 1
 ADDR_PROJECTED, ADDR_DIRECT = 0, 1
-_STATUS = {0: "SDM_OK", 1: "SDM_ERR_INVALID_ARG", 2: "SDM_ERR_UNSUPPORTED", 3: "SDM_ERR_OOM",
-           4: "SDM_ERR_CUDA", 5: "SDM_ERR_TIMEOUT", 6: "SDM_ERR_DEVICE"}
+_STATUS = {0: "SDM_OK", 1: "SDM_ERR_INVALID_ARG", 2: "SDM_ERR_UNSUPPORTED", 4: "SDM_ERR_CUDA",
+           5: "SDM_ERR_TIMEOUT", 6: "SDM_ERR_DEVICE"}
 
 
 class SdmError(RuntimeError):
@@ -100,6 +100,11 @@ def lib():
             L.sdm_recur_noalloc.restype = ctypes.c_int
             L.sdm_device_stats.argtypes = [ctypes.POINTER(ctypes.c_uint32), ctypes.c_int, _VP]
             L.sdm_device_stats.restype = ctypes.c_int
+            L.sdm_recur_plan.argtypes = [_SHP, ctypes.POINTER(ctypes.c_int32), ctypes.c_int]
+            L.sdm_recur_plan.restype = ctypes.c_int
+            L.sdm_test_recur_wait_timeout.argtypes = [_SHP, _I32P, _VP, _I32P, _VP, _VP, _VP, _VP, _VP, _VP, _VP,
+                                                      _SZ, ctypes.c_int64, _VP]
+            L.sdm_test_recur_wait_timeout.restype = ctypes.c_int
             for f in ("sdm_init_memory", "sdm_forward", "sdm_decode_step", "sdm_address", "sdm_recur",
                       "sdm_device_status"):
                 getattr(L, f).restype = ctypes.c_int
@@ -296,12 +301,32 @@ def recur_noalloc(shape: SdmShape, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem, 
 
 
 def device_status(stream=None) -> int:
-    """Read and clear the device status word (0 = clean).  Raises SdmError if it was set."""
+    """Read and clear the device status word (0 = clean; bit 2 = a bounded wait gave up).
+    Raises SdmError only if reading it failed."""
     code = ctypes.c_int32(0)
     st = lib().sdm_device_status(ctypes.byref(code), _stream(stream))
-    if st not in (0, 6):
+    if st not in (0, 5, 6):
         _check(st)
     return int(code.value)
+
+
+RECUR_PLAN_FIELDS = ("dch", "nsplit", "spt", "la", "split", "wpc")
+
+
+def recur_plan(shape: SdmShape) -> dict:
+    """sdm_recur_plan: the recurrence's launch plan for `shape` (host only)."""
+    arr = (ctypes.c_int32 * len(RECUR_PLAN_FIELDS))()
+    _check(lib().sdm_recur_plan(ctypes.byref(shape), arr, len(RECUR_PLAN_FIELDS)))
+    return {name: int(arr[i]) for i, name in enumerate(RECUR_PLAN_FIELDS)}
+
+
+def test_recur_wait_timeout(shape: SdmShape, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem, y, workspace,
+                            wait_cycles: int, stream=None):
+    """sdm_test_recur_wait_timeout: the writer/reader recurrence with a withheld hand-over and a
+    short wait limit (the bounded waits must run out and set status bit 2)."""
+    _check(lib().sdm_test_recur_wait_timeout(ctypes.byref(shape), _ptr(idx_w), _ptr(w_w), _ptr(idx_r), _ptr(w_r),
+                                             _ptr(v), _ptr(alpha), _ptr(beta), _ptr(mem), _ptr(y), _ptr(workspace),
+                                             _nbytes(workspace) or 0, int(wait_cycles), _stream(stream)))
 
 
 STAT_NAMES = ("half_band", "half_full", "comb_band", "comb_full", "select_retry", "comb_merge", "band_f64", "serial",

@@ -95,7 +95,7 @@ __global__ void __launch_bounds__(CK_THREADS) k_recur_chunk(const RecArgs a, int
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int64_t chain = blockIdx.x;
     const int64_t mrow0 = chain * a.N;                       // first memory row of the chain
-    bool bad = false;
+    bool bad = false, unsorted = false;
     for (int c0 = 0; c0 < T; c0 += C) {
         const int n = min(C, T - c0);
         const int64_t tok0 = chain * T + c0;
@@ -104,6 +104,8 @@ __global__ void __launch_bounds__(CK_THREADS) k_recur_chunk(const RecArgs a, int
             const int s = __ldg(a.idx_w + tok0 * kw + e);
             const bool ok = static_cast<uint32_t>(s) < N;
             bad |= !ok;
+            // the two-pointer merges and binary searches need strictly ascending lists
+            unsorted |= (e % kw) > 0 && __ldg(a.idx_w + tok0 * kw + e - 1) >= s;
             s_iw[e] = s;
             s_ww[e] = ok ? __ldg(a.w_w + tok0 * kw + e) : 0.f;
         }
@@ -111,13 +113,17 @@ __global__ void __launch_bounds__(CK_THREADS) k_recur_chunk(const RecArgs a, int
             const int s = __ldg(a.idx_r + tok0 * kr + e);
             const bool ok = static_cast<uint32_t>(s) < N;
             bad |= !ok;
+            unsorted |= (e % kr) > 0 && __ldg(a.idx_r + tok0 * kr + e - 1) >= s;
             s_ir[e] = s;
             s_wr[e] = ok ? __ldg(a.w_r + tok0 * kr + e) : 0.f;
         }
         for (int t = tid; t < n; t += CK_THREADS) {
             const float al = load_elem<D>(a.alpha, tok0 + t);
             s_al[t] = al;
-            s_la[t] = logf(al);
+            // log(alpha) floored at -80 (e^-80 < 2^-115): a gate of exactly 0, which the fp32
+            // gate formula reaches for large A softplus(.), then decays to below fp32 precision
+            // of any stored value instead of making lam = -inf and exp(-inf - -inf) = NaN
+            s_la[t] = al > 0.f ? fmaxf(logf(al), -80.f) : -80.f;
             s_be[t] = load_elem<D>(a.beta, tok0 + t);
         }
         for (int e = tid; e < n * dv; e += CK_THREADS) s_dV[e] = load_elem<D>(a.v, tok0 * dv + e);
@@ -237,6 +243,7 @@ __global__ void __launch_bounds__(CK_THREADS) k_recur_chunk(const RecArgs a, int
         __syncthreads();
     }
     if (bad && (threadIdx.x & 31) == 0) flag_error(a.err, ERR_BAD_INDEX);
+    if (unsorted) flag_error(a.err, ERR_UNSORTED);
 }
 
 cudaError_t launch_recur_chunkwise(int dtype, const RecArgs& a, int C, cudaStream_t stream) {

@@ -439,14 +439,14 @@ __device__ __forceinline__ void rec_mbar_arrive(uint32_t bar) {
     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];\n" ::"r"(bar) : "memory");
 }
 // Bounded wait for the completion of the phase with parity `par`; false on timeout or abort.
-__device__ __forceinline__ bool rec_mbar_wait(uint32_t bar, uint32_t par, volatile int* abort_flag) {
+__device__ __forceinline__ bool rec_mbar_wait(uint32_t bar, uint32_t par, volatile int* abort_flag, long long limit) {
     const long long t0 = clock64();
     while (true) {
         uint32_t ok;
         asm volatile("{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
                      : "=r"(ok) : "r"(bar), "r"(par) : "memory");
         if (ok) return true;
-        if (*abort_flag || clock64() - t0 > REC_WAIT_CYCLES) return false;
+        if (*abort_flag || clock64() - t0 > limit) return false;
     }
 }
 
@@ -593,6 +593,7 @@ __global__ void __launch_bounds__(64) k_recur_split(const RecArgs a, int nsplit,
     };
 
     bool bad = false, timed_out = false;
+    const long long wait_limit = a.wait_cycles > 0 ? a.wait_cycles : REC_WAIT_CYCLES;
     if (warp == 0) {
         // ------------------------------------------------------------------ writer
         float a_cur = 0.f, b_cur = 0.f, a_nxt = 0.f, b_nxt = 0.f;
@@ -663,7 +664,10 @@ __global__ void __launch_bounds__(64) k_recur_split(const RecArgs a, int nsplit,
                 packed[j] = pack16x2<D>(o);
             }
             // ring entry of token t - LA - 1 is free once the reader is done with token t - 1
-            if (t > 0 && !rec_mbar_wait(bar_read, static_cast<uint32_t>((t - 1) & 1), abort_flag)) { timed_out = true; break; }
+            if (t > 0 && !rec_mbar_wait(bar_read, static_cast<uint32_t>((t - 1) & 1), abort_flag, wait_limit)) {
+                timed_out = true;
+                break;
+            }
             const uint32_t wslot = my_wring + ws * KS * SLOTB;
 #pragma unroll
             for (int j = 0; j < SPT; ++j) {
@@ -671,7 +675,7 @@ __global__ void __launch_bounds__(64) k_recur_split(const RecArgs a, int nsplit,
                 sts128(wslot + j * SLOTB, packed[j], okw[j]);
             }
             __syncwarp();
-            if (lane == 0) rec_mbar_arrive(bar_written);
+            if (lane == 0 && !(a.hold_handover && t == 0)) rec_mbar_arrive(bar_written);
             prefetch(t, ms, rs);
             ms = ms + 1 == MR ? 0 : ms + 1;
             rs = rs + 1 == LA ? 0 : rs + 1;
@@ -690,7 +694,10 @@ __global__ void __launch_bounds__(64) k_recur_split(const RecArgs a, int nsplit,
             lds_vec<SPT>(m + 2 * KP + g * SPT, ir);
             lds_vec<SPT>(m + 3 * KP + g * SPT, *reinterpret_cast<int(*)[SPT]>(wr));
             lds_vec<SPT>(m + 4 * KP + g * SPT, hzv);
-            if (!rec_mbar_wait(bar_written, static_cast<uint32_t>(t & 1), abort_flag)) { timed_out = true; break; }
+            if (!rec_mbar_wait(bar_written, static_cast<uint32_t>(t & 1), abort_flag, wait_limit)) {
+                timed_out = true;
+                break;
+            }
             float2 yp[E2];
 #pragma unroll
             for (int e = 0; e < E2; ++e) yp[e] = make_float2(0.f, 0.f);

@@ -52,7 +52,7 @@ __global__ void __launch_bounds__(32 * BW_WARPS) k_recur_bwd(const RecArgs a, co
     const uint32_t N = static_cast<uint32_t>(a.N);
     const int64_t mbase = chain * a.N * dv;                              // element offset of the chain's memory
     float* G = dM + mbase;
-    bool bad = false;
+    bool bad = false, unsorted = false;
     for (int t = T - 1; t >= 0; --t) {
         const int64_t tok = chain * T + t;
         const float alpha = load_elem<D>(a.alpha, tok), beta = load_elem<D>(a.beta, tok);
@@ -62,6 +62,7 @@ __global__ void __launch_bounds__(32 * BW_WARPS) k_recur_bwd(const RecArgs a, co
         // ---- read of the post-write memory M_t
         for (int n = 0; n < kr; ++n) {
             const int32_t s = __ldg(a.idx_r + tok * kr + n);
+            unsorted |= n > 0 && __ldg(a.idx_r + tok * kr + n - 1) >= s;
             if (static_cast<uint32_t>(s) >= N) { bad = true; continue; }   // warp-uniform
             const float rho = __ldg(a.w_r + tok * kr + n);
             const int64_t row = mbase + static_cast<int64_t>(s) * dv;
@@ -87,6 +88,8 @@ __global__ void __launch_bounds__(32 * BW_WARPS) k_recur_bwd(const RecArgs a, co
         }
         for (int m = 0; m < kw; ++m) {
             const int32_t i = __ldg(a.idx_w + tok * kw + m);
+            // the write slots of a token must be distinct: checked as strictly ascending
+            unsorted |= m > 0 && __ldg(a.idx_w + tok * kw + m - 1) >= i;
             if (static_cast<uint32_t>(i) >= N) continue;                // no write, no log entry
             const float w = __ldg(a.w_w + tok * kw + m);
             const int64_t urow = (tok * kw + m) * dv;
@@ -144,6 +147,7 @@ __global__ void __launch_bounds__(32 * BW_WARPS) k_recur_bwd(const RecArgs a, co
         }
     }
     if (__any_sync(0xffffffffu, bad) && lane == 0) flag_error(a.err, ERR_BAD_INDEX);
+    if (__any_sync(0xffffffffu, unsorted) && lane == 0) flag_error(a.err, ERR_UNSORTED);
 }
 
 cudaError_t launch_recur_backward(int dtype, const RecArgs& a, const void* undo, const void* dy, float* dv,

@@ -346,7 +346,8 @@ sdm_status forward_impl(const char* who, const sdm_shape* s, const void* P_q, co
 // sdm_recur with an optional undo log (defined after the C entry points).
 sdm_status recur_impl(const char* who, const sdm_shape* s, const int32_t* idx_w, const float* w_w,
                       const int32_t* idx_r, const float* w_r, const void* v, const void* alpha, const void* beta,
-                      void* mem, void* y, void* undo, void* workspace, size_t workspace_bytes, sdm_stream_t stream);
+                      void* mem, void* y, void* undo, void* workspace, size_t workspace_bytes, sdm_stream_t stream,
+                      long long wait_cycles = 0, int hold_handover = 0);
 
 }  // namespace
 
@@ -636,7 +637,8 @@ namespace {
 
 sdm_status recur_impl(const char* who, const sdm_shape* s, const int32_t* idx_w, const float* w_w,
                       const int32_t* idx_r, const float* w_r, const void* v, const void* alpha, const void* beta,
-                      void* mem, void* y, void* undo, void* workspace, size_t workspace_bytes, sdm_stream_t stream) {
+                      void* mem, void* y, void* undo, void* workspace, size_t workspace_bytes, sdm_stream_t stream,
+                      long long wait_cycles, int hold_handover) {
     SDM_TRY(check_shape(s, false, nullptr));
     const size_t es = elem_bytes(s->dtype);
     const size_t bht = static_cast<size_t>(s->B) * s->H * s->T;
@@ -681,6 +683,8 @@ sdm_status recur_impl(const char* who, const sdm_shape* s, const int32_t* idx_w,
     r.N = s->N;
     r.err = err;
     r.undo = undo;
+    r.wait_cycles = wait_cycles;
+    r.hold_handover = hold_handover;
     cudaError_t e = sdm::launch_recur(s->dtype, r, static_cast<int32_t*>(workspace), reinterpret_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "recurrence launch");
     return ok();
@@ -717,10 +721,34 @@ sdm_status sdm_device_status(int32_t* code, sdm_stream_t stream) {
     if (e != cudaSuccess) return cuda_fail(e, "sdm_device_status");
     *code = host;
     if (host != 0)
-        return fail(SDM_ERR_DEVICE, "device status word = 0x%x (bit 0: slot index outside [0, N) skipped; "
+        return fail((host & sdm::ERR_TIMEOUT) ? SDM_ERR_TIMEOUT : SDM_ERR_DEVICE,
+                    "device status word = 0x%x (bit 0: slot index outside [0, N) skipped; "
                     "bit 1: slot list not strictly ascending; bit 2: bounded wait timed out; "
                     "bit 3: selection invariant failed)", host);
     return ok();
+}
+
+sdm_status sdm_recur_plan(const sdm_shape* s, int32_t* out, int n) {
+    SDM_TRY(check_shape(s, false, nullptr));
+    if (!out || n < 0 || n > 6) return fail(SDM_ERR_INVALID_ARG, "sdm_recur_plan: out must be non-NULL and n in [0, 6]");
+    const sdm::RecPlan p = sdm::rec_plan(s->dtype, s->B, s->H, s->T, s->d_v, s->k_write, s->k_read);
+    const int32_t v[6] = {p.dch, p.nsplit, p.spt, p.la, p.split, p.wpc};
+    for (int i = 0; i < n; ++i) out[i] = v[i];
+    return ok();
+}
+
+sdm_status sdm_test_recur_wait_timeout(const sdm_shape* s, const int32_t* idx_w, const float* w_w,
+                                       const int32_t* idx_r, const float* w_r, const void* v, const void* alpha,
+                                       const void* beta, void* mem, void* y, void* workspace, size_t workspace_bytes,
+                                       int64_t wait_cycles, sdm_stream_t stream) {
+    SDM_TRY(check_shape(s, false, nullptr));
+    if (wait_cycles < 1 || wait_cycles > (static_cast<int64_t>(1) << 32))
+        return fail(SDM_ERR_INVALID_ARG, "sdm_test_recur_wait_timeout: wait_cycles must be in [1, 2^32]");
+    const sdm::RecPlan p = sdm::rec_plan(s->dtype, s->B, s->H, s->T, s->d_v, s->k_write, s->k_read);
+    if (!p.split || static_cast<int64_t>(s->B) * s->H * s->T == 0)
+        return fail(SDM_ERR_UNSUPPORTED, "sdm_test_recur_wait_timeout: the writer/reader kernel does not serve this shape");
+    return recur_impl("sdm_test_recur_wait_timeout", s, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem, y, nullptr,
+                      workspace, workspace_bytes, stream, static_cast<long long>(wait_cycles), 1);
 }
 
 }  // extern "C"

@@ -63,6 +63,9 @@ struct RecArgs {
     int B, H, T, dv, kw, kr;
     int64_t N;
     int* err;
+    long long wait_cycles;                    // limit of every bounded device wait (0: the default)
+    int hold_handover;                        // test hook: the writer warp withholds its first
+                                              // hand-over, so the reader's wait runs out
 };
 // Launch geometry of the recurrence (depends only on the shape).
 struct RecPlan {

@@ -13,7 +13,9 @@
 //     anything is launched;
 //   * the array's address is looked up once per device (cudaGetSymbolAddress, with that
 //     device current) on the first call made with it current, and cached; that first call
-//     therefore does host-side set-up work and should come before any stream capture;
+//     therefore does host-side set-up work and should come before any stream capture.  A
+//     device reset (cudaDeviceReset) after that first call is not supported: the cached
+//     address would outlive the context it belongs to;
 //   * every entry of the table that the kernels read is written by the hazard kernel first
 //     in the same call, so nothing has to start at zero;
 //   * there is one array per device: calls that overlap on the GPU (different streams, or
@@ -65,15 +67,29 @@ extern "C" sdm_status sdm_recur_noalloc(const sdm_shape* s, const int32_t* idx_w
                                         const int32_t* idx_r, const float* w_r, const void* v, const void* alpha,
                                         const void* beta, void* mem, void* y, sdm_stream_t stream) {
     if (s == nullptr) return sdm::api_error(SDM_ERR_INVALID_ARG, "sdm_recur_noalloc: shape is NULL");
-    // size limit first: it needs no device and rejects before any CUDA call
-    if (s->B >= 0 && s->H >= 0 && s->T >= 0 && s->k_write >= 0 && s->k_read >= 0) {
-        const size_t need = sdm::rec_workspace_bytes(s->B, s->H, s->T, s->k_write, s->k_read);
-        if (need > kScratchBytes) {
+    // size limit first: it needs no device and rejects before any CUDA call.  The entry
+    // count B*H*T*kmax is checked factor by factor against the capacity, so it cannot wrap.
+    if (s->B < 0 || s->H < 0 || s->T < 0)
+        return sdm::api_error(SDM_ERR_INVALID_ARG, "sdm_recur_noalloc: B, H, T must be >= 0");
+    if (s->k_write < 1 || s->k_read < 1 || s->k_write > 64 || s->k_read > 64)
+        return sdm::api_error(SDM_ERR_UNSUPPORTED, "sdm_recur_noalloc: k_write and k_read must be in [1, 64]");
+    {
+        const int64_t cap = static_cast<int64_t>(kScratchBytes / sizeof(int32_t));
+        const int64_t factors[4] = {s->B, s->H, s->T, s->k_write > s->k_read ? s->k_write : s->k_read};
+        int64_t entries = 1;
+        bool fits = true;
+        for (int64_t f : factors) {
+            if (f == 0) { entries = 0; break; }
+            if (entries > cap / f) fits = false;     // entries * f > cap
+            if (!fits) break;
+            entries *= f;
+        }
+        if (!fits) {
             char buf[256];
             snprintf(buf, sizeof(buf),
-                     "sdm_recur_noalloc: hazard table needs %zu bytes > fixed scratch of %zu bytes "
-                     "(B*H*T*max(k_write,k_read) must be <= %zu); use sdm_recur with a workspace",
-                     need, kScratchBytes, kScratchBytes / sizeof(int32_t));
+                     "sdm_recur_noalloc: the hazard table does not fit the fixed scratch of %zu bytes "
+                     "(B*H*T*max(k_write,k_read) must be <= %lld); use sdm_recur with a workspace",
+                     kScratchBytes, static_cast<long long>(cap));
             return sdm::api_error(SDM_ERR_UNSUPPORTED, buf);
         }
     }

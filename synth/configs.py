@@ -66,9 +66,11 @@ class SdmConfig:
         return (2 * self.k_write + self.k_read) * self.d_v * s + 2 * self.d_k * s + 2 * self.d_v * s + 2 * s
 
     def recurrence_bytes_per_token_head(self) -> int:
-        """Algorithmic bytes of the fused recurrence alone: rows gathered/scattered, v, alpha, beta, y."""
+        """Algorithmic bytes of the fused recurrence alone: rows gathered/scattered, v, alpha, beta, y,
+        and the slot lists it is given (int32 index + fp32 weight per write and per read slot)."""
         s = self.elem_bytes
-        return (2 * self.k_write + self.k_read) * self.d_v * s + 2 * self.d_v * s + 2 * s
+        return ((2 * self.k_write + self.k_read) * self.d_v * s + 2 * self.d_v * s + 2 * s
+                + (self.k_write + self.k_read) * 8)
 
 
 TINY_FP32 = SdmConfig("tiny_fp32", B=1, H=1, T=256, d_k=64, d_v=64, N=4096, k_write=8, k_read=8,

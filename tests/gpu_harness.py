@@ -88,3 +88,32 @@ def touched_bits(touched, N: int) -> np.ndarray:
 
 def host(t, dtype: str) -> np.ndarray:
     return from_torch(t, dtype)
+
+
+# ------------------------------------------------------------------ elementwise comparison
+
+def storage_ulp(x: np.ndarray, dtype: str) -> np.ndarray:
+    """Unit in the last place of the storage dtype at |x| (bf16: 8 significant bits, fp32: 24)."""
+    mant = 7 if dtype == "bf16" else 23
+    ax = np.abs(np.asarray(x, np.float64))
+    e = np.floor(np.log2(np.where(ax > 0, ax, 1.0)))
+    return np.where(ax > 0, 2.0 ** (e - mant), 2.0 ** (-126 - mant))
+
+
+def elementwise(got: np.ndarray, ref: np.ndarray, dtype: str) -> dict:
+    """Per-element distance of stored values `got` from the oracle's stored values `ref` (both
+    float64 of storage numbers), rows along the last axis:
+      max_row_ulps  max |got - ref| in units of the ulp of the row's largest |ref|;
+      frac_gt1      fraction of elements more than one ulp of their own value apart (the
+                    ulp taken at max(|ref|, 2^-8 * row max), so that near-zero elements of a
+                    row are measured at the row's own resolution);
+      max_rel_row   max |got - ref| / row max of |ref|."""
+    got = np.asarray(got, np.float64)
+    ref = np.asarray(ref, np.float64)
+    rowmax = np.max(np.abs(ref), axis=-1, keepdims=True)
+    d = np.abs(got - ref)
+    u_row = storage_ulp(rowmax, dtype)
+    u_own = storage_ulp(np.maximum(np.abs(ref), rowmax * 2.0 ** -8), dtype)
+    return {"max_row_ulps": float(np.max(d / u_row)) if d.size else 0.0,
+            "frac_gt1": float(np.mean(d > u_own)) if d.size else 0.0,
+            "max_rel_row": float(np.max(d / np.where(rowmax > 0, rowmax, 1.0))) if d.size else 0.0}

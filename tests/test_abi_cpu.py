@@ -43,7 +43,7 @@ def test_library_exports_every_declared_symbol(sdm):
     L = sdm.lib()
     for name in declared_functions():
         assert hasattr(L, name), name
-    assert sdm.abi_version() == 1
+    assert sdm.abi_version() == 2
 
 
 def test_shape_struct_layout_matches_header(sdm):
@@ -226,3 +226,39 @@ def test_binding_fails_loudly_without_library(tmp_path, monkeypatch):
     monkeypatch.setattr(b, "_lib", None)
     with pytest.raises(RuntimeError, match="not found"):
         b.lib()
+
+
+def test_recur_plan_reports_the_launch_shape(sdm):
+    """sdm_recur_plan is host-only: the short-T parity shapes of the GPU tests reach the kernel
+    variant the bench runs at full size (the plan depends on T only through T == 1)."""
+    import synth
+    full = synth.LAYER_1P4B
+    mk = lambda c, T: sdm.SdmShape.make(c.B, c.H, T, c.d_k, c.d_v, c.N, c.k_write, c.k_read, c.dtype)
+    bench_plan = sdm.recur_plan(mk(full, full.T))
+    assert sdm.recur_plan(mk(full, 128)) == bench_plan
+    assert set(bench_plan) == set(sdm.RECUR_PLAN_FIELDS)
+    assert sdm.recur_plan(mk(full, 1))["la"] == 1 and bench_plan["la"] > 1
+    arr = (ctypes.c_int32 * 8)()
+    assert sdm.lib().sdm_recur_plan(ctypes.byref(mk(full, 16)), arr, 7) == 1 and "[0, 6]" in sdm.last_error()
+
+
+def test_wait_timeout_hook_rejects_shapes_without_the_handover(sdm):
+    L = sdm.lib()
+    args = [FAKE, FAKE + 0x100000, FAKE + 0x200000, FAKE + 0x300000, FAKE + 0x400000, FAKE + 0x500000,
+            FAKE + 0x600000, FAKE + 0x10000000, FAKE + 0x700000, FAKE + 0x40000000, 1 << 30]
+    fused = _shape(sdm, B=8, H=16, T=64, d_k=128, d_v=128, N=262144, k_write=32, k_read=32)
+    assert sdm.recur_plan(fused)["split"] == 0
+    assert L.sdm_test_recur_wait_timeout(ctypes.byref(fused), *args, 1000, None) == 2
+    assert "writer/reader" in sdm.last_error()
+    split = _shape(sdm, B=1, H=2, T=8, d_v=64, N=4096, k_write=8, k_read=8)
+    assert sdm.recur_plan(split)["split"] == 1
+    assert L.sdm_test_recur_wait_timeout(ctypes.byref(split), *args, 0, None) == 1 and "wait_cycles" in sdm.last_error()
+
+
+def test_noalloc_size_check_cannot_wrap(sdm):
+    """A shape whose entry count B*H*T*k overflows 64 bits is still rejected as too large."""
+    huge = sdm.SdmShape.make(2 ** 31 - 1, 2 ** 31 - 1, 2 ** 31 - 1, 8, 64, 4096, 64, 64, "bf16")
+    st = sdm.lib().sdm_recur_noalloc(ctypes.byref(huge), *[FAKE + i * 0x10000000 for i in range(9)], None)
+    assert st == 2 and "fixed scratch" in sdm.last_error()
+    neg = sdm.SdmShape.make(-1, 1, 1, 8, 64, 4096, 8, 8, "bf16")
+    assert sdm.lib().sdm_recur_noalloc(ctypes.byref(neg), *[FAKE] * 9, None) == 1

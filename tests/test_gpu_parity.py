@@ -5,6 +5,18 @@ slot weights within max relative error (per (b, h) slice, Frobenius norm)
 TOL["bf16"] = 2e-3 or TOL["f32"] = 1e-5; untouched memory rows bit-identical to
 M0; kernels that must agree with each other (split runs, decode steps, batch
 slices) agree bit for bit.
+
+Element by element (``_check_elementwise``), against the oracle's stored values:
+  bf16  every element of y and of the written rows within 2 ulps of its row's largest
+        magnitude, and at most 0.1% of the elements more than 1 ulp of their own value
+        apart.  The GPU works in fp32 and the oracle in float64; both round the same
+        stored values, so a difference is a rounding that flipped (fp32 error near a
+        rounding tie), or such a flip carried into later reads and writes of the row;
+  f32   every element within 1e-5 of its row's largest magnitude (the relative bar,
+        taken per element);
+  weights  relative error at most 2e-5 per weight: the softmax of fp32 scores whose
+        rounding error is a few fp32 ulps of |s| <= ~5 (about 1e-6), doubled by the
+        max-subtraction, plus the fp32 sum and expf.
 """
 import numpy as np
 import pytest
@@ -31,19 +43,44 @@ def sdm():
     return sdm
 
 
-def _check_slices(cfg, out, slices, T=None, check_untouched=True):
+W_REL = 2e-5          # per-weight relative bar (see the module docstring)
+
+
+def _check_elementwise(dtype, got, ref, what):
+    """Element-by-element bars of the module docstring; returns the measured distances."""
+    e = G.elementwise(got, ref, dtype)
+    if dtype == "bf16":
+        assert e["max_row_ulps"] <= 2.0 and e["frac_gt1"] <= 1e-3, (what, e)
+    else:
+        assert e["max_rel_row"] <= 1e-5, (what, e)
+    return e
+
+
+def _check_weights(got, ref, what):
+    got = np.asarray(got, np.float64)
+    rel = np.max(np.abs(got - ref) / np.abs(ref)) if ref.size else 0.0
+    assert rel <= W_REL, (what, float(rel))
+
+
+def _check_slices(cfg, out, slices, T=None, check_untouched=True, ref=None):
     tol = TOL[cfg.dtype]
-    ref = oracle_slices(cfg, slices, T=T)
+    ref = ref if ref is not None else oracle_slices(cfg, slices, T=T)
     y = out["y"]
     for (b, h), r in ref.items():
         assert np.array_equal(out["idx_w"][b, h].cpu().numpy(), r["idx_w"]), ("idx_w", b, h)
         assert np.array_equal(out["idx_r"][b, h].cpu().numpy(), r["idx_r"]), ("idx_r", b, h)
         assert rel_fro(out["w_w"][b, h].cpu().numpy(), r["w_w"]) <= tol
         assert rel_fro(out["w_r"][b, h].cpu().numpy(), r["w_r"]) <= tol
-        ey = rel_fro(O.to_f64(G.host(y[b, h], cfg.dtype), cfg.dtype), r["y"])
+        _check_weights(out["w_w"][b, h].cpu().numpy(), r["w_w"], ("w_w", b, h))
+        _check_weights(out["w_r"][b, h].cpu().numpy(), r["w_r"], ("w_r", b, h))
+        gy = O.to_f64(G.host(y[b, h], cfg.dtype), cfg.dtype)
+        ey = rel_fro(gy, r["y"])
         mem_bh = G.host(out["mem"][b, h], cfg.dtype)
-        em = rel_fro(O.to_f64(mem_bh[r["touched"]], cfg.dtype), r["M_touched"])
+        gm = O.to_f64(mem_bh[r["touched"]], cfg.dtype)
+        em = rel_fro(gm, r["M_touched"])
         assert ey <= tol and em <= tol, (b, h, ey, em)
+        _check_elementwise(cfg.dtype, gy, r["y"], ("y", b, h))
+        _check_elementwise(cfg.dtype, gm, r["M_touched"], ("written rows", b, h))
         if check_untouched:
             M0 = synth.head_inputs(cfg, h, which=("M0",))["M0"]
             mask = np.ones(cfg.N, bool)
@@ -740,10 +777,165 @@ def test_access_stats_wide_lists_match_the_oracle(sdm):
     np.testing.assert_allclose(got[4 + kw:], O.cumulative_mass(r64).sum(axis=0), rtol=2e-5)
 
 
+# ------------------------------------------------------------------ launch shapes of the large workloads
+
+def _bench_plan_equal(sdm, cfg):
+    """The recurrence plan of cfg equals that of cfg at its full T (the plan depends on T only
+    through T == 1), i.e. the short-T case runs the kernel variant of the full workload."""
+    full = synth.CONFIGS[cfg.name]
+    got = sdm.recur_plan(G.shape_of(cfg))
+    assert got == sdm.recur_plan(G.shape_of(full)), (got, sdm.recur_plan(G.shape_of(full)))
+    return got
+
+
+LAYER_SHORT = synth.LAYER_1P4B.with_(T=128)
+LAYER_SLICES = [(0, 0), (2, 9), (5, 4), (7, 15)]
+
+
+@pytest.mark.gpu
+def test_layer_geometry_runs_the_bench_kernel_and_matches_the_oracle(sdm):
+    """All 8 x 16 chains of the bench workload (N=262144, k=32, bf16) over 128 tokens: the
+    recurrence launches exactly as in the timed bench step (asserted through sdm_recur_plan),
+    and sampled slices match the oracle (indices bit-exact, values element by element)."""
+    cfg = LAYER_SHORT
+    plan = _bench_plan_equal(sdm, cfg)
+    assert plan["la"] > 1
+    dev = G.device_inputs(cfg)
+    out = G.run_forward(cfg, dev)
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    _check_slices(cfg, out, LAYER_SLICES)
+    del out, dev
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.gpu
+def test_layer_geometry_lazy_path_matches_broadcast_and_oracle(sdm):
+    """The copy-on-write path at the bench geometry (same kernel plan): y, slot lists and written
+    rows equal the broadcast path's bit for bit, and sampled slices match the oracle."""
+    cfg = LAYER_SHORT
+    _bench_plan_equal(sdm, cfg)
+    dev = G.device_inputs(cfg)
+    ref = G.run_forward(cfg, dev)
+    out = G.run_forward_lazy(cfg, dev)
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    for key in ("idx_w", "w_w", "idx_r", "w_r", "y"):
+        assert torch.equal(out[key], ref[key]), key
+    mask = torch.from_numpy(G.touched_bits(out["touched"], cfg.N)).to("cuda")
+    assert torch.equal(out["mem"][mask], ref["mem"][mask])
+    del ref
+    sdm.materialize(G.shape_of(cfg), dev["M0"], out["touched"], out["mem"])
+    torch.cuda.synchronize()
+    _check_slices(cfg, out, LAYER_SLICES[::2])
+    del out, dev, mask
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.gpu
+def test_long_context_geometry_matches_the_oracle(sdm):
+    """The long-context geometry (B=2, H=16, N=2^20: two 512-column chunks per half, so the
+    multi-chunk finalize passes run on the tensor-core path) over 256 tokens, with its full
+    workload's recurrence plan; sampled slices against the oracle."""
+    cfg = synth.LONG_CTX.with_(T=256)
+    _bench_plan_equal(sdm, cfg)
+    dev = G.device_inputs(cfg)
+    out = G.run_forward(cfg, dev)
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    _check_slices(cfg, out, [(0, 3), (1, 14)])
+    del out, dev
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.gpu
+def test_decode_steps_match_the_oracle(sdm):
+    """sdm_decode_step at the decode workload's batch (B=256 sequences, N=262144, k=32, bf16;
+    H=2 heads to bound the 34 GB state) for 64 consecutive steps from M0, sampled sequences
+    replayed by the oracle token by token: slots bit-exact, y and written rows element by element."""
+    cfg = synth.DECODE.with_(H=2, prefill_steps=0, decode_steps=64)
+    full = synth.full_inputs(cfg)
+    params = {n: synth.torch_io.to_torch(full[n], cfg.dtype) for n in ("M0", "P_q", "P_k")}
+    shape = G.shape_of(cfg, 1)
+    assert sdm.recur_plan(shape)["la"] == 1
+    mem = torch.empty((cfg.B, cfg.H, cfg.N, cfg.d_v), dtype=torch.bfloat16, device="cuda")
+    sdm.init_memory(shape, params["M0"], mem)
+    ws = G.workspace(shape)
+    slices = [(0, 0), (77, 1), (255, 1)]
+    rec = {s: {"y": [], "iw": [], "ir": [], "ww": [], "wr": []} for s in slices}
+    buf = {n: torch.empty((cfg.B, cfg.H, k), dtype=dt, device="cuda")
+           for n, k, dt in (("iw", cfg.k_write, torch.int32), ("ir", cfg.k_read, torch.int32),
+                            ("ww", cfg.k_write, torch.float32), ("wr", cfg.k_read, torch.float32))}
+    y = torch.empty((cfg.B, cfg.H, cfg.d_v), dtype=torch.bfloat16, device="cuda")
+    for t in range(cfg.tokens_per_seq):
+        st = {n: synth.torch_io.to_torch(np.ascontiguousarray(full[n][:, :, t]), cfg.dtype)
+              for n in ("q", "k", "v", "alpha", "beta")}
+        sdm.decode_step(shape, params["P_q"], params["P_k"], st["q"], st["k"], st["v"], st["alpha"], st["beta"],
+                        mem, y, ws, idx_w=buf["iw"], w_w=buf["ww"], idx_r=buf["ir"], w_r=buf["wr"])
+        for (b, h) in slices:
+            rec[(b, h)]["y"].append(y[b, h].clone())
+            for n in ("iw", "ir", "ww", "wr"):
+                rec[(b, h)][n].append(buf[n][b, h].clone())
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    ref = oracle_slices(cfg, slices)
+    for (b, h), r in ref.items():
+        got = {n: torch.stack(v).cpu().numpy() for n, v in rec[(b, h)].items() if n != "y"}
+        assert np.array_equal(got["iw"], r["idx_w"]) and np.array_equal(got["ir"], r["idx_r"]), (b, h)
+        _check_weights(got["ww"], r["w_w"], ("w_w", b, h))
+        _check_weights(got["wr"], r["w_r"], ("w_r", b, h))
+        yg = O.to_f64(G.host(torch.stack(rec[(b, h)]["y"]), cfg.dtype), cfg.dtype)
+        assert rel_fro(yg, r["y"]) <= TOL["bf16"]
+        _check_elementwise("bf16", yg, r["y"], ("y", b, h))
+        mem_bh = O.to_f64(G.host(mem[b, h], cfg.dtype), cfg.dtype)
+        assert rel_fro(mem_bh[r["touched"]], r["M_touched"]) <= TOL["bf16"]
+        _check_elementwise("bf16", mem_bh[r["touched"]], r["M_touched"], ("written rows", b, h))
+    del mem, params, ws
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.gpu
+def test_bounded_wait_runs_out_and_reports_timeout(sdm):
+    """The writer/reader recurrence with its first hand-over withheld (test hook) and a wait
+    limit of 2^21 SM cycles (about a millisecond): the readers' waits run out, every CTA
+    returns, status bit 2 is set and sdm_device_status reports SDM_ERR_TIMEOUT; afterwards
+    the context still runs the normal recurrence correctly."""
+    import ctypes
+    rng = np.random.default_rng(5)
+    B, H, T, N, dv, k = 1, 2, 8, 4096, 64, 8
+    shape = sdm.SdmShape.make(B, H, T, 8, dv, N, k, k, "bf16")
+    assert sdm.recur_plan(shape)["split"] == 1
+    idx = np.sort(np.stack([rng.choice(N, k, replace=False) for _ in range(B * H * T)]), axis=1)
+    i32 = torch.from_numpy(idx.astype(np.int32).reshape(B, H, T, k)).cuda()
+    w = torch.full((B, H, T, k), 1.0 / k, dtype=torch.float32, device="cuda")
+    v = torch.randn((B, H, T, dv), device="cuda").to(torch.bfloat16)
+    gate = torch.full((B, H, T), 0.5, dtype=torch.bfloat16, device="cuda")
+    mem = torch.zeros((B, H, N, dv), dtype=torch.bfloat16, device="cuda")
+    y = torch.empty((B, H, T, dv), dtype=torch.bfloat16, device="cuda")
+    ws = torch.empty(sdm.recur_workspace_bytes(shape), dtype=torch.uint8, device="cuda")
+    sdm.device_status()
+    sdm.test_recur_wait_timeout(shape, i32, w, i32, w, v, gate, gate, mem, y, ws, 1 << 21)
+    torch.cuda.synchronize()
+    code = ctypes.c_int32(0)
+    st = sdm.lib().sdm_device_status(ctypes.byref(code), None)
+    assert st == 5 and code.value & 4, (st, code.value)
+    assert sdm.device_status() == 0                      # cleared
+    # the same inputs through sdm_recur still give the oracle's result
+    y2, M2 = _recur(sdm, "bf16", idx[:T], np.full((T, k), 1.0 / k), idx[:T], np.full((T, k), 1.0 / k),
+                    O.to_f64(G.host(v[0, 0], "bf16"), "bf16"), np.full(T, 0.5), np.full(T, 0.5), np.zeros((N, dv)))
+    Mo = np.zeros((N, dv))
+    _, yo = O.recur(Mo, idx[:T], np.full((T, k), 1.0 / k), idx[:T], np.full((T, k), 1.0 / k),
+                    O.to_f64(G.host(v[0, 0], "bf16"), "bf16"), np.full(T, 0.5), np.full(T, 0.5), "bf16")
+    assert rel_fro(y2, yo) <= TOL["bf16"] and rel_fro(M2, Mo) <= TOL["bf16"]
+
+
 # ------------------------------------------------------------------ full-size workloads
 
+@pytest.mark.gpu
 @pytest.mark.fullsize
 def test_layer_1p4b_full_size_sampled_slices(sdm):
+    """The bench workload itself (B=8 H=16 T=4096 N=262144 k=32 bf16, the launch shape the
+    bench times), four sampled slices against the oracle over all 4096 tokens."""
     cfg = synth.LAYER_1P4B
     dev = G.device_inputs(cfg)
     out = G.run_forward(cfg, dev)

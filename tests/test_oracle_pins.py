@@ -516,6 +516,8 @@ def test_cumulative_mass_invariants_on_softmax_weights():
 
 def test_unique_fraction_counts():
     N = 64
+    # literal count: slots {3, 5, 9, 60} appear (with repeats), so 4 of 64 are unique
+    assert O.unique_fraction(np.array([[3, 5, 9], [5, 9, 60], [3, 3, 60]]), N) == 4 / 64
     assert O.unique_fraction(np.arange(N).reshape(8, 8), N) == 1.0
     assert O.unique_fraction(np.full((5, 3), 7), N) == 1.0 / N
     rng = np.random.default_rng(25)
@@ -572,6 +574,15 @@ def test_norm_gate_closed_forms_and_invariance():
     # eps: rows of zeros stay zero, and eps > 0 shrinks the norm
     assert np.all(O.norm_gate(np.zeros((2, dv)), g[:2], gamma, 1e-6) == 0)
     assert np.all(np.abs(O.norm_gate(y, g, gamma, 1e-2)) < np.abs(O.norm_gate(y, g, gamma, 0.0)))
+
+
+def test_head_mix_two_heads_by_hand():
+    """Two heads, one token, d_v = 2, d = 2, worked by hand: concat(z_0, z_1) = [1, 2, 3, 4];
+    W_o rows [1, 0, 0, 1] and [0, 1, -1, 0] give o = [1 + 4, 2 - 3] = [5, -1]; the heads
+    concatenated in the wrong order would give [5, 3]."""
+    z = np.array([[[1.0, 2.0]], [[3.0, 4.0]]])            # [H=2, T=1, d_v=2]
+    W = np.array([[1.0, 0.0, 0.0, 1.0], [0.0, 1.0, -1.0, 0.0]])
+    assert np.array_equal(O.head_mix(z, W), np.array([[5.0, -1.0]]))
 
 
 def test_head_mix_is_a_sum_over_heads():

@@ -1,5 +1,10 @@
 """sdm_recur_noalloc (fixed device scratch, no workspace) against sdm_recur.
 
+Some callers cannot allocate device memory for the library (a runtime whose own pool
+owns the device, a serving loop that must not call an allocator); this entry point
+takes its scratch from an array the library reserves statically.  It runs the same
+kernels as sdm_recur, so the results must be identical bit for bit.
+
 Collected last on purpose: it must give the same results whether it runs alone in a
 fresh process (first use of its scratch) or after every other test."""
 import ctypes
@@ -71,11 +76,11 @@ def test_noalloc_matches_workspace_entry_on_two_calls(sdm, name):
         sdm.recur_noalloc(shape, *args, mem_na, y_na)
         torch.cuda.synchronize()
         assert sdm.device_status() == 0
+        # same kernels on the same inputs: only the scratch differs, so the results must be
+        # identical bit for bit (a tolerance could hide a scratch-aliasing fault)
+        assert torch.equal(y_na, y_ws), t0
         ya, yb = (O.to_f64(G.host(x, cfg.dtype), cfg.dtype) for x in (y_ws, y_na))
         for b in range(B):
             for h in range(H):
                 assert rel_fro(yb[b, h], ya[b, h]) <= TOL[cfg.dtype], (t0, b, h)
-    ma, mb = (O.to_f64(G.host(x, cfg.dtype), cfg.dtype) for x in (mem_ws, mem_na))
-    for b in range(B):
-        for h in range(H):
-            assert rel_fro(mb[b, h], ma[b, h]) <= TOL[cfg.dtype], (b, h)
+    assert torch.equal(mem_na, mem_ws)
