@@ -223,6 +223,170 @@ def weak_scaling_value(B: int, T: int, world: int, ms_max: float) -> float:
     return tokens_step_of(B, T, world) / (ms_max * 1e-3)
 
 
+# ----------------------------------------------------------------------------- other workloads
+
+def device_inputs(cfg, seed: int):
+    """Inputs of a workload's shapes and value distributions (the generator recipe of synth),
+    drawn on the device with torch's generator: the bench legs of the other workloads time
+    the kernels on them; their parity with the oracle is covered by the tests on synth's
+    inputs."""
+    import torch
+    from synth.torch_io import torch_dtype
+    dt = torch_dtype(cfg.dtype)
+    g = torch.Generator(device="cuda").manual_seed(seed)
+    rn = lambda *sh: torch.randn(sh, generator=g, device="cuda", dtype=torch.float32)
+    B, H, T, dk, dv, S = cfg.B, cfg.H, cfg.T, cfg.d_k, cfg.d_v, cfg.S
+    unit = lambda x: x / x.norm(dim=-1, keepdim=True)
+    out = {"q": unit(rn(B, H, T, dk)).to(dt), "k": unit(rn(B, H, T, dk)).to(dt), "v": rn(B, H, T, dv).to(dt),
+           "alpha": torch.sigmoid(rn(B, H, T) + cfg.alpha_mu).to(dt), "beta": torch.sigmoid(rn(B, H, T)).to(dt),
+           "P_q": rn(H, 2 * S, dk).to(dt), "P_k": rn(H, 2 * S, dk).to(dt)}
+    M0 = torch.empty((H, cfg.N, dv), dtype=dt, device="cuda")
+    for h in range(H):                      # in per-head pieces: bounded fp32 temporaries
+        M0[h] = (rn(cfg.N, dv) * cfg.mem_std).to(dt)
+    out["M0"] = M0
+    return out
+
+
+def leg_scan(name: str, steps: int, warmup: int) -> dict:
+    """A scan workload's step (sdm_forward_m0: M0 broadcast beside the addressing, then the
+    recurrence) and its phases, on device-drawn inputs; inputs larger than L2."""
+    import torch
+    import paper_2607_07386_gb300 as sdm
+    from synth.torch_io import torch_dtype
+    cfg = synth.get_config(name)
+    dev = device_inputs(cfg, seed=cfg.seed)
+    B, H, T, N, dv = cfg.B, cfg.H, cfg.T, cfg.N, cfg.d_v
+    dt = torch_dtype(cfg.dtype)
+    shape = sdm.SdmShape.make(B, H, T, cfg.d_k, dv, N, cfg.k_write, cfg.k_read, cfg.dtype)
+    mem = torch.empty((B, H, N, dv), dtype=dt, device="cuda")
+    y = torch.empty((B, H, T, dv), dtype=dt, device="cuda")
+    ws = torch.empty(sdm.workspace_bytes(shape), dtype=torch.uint8, device="cuda")
+    lists = {n: torch.empty((B, H, T, k), dtype=tt, device="cuda")
+             for n, k, tt in (("idx_w", cfg.k_write, torch.int32), ("w_w", cfg.k_write, torch.float32),
+                              ("idx_r", cfg.k_read, torch.int32), ("w_r", cfg.k_read, torch.float32))}
+    st = torch.cuda.current_stream()
+
+    def step():
+        sdm.forward_m0(shape, dev["M0"], dev["P_q"], dev["P_k"], dev["q"], dev["k"], dev["v"], dev["alpha"],
+                       dev["beta"], mem, y, ws, stream=st)
+
+    def timed(fn, n):
+        for _ in range(warmup):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(st)
+        for _ in range(n):
+            fn()
+        e1.record(st)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / n
+
+    ms = timed(step, steps)
+    ms_addr = timed(lambda: sdm.address(shape, dev["P_q"], dev["P_k"], dev["q"], dev["k"], lists["idx_w"], lists["w_w"],
+                                        lists["idx_r"], lists["w_r"], ws, stream=st), steps)
+    ms_rec = timed(lambda: sdm.recur(shape, lists["idx_w"], lists["w_w"], lists["idx_r"], lists["w_r"], dev["v"],
+                                     dev["alpha"], dev["beta"], mem, y, ws, stream=st), steps)
+    ms_init = timed(lambda: sdm.init_memory(shape, dev["M0"], mem, st), steps)
+    if sdm.device_status(st) != 0:
+        raise RuntimeError(f"device status word set in the {name} leg")
+    peaks = _peaks()
+    rec_bytes = cfg.recurrence_bytes_per_token_head() * B * H * T
+    gbs = rec_bytes / (ms_rec * 1e-3) / 1e9
+    return {"workload": _workload_desc(cfg), "data": "synthetic (device-drawn, the workload's distributions)",
+            "tokens_per_s": B * T / (ms * 1e-3), "ms_per_step": ms,
+            "step": "sdm_forward_m0 (M0 broadcast beside the addressing, then the recurrence)",
+            "phase_ms": {"init_memory": ms_init, "address": ms_addr, "recurrence": ms_rec},
+            "recurrence_gbs": gbs, "recurrence_frac_of_measured": gbs / peaks["hbm_gbs"],
+            "recurrence_frac_of_8tbs": gbs / 8000.0, "recurrence_bytes": rec_bytes, "gpu_launches_per_step": 8}
+
+
+def leg_decode(steps: int, warmup: int) -> dict:
+    """The decode workload: B=256 sequences x H=16 heads, one token per call on the 275 GB
+    state, per-sequence memories pre-filled by 1024 decode steps from M0, then `steps`
+    consecutive steps replayed as one CUDA graph.  Each step has its own inputs (a pool of 64
+    input sets cycled, so no step re-reads the previous steps' rows from L2)."""
+    import torch
+    import paper_2607_07386_gb300 as sdm
+    cfg = synth.DECODE
+    B, H, N, dv, dk = cfg.B, cfg.H, cfg.N, cfg.d_v, cfg.d_k
+    pool = 64
+    dev = device_inputs(cfg.with_(T=pool), seed=cfg.seed)
+    shape = sdm.SdmShape.make(B, H, 1, dk, dv, N, cfg.k_write, cfg.k_read, cfg.dtype)
+    mem = torch.empty((B, H, N, dv), dtype=torch.bfloat16, device="cuda")
+    y = torch.empty((B, H, dv), dtype=torch.bfloat16, device="cuda")
+    ws = torch.empty(sdm.workspace_bytes(shape), dtype=torch.uint8, device="cuda")
+    per = [{n: dev[n][:, :, i].contiguous() for n in ("q", "k", "v", "alpha", "beta")} for i in range(pool)]
+    st = torch.cuda.Stream()
+    with torch.cuda.stream(st):
+        sdm.init_memory(shape, dev["M0"], mem, st)
+
+        def one(i):
+            x = per[i % pool]
+            sdm.decode_step(shape, dev["P_q"], dev["P_k"], x["q"], x["k"], x["v"], x["alpha"], x["beta"], mem, y, ws,
+                            stream=st)
+
+        for i in range(cfg.prefill_steps):
+            one(i)
+        for i in range(warmup):
+            one(i)
+        st.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(st)
+        for i in range(steps):
+            one(i)
+        e1.record(st)
+        st.synchronize()
+        direct_us = e0.elapsed_time(e1) / steps * 1e3
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=st):
+            for i in range(steps):
+                one(i)
+        graph.replay()
+        st.synchronize()
+        e0.record(st)
+        graph.replay()
+        e1.record(st)
+        st.synchronize()
+        graph_us = e0.elapsed_time(e1) / steps * 1e3
+    if sdm.device_status(st) != 0:
+        raise RuntimeError("device status word set in the decode leg")
+    per_step = cfg.algorithmic_bytes_per_token_head() * B * H
+    peaks = _peaks()
+    return {"workload": _workload_desc(cfg) + f" prefill={cfg.prefill_steps} timed={steps}",
+            "data": "synthetic (device-drawn, the workload's distributions)",
+            "us_per_step": graph_us, "us_per_step_direct_calls": direct_us,
+            "tokens_per_s": B / (graph_us * 1e-6), "algorithmic_bytes_per_step": per_step,
+            "gbs": per_step / (graph_us * 1e-6) / 1e9, "frac_of_measured": per_step / (graph_us * 1e-6) / 1e9 / peaks["hbm_gbs"],
+            "timing": f"{steps} consecutive steps captured in one CUDA graph, one replay timed with CUDA events"}
+
+
+def run_leg(args):
+    """`bench.py --leg NAME`: one workload leg in its own process, printing one JSON object."""
+    import torch
+    from paper_2607_07386_gb300.build import build
+    torch.cuda.set_device(0)
+    build()
+    res = leg_decode(args.steps, args.warmup) if args.leg == "decode" else leg_scan(args.leg, args.steps, args.warmup)
+    print(json.dumps(res), flush=True)
+
+
+def legs_in_subprocesses(names, warmup: int) -> dict:
+    """Each (leg, steps) in a child process (its own CUDA context and memory), after the main
+    leg has released its memory; a leg that fails reports its error instead of a result."""
+    out = {}
+    for name, st in names:
+        cmd = [sys.executable, os.path.abspath(__file__), "--leg", name, "--steps", str(st), "--warmup", str(warmup)]
+        try:
+            r = subprocess.run(cmd, capture_output=True, text=True, timeout=900)
+            lines = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+            out[name] = json.loads(lines[-1]) if r.returncode == 0 and lines else {
+                "error": f"exit {r.returncode}: " + (r.stderr.strip().splitlines() or ["?"])[-1][:300]}
+        except Exception as e:          # timeout or a crashed child: report it, keep the main line
+            out[name] = {"error": repr(e)[:300]}
+    return out
+
+
 def run_ours(args, cfg):
     import torch
     import paper_2607_07386_gb300 as sdm
@@ -479,6 +643,14 @@ def run_ours(args, cfg):
                      "frac_of_8tbs": step_bytes / (ms_step * 1e-3) / 1e9 / 8000.0},
         "clocks": clocks,
     }
+    if rank == 0 and world == 1 and not args.no_legs:
+        # the other workloads (scan workloads and decode), each in its own process once this
+        # process has released its device memory
+        del dev, mem, y, ws, idx_w, w_w, idx_r, w_r, bufs, ys
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+        line["workloads"] = legs_in_subprocesses(
+            [("small_bf16", max(args.steps, 10)), ("long_ctx", 3), ("decode", 1000)], args.warmup)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(cfg)
     if rank == 0:
@@ -495,12 +667,17 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--config", default="layer_1p4b", choices=sorted(synth.CONFIGS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-legs", action="store_true", help="skip the other workloads' legs")
+    ap.add_argument("--leg", default=None, help=argparse.SUPPRESS)   # internal: one workload leg
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
+    if args.leg:
+        run_leg(args)
+        return
     cfg = synth.get_config(args.config)
     if cfg.is_decode:
-        raise SystemExit("the decode workload is exercised by the tests; bench.py times the scan workloads")
+        raise SystemExit("the decode workload is timed by the decode leg of the default run")
     if args.impl == "reference":
         run_reference(args, cfg)
     else:

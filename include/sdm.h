@@ -315,19 +315,20 @@ sdm_status sdm_device_stats(uint32_t* counts, int n, sdm_stream_t stream);
 /* Launch plan of the recurrence kernels for `shape` (the paper has no counterpart; for
  * tests that must reach a given kernel variant, and for tuning).  Writes the first n
  * (<= 6) of, in order: the 16-byte chunks of a memory row each warp owns (its d-range),
- * the warps (d-ranges) per (b, h) chain, the slot positions each lane handles per token,
- * the look-ahead in tokens of the row prefetch, 1 if the writer/reader kernel runs (else
- * 0), and the warps per CTA of the fused kernel.  Host only: launches nothing. */
+ * the d-ranges per (b, h) chain, the slot positions each lane handles per token, the
+ * hazard window in tokens (row prefetches in flight ahead of the processed token), the
+ * warps per CTA that interleave the tokens of one (chain, d-range) (0 when T == 1: one
+ * warp, no look-ahead), and each such warp's prefetch depth in its own tokens.  Host
+ * only: launches nothing. */
 sdm_status sdm_recur_plan(const sdm_shape* shape, int32_t* out, int n);
 
 /* Test hook for the bounded device waits (the paper has no counterpart).  Runs sdm_recur
- * (same arguments and workspace) with every wait of the writer/reader recurrence kernel
- * limited to wait_cycles SM clock cycles (1 .. 2^32) and with the writer warps withholding
- * their first hand-over.  The readers' first wait therefore runs out; every CTA leaves its
- * token loop and returns, and bit 2 of the device status word is set (sdm_device_status
- * then returns SDM_ERR_TIMEOUT).  y and mem are left undefined.  Returns
- * SDM_ERR_UNSUPPORTED when the writer/reader kernel does not serve `shape` (sdm_recur_plan
- * field 4 is 0). */
+ * (same arguments and workspace) with every wait of the token-interleaved recurrence
+ * kernel limited to wait_cycles SM clock cycles (1 .. 2^32), and with the first warp of
+ * every CTA withholding the progress word of token 0.  The other warps' waits for it run
+ * out; every CTA leaves its token loop and returns, and bit 2 of the device status word is
+ * set (sdm_device_status then returns SDM_ERR_TIMEOUT).  y and mem are left undefined.
+ * Returns SDM_ERR_UNSUPPORTED when that kernel does not serve `shape` (T == 1). */
 sdm_status sdm_test_recur_wait_timeout(const sdm_shape* shape, const int32_t* idx_w, const float* w_w,
                                        const int32_t* idx_r, const float* w_r, const void* v,
                                        const void* alpha, const void* beta, void* mem, void* y,

@@ -310,7 +310,7 @@ def device_status(stream=None) -> int:
     return int(code.value)
 
 
-RECUR_PLAN_FIELDS = ("dch", "nsplit", "spt", "la", "split", "wpc")
+RECUR_PLAN_FIELDS = ("dch", "nsplit", "spt", "la", "w", "p")
 
 
 def recur_plan(shape: SdmShape) -> dict:
@@ -322,8 +322,8 @@ def recur_plan(shape: SdmShape) -> dict:
 
 def test_recur_wait_timeout(shape: SdmShape, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem, y, workspace,
                             wait_cycles: int, stream=None):
-    """sdm_test_recur_wait_timeout: the writer/reader recurrence with a withheld hand-over and a
-    short wait limit (the bounded waits must run out and set status bit 2)."""
+    """sdm_test_recur_wait_timeout: the token-interleaved recurrence with a withheld progress
+    word and a short wait limit (the bounded waits must run out and set status bit 2)."""
     _check(lib().sdm_test_recur_wait_timeout(ctypes.byref(shape), _ptr(idx_w), _ptr(w_w), _ptr(idx_r), _ptr(w_r),
                                              _ptr(v), _ptr(alpha), _ptr(beta), _ptr(mem), _ptr(y), _ptr(workspace),
                                              _nbytes(workspace) or 0, int(wait_cycles), _stream(stream)))

@@ -732,7 +732,7 @@ sdm_status sdm_recur_plan(const sdm_shape* s, int32_t* out, int n) {
     SDM_TRY(check_shape(s, false, nullptr));
     if (!out || n < 0 || n > 6) return fail(SDM_ERR_INVALID_ARG, "sdm_recur_plan: out must be non-NULL and n in [0, 6]");
     const sdm::RecPlan p = sdm::rec_plan(s->dtype, s->B, s->H, s->T, s->d_v, s->k_write, s->k_read);
-    const int32_t v[6] = {p.dch, p.nsplit, p.spt, p.la, p.split, p.wpc};
+    const int32_t v[6] = {p.dch, p.nsplit, p.spt, p.la, p.w, p.p};
     for (int i = 0; i < n; ++i) out[i] = v[i];
     return ok();
 }
@@ -745,8 +745,8 @@ sdm_status sdm_test_recur_wait_timeout(const sdm_shape* s, const int32_t* idx_w,
     if (wait_cycles < 1 || wait_cycles > (static_cast<int64_t>(1) << 32))
         return fail(SDM_ERR_INVALID_ARG, "sdm_test_recur_wait_timeout: wait_cycles must be in [1, 2^32]");
     const sdm::RecPlan p = sdm::rec_plan(s->dtype, s->B, s->H, s->T, s->d_v, s->k_write, s->k_read);
-    if (!p.split || static_cast<int64_t>(s->B) * s->H * s->T == 0)
-        return fail(SDM_ERR_UNSUPPORTED, "sdm_test_recur_wait_timeout: the writer/reader kernel does not serve this shape");
+    if (p.w < 2 || static_cast<int64_t>(s->B) * s->H * s->T == 0)
+        return fail(SDM_ERR_UNSUPPORTED, "sdm_test_recur_wait_timeout: the token-interleaved kernel does not serve this shape");
     return recur_impl("sdm_test_recur_wait_timeout", s, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem, y, nullptr,
                       workspace, workspace_bytes, stream, static_cast<long long>(wait_cycles), 1);
 }

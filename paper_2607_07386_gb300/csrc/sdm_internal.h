@@ -63,21 +63,22 @@ struct RecArgs {
     int B, H, T, dv, kw, kr;
     int64_t N;
     int* err;
+    const int32_t* firstw;                    // lazy initial memory: first writer of each slot in
+                                              // this call ([B*H, N]), or nullptr
     long long wait_cycles;                    // limit of every bounded device wait (0: the default)
-    int hold_handover;                        // test hook: the writer warp withholds its first
-                                              // hand-over, so the reader's wait runs out
+    int hold_handover;                        // test hook: the first warp withholds its first
+                                              // progress word, so the other warps' waits run out
 };
 // Launch geometry of the recurrence (depends only on the shape).
 struct RecPlan {
-    int dch;      // 16-byte chunks of a row per CTA
-    int nsplit;   // CTAs per chain
-    int threads;  // threads per CTA
-    int spt;      // slots per thread per token
-    int la;       // lookahead depth (tokens whose gathers are in flight)
+    int dch;      // 16-byte chunks of a row per warp (its d-range)
+    int nsplit;   // d-ranges per chain
+    int spt;      // slot positions per lane per token
+    int la;       // hazard window in tokens (prefetches in flight ahead of the processed token)
     int kmax;     // max(k_write, k_read)
-    int split;    // writer and reader warps per (chain, d-range) (look-ahead > 1 only)
-    int wpc;      // warps per CTA of the fused kernel (consecutive d-ranges of a chain)
-    size_t smem;  // dynamic shared memory per CTA
+    int w;        // warps per CTA interleaving the tokens of one (chain, d-range); 0: one token
+                  // per chain (T == 1), one warp per (chain, d-range), no look-ahead
+    int p;        // prefetch depth of each interleaving warp, in its own tokens
 };
 RecPlan rec_plan(int dtype, int B, int H, int T, int dv, int kw, int kr);
 // Scratch of the recurrence: the hazard table [B, H, T, max(kw, kr)] int32.

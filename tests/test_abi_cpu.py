@@ -242,17 +242,17 @@ def test_recur_plan_reports_the_launch_shape(sdm):
     assert sdm.lib().sdm_recur_plan(ctypes.byref(mk(full, 16)), arr, 7) == 1 and "[0, 6]" in sdm.last_error()
 
 
-def test_wait_timeout_hook_rejects_shapes_without_the_handover(sdm):
+def test_wait_timeout_hook_rejects_shapes_without_interleaved_warps(sdm):
     L = sdm.lib()
     args = [FAKE, FAKE + 0x100000, FAKE + 0x200000, FAKE + 0x300000, FAKE + 0x400000, FAKE + 0x500000,
             FAKE + 0x600000, FAKE + 0x10000000, FAKE + 0x700000, FAKE + 0x40000000, 1 << 30]
-    fused = _shape(sdm, B=8, H=16, T=64, d_k=128, d_v=128, N=262144, k_write=32, k_read=32)
-    assert sdm.recur_plan(fused)["split"] == 0
-    assert L.sdm_test_recur_wait_timeout(ctypes.byref(fused), *args, 1000, None) == 2
-    assert "writer/reader" in sdm.last_error()
-    split = _shape(sdm, B=1, H=2, T=8, d_v=64, N=4096, k_write=8, k_read=8)
-    assert sdm.recur_plan(split)["split"] == 1
-    assert L.sdm_test_recur_wait_timeout(ctypes.byref(split), *args, 0, None) == 1 and "wait_cycles" in sdm.last_error()
+    one = _shape(sdm, B=8, H=16, T=1, d_k=128, d_v=128, N=262144, k_write=32, k_read=32)
+    assert sdm.recur_plan(one)["w"] == 0
+    assert L.sdm_test_recur_wait_timeout(ctypes.byref(one), *args, 1000, None) == 2
+    assert "token-interleaved" in sdm.last_error()
+    many = _shape(sdm, B=1, H=2, T=8, d_v=64, N=4096, k_write=8, k_read=8)
+    assert sdm.recur_plan(many)["w"] >= 2
+    assert L.sdm_test_recur_wait_timeout(ctypes.byref(many), *args, 0, None) == 1 and "wait_cycles" in sdm.last_error()
 
 
 def test_noalloc_size_check_cannot_wrap(sdm):
