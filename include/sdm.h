@@ -324,10 +324,10 @@ sdm_status sdm_recur_plan(const sdm_shape* shape, int32_t* out, int n);
 
 /* Test hook for the bounded device waits (the paper has no counterpart).  Runs sdm_recur
  * (same arguments and workspace) with every wait of the token-interleaved recurrence
- * kernel limited to wait_cycles SM clock cycles (1 .. 2^32), and with the first warp of
- * every CTA withholding the progress word of token 0.  The other warps' waits for it run
- * out; every CTA leaves its token loop and returns, and bit 2 of the device status word is
- * set (sdm_device_status then returns SDM_ERR_TIMEOUT).  y and mem are left undefined.
+ * kernel limited to wait_cycles SM clock cycles (1 .. 2^32), with the first warp of every
+ * CTA withholding the progress word of token 0 and every later token waiting for it.  Those
+ * waits run out; every CTA leaves its token loop and returns, and bit 2 of the device status
+ * word is set (sdm_device_status then returns SDM_ERR_TIMEOUT).  y and mem are left undefined.
  * Returns SDM_ERR_UNSUPPORTED when that kernel does not serve `shape` (T == 1). */
 sdm_status sdm_test_recur_wait_timeout(const sdm_shape* shape, const int32_t* idx_w, const float* w_w,
                                        const int32_t* idx_r, const float* w_r, const void* v,

@@ -134,7 +134,8 @@ __global__ void __launch_bounds__(32) k_recur_one(const RecArgs a, int nsplit, i
     cp_async_commit();
     cp_async_wait<0>();
     __syncwarp();
-    // ---- codes: read slot written by this token (1 + its write position), fresh flags
+    // ---- hazard words (layout of sdm_internal.h): read slot written by this token (code 1 +
+    // its write position), fresh flags
     bool unsorted = false;
     for (int p = lane; p < kmax; p += 32) {
         int code = 0;
@@ -147,13 +148,13 @@ __global__ void __launch_bounds__(32) k_recur_one(const RecArgs a, int nsplit, i
                 if (m[mid] < s) lo = mid + 1; else hi = mid;
             }
             int rc = (lo < kw && m[lo] == s) ? 1 + lo : 0;
-            if (a.firstw && static_cast<uint32_t>(s) < N && __ldg(a.firstw + chain * a.N + s) >= 0) rc |= 0x8000;
-            code |= rc << 16;
+            if (a.firstw && static_cast<uint32_t>(s) < N && __ldg(a.firstw + chain * a.N + s) >= 0) rc |= HZ_R_FRESH >> HZ_R_SHIFT;
+            code |= rc << HZ_R_SHIFT;
         }
         if (p < kw) {
             const int s = m[p];
             unsorted |= p > 0 && m[p - 1] >= s;
-            if (a.firstw && static_cast<uint32_t>(s) < N && __ldg(a.firstw + chain * a.N + s) >= 0) code |= 0x8000;
+            if (a.firstw && static_cast<uint32_t>(s) < N && __ldg(a.firstw + chain * a.N + s) >= 0) code |= HZ_W_FRESH;
         }
         m[4 * KP + p] = code;
     }
@@ -174,11 +175,11 @@ __global__ void __launch_bounds__(32) k_recur_one(const RecArgs a, int nsplit, i
         okw[j] = mw && static_cast<uint32_t>(iw[j]) < N;
         okr[j] = mr && static_cast<uint32_t>(ir[j]) < N;
         bad |= (mw && !okw[j]) || (mr && !okr[j]);
-        const char* bw = (hzv[j] & 0x8000) ? M0c : Mc;
-        const char* br = hzv[j] < 0 ? M0c : Mc;
+        const char* bw = (hzv[j] & HZ_W_FRESH) ? M0c : Mc;
+        const char* br = (hzv[j] & HZ_R_FRESH) ? M0c : Mc;
         cp_async16z(my_rows + j * SLOTB, bw + static_cast<uint64_t>(okw[j] ? iw[j] : 0) * rowbytes, okw[j] ? 16 : 0);
         cp_async16z(my_rows + (KS + j) * SLOTB, br + static_cast<uint64_t>(okr[j] ? ir[j] : 0) * rowbytes, okr[j] ? 16 : 0);
-        fix |= okr[j] && ((hzv[j] >> 16) & 0x7fff) != 0;
+        fix |= okr[j] && hz_rcode(hzv[j]) != 0;
     }
     cp_async_commit();
     const float alpha = load_elem<D>(a.alpha, tok), beta = load_elem<D>(a.beta, tok);
@@ -192,7 +193,7 @@ __global__ void __launch_bounds__(32) k_recur_one(const RecArgs a, int nsplit, i
     const float2 alpha2 = make_float2(alpha, alpha);
 #pragma unroll
     for (int j = 0; j < SPT; ++j) {
-        const bool rfix = okr[j] && ((hzv[j] >> 16) & 0x7fff) != 0;
+        const bool rfix = okr[j] && hz_rcode(hzv[j]) != 0;
         const uint4 mwv = lds128(my_rows + j * SLOTB);
         if (undo_c && okw[j]) *reinterpret_cast<uint4*>(undo_c + (tok * kw + g * SPT + j) * static_cast<int64_t>(rowbytes)) = mwv;
         const uint4 mrv = lds128(my_rows + (KS + j) * SLOTB);
@@ -243,7 +244,7 @@ __global__ void __launch_bounds__(32) k_recur_one(const RecArgs a, int nsplit, i
         for (int e = 0; e < E; ++e) yc[e] = 0.f;
 #pragma unroll
         for (int j = 0; j < SPT; ++j) {
-            const int hr = okr[j] ? ((hzv[j] >> 16) & 0x7fff) : 0;
+            const int hr = okr[j] ? hz_rcode(hzv[j]) : 0;
             if (hr != 0) {
                 const int np = hr - 1;
                 float f[E], o[E];

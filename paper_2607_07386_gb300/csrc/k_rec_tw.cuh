@@ -15,8 +15,10 @@
 //     token writes recomputes the written value from the same operands, bit for bit;
 //   * write after write: a token that writes a slot an earlier token of the window wrote has
 //     a write-gather hazard on it, so it waits for that writer before it writes;
-//   * write after read: a token stores its rows only once every earlier token has gathered
-//     (the other warps' gather words), so no earlier gather sees a later write.
+//   * write after read: when a token of the window read-gathers a slot that token t writes,
+//     t stores its rows only once every token up to that reader has gathered (the warps'
+//     gather words), so no earlier gather sees a later write.  Readers older than the window
+//     were done before t's rows were prefetched.
 // Every wait is bounded: on timeout the CTA sets the timeout bit and leaves.
 #pragma once
 #include "sdm_internal.h"
@@ -44,6 +46,7 @@ __device__ __forceinline__ bool tw_wait_done(volatile int* prog, int ww, int u, 
     const long long t0 = clock64();
     while (prog[ww] < u) {
         if (*abort_flag || clock64() - t0 > limit) return false;
+        __nanosleep(64);                 // leave the issue slots to the warps doing work
     }
     return true;
 }
@@ -160,8 +163,8 @@ __global__ void __launch_bounds__(32 * W) k_recur_tw(const RecArgs a, int nsplit
             if (!lazy) hc[j] = 0;
             const bool ow = my_w[j] && static_cast<uint32_t>(iw[j]) < N;
             const bool orr = my_r[j] && static_cast<uint32_t>(ir[j]) < N;
-            const char* bw = (hc[j] & 0x8000) ? M0c : Mc;
-            const char* br = hc[j] < 0 ? M0c : Mc;
+            const char* bw = (hc[j] & HZ_W_FRESH) ? M0c : Mc;
+            const char* br = (hc[j] & HZ_R_FRESH) ? M0c : Mc;
             const uint32_t at = rows_t + ((g * SPT + j) * DCH + c) * 16;
             cp_async16z(at, bw + static_cast<uint64_t>(ow ? iw[j] : 0) * rowbytes, ow ? 16 : 0);
             cp_async16z(at + KS * SLOTB, br + static_cast<uint64_t>(orr ? ir[j] : 0) * rowbytes, orr ? 16 : 0);
@@ -214,21 +217,24 @@ __global__ void __launch_bounds__(32 * W) k_recur_tw(const RecArgs a, int nsplit
 
         // ---- stale prefetches (rare): wait for the writer token, reload the row from memory
         bool okw[SPT], okr[SPT], stale = false, fix = false;
+        int war_u = -1;                                  // latest earlier reader of a write slot
 #pragma unroll
         for (int j = 0; j < SPT; ++j) {
             okw[j] = my_w[j] && static_cast<uint32_t>(iw[j]) < N;
             okr[j] = my_r[j] && static_cast<uint32_t>(ir[j]) < N;
             bad |= (my_w[j] && !okw[j]) || (my_r[j] && !okr[j]);
-            const int hw = okw[j] ? (hzv[j] & 0x7fff) : 0;
-            const int hr = okr[j] ? ((hzv[j] >> 16) & 0x7fff) : 0;
+            const int hw = okw[j] ? hz_wcode(hzv[j]) : 0;
+            const int hr = okr[j] ? hz_rcode(hzv[j]) : 0;
             stale |= hw != 0 || hr > 64;                 // read codes 1..64: written by this token
             fix |= hr != 0 && hr <= 64;
+            const int war = okw[j] ? hz_war(hzv[j]) : 0;
+            war_u = war ? max(war_u, t - war) : war_u;
         }
         if (__any_sync(0xffffffffu, stale)) {
 #pragma unroll
             for (int j = 0; j < SPT; ++j) {
-                const int hw = okw[j] ? (hzv[j] & 0x7fff) : 0;
-                const int hr = okr[j] ? ((hzv[j] >> 16) & 0x7fff) : 0;
+                const int hw = okw[j] ? hz_wcode(hzv[j]) : 0;
+                const int hr = okr[j] ? hz_rcode(hzv[j]) : 0;
                 if (hw != 0) {
                     const int u = t - ((hw - 1) >> 6);
                     if (!tw_wait_done(prog, u % W, u, abort_flag, limit)) timed_out = true;
@@ -259,7 +265,7 @@ __global__ void __launch_bounds__(32 * W) k_recur_tw(const RecArgs a, int nsplit
         const float2 alpha2 = make_float2(alpha, alpha);
 #pragma unroll
         for (int j = 0; j < SPT; ++j) {
-            const int hr = okr[j] ? ((hzv[j] >> 16) & 0x7fff) : 0;
+            const int hr = okr[j] ? hz_rcode(hzv[j]) : 0;
             const bool rfix = hr != 0 && hr <= 64;
             const uint4 mw = lds128(my_rows + j * SLOTB);
             if (undo_c && okw[j])
@@ -293,10 +299,12 @@ __global__ void __launch_bounds__(32 * W) k_recur_tw(const RecArgs a, int nsplit
         unpack16x2<D>(lds128(mslot + 5 * KP * 4 + c * 16), d2);
 #pragma unroll
         for (int e = 0; e < E2; ++e) d2[e] = __fadd2_rn(d2[e], make_float2(-pp[e].x, -pp[e].y));
-        {
+        if (a.hold_handover && t > 0) war_u = max(war_u, 0);   // (test hook: every later token waits)
+        war_u = __reduce_max_sync(0xffffffffu, war_u);
+        if (war_u >= 0) {                                // (rare) every token up to that reader gathered
             bool ok = true;
 #pragma unroll
-            for (int v = 0; v < W; ++v) ok &= tw_wait_done(gath, v, t - W + 1, abort_flag, limit);
+            for (int v = 0; v < W; ++v) ok &= tw_wait_done(gath, v, war_u - W + 1, abort_flag, limit);
             if (!ok) timed_out = true;
             if (__any_sync(0xffffffffu, timed_out)) break;
             __threadfence_block();
@@ -321,7 +329,7 @@ __global__ void __launch_bounds__(32 * W) k_recur_tw(const RecArgs a, int nsplit
             for (int e = 0; e < E; ++e) yc[e] = 0.f;
 #pragma unroll
             for (int j = 0; j < SPT; ++j) {
-                const int hr = okr[j] ? ((hzv[j] >> 16) & 0x7fff) : 0;
+                const int hr = okr[j] ? hz_rcode(hzv[j]) : 0;
                 if (hr != 0 && hr <= 64) {
                     const int np = hr - 1;
                     float f[E], o[E];

@@ -69,6 +69,25 @@ struct RecArgs {
     int hold_handover;                        // test hook: the first warp withholds its first
                                               // progress word, so the other warps' waits run out
 };
+// Hazard word of a (token t, list position n) pair: written by the hazard pass (k_hazard.cu),
+// read by the recurrence kernels.
+//   bits  0-10  write-gather code: 0 = no token of the window [t - LA, t - 1] wrote the slot,
+//               else 1 + delta * 64 + n' (the latest writer t - delta, its list position n')
+//   bit   11    the write slot is fresh (lazy memory: not written before t; gather M0's row)
+//   bits 12-22  read-gather code, as above with delta in [0, LA] (delta = 0: this token)
+//   bit   23    the read slot is fresh
+//   bits 24-29  write after read: t - u for the latest token u of the window that
+//               read-gathers the write slot (0: none)
+constexpr int HZ_CODE_MASK = 0x7ff;
+constexpr int HZ_W_FRESH = 1 << 11;
+constexpr int HZ_R_SHIFT = 12;
+constexpr int HZ_R_FRESH = 1 << 23;
+constexpr int HZ_WAR_SHIFT = 24;
+constexpr int HZ_MAX_LA = 30;           // 1 + 30 * 64 + 63 < 2^11, and distances < 64
+__host__ __device__ __forceinline__ int hz_wcode(int h) { return h & HZ_CODE_MASK; }
+__host__ __device__ __forceinline__ int hz_rcode(int h) { return (h >> HZ_R_SHIFT) & HZ_CODE_MASK; }
+__host__ __device__ __forceinline__ int hz_war(int h) { return (h >> HZ_WAR_SHIFT) & 63; }
+
 // Launch geometry of the recurrence (depends only on the shape).
 struct RecPlan {
     int dch;      // 16-byte chunks of a row per warp (its d-range)
