@@ -147,11 +147,13 @@ def _oracle_step(pool, cfg, slices, T):
     return max(pool.map(timed_worker, [(cfg, b, h, T) for b, h in slices]))
 
 
-# The oracle sample, the same for the cpu_baseline key and the reference arm: each step runs
-# one (b, h) slice per host core over the slice's first ORACLE_T tokens.  Both legs measure
-# this one sample size, so they time the same work (the oracle's per-slice set-up, a float64
-# copy of the head's M0, is amortised over the same number of tokens).
-ORACLE_T = 512
+# The oracle sample, the same unit of work for the cpu_baseline key and the reference arm: one
+# (b, h) slice per host core over the slice's first ORACLE_T tokens.  Both legs time this unit
+# (the oracle's per-slice set-up, a float64 copy of the head's M0, is amortised over the same
+# number of tokens), so their tokens/s agree; the cpu_baseline key repeats it CPU_REPEATS
+# times for a 10-30 s sample, the reference arm once per step.
+ORACLE_T = 1024
+CPU_REPEATS = 12
 
 
 def _oracle_sample(cfg, pool, cores, steps, seed):
@@ -164,14 +166,16 @@ def _oracle_sample(cfg, pool, cores, steps, seed):
 
 
 def cpu_baseline(cfg):
-    """Oracle throughput on a bounded sample: one (b, h) slice x ORACLE_T tokens per core;
-    tokens/s per layer = slice-tokens / H / time (slices are independent, so per-core work adds up)."""
+    """Oracle throughput on a bounded sample: CPU_REPEATS rounds of one (b, h) slice x ORACLE_T
+    tokens per core; tokens/s per layer = slice-tokens / H / time (slices are independent, so
+    per-core work adds up)."""
     cores = os.cpu_count() or 1
     with _oracle_pool(cores) as pool:
-        value, times = _oracle_sample(cfg, pool, cores, 1, 0)
+        value, times = _oracle_sample(cfg, pool, cores, CPU_REPEATS, 0)
     return {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
-            "sample": f"{cores} (b,h) slices x first {ORACLE_T} tokens of {cfg.name}, one float64 worker per core, "
-                      f"{times[0]:.1f} s (slowest worker, input generation excluded)"}
+            "sample": f"{CPU_REPEATS} rounds of {cores} (b,h) slices x first {ORACLE_T} tokens of {cfg.name}, one "
+                      f"float64 worker per core, {sum(times):.1f} s (slowest worker per round, input generation "
+                      "excluded); the reference arm times the same unit"}
 
 
 def run_reference(args, cfg):

@@ -68,6 +68,14 @@ __device__ __forceinline__ void sts128(uint32_t addr, const uint4& v, bool pred)
 __device__ __forceinline__ void cp_async16z(uint32_t dst, const void* src, int src_bytes) {
     asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
 }
+// The same for a piece of a memory row; when whole256 (rows a multiple of 256 bytes), L2
+// fetches the whole aligned 256-byte region around it.
+__device__ __forceinline__ void cp_async16z_row(uint32_t dst, const void* src, int src_bytes, bool whole256) {
+    if (whole256)
+        asm volatile("cp.async.cg.shared.global.L2::256B [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+    else
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
 
 // ------------------------------------------------------------------------------------------
 // One token per chain (a decode step, T == 1): one warp per (chain, d-range), no look-ahead and
@@ -104,6 +112,7 @@ __global__ void __launch_bounds__(32) k_recur_one(const RecArgs a, int nsplit, i
     const int64_t chain = gw / nsplit;
     const int split = static_cast<int>(gw - chain * nsplit);
     const uint32_t rowbytes = static_cast<uint32_t>(a.dv) * D::BYTES;
+    const bool row256 = rowbytes % 256 == 0;
     const int64_t dbyte = static_cast<int64_t>(split * DCH) * 16;
     const char* Mc = static_cast<const char*>(a.mem) + chain * a.N * static_cast<int64_t>(rowbytes) + dbyte + c * 16;
     char* Mw = const_cast<char*>(Mc);
@@ -177,8 +186,8 @@ __global__ void __launch_bounds__(32) k_recur_one(const RecArgs a, int nsplit, i
         bad |= (mw && !okw[j]) || (mr && !okr[j]);
         const char* bw = (hzv[j] & HZ_W_FRESH) ? M0c : Mc;
         const char* br = (hzv[j] & HZ_R_FRESH) ? M0c : Mc;
-        cp_async16z(my_rows + j * SLOTB, bw + static_cast<uint64_t>(okw[j] ? iw[j] : 0) * rowbytes, okw[j] ? 16 : 0);
-        cp_async16z(my_rows + (KS + j) * SLOTB, br + static_cast<uint64_t>(okr[j] ? ir[j] : 0) * rowbytes, okr[j] ? 16 : 0);
+        cp_async16z_row(my_rows + j * SLOTB, bw + static_cast<uint64_t>(okw[j] ? iw[j] : 0) * rowbytes, okw[j] ? 16 : 0, row256);
+        cp_async16z_row(my_rows + (KS + j) * SLOTB, br + static_cast<uint64_t>(okr[j] ? ir[j] : 0) * rowbytes, okr[j] ? 16 : 0, row256);
         fix |= okr[j] && hz_rcode(hzv[j]) != 0;
     }
     cp_async_commit();

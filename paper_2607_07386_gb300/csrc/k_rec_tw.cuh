@@ -90,6 +90,7 @@ __global__ void __launch_bounds__(32 * W) k_recur_tw(const RecArgs a, int nsplit
     const int64_t chain = blockIdx.x / nsplit;
     const int split = static_cast<int>(blockIdx.x - chain * nsplit);
     const uint32_t rowbytes = static_cast<uint32_t>(a.dv) * D::BYTES;
+    const bool row256 = rowbytes % 256 == 0;
     const int64_t dbyte = static_cast<int64_t>(split * DCH) * 16;
     const char* Mc = static_cast<const char*>(a.mem) + chain * a.N * static_cast<int64_t>(rowbytes) + dbyte + c * 16;
     char* Mw = const_cast<char*>(Mc);
@@ -150,7 +151,10 @@ __global__ void __launch_bounds__(32 * W) k_recur_tw(const RecArgs a, int nsplit
         if (lane < DCH) cp_async16z(slot_addr + 5 * KP * 4 + lane * 16, vrange + static_cast<int64_t>(t) * rowbytes + lane * 16, 16);
     };
     // rows that token t gathers (own slots, own chunk) into rows slot `rows_t`; zero-filled for
-    // invalid slots; fresh slots of the lazy memory come from M0
+    // invalid slots; fresh slots of the lazy memory come from M0.  Each 16-byte piece asks L2 to
+    // fetch the whole aligned 256-byte region around it (the row, at d_v = 128 bf16), so DRAM
+    // moves rows as whole bursts and the other d-ranges' pieces of a row hit L2 (random 64-byte
+    // pieces alone reach less than half of the bandwidth of whole 256-byte rows).
     auto copy_rows = [&](int t, uint32_t meta_addr, uint32_t rows_t) {
         if (t >= T) return;
         const int* m = reinterpret_cast<const int*>(meta_gen + (meta_addr - meta0));
@@ -166,8 +170,8 @@ __global__ void __launch_bounds__(32 * W) k_recur_tw(const RecArgs a, int nsplit
             const char* bw = (hc[j] & HZ_W_FRESH) ? M0c : Mc;
             const char* br = (hc[j] & HZ_R_FRESH) ? M0c : Mc;
             const uint32_t at = rows_t + ((g * SPT + j) * DCH + c) * 16;
-            cp_async16z(at, bw + static_cast<uint64_t>(ow ? iw[j] : 0) * rowbytes, ow ? 16 : 0);
-            cp_async16z(at + KS * SLOTB, br + static_cast<uint64_t>(orr ? ir[j] : 0) * rowbytes, orr ? 16 : 0);
+            cp_async16z_row(at, bw + static_cast<uint64_t>(ow ? iw[j] : 0) * rowbytes, ow ? 16 : 0, row256);
+            cp_async16z_row(at + KS * SLOTB, br + static_cast<uint64_t>(orr ? ir[j] : 0) * rowbytes, orr ? 16 : 0, row256);
         }
     };
     // own tokens: t = w + i * W, i = 0, 1, ...
