@@ -317,8 +317,8 @@ sdm_status sdm_device_stats(uint32_t* counts, int n, sdm_stream_t stream);
  * (<= 6) of, in order: the 16-byte chunks of a memory row each warp owns (its d-range),
  * the d-ranges per (b, h) chain, the slot positions each lane handles per token, the
  * hazard window in tokens (row prefetches in flight ahead of the processed token), the
- * warps per CTA that interleave the tokens of one (chain, d-range) (0 when T == 1: one
- * warp, no look-ahead), and each such warp's prefetch depth in its own tokens.  Host
+ * token phases: warps that interleave the tokens of one (chain, d-range) (0 when T == 1:
+ * one warp, no look-ahead), and each such warp's prefetch depth in its own tokens.  Host
  * only: launches nothing. */
 sdm_status sdm_recur_plan(const sdm_shape* shape, int32_t* out, int n);
 

@@ -345,6 +345,54 @@ def test_recur_high_collision_rate(sdm, dtype, N, k, T):
     assert rel_fro(y, yo) <= TOL[dtype] and rel_fro(M, Mo) <= TOL[dtype]
 
 
+@pytest.mark.parametrize("N,k,T", [(300, 32, 150), (4096, 32, 97), (2 ** 18, 32, 64)])
+def test_interleaved_recurrence_with_collisions_on_many_chains(sdm, N, k, T):
+    """The token-interleaved recurrence on 96 chains (d_v = 128 bf16, k = 32, several token
+    phases per chain): with N = 300 almost every token re-reads and rewrites rows of the tokens
+    just before it (stale-row reloads after their writer, write-after-read waits, reads of
+    slots the token itself writes); sampled chains against the oracle."""
+    B, H, dv = 8, 12, 128
+    shape = sdm.SdmShape.make(B, H, T, 32, dv, N, k, k, "bf16")
+    assert sdm.recur_plan(shape)["w"] >= 4
+    rng = np.random.default_rng(N + T)
+    C = B * H
+    sampled = (0, 37, C - 1)
+    # the memory is drawn on the device (the 2^18-slot case holds 6.4 GB); the sampled chains'
+    # initial rows come back for the oracle
+    gen = torch.Generator(device="cuda").manual_seed(N + T)
+    mem = (torch.randn((B, H, N, dv), generator=gen, device="cuda") * 0.3).to(torch.bfloat16)
+    M0s = {c: O.to_f64(G.host(mem[c // H, c % H], "bf16"), "bf16") for c in sampled}
+    iw = np.stack([np.sort(rng.choice(N, k, replace=False)) for _ in range(C * T)]).reshape(B, H, T, k)
+    ir = np.stack([np.sort(rng.choice(N, k, replace=False)) for _ in range(C * T)]).reshape(B, H, T, k)
+    ww = rng.dirichlet(np.ones(k), C * T).astype(np.float32).reshape(B, H, T, k)
+    wr = rng.dirichlet(np.ones(k), C * T).astype(np.float32).reshape(B, H, T, k)
+    a = O.round_storage(1 / (1 + np.exp(-rng.standard_normal((B, H, T)) - 2)), "bf16")
+    b = O.round_storage(1 / (1 + np.exp(-rng.standard_normal((B, H, T)))), "bf16")
+    V = O.round_storage(rng.standard_normal((B, H, T, dv)), "bf16")
+    st = lambda x: to_torch(O.to_bf16_bits(x), "bf16")
+    cu = lambda x: torch.from_numpy(np.ascontiguousarray(x)).cuda()
+    y = torch.empty((B, H, T, dv), dtype=torch.bfloat16, device="cuda")
+    ws = torch.empty(sdm.recur_workspace_bytes(shape), dtype=torch.uint8, device="cuda")
+    sdm.recur(shape, cu(iw.astype(np.int32)), cu(ww), cu(ir.astype(np.int32)), cu(wr), st(V), st(a), st(b), mem, y, ws)
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    gy = O.to_f64(G.host(y, "bf16"), "bf16")
+    for c in sampled:
+        bb, hh = divmod(c, H)
+        gm = O.to_f64(G.host(mem[bb, hh], "bf16"), "bf16")
+        Mo = M0s[c].copy()
+        _, yo = O.recur(Mo, iw[bb, hh], ww[bb, hh].astype(np.float64), ir[bb, hh], wr[bb, hh].astype(np.float64),
+                        V[bb, hh], a[bb, hh], b[bb, hh], "bf16")
+        assert rel_fro(gy[bb, hh], yo) <= TOL["bf16"] and rel_fro(gm, Mo) <= TOL["bf16"], c
+        _check_elementwise("bf16", gy[bb, hh], yo, ("y", c))
+        touched = np.unique(iw[bb, hh])
+        _check_elementwise("bf16", gm[touched], Mo[touched], ("written rows", c))
+        untouched = np.setdiff1d(np.arange(N), touched)
+        assert np.array_equal(gm[untouched], M0s[c][untouched])
+    del mem, y, ws
+    torch.cuda.empty_cache()
+
+
 def test_unsorted_slot_list_is_reported(sdm):
     N, dv, T = 64, 32, 3
     idx = np.array([[3, 1], [2, 5], [4, 6]])
