@@ -322,6 +322,17 @@ sdm_status sdm_device_stats(uint32_t* counts, int n, sdm_stream_t stream);
  * only: launches nothing. */
 sdm_status sdm_recur_plan(const sdm_shape* shape, int32_t* out, int n);
 
+/* Test hook of the tensor-core score kernel (the paper has no counterpart): the raw fp32
+ * scores s = P x (Sec. 3.1 item 1) the selection starts from, as the tcgen05 MMA accumulates
+ * them, written to scores [2][H][B*T][2 sqrt(N)] float32 (side 0: q with P_q, side 1: k with
+ * P_k; token index b*T + t; columns of both halves).  For testing the error bound the
+ * selection certifies with.  Same arguments as sdm_address otherwise (workspace of
+ * sdm_workspace_bytes).  Returns SDM_ERR_UNSUPPORTED for shapes that do not take the
+ * tensor-core path (bf16, PROJECTED, d_k 64 or 128, k <= 32). */
+sdm_status sdm_test_scores(const sdm_shape* shape, const void* P_q, const void* P_k, const void* q,
+                           const void* k, float* scores, void* workspace, size_t workspace_bytes,
+                           sdm_stream_t stream);
+
 /* Test hook for the bounded device waits (the paper has no counterpart).  Runs sdm_recur
  * (same arguments and workspace) with every wait of the token-interleaved recurrence
  * kernel limited to wait_cycles SM clock cycles (1 .. 2^32), with the first warp of every

@@ -11,5 +11,5 @@ from ._binding import (  # noqa: F401
     recur_workspace_bytes, workspace_bytes, RECUR_NOALLOC_SCRATCH_BYTES, forward_lazy, lazy_workspace_bytes,
     materialize, touched_words, access_stats, access_stats_workspace_bytes, gates, norm_gate,
     undo_log_bytes, recur_undo, recur_backward, recur_chunkwise, recur_plan, test_recur_wait_timeout,
-    RECUR_PLAN_FIELDS,
+    RECUR_PLAN_FIELDS, test_scores,
 )

@@ -100,6 +100,8 @@ def lib():
             L.sdm_recur_noalloc.restype = ctypes.c_int
             L.sdm_device_stats.argtypes = [ctypes.POINTER(ctypes.c_uint32), ctypes.c_int, _VP]
             L.sdm_device_stats.restype = ctypes.c_int
+            L.sdm_test_scores.argtypes = [_SHP, _VP, _VP, _VP, _VP, _VP, _VP, _SZ, _VP]
+            L.sdm_test_scores.restype = ctypes.c_int
             L.sdm_recur_plan.argtypes = [_SHP, ctypes.POINTER(ctypes.c_int32), ctypes.c_int]
             L.sdm_recur_plan.restype = ctypes.c_int
             L.sdm_test_recur_wait_timeout.argtypes = [_SHP, _I32P, _VP, _I32P, _VP, _VP, _VP, _VP, _VP, _VP, _VP,
@@ -308,6 +310,12 @@ def device_status(stream=None) -> int:
     if st not in (0, 5, 6):
         _check(st)
     return int(code.value)
+
+
+def test_scores(shape: SdmShape, P_q, P_k, q, k, scores, workspace, stream=None):
+    """sdm_test_scores: raw tensor-core scores [2, H, B*T, 2 sqrt(N)] float32 into `scores`."""
+    _check(lib().sdm_test_scores(ctypes.byref(shape), _ptr(P_q), _ptr(P_k), _ptr(q), _ptr(k), _ptr(scores),
+                                 _ptr(workspace), _nbytes(workspace) or 0, _stream(stream)))
 
 
 RECUR_PLAN_FIELDS = ("dch", "nsplit", "spt", "la", "w", "p")

@@ -157,6 +157,7 @@ struct MmaLaunch {
     float* part_v;
     int* part_i;
     int* err;
+    float* raw;                 // test hook: the raw fp32 scores [2H][B*T][2S] instead of the lists
 };
 
 // COLS: TMEM columns (fp32 accumulators) = maximum chunk width (512: one CTA per SM;
@@ -243,6 +244,24 @@ __global__ void __launch_bounds__(MM_THREADS, 1) k_addr_mma(const __grid_constan
     const bool valid = ok && b < a.B && t < a.T;
     const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
     const int nblk32 = npad / 32 + ((npad & 31) ? 1 : 0);   // 32-column blocks with columns
+
+    if (a.raw != nullptr) {
+        // test hook: the accumulators themselves, one token row per thread, no selection
+        float* dst = a.raw + (static_cast<int64_t>(blockIdx.z) * BT + static_cast<int64_t>(b) * a.T + t) * (2 * a.S) + hf * a.S + c0;
+#pragma unroll 1
+        for (int cb = 0; cb < nblk32; ++cb) {
+            float v[32];
+            tmem_ld32(trow + cb * 32, v);                        // warp-collective: every lane loads
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+                if (valid && cb * 32 + j < np) dst[cb * 32 + j] = v[j];
+        }
+        if (!ok && tid == 0) flag_error(a.err, ERR_TIMEOUT);
+        asm volatile("tcgen05.fence::before_thread_sync;\n" ::: "memory");
+        __syncthreads();
+        if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;\n" ::"r"(tmem), "r"(COLS) : "memory");
+        return;
+    }
 
     // 1-2. top-2 of each column class mod 32; threshold = L-th largest of those 64 values
     // (>= L distinct columns reach it, so it is a lower bound on the L-th largest score)
@@ -406,6 +425,7 @@ cudaError_t launch_address_mma(const AddrPlan& plan, const AddrArgs& aa, cudaStr
     a.part_v = aa.part_v;
     a.part_i = aa.part_i;
     a.err = aa.err;
+    a.raw = aa.raw;
 
     CUtensorMap maps[4];
     for (int s = 0; s < 2; ++s) {

@@ -175,6 +175,24 @@ Layout layout_for(const sdm_shape* s, int64_t S, bool lazy = false) {
     return L;
 }
 
+// |fp32 score - float64 score| <= c * sum_d |P_jd x_d| <= c * max_j ||P_j|| * ||x||.
+//   FFMA path (sequential fp32 fused multiply-adds in d order): c = (d_k + 4) 2^-24, the
+//   classical gamma_{d_k} bound with the float64 reference's own rounding as margin.
+//   Tensor cores (tcgen05.mma kind::f16, bf16 operands, fp32 accumulation, K = 16 per
+//   instruction): every product of two bf16 numbers is exact in fp32.  One instruction adds
+//   16 products to the accumulator D; modelling it as an alignment of the 17 terms to the
+//   largest exponent e with at least 24 significant bits kept (each term off by less than
+//   2^(e-23) <= 2^-23 max|term|) and a rounding or truncation of the result to fp32 (off by
+//   at most 2^-23 |D'|) bounds its error by 18 * 2^-23 (|D| + sum of the block's |products|).
+//   |D| before block i is at most the sum of the earlier blocks' |products|, so over the
+//   d_k / 16 instructions the error is at most 18 (d_k / 16) 2^-23 sum_d |P_jd x_d|, plus
+//   2^-40 of slack for the float64 reference (d_k 2^-53).  The model allows more error than
+//   round-to-nearest accumulation could make; the GPU test of the raw scores checks it.
+double score_bound_constant(int dk, bool mma) {
+    if (!mma) return (dk + 4) * 0x1p-24;
+    return 18.0 * ((dk + 15) / 16) * 0x1p-23 + 0x1p-40;
+}
+
 // Addressing into the given (or workspace) index/weight buffers.
 sdm_status run_address(const sdm_shape* s, int64_t S, const Layout& L, const void* P_q, const void* P_k, const void* q,
                        const void* k, int32_t* idx_w, float* w_w, int32_t* idx_r, float* w_r, char* ws,
@@ -190,10 +208,7 @@ sdm_status run_address(const sdm_shape* s, int64_t S, const Layout& L, const voi
     a.B = s->B; a.H = s->H; a.T = s->T; a.dk = s->d_k; a.S = static_cast<int>(S);
     a.ncc = L.plan.ncc;
     a.cw = L.plan.cw;
-    // |fp32 score - float64 score| <= cbound * max_j ||P_j|| * ||x||: (d_k + 4) * 2^-24 covers sequential
-    // fp32 FMA accumulation plus the float64 reference's own rounding; the tensor-core path
-    // (blocked accumulation, truncating adds) is given 4x that margin.
-    a.cbound = static_cast<float>((s->d_k + 4) * 0x1p-24 * (L.plan.mma ? 4.0 : 1.0));
+    a.cbound = static_cast<float>(score_bound_constant(s->d_k, L.plan.mma));
     a.part_v = reinterpret_cast<float*>(ws + L.part_v);
     a.part_i = reinterpret_cast<int*>(ws + L.part_i);
     a.pnorm = reinterpret_cast<float*>(ws + L.pnorm);
@@ -725,6 +740,37 @@ sdm_status sdm_device_status(int32_t* code, sdm_stream_t stream) {
                     "device status word = 0x%x (bit 0: slot index outside [0, N) skipped; "
                     "bit 1: slot list not strictly ascending; bit 2: bounded wait timed out; "
                     "bit 3: selection invariant failed)", host);
+    return ok();
+}
+
+sdm_status sdm_test_scores(const sdm_shape* s, const void* P_q, const void* P_k, const void* q, const void* k,
+                           float* scores, void* workspace, size_t workspace_bytes, sdm_stream_t stream) {
+    int64_t S = 0;
+    SDM_TRY(check_shape(s, true, &S));
+    if (static_cast<size_t>(s->B) * s->H * s->T == 0) return ok();
+    const Layout L = layout_for(s, S);
+    if (!L.plan.mma) return fail(SDM_ERR_UNSUPPORTED, "sdm_test_scores: the shape does not take the tensor-core score path");
+    SDM_TRY(check_vec(P_q, "P_q", 16));
+    SDM_TRY(check_vec(P_k, "P_k", 16));
+    SDM_TRY(check_vec(q, "q", 16));
+    SDM_TRY(check_vec(k, "k", 16));
+    SDM_TRY(check_vec(scores, "scores", 4));
+    if (!workspace || !aligned(workspace, 256) || workspace_bytes < L.total)
+        return fail(SDM_ERR_INVALID_ARG, "sdm_test_scores: workspace must be >= sdm_workspace_bytes and 256-byte aligned");
+    int* err = nullptr;
+    SDM_TRY(status_word(&err));
+    char* ws = static_cast<char*>(workspace);
+    sdm::AddrArgs a{};
+    a.P[0] = P_q; a.P[1] = P_k; a.X[0] = q; a.X[1] = k;
+    a.kk[0] = s->k_read; a.kk[1] = s->k_write;
+    a.B = s->B; a.H = s->H; a.T = s->T; a.dk = s->d_k; a.S = static_cast<int>(S);
+    a.ncc = L.plan.ncc; a.cw = L.plan.cw;
+    a.part_v = reinterpret_cast<float*>(ws + L.part_v);
+    a.part_i = reinterpret_cast<int*>(ws + L.part_i);
+    a.err = err;
+    a.raw = scores;
+    cudaError_t e = sdm::launch_address_mma(L.plan, a, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "sdm_test_scores launch");
     return ok();
 }
 

@@ -32,6 +32,8 @@ struct AddrArgs {
     int* queue;            // workspace [2 + 2 (2 H B T)]: counts of queues A and B, then their
                            // token-side ids (nullptr: one pass does everything)
     int* err;              // device status word
+    float* raw;            // test hook of the tensor-core score kernel: raw fp32 scores
+                           // [2H][B*T][2S] instead of the per-chunk lists (nullptr normally)
 };
 
 // Geometry of the PKM partial lists for a shape (depends only on the shape).

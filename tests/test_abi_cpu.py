@@ -262,3 +262,10 @@ def test_noalloc_size_check_cannot_wrap(sdm):
     assert st == 2 and "fixed scratch" in sdm.last_error()
     neg = sdm.SdmShape.make(-1, 1, 1, 8, 64, 4096, 8, 8, "bf16")
     assert sdm.lib().sdm_recur_noalloc(ctypes.byref(neg), *[FAKE] * 9, None) == 1
+
+
+def test_score_hook_rejects_shapes_off_the_tensor_core_path(sdm):
+    s = _shape(sdm, dtype="f32")
+    st = sdm.lib().sdm_test_scores(ctypes.byref(s), FAKE, FAKE + 0x100000, FAKE + 0x200000, FAKE + 0x300000,
+                                   FAKE + 0x400000, FAKE + 0x40000000, 1 << 30, None)
+    assert st == 2 and "tensor-core" in sdm.last_error()

@@ -150,6 +150,42 @@ def test_address_matches_oracle(sdm, name):
             assert rel_fro(out["w_r"][b, h].cpu().numpy(), wr) <= tol
 
 
+def test_tensor_core_scores_within_the_derived_bound(sdm):
+    """The raw tcgen05 scores (test hook sdm_test_scores) of 4.2M (token, column) pairs at the
+    bench geometry (d_k = 128, 2 sqrt(N) = 1024 columns per side) against float64 sums of the
+    exact products: every |s_gpu - s| <= 18 (d_k / 16) 2^-23 sum_d |P_jd x_d|, the bound the
+    certification uses (model of blocked fp32 accumulation; see score_bound_constant).  Tokens
+    of three kinds: unit Gaussian, heavy-tailed (a few components dominate, so small products
+    are aligned to a large one), and columns with alternating signs (cancelling sums)."""
+    B, H, T, dk, S = 1, 2, 1024, 128, 512
+    shape = sdm.SdmShape.make(B, H, T, dk, 128, S * S, 32, 32, "bf16")
+    rng = np.random.default_rng(91)
+    g = rng.standard_normal((2, H, T, dk))
+    g[:, :, T // 3:2 * T // 3] = g[:, :, T // 3:2 * T // 3] ** 3          # heavy-tailed tokens
+    X = O.round_storage(g / np.linalg.norm(g, axis=-1, keepdims=True), "bf16")
+    P = rng.standard_normal((2, H, 2 * S, dk))
+    P[:, :, :64] = np.abs(P[:, :, :64]) * np.where(np.arange(dk) % 2 == 0, 1.0, -1.0)   # cancelling columns
+    P = O.round_storage(P, "bf16")
+    st = lambda x: to_torch(O.to_bf16_bits(x), "bf16")
+    out = torch.empty((2, H, B * T, 2 * S), dtype=torch.float32, device="cuda")
+    ws = G.workspace(shape)
+    sdm.test_scores(shape, st(P[0]), st(P[1]), st(X[0][None]), st(X[1][None]), out, ws)
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    got = out.cpu().numpy().astype(np.float64)
+    c = 18.0 * (dk // 16) * 2.0 ** -23 + 2.0 ** -40
+    worst = 0.0
+    for side in range(2):
+        for h in range(H):
+            ref = X[side, h] @ P[side, h].T                                  # [T, 2S], exact products
+            bound = c * (np.abs(X[side, h]) @ np.abs(P[side, h]).T)
+            err = np.abs(got[side, h] - ref)
+            assert np.all(err <= bound), (side, h, float((err / bound).max()))
+            worst = max(worst, float((err / bound).max()))
+    assert worst < 1.0
+    print(f"max |error| / bound over {2 * H * T * 2 * S} pairs: {worst:.3e}")
+
+
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
 def test_address_integer_ties(sdm, dtype):
     """Small-integer keys and projections: many exactly equal scores, so the selection
