@@ -34,12 +34,18 @@ __host__ __device__ inline int hz_table_log2(int tile, int la, int kw, int kr) {
     return lg;
 }
 
+// Shared memory of a CTA: the table, then the window's slot lists (write, then read) as int32.
+__host__ __device__ inline size_t hz_smem_bytes(int tile, int la, int kw, int kr) {
+    return (static_cast<size_t>(8) << hz_table_log2(tile, la, kw, kr)) + static_cast<size_t>(tile + la) * (kw + kr) * 4;
+}
+
 // Largest tile (64, 32 or 16 tokens) whose table fits the target size.
 int hz_tile(int la, int kw, int kr) {
     for (int tile = 64; tile > 16; tile >>= 1)
-        if ((static_cast<size_t>(8) << hz_table_log2(tile, la, kw, kr)) <= HZ_TABLE_TARGET) return tile;
+        if (hz_smem_bytes(tile, la, kw, kr) <= HZ_TABLE_TARGET + 32 * 1024) return tile;
     return 16;
 }
+
 
 __device__ __forceinline__ uint32_t hz_hash(uint32_t s, int lg) { return (s * 0x9E3779B1u) >> (32 - lg); }
 
@@ -55,7 +61,24 @@ __global__ void __launch_bounds__(HZ_THREADS) k_hazard(const RecArgs a, int LA, 
     const int t1 = min(a.T, t0 + tile);
     const int w0 = max(0, t0 - LA);                         // first token of the window
     const int64_t tokbase = chain * a.T;
+    // the window's lists in shared memory: sw [t1 - w0][kw], then sr [t1 - w0][kr]
+    int32_t* sw = reinterpret_cast<int32_t*>(tab + (mask + 1));
+    int32_t* sr = sw + (t1 - w0) * kw;
 
+    // stage the lists (contiguous per chain: one block of each), clear the table
+    {
+        const int nw = (t1 - w0) * kw, nr = (t1 - w0) * kr;
+        const int32_t* gw = a.idx_w + (tokbase + w0) * kw;
+        const int32_t* gr = a.idx_r + (tokbase + w0) * kr;
+        const bool v4 = ((reinterpret_cast<uintptr_t>(gw) | reinterpret_cast<uintptr_t>(gr)) & 15) == 0 && nw % 4 == 0 && nr % 4 == 0;
+        if (v4) {
+            for (int i = threadIdx.x; i < nw / 4; i += HZ_THREADS) reinterpret_cast<int4*>(sw)[i] = __ldg(reinterpret_cast<const int4*>(gw) + i);
+            for (int i = threadIdx.x; i < nr / 4; i += HZ_THREADS) reinterpret_cast<int4*>(sr)[i] = __ldg(reinterpret_cast<const int4*>(gr) + i);
+        } else {
+            for (int i = threadIdx.x; i < nw; i += HZ_THREADS) sw[i] = __ldg(gw + i);
+            for (int i = threadIdx.x; i < nr; i += HZ_THREADS) sr[i] = __ldg(gr + i);
+        }
+    }
     for (int i = threadIdx.x; i <= static_cast<int>(mask); i += HZ_THREADS) tab[i] = HZ_EMPTY;
     __syncthreads();
     // insert the write and read entries of tokens [w0, t1)
@@ -65,7 +88,7 @@ __global__ void __launch_bounds__(HZ_THREADS) k_hazard(const RecArgs a, int LA, 
         const int u = w0 + e / kk, q = e - (e / kk) * kk;
         const bool rd = q >= kw;
         const int n = rd ? q - kw : q;
-        const int32_t s = __ldg((rd ? a.idx_r + (tokbase + u) * kr : a.idx_w + (tokbase + u) * kw) + n);
+        const int32_t s = rd ? sr[(u - w0) * kr + n] : sw[(u - w0) * kw + n];
         const unsigned long long word = (static_cast<unsigned long long>(static_cast<uint32_t>(s)) << 32) |
                                         (rd ? 0x80000000ull : 0ull) |
                                         (static_cast<unsigned long long>(u - w0) << 16) | static_cast<unsigned>(n);
@@ -88,9 +111,9 @@ __global__ void __launch_bounds__(HZ_THREADS) k_hazard(const RecArgs a, int LA, 
         for (int side = 0; side < 2; ++side) {                      // 0: write slot, 1: read slot
             const int k = side ? kr : kw;
             if (n >= k) continue;
-            const int32_t* lst = (side ? a.idx_r : a.idx_w) + tok * k;
-            const int32_t s = __ldg(lst + n);
-            if (n > 0 && __ldg(lst + n - 1) >= s) unsorted = true;
+            const int32_t* lst = (side ? sr : sw) + (t - w0) * k;
+            const int32_t s = lst[n];
+            if (n > 0 && lst[n - 1] >= s) unsorted = true;
             const int hi = side ? t : t - 1;                         // writers u in [t - LA, hi]
             int best_w = -1, best_n = 0, best_r = -1;
             uint32_t h = hz_hash(static_cast<uint32_t>(s), lg);
@@ -124,7 +147,7 @@ cudaError_t launch_hazard(const RecArgs& a, int la, int kmax, int32_t* hz, cudaS
     const int64_t chains = static_cast<int64_t>(a.B) * a.H;
     const int tile = hz_tile(la, a.kw, a.kr);
     const int ntiles = (a.T + tile - 1) / tile;
-    const size_t smem = static_cast<size_t>(8) << hz_table_log2(tile, la, a.kw, a.kr);
+    const size_t smem = hz_smem_bytes(tile, la, a.kw, a.kr);
     if (smem > 48 * 1024) {
         cudaError_t e = cudaFuncSetAttribute(k_hazard, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
         if (e != cudaSuccess) return e;
