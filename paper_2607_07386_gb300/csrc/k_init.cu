@@ -7,7 +7,7 @@
 namespace sdm {
 
 constexpr int INIT_THREADS = 256;
-constexpr int INIT_UNROLL = 4;
+constexpr int INIT_UNROLL = 8;
 
 __global__ void __launch_bounds__(INIT_THREADS) k_init_memory(const uint4* __restrict__ M0, uint4* __restrict__ mem,
                                                               int64_t nvec, int B) {

@@ -67,7 +67,7 @@ struct SideStream {
     cudaEvent_t fork = nullptr, join = nullptr;
 };
 SideStream g_side[kMaxDevices];
-constexpr int kCopyCtasPerSm = 2;     // M0 copy CTAs per SM beside the addressing
+constexpr int kCopyCtasPerSm = 4;     // M0 copy CTAs per SM beside the addressing
 std::mutex g_side_mutex[kMaxDevices];
 
 sdm_status side_stream(int* dev_out, SideStream** out) {
