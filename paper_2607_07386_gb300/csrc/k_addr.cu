@@ -1255,35 +1255,37 @@ size_t addr_partial_bytes(const AddrPlan& plan, int B, int H, int T) {
 
 // ------------------------------------------------------------------------------------------
 // Certified pass, one thread per token-side (one column chunk per half, k <= 32).  Same
-// decisions as the warp pass (MODE 0), with the outer-sum candidates taken from a binary
-// max-heap of the k row heads A1[i] + A2[j_i] in shared memory (the rows start sorted, so the
-// array of first heads already is a heap): k + 1 pops give the k-th and (k+1)-th values.
-// Exact tie order is irrelevant here: a certified boundary has a positive gap, so equal
-// values never straddle it.  Token-sides with an uncertified boundary go to queue A.
+// decisions as the warp pass (MODE 0).  The outer sums A1[i] + A2[j] (i, j < k: only they can
+// hold the k largest once both half boundaries are certified) are taken in descending order
+// from a frontier held in registers: with both lists descending the taken cells form a
+// staircase (row i holds the cells j < m_i, m non-increasing) and the next largest sum is one
+// of its outer corners, at most 8 of them while at most 35 cells are taken.  k + 1 steps give
+// the k-th and (k+1)-th values; the selected cells are the staircase after k steps.  Exact
+// tie order is irrelevant: a certified boundary has a positive gap, so equal values never
+// straddle it.  Token-sides with an uncertified boundary go to queue A.
 // ------------------------------------------------------------------------------------------
 constexpr int FT_THREADS = 64;
+constexpr int FT_FRONT = 8;       // frontier cells (outer corners of a staircase of <= 35 cells)
 
-// Shared bytes per thread: values and popped candidates as 32-bit words, list indices and
-// heap positions as 16-bit (one column chunk per half: indices < 512).
-__host__ __device__ constexpr int ft_bytes(int km) { return 4 * (km + 1) * 4 + 4 * km + 2 * km * 3; }
+// Shared bytes per thread: the first k + 1 values of each half list (32-bit), the first k list
+// indices (16-bit: one column chunk per half, indices < 512) and the staircase row counts
+// (bytes, k + 1 of them, padded to a word).
+__host__ __device__ constexpr int ft_bytes(int km) { return 2 * 4 * (km + 1) + 2 * 2 * km + ((km + 4) & ~3); }
 
 template <class D, int L>
-__global__ void __launch_bounds__(FT_THREADS) k_addr_finalize_thread(const AddrArgs a) {
+__global__ void __launch_bounds__(FT_THREADS, 8) k_addr_finalize_thread(const AddrArgs a) {
     constexpr int KM = L - 4;                     // largest k served
-    constexpr int LOG = KM <= 8 ? 3 : KM <= 16 ? 4 : 5;
+    static_assert(KM <= 32, "frontier bound holds for k <= 32");
     extern __shared__ float fts[];
     const int tid = threadIdx.x;
     constexpr int W = FT_THREADS;
     // per-thread columns [element][FT_THREADS]: conflict-free for any element index
     float* const A1v = fts + tid;                                             // [KM + 1]
     float* const A2v = fts + (KM + 1) * W + tid;                              // [KM + 1]
-    float* const ov = fts + 2 * (KM + 1) * W + tid;                           // [KM + 1] popped values
-    int* const os = reinterpret_cast<int*>(fts) + 3 * (KM + 1) * W + tid;     // [KM + 1] popped slots
-    float* const hv = fts + 4 * (KM + 1) * W + tid;                           // [KM] heap values
-    unsigned short* const h16 = reinterpret_cast<unsigned short*>(fts + (4 * (KM + 1) + KM) * W);
+    unsigned short* const h16 = reinterpret_cast<unsigned short*>(fts + 2 * (KM + 1) * W);
     unsigned short* const A1i = h16 + tid;                                    // [KM]
     unsigned short* const A2i = h16 + KM * W + tid;                           // [KM]
-    unsigned short* const hp = h16 + 2 * KM * W + tid;                        // [KM] row | col << 8
+    unsigned char* const m8 = reinterpret_cast<unsigned char*>(h16 + 2 * KM * W) + tid;   // [KM + 1]
 
     const uint32_t BT = static_cast<uint32_t>(a.B) * static_cast<uint32_t>(a.T);
     const uint32_t items = 2u * static_cast<uint32_t>(a.H) * BT;      // < 2^31 (a queue exists)
@@ -1358,51 +1360,68 @@ __global__ void __launch_bounds__(FT_THREADS) k_addr_finalize_thread(const AddrA
     }
     const float e2c = __fadd_ru(__fmul_ru(2.f, e2), __fmul_ru(0x1p-21f, __fadd_ru(amax[0], amax[1])));
 
-    // k-way merge of the rows i (head A1[i] + A2[j_i]) through a max-heap of size k
-    const float a20 = A2v[0];
-    for (int i = 0; i < k; ++i) { hv[i * W] = A1v[i * W] + a20; hp[i * W] = static_cast<unsigned short>(i); }
-    for (int r = 0; r <= k; ++r) {
-        const float v = hv[0];
-        const int pk = hp[0];
-        const int i = pk & 255, j = pk >> 8;
-        ov[r * W] = v;
-        os[r * W] = static_cast<int>(A1i[i * W]) * S + static_cast<int>(A2i[(j < k ? j : 0) * W]);
-        const int j1 = j + 1;
-        const float nv = j1 < k ? A1v[i * W] + A2v[j1 * W] : -INFINITY;
-        const unsigned short np = static_cast<unsigned short>(i | (j1 << 8));
-        int pos = 0;
-        bool done = false;
+    // staircase walk: k + 1 steps, each taking the largest frontier cell
 #pragma unroll
-        for (int lvl = 0; lvl < LOG; ++lvl) {
-            const int c = 2 * pos + 1;
-            const float v1 = c < k ? hv[c * W] : -INFINITY;
-            const float v2 = c + 1 < k ? hv[(c + 1) * W] : -INFINITY;
-            const int cm = v2 > v1 ? c + 1 : c;
-            const float vm = fmaxf(v1, v2);
-            if (!done && vm > nv) {
-                hv[pos * W] = vm;
-                hp[pos * W] = hp[cm * W];
-                pos = cm;
-            } else {
-                done = true;
-            }
+    for (int i = 0; i <= KM; ++i)
+        if (i <= k) m8[i * W] = 0;
+    float fv[FT_FRONT];
+    int fij[FT_FRONT];                            // i | j << 8
+#pragma unroll
+    for (int f = 0; f < FT_FRONT; ++f) { fv[f] = -INFINITY; fij[f] = 0; }
+    const float vmax = A1v[0] + A2v[0];
+    fv[0] = vmax;
+    float ck = -INFINITY, ck1 = -INFINITY;
+    bool full = false;
+    for (int r = 0; r <= k; ++r) {
+        float bv = fv[0];
+        int bf = 0;
+#pragma unroll
+        for (int f = 1; f < FT_FRONT; ++f) {
+            const bool gt = fv[f] > bv;
+            bv = gt ? fv[f] : bv;
+            bf = gt ? f : bf;
         }
-        hv[pos * W] = nv;
-        hp[pos * W] = np;
+        if (r == k) { ck1 = bv; break; }
+        ck = bv;                                   // the k-th value after the last step
+        int bij = 0;
+#pragma unroll
+        for (int f = 0; f < FT_FRONT; ++f) bij = f == bf ? fij[f] : bij;
+        const int i = bij & 255, j = bij >> 8;
+        m8[i * W] = static_cast<unsigned char>(j + 1);
+        // (i, j + 1) becomes a corner once row i - 1 holds more than j + 1 cells
+        const bool right = j + 1 < k && (i == 0 || m8[(i - 1) * W] > j + 1);
+        // (i + 1, j) becomes a corner when row i + 1 holds exactly j cells
+        const bool down = i + 1 < k && m8[(i + 1) * W] == j;
+        const float rv = right ? A1v[i * W] + A2v[(j + 1) * W] : -INFINITY;
+        const float dv = down ? A1v[(i + 1) * W] + A2v[j * W] : -INFINITY;
+#pragma unroll
+        for (int f = 0; f < FT_FRONT; ++f)
+            if (f == bf) { fv[f] = rv; fij[f] = i | ((j + 1) << 8); }
+        bool placed = !down || dv == -INFINITY;
+#pragma unroll
+        for (int f = 0; f < FT_FRONT; ++f) {
+            const bool here = !placed && fv[f] == -INFINITY;
+            fv[f] = here ? dv : fv[f];
+            fij[f] = here ? ((i + 1) | (j << 8)) : fij[f];
+            placed |= here;
+        }
+        full |= !placed;
     }
-    if (!(__fsub_rd(ov[(k - 1) * W], ov[k * W]) > e2c)) { defer(); return; }
-
-    // softmax over the k selected scores, then ascending slot order (bitonic network)
-    const float vmax = ov[0];
+    // (-inf cells are padding past a short half list; they only ever supply the (k+1)-th value)
+    if (full || !(__fsub_rd(ck, ck1) > e2c)) { defer(); return; }
+    // softmax over the k selected scores (the staircase, row by row), then ascending slot order
+    // (bitonic network)
     float ew[KM];
     int sl[KM];
     float zsum = 0.f;
+    int ci = 0, cj = 0, mi = m8[0];
 #pragma unroll
     for (int r = 0; r < KM; ++r) {
         if (r < k) {
-            ew[r] = expf(ov[r * W] - vmax);
-            sl[r] = os[r * W];
+            ew[r] = expf((A1v[ci * W] + A2v[cj * W]) - vmax);
+            sl[r] = static_cast<int>(A1i[ci * W]) * S + static_cast<int>(A2i[cj * W]);
             zsum += ew[r];
+            if (++cj == mi) { ++ci; cj = 0; mi = m8[ci * W]; }
         } else {
             ew[r] = 0.f;
             sl[r] = INT_MAX;
@@ -1424,14 +1443,12 @@ __global__ void __launch_bounds__(FT_THREADS) k_addr_finalize_thread(const AddrA
                     sl[jx] = sw ? si : sl[jx]; ew[jx] = sw ? ei : ew[jx];
                 }
             }
-    const float inv = 1.f / zsum;
     const int64_t tokoff = ((static_cast<int64_t>(b) * a.H + h) * a.T + t) * k;
     int32_t* oi = a.idx[side] + tokoff;
     float* ow = a.w[side] + tokoff;
 #pragma unroll
     for (int r = 0; r < KM; ++r)
         if (r < k) { oi[r] = sl[r]; ow[r] = ew[r] / zsum; }
-    (void)inv;
 }
 
 // ------------------------------------------------------------------------------------------
@@ -1481,230 +1498,231 @@ __global__ void __launch_bounds__(BT_THREADS) k_addr_band_thread(const AddrArgs 
 
     const uint32_t BT = static_cast<uint32_t>(a.B) * static_cast<uint32_t>(a.T);
     const uint32_t nq = static_cast<uint32_t>(*reinterpret_cast<volatile int*>(a.queue));
-    const uint32_t q = blockIdx.x * BT_THREADS + tid;
-    if (q >= nq) return;
     const uint32_t all = 2u * static_cast<uint32_t>(a.H) * BT;
-    const uint32_t item = static_cast<uint32_t>(a.queue[2 + q]);
-    int* const qb = a.queue + 2 + all;
-    auto defer = [&]() { qb[atomicAdd(a.queue + 1, 1)] = static_cast<int>(item); };
-    const uint32_t z = item / BT, u = item - z * BT;
-    const int side = static_cast<int>(z) / a.H, h = static_cast<int>(z) % a.H;
-    const int k = a.kk[side];
-    const int S = a.S;
-    const uint32_t b = u / static_cast<uint32_t>(a.T), t = u - b * static_cast<uint32_t>(a.T);
-    const void* X = a.X[side];
-    const void* P = a.P[side];
-    const int64_t xoff = ((static_cast<int64_t>(b) * a.H + h) * a.T + t) * a.dk;
-    const int64_t prow0 = static_cast<int64_t>(h) * 2 * S;
-
-    float e2 = 0.f;
-    if (P != nullptr) {
-        float ss = 0.f;
-        const char* xr = static_cast<const char*>(X) + xoff * D::BYTES;
-        if ((reinterpret_cast<uintptr_t>(xr) & 15) == 0 && (a.dk * D::BYTES) % 16 == 0) {
-            const int nq = a.dk * D::BYTES / 16;
-            for (int q0 = 0; q0 < nq; q0 += 4) {
-                uint4 xq[4];
-#pragma unroll
-                for (int u = 0; u < 4; ++u)
-                    if (q0 + u < nq) xq[u] = __ldg(reinterpret_cast<const uint4*>(xr) + q0 + u);
-#pragma unroll
-                for (int u = 0; u < 4; ++u)
-                    if (q0 + u < nq) {
-                        float f[D::E];
-                        unpack16<D>(xq[u], f);
-#pragma unroll
-                        for (int e = 0; e < D::E; ++e) ss = fmaf(f[e], f[e], ss);
-                    }
-            }
-        } else {
-            for (int d = 0; d < a.dk; ++d) {
-                const float xv = load_elem<D>(X, xoff + d);
-                ss = fmaf(xv, xv, ss);
-            }
-        }
-        e2 = __fmul_ru(__fmul_ru(__fmul_ru(2.f * a.cbound, a.pnorm[side * a.H + h]), sqrtf(ss)), 1.f + 0x1p-12f);
-    }
     uint32_t stat_hb = 0, stat_he = 0, stat_cb = 0, stat_ce = 0;
+    // grid-stride over queue A (the grid is sized to the SMs, not to the longest queue)
+    for (uint32_t q = blockIdx.x * BT_THREADS + tid; q < nq; q += gridDim.x * BT_THREADS) {
+        const uint32_t item = static_cast<uint32_t>(a.queue[2 + q]);
+        int* const qb = a.queue + 2 + all;
+        auto defer = [&]() { qb[atomicAdd(a.queue + 1, 1)] = static_cast<int>(item); };
+        const uint32_t z = item / BT, u = item - z * BT;
+        const int side = static_cast<int>(z) / a.H, h = static_cast<int>(z) % a.H;
+        const int k = a.kk[side];
+        const int S = a.S;
+        const uint32_t b = u / static_cast<uint32_t>(a.T), t = u - b * static_cast<uint32_t>(a.T);
+        const void* X = a.X[side];
+        const void* P = a.P[side];
+        const int64_t xoff = ((static_cast<int64_t>(b) * a.H + h) * a.T + t) * a.dk;
+        const int64_t prow0 = static_cast<int64_t>(h) * 2 * S;
 
-    float amax[2];
-    for (int hf = 0; hf < 2; ++hf) {
-        const int64_t base = part_at(static_cast<int>(z), 1, hf, BT, u, L, 0);
-        float* Av = hf ? A2v : A1v;
-        int* Ai = hf ? A2i : A1i;
-        const float4* pv = reinterpret_cast<const float4*>(a.part_v + base);   // L % 4 == 0, 16-byte aligned
-        const int4* pi = reinterpret_cast<const int4*>(a.part_i + base);
+        float e2 = 0.f;
+        if (P != nullptr) {
+            float ss = 0.f;
+            const char* xr = static_cast<const char*>(X) + xoff * D::BYTES;
+            if ((reinterpret_cast<uintptr_t>(xr) & 15) == 0 && (a.dk * D::BYTES) % 16 == 0) {
+                const int nq = a.dk * D::BYTES / 16;
+                for (int q0 = 0; q0 < nq; q0 += 4) {
+                    uint4 xq[4];
 #pragma unroll
-        for (int q4 = 0; q4 < L / 4; ++q4) {
-            const float4 v4 = __ldg(pv + q4);
-            const int4 i4 = __ldg(pi + q4);
-            Av[(4 * q4) * W] = v4.x; Av[(4 * q4 + 1) * W] = v4.y; Av[(4 * q4 + 2) * W] = v4.z; Av[(4 * q4 + 3) * W] = v4.w;
-            Ai[(4 * q4) * W] = i4.x; Ai[(4 * q4 + 1) * W] = i4.y; Ai[(4 * q4 + 2) * W] = i4.z; Ai[(4 * q4 + 3) * W] = i4.w;
+                    for (int u = 0; u < 4; ++u)
+                        if (q0 + u < nq) xq[u] = __ldg(reinterpret_cast<const uint4*>(xr) + q0 + u);
+#pragma unroll
+                    for (int u = 0; u < 4; ++u)
+                        if (q0 + u < nq) {
+                            float f[D::E];
+                            unpack16<D>(xq[u], f);
+#pragma unroll
+                            for (int e = 0; e < D::E; ++e) ss = fmaf(f[e], f[e], ss);
+                        }
+                }
+            } else {
+                for (int d = 0; d < a.dk; ++d) {
+                    const float xv = load_elem<D>(X, xoff + d);
+                    ss = fmaf(xv, xv, ss);
+                }
+            }
+            e2 = __fmul_ru(__fmul_ru(__fmul_ru(2.f * a.cbound, a.pnorm[side * a.H + h]), sqrtf(ss)), 1.f + 0x1p-12f);
         }
-        const float vk = Av[(k - 1) * W], vk1 = Av[k * W];
-        if (!(S <= k || __fsub_rd(vk, vk1) > e2)) {
-            // band of the half boundary
-            ++stat_hb;
-            const float lo = __fsub_rd(vk, e2), hi = __fadd_ru(vk1, e2);
-            if (S > L && Av[(L - 1) * W] >= lo) { defer(); goto done; }
-            int cin = 0, m = 0;
-            for (int p = 0; p < L; ++p) {        // (-inf padding never enters a band)
-                const float v = Av[p * W];
-                cin += v > hi ? 1 : 0;
-                m += (v >= lo && v <= hi && v != -INFINITY) ? 1 : 0;
-            }
-            if (m > BT_BAND) { defer(); goto done; }
-            stat_he += m;
-            for (int e = 0; e < m; ++e) {
-                const FF f = ff_score_thread<D>(P, X, xoff, prow0, a.dk, S, hf, Ai[(cin + e) * W]);
-                bh[e * W] = f.h; bl[e * W] = f.l; bb[e * W] = f.b;
-            }
-            bool unsure = false;
-            for (int e = 0; e < m; ++e) {
-                const FF fe{bh[e * W], bl[e * W], bb[e * W]};
-                const int ie = Ai[(cin + e) * W];
-                int rank = 0;
-                for (int f = 0; f < m; ++f) {
-                    if (f == e) continue;
-                    const FF ff{bh[f * W], bl[f * W], bb[f * W]};
-                    const int c = ff_cmp(ff, fe, unsure);
-                    rank += (c > 0 || (c == 0 && Ai[(cin + f) * W] < ie)) ? 1 : 0;
-                }
-                bc[e * W] = rank < k - cin ? 1 : 0;
-            }
-            if (unsure) { defer(); goto done; }
-            // chosen band entries, in list order, after the certain prefix
-            int q2 = cin;
-            for (int e = 0; e < m; ++e) {
-                if (bc[e * W]) {
-                    const float v = Av[(cin + e) * W];
-                    const int ix = Ai[(cin + e) * W];
-                    Av[q2 * W] = v; Ai[q2 * W] = ix;       // q2 <= cin + e: in-place compaction
-                    ++q2;
-                }
-            }
-        }
-        amax[hf] = fmaxf(fabsf(Av[0]), fabsf(Av[(k - 1) * W]));
-    }
-    {
-        const float e2c = __fadd_ru(__fmul_ru(2.f, e2), __fmul_ru(0x1p-21f, __fadd_ru(amax[0], amax[1])));
-        // outer-sum candidates by a max-heap of the row heads (k+4 of them, 64 if the band needs)
-        const float a20 = A2v[0];
-        for (int i = 0; i < k; ++i) { hv[i * W] = A1v[i * W] + a20; hp[i * W] = i; }
-        const int kk2 = k * k;
-        int npop = 0;
-        auto pops = [&](int upto) {
-            for (; npop < upto; ++npop) {
-                const float v = hv[0];
-                const int pk = hp[0];
-                const int i = pk & 255, j = pk >> 8;
-                ov[npop * W] = v;
-                os[npop * W] = (j < k) ? A1i[i * W] * S + A2i[j * W] : INT_MAX;
-                const int j1 = j + 1;
-                const float nv = j1 < k ? A1v[i * W] + A2v[j1 * W] : -INFINITY;
-                const int np = i | (j1 << 8);
-                int pos = 0;
-                bool stop = false;
+
+        float amax[2];
+        for (int hf = 0; hf < 2; ++hf) {
+            const int64_t base = part_at(static_cast<int>(z), 1, hf, BT, u, L, 0);
+            float* Av = hf ? A2v : A1v;
+            int* Ai = hf ? A2i : A1i;
+            const float4* pv = reinterpret_cast<const float4*>(a.part_v + base);   // L % 4 == 0, 16-byte aligned
+            const int4* pi = reinterpret_cast<const int4*>(a.part_i + base);
 #pragma unroll
-                for (int lvl = 0; lvl < LOG; ++lvl) {
-                    const int c = 2 * pos + 1;
-                    const float v1 = c < k ? hv[c * W] : -INFINITY;
-                    const float v2 = c + 1 < k ? hv[(c + 1) * W] : -INFINITY;
-                    const int cm = v2 > v1 ? c + 1 : c;
-                    const float vm = fmaxf(v1, v2);
-                    if (!stop && vm > nv) { hv[pos * W] = vm; hp[pos * W] = hp[cm * W]; pos = cm; }
-                    else stop = true;
+            for (int q4 = 0; q4 < L / 4; ++q4) {
+                const float4 v4 = __ldg(pv + q4);
+                const int4 i4 = __ldg(pi + q4);
+                Av[(4 * q4) * W] = v4.x; Av[(4 * q4 + 1) * W] = v4.y; Av[(4 * q4 + 2) * W] = v4.z; Av[(4 * q4 + 3) * W] = v4.w;
+                Ai[(4 * q4) * W] = i4.x; Ai[(4 * q4 + 1) * W] = i4.y; Ai[(4 * q4 + 2) * W] = i4.z; Ai[(4 * q4 + 3) * W] = i4.w;
+            }
+            const float vk = Av[(k - 1) * W], vk1 = Av[k * W];
+            if (!(S <= k || __fsub_rd(vk, vk1) > e2)) {
+                // band of the half boundary
+                ++stat_hb;
+                const float lo = __fsub_rd(vk, e2), hi = __fadd_ru(vk1, e2);
+                if (S > L && Av[(L - 1) * W] >= lo) { defer(); goto next; }
+                int cin = 0, m = 0;
+                for (int p = 0; p < L; ++p) {        // (-inf padding never enters a band)
+                    const float v = Av[p * W];
+                    cin += v > hi ? 1 : 0;
+                    m += (v >= lo && v <= hi && v != -INFINITY) ? 1 : 0;
                 }
-                hv[pos * W] = nv;
-                hp[pos * W] = np;
-            }
-        };
-        const int len0 = kk2 < L ? kk2 : L;
-        pops(len0 > k + 1 ? len0 : k + 1);
-        int len = npop;
-        const float ck = ov[(k - 1) * W], ck1 = k < npop ? ov[k * W] : -INFINITY;
-        int nsel = k;                              // selected: candidates [0, k) unless a band is resolved
-        if (!(ck1 == -INFINITY || __fsub_rd(ck, ck1) > e2c)) {
-            ++stat_cb;
-            const float lo = __fsub_rd(ck, e2c), hi = __fadd_ru(ck1, e2c);
-            // a band reaching the last kept candidate (merge to be extended): queue B
-            const bool all_cands = len >= kk2;
-            if (!all_cands && ov[(len - 1) * W] != -INFINITY && ov[(len - 1) * W] >= lo) { defer(); goto done; }
-            int cin = 0, m = 0;
-            for (int p = 0; p < len; ++p) {      // (exhausted rows, -inf, never enter a band)
-                const float v = ov[p * W];
-                cin += v > hi ? 1 : 0;
-                m += (v >= lo && v <= hi && v != -INFINITY) ? 1 : 0;
-            }
-            if (m > BT_BAND) { defer(); goto done; }
-            stat_ce += m;
-            for (int e = 0; e < m; ++e) {
-                const int f = os[(cin + e) * W];
-                const FF s1 = ff_score_thread<D>(P, X, xoff, prow0, a.dk, S, 0, f / S);
-                const FF s2 = ff_score_thread<D>(P, X, xoff, prow0, a.dk, S, 1, f % S);
-                const FF sm = ff_add(s1, s2, P == nullptr);
-                bh[e * W] = sm.h; bl[e * W] = sm.l; bb[e * W] = sm.b;
-            }
-            bool unsure = false;
-            for (int e = 0; e < m; ++e) {
-                const FF fe{bh[e * W], bl[e * W], bb[e * W]};
-                const int ie = os[(cin + e) * W];
-                int rank = 0;
-                for (int f = 0; f < m; ++f) {
-                    if (f == e) continue;
-                    const FF ff{bh[f * W], bl[f * W], bb[f * W]};
-                    const int c = ff_cmp(ff, fe, unsure);
-                    rank += (c > 0 || (c == 0 && os[(cin + f) * W] < ie)) ? 1 : 0;
+                if (m > BT_BAND) { defer(); goto next; }
+                stat_he += m;
+                for (int e = 0; e < m; ++e) {
+                    const FF f = ff_score_thread<D>(P, X, xoff, prow0, a.dk, S, hf, Ai[(cin + e) * W]);
+                    bh[e * W] = f.h; bl[e * W] = f.l; bb[e * W] = f.b;
                 }
-                bc[e * W] = rank < k - cin ? 1 : 0;
-            }
-            if (unsure) { defer(); goto done; }
-            int q2 = cin;
-            for (int e = 0; e < m; ++e) {
-                if (bc[e * W]) {
-                    const float v = ov[(cin + e) * W];
-                    const int f = os[(cin + e) * W];
-                    ov[q2 * W] = v; os[q2 * W] = f;
-                    ++q2;
+                bool unsure = false;
+                for (int e = 0; e < m; ++e) {
+                    const FF fe{bh[e * W], bl[e * W], bb[e * W]};
+                    const int ie = Ai[(cin + e) * W];
+                    int rank = 0;
+                    for (int f = 0; f < m; ++f) {
+                        if (f == e) continue;
+                        const FF ff{bh[f * W], bl[f * W], bb[f * W]};
+                        const int c = ff_cmp(ff, fe, unsure);
+                        rank += (c > 0 || (c == 0 && Ai[(cin + f) * W] < ie)) ? 1 : 0;
+                    }
+                    bc[e * W] = rank < k - cin ? 1 : 0;
                 }
-            }
-            nsel = q2;                             // = k
-        }
-        // softmax over the k selected scores, then ascending slot order
-        float vmax = -INFINITY;
-        for (int r = 0; r < nsel; ++r) vmax = fmaxf(vmax, ov[r * W]);
-        float ew[KM];
-        int sl[KM];
-        float zsum = 0.f;
-#pragma unroll
-        for (int r = 0; r < KM; ++r) {
-            if (r < k) { ew[r] = expf(ov[r * W] - vmax); sl[r] = os[r * W]; zsum += ew[r]; }
-            else { ew[r] = 0.f; sl[r] = INT_MAX; }
-        }
-#pragma unroll
-        for (int size = 2; size <= KM; size <<= 1)
-#pragma unroll
-            for (int stride = size >> 1; stride > 0; stride >>= 1)
-#pragma unroll
-                for (int i = 0; i < KM; ++i) {
-                    const int jx = i ^ stride;
-                    if (jx > i) {
-                        const bool up = (i & size) == 0;
-                        const bool sw = up ? (sl[i] > sl[jx]) : (sl[i] < sl[jx]);
-                        const int si = sl[i];
-                        const float ei = ew[i];
-                        sl[i] = sw ? sl[jx] : si;  ew[i] = sw ? ew[jx] : ei;
-                        sl[jx] = sw ? si : sl[jx]; ew[jx] = sw ? ei : ew[jx];
+                if (unsure) { defer(); goto next; }
+                // chosen band entries, in list order, after the certain prefix
+                int q2 = cin;
+                for (int e = 0; e < m; ++e) {
+                    if (bc[e * W]) {
+                        const float v = Av[(cin + e) * W];
+                        const int ix = Ai[(cin + e) * W];
+                        Av[q2 * W] = v; Ai[q2 * W] = ix;       // q2 <= cin + e: in-place compaction
+                        ++q2;
                     }
                 }
-        const int64_t tokoff = ((static_cast<int64_t>(b) * a.H + h) * a.T + t) * k;
-        int32_t* oi = a.idx[side] + tokoff;
-        float* ow = a.w[side] + tokoff;
+            }
+            amax[hf] = fmaxf(fabsf(Av[0]), fabsf(Av[(k - 1) * W]));
+        }
+        {
+            const float e2c = __fadd_ru(__fmul_ru(2.f, e2), __fmul_ru(0x1p-21f, __fadd_ru(amax[0], amax[1])));
+            // outer-sum candidates by a max-heap of the row heads (k+4 of them, 64 if the band needs)
+            const float a20 = A2v[0];
+            for (int i = 0; i < k; ++i) { hv[i * W] = A1v[i * W] + a20; hp[i * W] = i; }
+            const int kk2 = k * k;
+            int npop = 0;
+            auto pops = [&](int upto) {
+                for (; npop < upto; ++npop) {
+                    const float v = hv[0];
+                    const int pk = hp[0];
+                    const int i = pk & 255, j = pk >> 8;
+                    ov[npop * W] = v;
+                    os[npop * W] = (j < k) ? A1i[i * W] * S + A2i[j * W] : INT_MAX;
+                    const int j1 = j + 1;
+                    const float nv = j1 < k ? A1v[i * W] + A2v[j1 * W] : -INFINITY;
+                    const int np = i | (j1 << 8);
+                    int pos = 0;
+                    bool stop = false;
 #pragma unroll
-        for (int r = 0; r < KM; ++r)
-            if (r < k) { oi[r] = sl[r]; ow[r] = ew[r] / zsum; }
+                    for (int lvl = 0; lvl < LOG; ++lvl) {
+                        const int c = 2 * pos + 1;
+                        const float v1 = c < k ? hv[c * W] : -INFINITY;
+                        const float v2 = c + 1 < k ? hv[(c + 1) * W] : -INFINITY;
+                        const int cm = v2 > v1 ? c + 1 : c;
+                        const float vm = fmaxf(v1, v2);
+                        if (!stop && vm > nv) { hv[pos * W] = vm; hp[pos * W] = hp[cm * W]; pos = cm; }
+                        else stop = true;
+                    }
+                    hv[pos * W] = nv;
+                    hp[pos * W] = np;
+                }
+            };
+            const int len0 = kk2 < L ? kk2 : L;
+            pops(len0 > k + 1 ? len0 : k + 1);
+            int len = npop;
+            const float ck = ov[(k - 1) * W], ck1 = k < npop ? ov[k * W] : -INFINITY;
+            int nsel = k;                              // selected: candidates [0, k) unless a band is resolved
+            if (!(ck1 == -INFINITY || __fsub_rd(ck, ck1) > e2c)) {
+                ++stat_cb;
+                const float lo = __fsub_rd(ck, e2c), hi = __fadd_ru(ck1, e2c);
+                // a band reaching the last kept candidate (merge to be extended): queue B
+                const bool all_cands = len >= kk2;
+                if (!all_cands && ov[(len - 1) * W] != -INFINITY && ov[(len - 1) * W] >= lo) { defer(); goto next; }
+                int cin = 0, m = 0;
+                for (int p = 0; p < len; ++p) {      // (exhausted rows, -inf, never enter a band)
+                    const float v = ov[p * W];
+                    cin += v > hi ? 1 : 0;
+                    m += (v >= lo && v <= hi && v != -INFINITY) ? 1 : 0;
+                }
+                if (m > BT_BAND) { defer(); goto next; }
+                stat_ce += m;
+                for (int e = 0; e < m; ++e) {
+                    const int f = os[(cin + e) * W];
+                    const FF s1 = ff_score_thread<D>(P, X, xoff, prow0, a.dk, S, 0, f / S);
+                    const FF s2 = ff_score_thread<D>(P, X, xoff, prow0, a.dk, S, 1, f % S);
+                    const FF sm = ff_add(s1, s2, P == nullptr);
+                    bh[e * W] = sm.h; bl[e * W] = sm.l; bb[e * W] = sm.b;
+                }
+                bool unsure = false;
+                for (int e = 0; e < m; ++e) {
+                    const FF fe{bh[e * W], bl[e * W], bb[e * W]};
+                    const int ie = os[(cin + e) * W];
+                    int rank = 0;
+                    for (int f = 0; f < m; ++f) {
+                        if (f == e) continue;
+                        const FF ff{bh[f * W], bl[f * W], bb[f * W]};
+                        const int c = ff_cmp(ff, fe, unsure);
+                        rank += (c > 0 || (c == 0 && os[(cin + f) * W] < ie)) ? 1 : 0;
+                    }
+                    bc[e * W] = rank < k - cin ? 1 : 0;
+                }
+                if (unsure) { defer(); goto next; }
+                int q2 = cin;
+                for (int e = 0; e < m; ++e) {
+                    if (bc[e * W]) {
+                        const float v = ov[(cin + e) * W];
+                        const int f = os[(cin + e) * W];
+                        ov[q2 * W] = v; os[q2 * W] = f;
+                        ++q2;
+                    }
+                }
+                nsel = q2;                             // = k
+            }
+            // softmax over the k selected scores, then ascending slot order
+            float vmax = -INFINITY;
+            for (int r = 0; r < nsel; ++r) vmax = fmaxf(vmax, ov[r * W]);
+            float ew[KM];
+            int sl[KM];
+            float zsum = 0.f;
+#pragma unroll
+            for (int r = 0; r < KM; ++r) {
+                if (r < k) { ew[r] = expf(ov[r * W] - vmax); sl[r] = os[r * W]; zsum += ew[r]; }
+                else { ew[r] = 0.f; sl[r] = INT_MAX; }
+            }
+#pragma unroll
+            for (int size = 2; size <= KM; size <<= 1)
+#pragma unroll
+                for (int stride = size >> 1; stride > 0; stride >>= 1)
+#pragma unroll
+                    for (int i = 0; i < KM; ++i) {
+                        const int jx = i ^ stride;
+                        if (jx > i) {
+                            const bool up = (i & size) == 0;
+                            const bool sw = up ? (sl[i] > sl[jx]) : (sl[i] < sl[jx]);
+                            const int si = sl[i];
+                            const float ei = ew[i];
+                            sl[i] = sw ? sl[jx] : si;  ew[i] = sw ? ew[jx] : ei;
+                            sl[jx] = sw ? si : sl[jx]; ew[jx] = sw ? ei : ew[jx];
+                        }
+                    }
+            const int64_t tokoff = ((static_cast<int64_t>(b) * a.H + h) * a.T + t) * k;
+            int32_t* oi = a.idx[side] + tokoff;
+            float* ow = a.w[side] + tokoff;
+#pragma unroll
+            for (int r = 0; r < KM; ++r)
+                if (r < k) { oi[r] = sl[r]; ow[r] = ew[r] / zsum; }
+        }
+    next:;
     }
-done:
     if (stat_hb) stat_add(a.err, STAT_HALF_BAND, stat_hb);
     if (stat_he) stat_add(a.err, STAT_HALF_BAND_ENTRIES, stat_he);
     if (stat_cb) stat_add(a.err, STAT_COMB_BAND, stat_cb);
@@ -1751,7 +1769,12 @@ static cudaError_t launch_finalize(const AddrArgs& a, cudaStream_t stream) {
                                          static_cast<int>(smb));
                 if (e != cudaSuccess) return e;
                 const int64_t items = 2 * a.H * BT;       // upper bound of the queue length
-                k_addr_band_thread<D, L><<<static_cast<unsigned>((items + BT_THREADS - 1) / BT_THREADS), BT_THREADS,
+                int per_sm_b = 0;
+                e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm_b, k_addr_band_thread<D, L>, BT_THREADS, smb);
+                if (e != cudaSuccess) return e;
+                const int64_t need_b = (items + BT_THREADS - 1) / BT_THREADS;
+                const int64_t full_b = static_cast<int64_t>(sms) * (per_sm_b > 0 ? per_sm_b : 1);
+                k_addr_band_thread<D, L><<<static_cast<unsigned>(need_b < full_b ? need_b : full_b), BT_THREADS,
                                            smb, stream>>>(a);
             } else {
                 k_addr_finalize<D, L, FIN_BAND><<<grid, FW_WARPS * 32, 0, stream>>>(a);
