@@ -365,13 +365,106 @@ def leg_decode(steps: int, warmup: int) -> dict:
             "timing": f"{steps} consecutive steps captured in one CUDA graph, one replay timed with CUDA events"}
 
 
+def leg_next(steps: int, warmup: int) -> dict:
+    """The rows beyond the token-serial forward, timed at the layer_1p4b geometry on the same
+    device-drawn inputs: the chunkwise (WY) forward (App. A.1) at C = 16 and 32, the forward
+    that also writes the undo log, and the backward that walks the tokens in reverse and
+    restores the memory from that log (App. A.3).  Each call is bracketed by its own CUDA
+    events; the zeroing of dM between backward calls is outside them."""
+    import torch
+    import paper_2607_07386_gb300 as sdm
+    from synth.torch_io import torch_dtype
+    cfg = synth.LAYER_1P4B
+    dev = device_inputs(cfg, seed=cfg.seed)
+    B, H, T, N, dv = cfg.B, cfg.H, cfg.T, cfg.N, cfg.d_v
+    dt = torch_dtype(cfg.dtype)
+    shape = sdm.SdmShape.make(B, H, T, cfg.d_k, dv, N, cfg.k_write, cfg.k_read, cfg.dtype)
+    st = torch.cuda.current_stream()
+    mem = torch.empty((B, H, N, dv), dtype=dt, device="cuda")
+    y = torch.empty((B, H, T, dv), dtype=dt, device="cuda")
+    ws = torch.empty(max(sdm.workspace_bytes(shape), sdm.recur_workspace_bytes(shape)), dtype=torch.uint8, device="cuda")
+    lists = {n: torch.empty((B, H, T, k), dtype=tt, device="cuda")
+             for n, k, tt in (("idx_w", cfg.k_write, torch.int32), ("w_w", cfg.k_write, torch.float32),
+                              ("idx_r", cfg.k_read, torch.int32), ("w_r", cfg.k_read, torch.float32))}
+    sdm.address(shape, dev["P_q"], dev["P_k"], dev["q"], dev["k"], lists["idx_w"], lists["w_w"], lists["idx_r"],
+                lists["w_r"], ws, stream=st)
+    sdm.init_memory(shape, dev["M0"], mem, st)
+    L = (lists["idx_w"], lists["w_w"], lists["idx_r"], lists["w_r"], dev["v"], dev["alpha"], dev["beta"])
+
+    def timed(fn, n, between=None):
+        tot = 0.0
+        for i in range(warmup + n):
+            if between is not None:
+                between()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(st)
+            fn()
+            e1.record(st)
+            e1.synchronize()
+            if i >= warmup:
+                tot += e0.elapsed_time(e1)
+        return tot / n
+
+    out = {"workload": _workload_desc(cfg), "data": "synthetic (device-drawn, the workload's distributions)"}
+    rec_bytes = cfg.recurrence_bytes_per_token_head() * B * H * T
+    for C in (16, 32):
+        ms = timed(lambda: sdm.recur_chunkwise(shape, *L, mem, y, C, stream=st), steps)
+        out[f"chunkwise_c{C}"] = {"ms": ms, "tokens_per_s": B * T / (ms * 1e-3),
+                                  "gbs_of_recurrence_bytes": rec_bytes / (ms * 1e-3) / 1e9}
+    undo = torch.empty(sdm.undo_log_bytes(shape), dtype=torch.uint8, device="cuda")
+    ms_u = timed(lambda: sdm.recur_undo(shape, *L, mem, y, undo, ws, stream=st), steps)
+    dy = torch.randn((B, H, T, dv), device="cuda").to(dt)
+    grads = {"dv": torch.empty((B, H, T, dv), device="cuda"), "dalpha": torch.empty((B, H, T), device="cuda"),
+             "dbeta": torch.empty((B, H, T), device="cuda"), "dw_w": torch.empty((B, H, T, cfg.k_write), device="cuda"),
+             "dw_r": torch.empty((B, H, T, cfg.k_read), device="cuda")}
+    dM = torch.empty((B, H, N, dv), device="cuda")
+    # each backward restores mem to the state before the forward: one undo forward before each
+    def fwd_then_zero():
+        sdm.recur_undo(shape, *L, mem, y, undo, ws, stream=st)
+        dM.zero_()
+    ms_b = timed(lambda: sdm.recur_backward(shape, *L, mem, undo, dy, grads["dv"], grads["dalpha"], grads["dbeta"],
+                                            grads["dw_w"], grads["dw_r"], dM, stream=st), steps, between=fwd_then_zero)
+    undo_bytes = undo.numel()
+    out["forward_with_undo_log"] = {"ms": ms_u, "tokens_per_s": B * T / (ms_u * 1e-3), "undo_log_bytes": undo_bytes}
+    out["backward"] = {"ms": ms_b, "tokens_per_s": B * T / (ms_b * 1e-3)}
+    rows = B * H * T * cfg.k_write
+    scales = torch.empty(rows, dtype=torch.float32, device="cuda")
+    for kind in ("fp8", "int4"):
+        codes = torch.empty(sdm.undo_code_bytes(shape, kind), dtype=torch.uint8, device="cuda")
+        sdm.recur_undo(shape, *L, mem, y, undo, ws, stream=st)
+        ms_q = timed(lambda: sdm.undo_quantize(shape, undo, kind, codes, scales, stream=st), steps)
+        q_bytes = undo_bytes + codes.numel() + rows * 4
+        sdm.recur_backward_q(shape, *L, mem, kind, codes, scales, dy, grads["dv"], grads["dalpha"], grads["dbeta"],
+                             grads["dw_w"], grads["dw_r"], dM, stream=st)     # back to M_0
+
+        def fwd_quant_zero():
+            sdm.recur_undo(shape, *L, mem, y, undo, ws, stream=st)
+            sdm.undo_quantize(shape, undo, kind, codes, scales, stream=st)
+            dM.zero_()
+        ms_bq = timed(lambda: sdm.recur_backward_q(shape, *L, mem, kind, codes, scales, dy, grads["dv"], grads["dalpha"],
+                                                   grads["dbeta"], grads["dw_w"], grads["dw_r"], dM, stream=st),
+                      steps, between=fwd_quant_zero)
+        out[f"snapshot_{kind}"] = {"quantize_ms": ms_q, "quantize_gbs": q_bytes / (ms_q * 1e-3) / 1e9,
+                                   "snapshot_bytes": codes.numel() + rows * 4, "backward_ms": ms_bq}
+        del codes
+    if sdm.device_status(st) != 0:
+        raise RuntimeError("device status word set in the next-rows leg")
+    out["timing"] = f"{warmup} untimed + {steps} timed calls each, CUDA events around each call"
+    return out
+
+
 def run_leg(args):
     """`bench.py --leg NAME`: one workload leg in its own process, printing one JSON object."""
     import torch
     from paper_2607_07386_gb300.build import build
     torch.cuda.set_device(0)
     build()
-    res = leg_decode(args.steps, args.warmup) if args.leg == "decode" else leg_scan(args.leg, args.steps, args.warmup)
+    if args.leg == "decode":
+        res = leg_decode(args.steps, args.warmup)
+    elif args.leg == "next_rows":
+        res = leg_next(args.steps, args.warmup)
+    else:
+        res = leg_scan(args.leg, args.steps, args.warmup)
     print(json.dumps(res), flush=True)
 
 
@@ -654,7 +747,7 @@ def run_ours(args, cfg):
         torch.cuda.synchronize()
         torch.cuda.empty_cache()
         line["workloads"] = legs_in_subprocesses(
-            [("small_bf16", max(args.steps, 10)), ("long_ctx", 3), ("decode", 1000)], args.warmup)
+            [("small_bf16", max(args.steps, 10)), ("long_ctx", 3), ("decode", 1000), ("next_rows", 2)], args.warmup)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(cfg)
     if rank == 0:

@@ -266,6 +266,38 @@ sdm_status sdm_recur_backward(const sdm_shape* shape, const int32_t* idx_w, cons
                               const void* dy, float* dv, float* dalpha, float* dbeta, float* dw_w,
                               float* dw_r, float* dM, sdm_stream_t stream);
 
+/* Quantised snapshots of the undo log (App. A.3: for long sequences the log can be kept as fp8
+ * or int4, which the paper reports does not hurt training).  Row r of the log (r = ((b*H + h)*T
+ * + t)*k_write + n, d_v elements) is kept as one float32 scale s_r = fl32(max|row| / top), 1 for
+ * an all-zero row, and d_v codes q = round(fl32(row / s_r)), every step a correctly rounded
+ * float32 operation: SDM_UNDO_FP8 codes are e4m3 values (top 448, round to nearest even, one
+ * byte per element); SDM_UNDO_INT4 codes are the integers -7..7 (top 7, ties to even), two per
+ * byte, element 2i in the low nibble, two's complement. */
+enum { SDM_UNDO_FP8 = 1, SDM_UNDO_INT4 = 2 };
+
+/* Bytes of the codes of a quantised log: B*H*T*k_write rows of d_v (fp8) or d_v / 2 (int4)
+ * bytes; the scales take B*H*T*k_write floats more.  0 for an invalid shape or kind. */
+size_t sdm_undo_code_bytes(const sdm_shape* shape, int kind);
+
+/* Quantises the undo log of sdm_recur_undo (stored rows, [B, H, T, k_write, d_v]) into codes
+ * and scales as above (caller-owned device buffers; codes 16-byte aligned, none of the three
+ * overlapping).  Rows of write entries whose slot index is out of range were never written by
+ * the forward; their codes are unspecified and the backward never reads them.  d_v must be a
+ * multiple of 32, at most 256. */
+sdm_status sdm_undo_quantize(const sdm_shape* shape, const void* undo, int kind, void* codes,
+                             float* scales, sdm_stream_t stream);
+
+/* sdm_recur_backward with the log read back from a quantised snapshot: each logged row is taken
+ * as the stored value (storage dtype rounding) of q * s_r, both in the chain rule and in the
+ * undo, so mem returns to M_0 only up to the snapshot's quantisation.  Arguments and outputs as
+ * in sdm_recur_backward, with (kind, codes, scales) from sdm_undo_quantize in place of undo. */
+sdm_status sdm_recur_backward_q(const sdm_shape* shape, const int32_t* idx_w, const float* w_w,
+                                const int32_t* idx_r, const float* w_r, const void* v,
+                                const void* alpha, const void* beta, void* mem, int kind,
+                                const void* codes, const float* scales, const void* dy, float* dv,
+                                float* dalpha, float* dbeta, float* dw_w, float* dw_r, float* dM,
+                                sdm_stream_t stream);
+
 /* Reads (host pointer `code`, synchronising on `stream`) and clears the device
  * status word of the current device: 0 = no fault; bit 0 = a slot index outside
  * [0, N) was skipped; bit 1 = a slot list given to the recurrence (forward, chunkwise

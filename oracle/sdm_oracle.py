@@ -73,7 +73,7 @@ __all__ = [
     "recur", "forward_slice", "state_elements_per_layer", "n_global_layers",
     "touched_mask", "recur_lazy", "materialize", "eff_keys_fraction", "cumulative_mass", "unique_fraction",
     "softplus", "gates", "norm_gate", "head_mix", "sparse_ip", "recur_chunkwise",
-    "recur_forward_undo", "recur_backward", "round_e4m3", "quantize_undo",
+    "recur_forward_undo", "recur_backward", "round_e4m3", "quantize_undo", "undo_codes",
 ]
 
 
@@ -380,20 +380,46 @@ def round_e4m3(x: np.ndarray) -> np.ndarray:
     return np.rint(x / q) * q
 
 
-def quantize_undo(undo: np.ndarray, kind: str) -> np.ndarray:
+def quantize_undo(undo: np.ndarray, kind: str, arith: str = "f64") -> np.ndarray:
     """The undo log as a quantised snapshot would give it back (App. A.3: fp8 or int4 snapshots
     for long sequences), one scale per logged row: "fp8" rounds row / s to e4m3 with
     s = max|row| / 448; "int4" rounds row / s to the integers -7..7 with s = max|row| / 7;
-    "exact" returns the log unchanged."""
+    "exact" returns the log unchanged.
+
+    arith="f64" does the arithmetic in float64.  arith="f32" takes every step in float32 with
+    correctly rounded operations (the scale, the division by it and the dequantising product
+    q * s), so that the codes are decided in the precision a float32 implementation uses:
+    the values equal ``undo_codes``' codes times their scales, rounded to float32."""
     u = np.asarray(undo, dtype=np.float64)
     if kind == "exact":
         return u.copy()
+    if arith == "f32":
+        codes, scale = undo_codes(u, kind)
+        return (codes.astype(np.float32) * scale[..., None]).astype(np.float64)
     top = {"fp8": 448.0, "int4": 7.0}[kind]
     amax = np.max(np.abs(u), axis=-1, keepdims=True)
     scale = np.where(amax > 0, amax / top, 1.0)
     y = u / scale
     q = round_e4m3(y) if kind == "fp8" else np.clip(np.rint(y), -7, 7)
     return q * scale
+
+
+def undo_codes(undo: np.ndarray, kind: str):
+    """The quantised snapshot itself, in float32 arithmetic: per logged row the scale
+    s = fl32(max|row| / top) (1 for an all-zero row) and the codes q = round(fl32(row / s)),
+    e4m3 values for "fp8" (top 448, ties to even) and integers -7..7 for "int4" (top 7, ties
+    to even).  The rows must be float32-representable (stored values).  Returns (codes as
+    float64 [..., d_v], scales as float32 [...])."""
+    u = np.asarray(undo, dtype=np.float64)
+    u32 = u.astype(np.float32)
+    if not np.array_equal(u32.astype(np.float64), u):
+        raise ValueError("undo_codes: the logged rows must be float32 values")
+    top = np.float32({"fp8": 448.0, "int4": 7.0}[kind])
+    amax = np.max(np.abs(u32), axis=-1)
+    scale = np.where(amax > 0, amax / top, np.float32(1.0)).astype(np.float32)
+    y = (u32 / scale[..., None]).astype(np.float32).astype(np.float64)
+    q = round_e4m3(np.clip(y, -448.0, 448.0)) if kind == "fp8" else np.clip(np.rint(y), -7, 7)
+    return q, scale
 
 
 # --------------------------------------------------------------------------------------

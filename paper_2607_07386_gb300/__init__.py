@@ -10,6 +10,6 @@ from ._binding import (  # noqa: F401
     decode_step, device_stats, device_status, forward, forward_m0, init_memory, last_error, lib, lib_path, recur, recur_noalloc,
     recur_workspace_bytes, workspace_bytes, RECUR_NOALLOC_SCRATCH_BYTES, forward_lazy, lazy_workspace_bytes,
     materialize, touched_words, access_stats, access_stats_workspace_bytes, gates, norm_gate,
-    undo_log_bytes, recur_undo, recur_backward, recur_chunkwise, recur_plan, test_recur_wait_timeout,
+    undo_log_bytes, recur_undo, recur_backward, undo_code_bytes, undo_quantize, recur_backward_q, recur_chunkwise, recur_plan, test_recur_wait_timeout,
     RECUR_PLAN_FIELDS, test_scores,
 )

@@ -83,6 +83,13 @@ def lib():
             L.sdm_recur_backward.argtypes = [_SHP, _I32P, _VP, _I32P, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP,
                                              _VP, _VP, _VP, _VP, _VP]
             L.sdm_recur_backward.restype = ctypes.c_int
+            L.sdm_undo_code_bytes.restype = ctypes.c_size_t
+            L.sdm_undo_code_bytes.argtypes = [_SHP, ctypes.c_int]
+            L.sdm_undo_quantize.argtypes = [_SHP, _VP, ctypes.c_int, _VP, _VP, _VP]
+            L.sdm_undo_quantize.restype = ctypes.c_int
+            L.sdm_recur_backward_q.argtypes = [_SHP, _I32P, _VP, _I32P, _VP, _VP, _VP, _VP, _VP, ctypes.c_int, _VP,
+                                               _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP]
+            L.sdm_recur_backward_q.restype = ctypes.c_int
             L.sdm_gates.argtypes = [_SHP, ctypes.c_int32, _VP, _VP, _VP, _VP, _VP, _VP, _VP, _VP]
             L.sdm_gates.restype = ctypes.c_int
             L.sdm_norm_gate.argtypes = [_SHP, _VP, _VP, _VP, ctypes.c_float, _VP, _VP]
@@ -242,6 +249,33 @@ def recur_backward(shape: SdmShape, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem,
     _check(lib().sdm_recur_backward(ctypes.byref(shape), _ptr(idx_w), _ptr(w_w), _ptr(idx_r), _ptr(w_r), _ptr(v),
                                     _ptr(alpha), _ptr(beta), _ptr(mem), _ptr(undo), _ptr(dy), _ptr(dv),
                                     _ptr(dalpha), _ptr(dbeta), _ptr(dw_w), _ptr(dw_r), _ptr(dM), _stream(stream)))
+
+
+UNDO_KINDS = {"fp8": 1, "int4": 2}
+
+
+def undo_code_bytes(shape: SdmShape, kind: str) -> int:
+    """Bytes of the codes of a quantised undo log ("fp8" or "int4"); the scales are
+    B*H*T*k_write float32 more."""
+    n = lib().sdm_undo_code_bytes(ctypes.byref(shape), UNDO_KINDS[kind])
+    if n == 0 and shape.B * shape.H * shape.T * shape.k_write > 0:
+        raise SdmError(1, last_error())
+    return n
+
+
+def undo_quantize(shape: SdmShape, undo, kind: str, codes, scales, stream=None):
+    """sdm_undo_quantize: fp8 / int4 snapshot of the undo log, one float32 scale per row."""
+    _check(lib().sdm_undo_quantize(ctypes.byref(shape), _ptr(undo), UNDO_KINDS[kind], _ptr(codes), _ptr(scales),
+                                   _stream(stream)))
+
+
+def recur_backward_q(shape: SdmShape, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem, kind: str, codes, scales, dy, dv,
+                     dalpha, dbeta, dw_w, dw_r, dM, stream=None):
+    """sdm_recur_backward_q: sdm_recur_backward reading the log from a quantised snapshot."""
+    _check(lib().sdm_recur_backward_q(ctypes.byref(shape), _ptr(idx_w), _ptr(w_w), _ptr(idx_r), _ptr(w_r), _ptr(v),
+                                      _ptr(alpha), _ptr(beta), _ptr(mem), UNDO_KINDS[kind], _ptr(codes), _ptr(scales),
+                                      _ptr(dy), _ptr(dv), _ptr(dalpha), _ptr(dbeta), _ptr(dw_w), _ptr(dw_r), _ptr(dM),
+                                      _stream(stream)))
 
 
 def gates(shape: SdmShape, d_model: int, x, W_a, W_b, b_dt, A, alpha, beta, stream=None):

@@ -67,7 +67,7 @@ struct SideStream {
     cudaEvent_t fork = nullptr, join = nullptr;
 };
 SideStream g_side[kMaxDevices];
-constexpr int kCopyCtasPerSm = 4;     // M0 copy CTAs per SM beside the addressing
+constexpr int kCopyCtasPerSm = 1;     // M0 copy CTAs per SM beside the addressing
 std::mutex g_side_mutex[kMaxDevices];
 
 sdm_status side_stream(int* dev_out, SideStream** out) {
@@ -364,6 +364,12 @@ sdm_status recur_impl(const char* who, const sdm_shape* s, const int32_t* idx_w,
                       void* mem, void* y, void* undo, void* workspace, size_t workspace_bytes, sdm_stream_t stream,
                       long long wait_cycles = 0, int hold_handover = 0);
 
+// sdm_recur_backward over a stored log (kind 0) or a quantised snapshot (kind 1, 2).
+sdm_status backward_impl(const char* who, const sdm_shape* s, const int32_t* idx_w, const float* w_w,
+                         const int32_t* idx_r, const float* w_r, const void* v, const void* alpha, const void* beta,
+                         void* mem, int kind, const void* log, const float* scales, const void* dy, float* dv,
+                         float* dalpha, float* dbeta, float* dw_w, float* dw_r, float* dM, sdm_stream_t stream);
+
 }  // namespace
 
 extern "C" {
@@ -593,9 +599,60 @@ sdm_status sdm_recur_backward(const sdm_shape* s, const int32_t* idx_w, const fl
                               const float* w_r, const void* v, const void* alpha, const void* beta, void* mem,
                               const void* undo, const void* dy, float* dv, float* dalpha, float* dbeta, float* dw_w,
                               float* dw_r, float* dM, sdm_stream_t stream) {
+    return backward_impl("sdm_recur_backward", s, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem, 0, undo, nullptr,
+                         dy, dv, dalpha, dbeta, dw_w, dw_r, dM, stream);
+}
+
+size_t sdm_undo_code_bytes(const sdm_shape* s, int kind) {
+    if (check_shape(s, false, nullptr) != SDM_OK || (kind != SDM_UNDO_FP8 && kind != SDM_UNDO_INT4)) return 0;
+    const size_t rows = static_cast<size_t>(s->B) * s->H * s->T * s->k_write;
+    return rows * (kind == SDM_UNDO_FP8 ? s->d_v : s->d_v / 2);
+}
+
+sdm_status sdm_undo_quantize(const sdm_shape* s, const void* undo, int kind, void* codes, float* scales,
+                             sdm_stream_t stream) {
+    SDM_TRY(check_shape(s, false, nullptr));
+    if (kind != SDM_UNDO_FP8 && kind != SDM_UNDO_INT4)
+        return fail(SDM_ERR_INVALID_ARG, "sdm_undo_quantize: kind must be SDM_UNDO_FP8 or SDM_UNDO_INT4 (kind=%d)", kind);
+    if (s->d_v % 32 != 0 || s->d_v > 256)
+        return fail(SDM_ERR_UNSUPPORTED, "sdm_undo_quantize: d_v must be a multiple of 32, at most 256 (d_v=%d)", s->d_v);
+    const size_t rows = static_cast<size_t>(s->B) * s->H * s->T * s->k_write;
+    if (rows == 0) return ok();
+    const size_t es = elem_bytes(s->dtype);
+    SDM_TRY(check_vec(undo, "undo", 16));
+    SDM_TRY(check_vec(codes, "codes", 16));
+    SDM_TRY(check_vec(scales, "scales", 4));
+    const Range in{undo, rows * s->d_v * es, "undo"};
+    const Range oc{codes, sdm_undo_code_bytes(s, kind), "codes"}, os{scales, rows * 4, "scales"};
+    if (overlaps(oc, in) || overlaps(os, in) || overlaps(oc, os))
+        return fail(SDM_ERR_INVALID_ARG, "sdm_undo_quantize: undo, codes and scales must not overlap");
+    cudaError_t e = sdm::launch_undo_quantize(s->dtype, kind, undo, static_cast<int64_t>(rows), s->d_v, codes, scales,
+                                              reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "undo quantize launch");
+    return ok();
+}
+
+sdm_status sdm_recur_backward_q(const sdm_shape* s, const int32_t* idx_w, const float* w_w, const int32_t* idx_r,
+                                const float* w_r, const void* v, const void* alpha, const void* beta, void* mem,
+                                int kind, const void* codes, const float* scales, const void* dy, float* dv,
+                                float* dalpha, float* dbeta, float* dw_w, float* dw_r, float* dM, sdm_stream_t stream) {
+    if (kind != SDM_UNDO_FP8 && kind != SDM_UNDO_INT4)
+        return fail(SDM_ERR_INVALID_ARG, "sdm_recur_backward_q: kind must be SDM_UNDO_FP8 or SDM_UNDO_INT4 (kind=%d)", kind);
+    return backward_impl("sdm_recur_backward_q", s, idx_w, w_w, idx_r, w_r, v, alpha, beta, mem, kind, codes, scales,
+                         dy, dv, dalpha, dbeta, dw_w, dw_r, dM, stream);
+}
+
+}  // extern "C"
+
+namespace {
+
+sdm_status backward_impl(const char* who, const sdm_shape* s, const int32_t* idx_w, const float* w_w,
+                         const int32_t* idx_r, const float* w_r, const void* v, const void* alpha, const void* beta,
+                         void* mem, int kind, const void* log, const float* scales, const void* dy, float* dv,
+                         float* dalpha, float* dbeta, float* dw_w, float* dw_r, float* dM, sdm_stream_t stream) {
     SDM_TRY(check_shape(s, false, nullptr));
     if (s->d_v % 32 != 0 || s->d_v > 256)
-        return fail(SDM_ERR_UNSUPPORTED, "sdm_recur_backward: d_v must be a multiple of 32, at most 256 (d_v=%d)", s->d_v);
+        return fail(SDM_ERR_UNSUPPORTED, "%s: d_v must be a multiple of 32, at most 256 (d_v=%d)", who, s->d_v);
     const size_t es = elem_bytes(s->dtype);
     const size_t bht = static_cast<size_t>(s->B) * s->H * s->T;
     if (bht == 0) return ok();
@@ -607,7 +664,8 @@ sdm_status sdm_recur_backward(const sdm_shape* s, const int32_t* idx_w, const fl
     SDM_TRY(check_vec(alpha, "alpha", es));
     SDM_TRY(check_vec(beta, "beta", es));
     SDM_TRY(check_vec(mem, "mem", 16));
-    SDM_TRY(check_vec(undo, "undo", 16));
+    SDM_TRY(check_vec(log, kind == 0 ? "undo" : "codes", 16));
+    if (kind != 0) SDM_TRY(check_vec(scales, "scales", 4));
     SDM_TRY(check_vec(dy, "dy", es));
     SDM_TRY(check_vec(dv, "dv", 4));
     SDM_TRY(check_vec(dalpha, "dalpha", 4));
@@ -617,6 +675,7 @@ sdm_status sdm_recur_backward(const sdm_shape* s, const int32_t* idx_w, const fl
     SDM_TRY(check_vec(dM, "dM", 4));
     const size_t rowb = static_cast<size_t>(s->d_v) * es;
     const size_t memb = static_cast<size_t>(s->B) * s->H * static_cast<size_t>(s->N) * rowb;
+    const size_t logb = kind == 0 ? bht * s->k_write * rowb : sdm_undo_code_bytes(s, kind);
     const Range outs[] = {{mem, memb, "mem"}, {dv, bht * s->d_v * 4, "dv"}, {dalpha, bht * 4, "dalpha"},
                           {dbeta, bht * 4, "dbeta"}, {dw_w, bht * s->k_write * 4, "dw_w"},
                           {dw_r, bht * s->k_read * 4, "dw_r"},
@@ -624,13 +683,14 @@ sdm_status sdm_recur_backward(const sdm_shape* s, const int32_t* idx_w, const fl
     const Range ins[] = {{idx_w, bht * s->k_write * 4, "idx_w"}, {w_w, bht * s->k_write * 4, "w_w"},
                          {idx_r, bht * s->k_read * 4, "idx_r"}, {w_r, bht * s->k_read * 4, "w_r"},
                          {v, bht * rowb, "v"}, {alpha, bht * es, "alpha"}, {beta, bht * es, "beta"},
-                         {undo, bht * s->k_write * rowb, "undo"}, {dy, bht * rowb, "dy"}};
+                         {log, logb, kind == 0 ? "undo" : "codes"},
+                         {scales, kind == 0 ? 0 : bht * s->k_write * 4, "scales"}, {dy, bht * rowb, "dy"}};
     for (size_t i = 0; i < sizeof(outs) / sizeof(outs[0]); ++i) {
         for (const Range& r : ins)
-            if (overlaps(outs[i], r)) return fail(SDM_ERR_INVALID_ARG, "sdm_recur_backward: %s overlaps %s", outs[i].name, r.name);
+            if (overlaps(outs[i], r)) return fail(SDM_ERR_INVALID_ARG, "%s: %s overlaps %s", who, outs[i].name, r.name);
         for (size_t j = i + 1; j < sizeof(outs) / sizeof(outs[0]); ++j)
             if (overlaps(outs[i], outs[j]))
-                return fail(SDM_ERR_INVALID_ARG, "sdm_recur_backward: %s overlaps %s", outs[i].name, outs[j].name);
+                return fail(SDM_ERR_INVALID_ARG, "%s: %s overlaps %s", who, outs[i].name, outs[j].name);
     }
     int* err = nullptr;
     SDM_TRY(status_word(&err));
@@ -640,15 +700,12 @@ sdm_status sdm_recur_backward(const sdm_shape* s, const int32_t* idx_w, const fl
     r.B = s->B; r.H = s->H; r.T = s->T; r.dv = s->d_v; r.kw = s->k_write; r.kr = s->k_read;
     r.N = s->N;
     r.err = err;
-    cudaError_t e = sdm::launch_recur_backward(s->dtype, r, undo, dy, dv, dalpha, dbeta, dw_w, dw_r, dM,
+    cudaError_t e = sdm::launch_recur_backward(s->dtype, r, kind, kind == 0 ? log : nullptr, kind == 0 ? nullptr : log,
+                                               scales, dy, dv, dalpha, dbeta, dw_w, dw_r, dM,
                                                reinterpret_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "backward launch");
     return ok();
 }
-
-}  // extern "C"
-
-namespace {
 
 sdm_status recur_impl(const char* who, const sdm_shape* s, const int32_t* idx_w, const float* w_w,
                       const int32_t* idx_r, const float* w_r, const void* v, const void* alpha, const void* beta,

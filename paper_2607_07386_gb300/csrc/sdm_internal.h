@@ -111,9 +111,15 @@ cudaError_t launch_recur(int dtype, const RecArgs& a, int32_t* hz_ws, cudaStream
                          const int32_t* firstw = nullptr);
 
 // Backward of the recurrence with in-place undo (k_recur_bwd.cu).  a.mem holds M_T on entry and
-// M_0 on return; dM ([B, H, N, dv] fp32, zero on entry) receives dL/dM_0 per chain.
-cudaError_t launch_recur_backward(int dtype, const RecArgs& a, const void* undo, const void* dy, float* dv,
-                                  float* dalpha, float* dbeta, float* dw_w, float* dw_r, float* dM, cudaStream_t stream);
+// M_0 on return; dM ([B, H, N, dv] fp32, zero on entry) receives dL/dM_0 per chain.  kind 0:
+// the log is `undo` (stored rows); kind 1 / 2: fp8 / int4 codes with one float32 scale per row.
+cudaError_t launch_recur_backward(int dtype, const RecArgs& a, int kind, const void* undo, const void* codes,
+                                  const float* scales, const void* dy, float* dv, float* dalpha, float* dbeta,
+                                  float* dw_w, float* dw_r, float* dM, cudaStream_t stream);
+// Quantised snapshot of an undo log of `rows` rows of dv storage elements (kind 1: fp8 e4m3 codes,
+// dv bytes per row; kind 2: int4 codes, dv / 2 bytes per row), one float32 scale per row.
+cudaError_t launch_undo_quantize(int dtype, int kind, const void* undo, int64_t rows, int dv, void* codes,
+                                 float* scales, cudaStream_t stream);
 
 // Chunkwise (WY) form of the recurrence (k_chunk.cu), chunks of C <= 32 tokens; d_v <= 256.
 cudaError_t launch_recur_chunkwise(int dtype, const RecArgs& a, int C, cudaStream_t stream);

@@ -705,6 +705,150 @@ def test_recur_backward_with_undo_matches_the_oracle(sdm, dtype):
             assert e <= tol, (dtype, c, name, e)
 
 
+def _host_undo_log(rng, rows: int, dv: int, dtype: str) -> np.ndarray:
+    """Seeded stand-in for an undo log: rows of stored values with magnitudes spread over many
+    binades, a zero row, a row whose scale is 1 with entries at rounding ties, a row with a
+    single non-zero entry."""
+    u = rng.standard_normal((rows, dv)) * np.exp(2.0 * rng.standard_normal((rows, 1)))
+    u[0] = 0.0
+    u[1] = 0.0
+    u[1, :6] = [448.0, 1.0625, -1.1875, 3.5, 2.5, -0.5]
+    u[2] = 0.0
+    u[2, 5] = -3.0
+    return O.round_storage(u, dtype)
+
+
+def _decode_codes(codes: np.ndarray, kind: str, rows: int, dv: int) -> np.ndarray:
+    """The code values of sdm_undo_quantize's byte layout (fp8: e4m3 bytes; int4: two's
+    complement nibbles, element 2i low), as float64 [rows, dv]."""
+    if kind == "fp8":
+        t = torch.from_numpy(codes.reshape(rows, dv).copy()).view(torch.float8_e4m3fn)
+        return t.to(torch.float64).numpy()
+    b = codes.reshape(rows, dv // 2).astype(np.int32)
+    lo, hi = b & 15, b >> 4
+    q = np.empty((rows, dv), dtype=np.int32)
+    q[:, 0::2] = np.where(lo > 7, lo - 16, lo)
+    q[:, 1::2] = np.where(hi > 7, hi - 16, hi)
+    return q.astype(np.float64)
+
+
+def _encode_codes(q: np.ndarray, kind: str) -> np.ndarray:
+    """Inverse of ``_decode_codes``: bytes of the code values q [rows, dv]."""
+    if kind == "fp8":
+        return torch.from_numpy(q.astype(np.float32)).to(torch.float8_e4m3fn).view(torch.uint8).numpy().ravel()
+    qi = q.astype(np.int32) & 15
+    return (qi[:, 0::2] | (qi[:, 1::2] << 4)).astype(np.uint8).ravel()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("kind", ["fp8", "int4"])
+def test_undo_quantize_codes_match_the_oracle(sdm, kind, dtype):
+    """sdm_undo_quantize on a seeded log gives the oracle's float32-arithmetic codes and scales
+    bit for bit (both sides decide each code in float32: App. A.3's snapshots, one scale per
+    logged row)."""
+    if kind == "fp8" and not hasattr(torch, "float8_e4m3fn"):
+        pytest.skip("torch without float8")
+    B, H, T, kw, dv = 2, 3, 37, 8, (128 if dtype == "bf16" else 64)
+    rows = B * H * T * kw
+    rng = np.random.default_rng(90)
+    log = _host_undo_log(rng, rows, dv, dtype)
+    shape = sdm.SdmShape.make(B, H, T, 32, dv, 1000, kw, kw, dtype)
+    st = lambda x: to_torch(O.to_bf16_bits(x) if dtype == "bf16" else x.astype(np.float32), dtype)
+    tlog = st(log)
+    codes = torch.empty(sdm.undo_code_bytes(shape, kind), dtype=torch.uint8, device="cuda")
+    scales = torch.empty(rows, dtype=torch.float32, device="cuda")
+    sdm.undo_quantize(shape, tlog, kind, codes, scales)
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    q_ref, s_ref = O.undo_codes(log, kind)
+    got_s = scales.cpu().numpy()
+    assert np.array_equal(got_s, s_ref), np.flatnonzero(got_s != s_ref)[:10]
+    got_q = _decode_codes(codes.cpu().numpy(), kind, rows, dv)
+    bad = np.argwhere(got_q != q_ref)
+    assert bad.size == 0, (bad[:10], got_q[tuple(bad[0])], q_ref[tuple(bad[0])])
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("kind", ["fp8", "int4"])
+def test_recur_backward_from_quantized_snapshot_matches_the_oracle(sdm, kind, dtype):
+    """sdm_recur_backward_q from the oracle's snapshot of the oracle's forward: the restored
+    memory equals the oracle's restore (each row the stored value of q * s) bit for bit, and
+    the six gradients match the oracle's backward through the same log within the bars of the
+    exact backward.  Then the whole chain on the GPU (sdm_recur_undo, sdm_undo_quantize,
+    sdm_recur_backward_q) runs clean."""
+    if kind == "fp8" and not hasattr(torch, "float8_e4m3fn"):
+        pytest.skip("torch without float8")
+    B, H, N, T, kw, kr = 2, 1, 400, 90, 8, 20
+    dv = 128 if dtype == "bf16" else 64
+    rng = np.random.default_rng(91)
+    M0 = O.round_storage(rng.standard_normal((B * H, N, dv)) * 0.3, dtype)
+    iw = np.stack([np.sort(rng.choice(N, kw, replace=False)) for _ in range(B * H * T)]).reshape(B, H, T, kw)
+    ir = np.stack([np.sort(rng.choice(N, kr, replace=False)) for _ in range(B * H * T)]).reshape(B, H, T, kr)
+    ww = rng.dirichlet(np.ones(kw), B * H * T).astype(np.float32).reshape(B, H, T, kw)
+    wr = rng.dirichlet(np.ones(kr), B * H * T).astype(np.float32).reshape(B, H, T, kr)
+    a = O.round_storage(1 / (1 + np.exp(-rng.standard_normal((B, H, T)) - 2)), dtype)
+    b = O.round_storage(1 / (1 + np.exp(-rng.standard_normal((B, H, T)))), dtype)
+    V = O.round_storage(rng.standard_normal((B, H, T, dv)), dtype)
+    dY = O.round_storage(rng.standard_normal((B, H, T, dv)), dtype)
+    st = lambda x: to_torch(O.to_bf16_bits(x) if dtype == "bf16" else x.astype(np.float32), dtype)
+    cu = lambda x: torch.from_numpy(np.ascontiguousarray(x)).cuda()
+    shape = sdm.SdmShape.make(B, H, T, 32, dv, N, kw, kr, dtype)
+    tiw, tir, tww, twr = cu(iw.astype(np.int32)), cu(ir.astype(np.int32)), cu(ww), cu(wr)
+    tv, ta, tb, tdy = st(V), st(a), st(b), st(dY)
+    # the oracle's forward: M_T and the log; its snapshot; the backward through it
+    MT, logs, refs, restored = [], [], [], []
+    for c in range(B * H):
+        bb, hh = divmod(c, H)
+        Mo = M0[c].copy()
+        _, und = O.recur_forward_undo(Mo, iw[bb, hh], ww[bb, hh].astype(np.float64), ir[bb, hh],
+                                      wr[bb, hh].astype(np.float64), V[bb, hh], a[bb, hh], b[bb, hh], dtype)
+        MT.append(Mo.copy())
+        logs.append(und)
+        deq = O.round_storage(O.quantize_undo(und, kind, "f32"), dtype)
+        Mr = Mo.copy()
+        refs.append(O.recur_backward(Mr, deq, iw[bb, hh], ww[bb, hh].astype(np.float64), ir[bb, hh],
+                                     wr[bb, hh].astype(np.float64), V[bb, hh], a[bb, hh], b[bb, hh], dY[bb, hh]))
+        restored.append(Mr)
+    rows = B * H * T * kw
+    q, sc = O.undo_codes(np.stack(logs).reshape(rows, dv), kind)
+    codes = cu(_encode_codes(q, kind))
+    scales = cu(sc.astype(np.float32))
+    assert codes.numel() == sdm.undo_code_bytes(shape, kind)
+    mem = st(np.stack(MT).reshape(B, H, N, dv))
+    f32 = lambda *s_: torch.zeros(s_, dtype=torch.float32, device="cuda")
+    g_dv, g_da, g_db = f32(B, H, T, dv), f32(B, H, T), f32(B, H, T)
+    g_ww, g_wr, g_dM = f32(B, H, T, kw), f32(B, H, T, kr), f32(B, H, N, dv)
+    sdm.recur_backward_q(shape, tiw, tww, tir, twr, tv, ta, tb, mem, kind, codes, scales, tdy, g_dv, g_da, g_db,
+                         g_ww, g_wr, g_dM)
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    assert torch.equal(mem, st(np.stack(restored).reshape(B, H, N, dv)))
+    tol = 1e-4 if dtype == "f32" else 5e-3
+    for c in range(B * H):
+        bb, hh = divmod(c, H)
+        for name, got in (("dv", g_dv), ("dalpha", g_da), ("dbeta", g_db), ("dw_w", g_ww), ("dw_r", g_wr),
+                          ("dM0", g_dM)):
+            e = rel_fro(got[bb, hh].cpu().numpy().astype(np.float64), refs[c][name])
+            assert e <= tol, (kind, dtype, c, name, e)
+    # the chain on the GPU alone
+    mem = st(M0.reshape(B, H, N, dv))
+    y = torch.empty((B, H, T, dv), dtype=mem.dtype, device="cuda")
+    undo = torch.empty(sdm.undo_log_bytes(shape), dtype=torch.uint8, device="cuda")
+    rws = torch.empty(sdm.recur_workspace_bytes(shape), dtype=torch.uint8, device="cuda")
+    sdm.recur_undo(shape, tiw, tww, tir, twr, tv, ta, tb, mem, y, undo, rws)
+    sdm.undo_quantize(shape, undo, kind, codes, scales)
+    for t_ in (g_dv, g_da, g_db, g_ww, g_wr, g_dM):
+        t_.zero_()
+    sdm.recur_backward_q(shape, tiw, tww, tir, twr, tv, ta, tb, mem, kind, codes, scales, tdy, g_dv, g_da, g_db,
+                         g_ww, g_wr, g_dM)
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    for c in range(B * H):
+        bb, hh = divmod(c, H)
+        e = rel_fro(g_dv[bb, hh].cpu().numpy().astype(np.float64), refs[c]["dv"])
+        assert e <= 10 * tol, (kind, dtype, c, e)
+
+
 # ------------------------------------------------------------------ gates and output epilogue
 
 def _storage_ulp(ref: np.ndarray, dtype: str) -> np.ndarray:

@@ -430,6 +430,45 @@ def test_quantized_undo_log_bounds_and_effect_on_gradients():
     assert 0 < err["fp8"] < err["int4"] and err["fp8"] < 0.1
 
 
+def test_undo_codes_in_float32_arithmetic():
+    """The snapshot codes as a float32 implementation decides them: hand-worked int4 row with
+    ties to even, the row maximum always coded as the top value, codes inside the format, the
+    float64 path reproduced exactly where the scale is a power of two (every step exact), and
+    the half-step error bound of the float32 dequantised rows."""
+    # s = 7 / 7 = 1: codes are the integers nearest the entries, ties to even
+    row = np.array([[7.0, 3.5, -3.5, 0.5, 1.5, 2.5, -6.5, 0.0]])
+    q, sc = O.undo_codes(row, "int4")
+    assert sc.tolist() == [1.0]
+    assert q.tolist() == [[7, 4, -4, 0, 2, 2, -6, 0]]
+    # fp8: max 448 -> s = 1; 1.0625 lies halfway between 1 and 1.125 (4 significant bits): to even
+    row = np.array([[448.0, 1.0625, 1.1875, -2.0 ** -9, 3.0 * 2.0 ** -10, 0.0]])
+    q, sc = O.undo_codes(row, "fp8")
+    assert sc.tolist() == [1.0]
+    assert q.tolist() == [[448.0, 1.0, 1.25, -2.0 ** -9, 2.0 ** -8, 0.0]]
+    # zero rows: scale 1, codes 0
+    q, sc = O.undo_codes(np.zeros((2, 5)), "fp8")
+    assert sc.tolist() == [1.0, 1.0] and not q.any()
+    rng = np.random.default_rng(66)
+    u = (rng.standard_normal((40, 9, 32)) * np.exp(3 * rng.standard_normal((40, 9, 1)))).astype(np.float32)
+    u = u.astype(np.float64)
+    for kind, top in (("fp8", 448.0), ("int4", 7.0)):
+        q, sc = O.undo_codes(u, kind)
+        assert sc.dtype == np.float32
+        amax = np.abs(u).max(axis=-1)
+        assert np.all(np.abs(q).max(axis=-1) == top)                     # the row maximum codes as +-top
+        if kind == "int4":
+            assert np.array_equal(q, np.round(q)) and np.abs(q).max() <= 7
+        else:
+            assert np.array_equal(O.round_e4m3(q), q)
+        deq = O.quantize_undo(u, kind, "f32")
+        step = amax * (2.0 ** -4 if kind == "fp8" else 1.0 / 14.0)
+        assert np.all(np.abs(deq - u) <= step[..., None] * (1 + 2.0 ** -20) + 1e-300)
+        # rows scaled so that max|row| = top * 2^e: the scale is a power of two, every step exact
+        p2 = (u / amax[..., None] * top).astype(np.float32).astype(np.float64)
+        p2 = p2 * 2.0 ** rng.integers(-8, 8, amax.shape)[..., None]
+        assert np.array_equal(O.quantize_undo(p2, kind, "f32"), O.quantize_undo(p2, kind))
+
+
 # ------------------------------------------------------------------ lazy M0 (copy-on-write)
 
 def test_lazy_overlay_equals_dense_masked_form():
