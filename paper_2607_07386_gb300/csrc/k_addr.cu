@@ -1763,7 +1763,10 @@ static cudaError_t launch_finalize(const AddrArgs& a, cudaStream_t stream) {
             } else {
                 k_addr_finalize<D, L, FIN_FAST><<<grid, FW_WARPS * 32, 0, stream>>>(a);
             }
-            if (a.ncc == 1) {                    // band pass, one thread per queued token-side
+            // band pass: one thread per queued token-side on large problems; a warp per item when
+            // the problem is small (decode): there the queue is short and each item's serial
+            // rescoring, not the item count, sets the pass's length
+            if (a.ncc == 1 && 2 * a.H * BT >= 32768) {
                 const size_t smb = static_cast<size_t>(bt_words(L)) * BT_THREADS * sizeof(float);
                 e = cudaFuncSetAttribute(k_addr_band_thread<D, L>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smb));

@@ -223,14 +223,17 @@ def _clustered_projection(rng, S, dk, x0, n_hi, cluster, dup):
 
 
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
-def test_address_clustered_scores_take_every_band_path(sdm, dtype):
+@pytest.mark.parametrize("B", [1, 176])
+def test_address_clustered_scores_take_every_band_path(sdm, dtype, B):
     """Scores clustered within the fp32 error bound around the top-k boundary.  Head 0: a
     cluster wide enough that the band leaves the kept list (whole-half rescan); head 1:
     duplicated rows inside the band (exact ties, decided in float64).  Indices must equal
-    the float64 definition's; the event counters show which paths decided."""
+    the float64 definition's; the event counters show which paths decided.  B = 176 repeats
+    the sequence to 33,792 token-sides, past the size where the band pass turns from a warp
+    per item to a thread per item (every copy must give the same lists)."""
     S, dk, T = 64, 64, 48
     x0 = 2.0 ** -10 if dtype == "bf16" else 2.0 ** -14
-    cfg = synth.SdmConfig("clustered", B=1, H=2, T=T, d_k=dk, d_v=16, N=S * S, k_write=16, k_read=8,
+    cfg = synth.SdmConfig("clustered", B=B, H=2, T=T, d_k=dk, d_v=16, N=S * S, k_write=16, k_read=8,
                           dtype=dtype, seed=7, alpha_mu=3.0)
     rng = np.random.default_rng(11)
     full = {}
@@ -241,10 +244,10 @@ def test_address_clustered_scores_take_every_band_path(sdm, dtype):
                       _clustered_projection(rng, S, dk, x0, 13, 3, 2) for _ in range(2)]
             heads.append(np.concatenate(halves))
         full[name] = np.stack(heads)
-    X = np.zeros((1, 2, T, dk))
+    X = np.zeros((B, 2, T, dk))
     X[..., 0] = x0
     X[..., 1] = 1.0
-    X[..., 2:] = rng.standard_normal((1, 2, T, dk - 2)) * 0.0     # keep the scores exact
+    X[..., 2:] = rng.standard_normal((B, 2, T, dk - 2)) * 0.0     # keep the scores exact
     full["q"], full["k"] = X.copy(), X.copy()
     full = {n: synth.round_f64_to_storage(a, dtype) for n, a in full.items()}
     dev = {n: synth.torch_io.to_torch(a, dtype) for n, a in full.items()}
@@ -258,6 +261,8 @@ def test_address_clustered_scores_take_every_band_path(sdm, dtype):
         ir, _, _ = O.address(f(full["P_q"][h]), f(full["q"][0, h]), S * S, 8)
         assert np.array_equal(out["idx_w"][0, h].cpu().numpy(), iw), h
         assert np.array_equal(out["idx_r"][0, h].cpu().numpy(), ir), h
+    for n in ("idx_w", "idx_r"):
+        assert torch.equal(out[n], out[n][:1].expand_as(out[n])), n
     assert st["half_band"] > 0 and st["half_full"] > 0 and st["band_f64"] > 0, st
 
 
