@@ -38,10 +38,10 @@ UNIT = "tokens/s"
 
 
 # DRAM bytes per token-head moved by the recurrence phase (hazard pass + recurrence), from an
-# ncu capture of dram__bytes_read.sum + dram__bytes_write.sum at the layer geometry with B=2,
-# the same kernels as at B=8 (profiles/recurrence_layer_1p4b_dram_traffic.txt):
-# 3,205,865,728 B / 131,072 token-heads.
-RECUR_DRAM_BYTES_PER_TOKEN_HEAD = 3205865728 / 131072
+# ncu capture of dram__bytes_read.sum + dram__bytes_write.sum of the hazard pass and the
+# recurrence on the layer_1p4b workload itself (profiles/recurrence_layer_1p4b.md):
+# (134.24 MB + 38.05 MB) + (10.45 GB + 4.35 GB) over 524,288 token-heads.
+RECUR_DRAM_BYTES_PER_TOKEN_HEAD = (134.24e6 + 38.05e6 + 10.45e9 + 4.35e9) / 524288
 
 
 def _peaks():
@@ -617,8 +617,10 @@ def run_ours(args, cfg):
         b_o = torch.empty_like(a_o)
         z = torch.empty((B, T, H, dv), dtype=dt, device="cuda")
         W_o = (torch.randn(d_model, H * dv, device="cuda") / (H * dv) ** 0.5).to(dt)
+        o_mix = torch.empty((B * T, d_model), dtype=dt, device="cuda")
         runs = {"gates": lambda: sdm.gates(shape, d_model, lx, lwa, lwb, lbdt, lA, a_o, b_o, stream=stream),
                 "norm_gate": lambda: sdm.norm_gate(shape, y, lg, lgam, 1e-6, z, stream=stream),
+                "head_mix": lambda: sdm.head_mix(shape, d_model, z.view(B * T, H * dv), W_o, o_mix, stream=stream),
                 "w_o_gemm": lambda: torch.matmul(z.view(B * T, H * dv), W_o.t())}
         ms = {}
         for name, fn in runs.items():
@@ -636,16 +638,20 @@ def run_ours(args, cfg):
         n_bytes = 3 * B * H * T * dv * es + dv * 4
         w_flop = 2.0 * B * T * (H * dv) * d_model
         around = {
-            "note": "sdm_gates and sdm_norm_gate (library kernels) and the W_o head-mixing GEMM (torch/cuBLAS), "
-                    "each timed alone; inputs larger than L2",
+            "note": "sdm_gates, sdm_norm_gate and sdm_head_mix (library kernels; the gates and the head mix on "
+                    "the tensor cores), each timed alone, with cuBLAS's GEMM of the same head mix beside them for "
+                    "comparison; inputs larger than L2",
             "d_model": d_model,
             "gates": {"ms": ms["gates"], "gbs": g_bytes / (ms["gates"] * 1e-3) / 1e9,
                       "gflops": 4.0 * B * T * H * d_model / (ms["gates"] * 1e-3) / 1e9},
             "norm_gate": {"ms": ms["norm_gate"], "gbs": n_bytes / (ms["norm_gate"] * 1e-3) / 1e9,
                           "frac_of_measured_hbm": n_bytes / (ms["norm_gate"] * 1e-3) / 1e9 / _peaks()["hbm_gbs"]},
+            "head_mix": {"ms": ms["head_mix"], "tflops": w_flop / (ms["head_mix"] * 1e-3) / 1e12,
+                         "frac_of_measured_bf16": w_flop / (ms["head_mix"] * 1e-3) / 1e12 / _peaks()["bf16_tflops"]},
+            "gates_tensor_cores": sdm.gates_tensor_cores(shape, d_model),
             "w_o_gemm_cublas": {"ms": ms["w_o_gemm"], "tflops": w_flop / (ms["w_o_gemm"] * 1e-3) / 1e12},
         }
-        del lx, lwa, lwb, lg, a_o, b_o, z, W_o
+        del lx, lwa, lwb, lg, a_o, b_o, z, W_o, o_mix
 
     # ---- end to end through the public API with host buffers (pinned), copies inside the region
     h2d = sum(t.numel() * t.element_size() for t in host_pinned.values())
@@ -723,14 +729,11 @@ def run_ours(args, cfg):
         "e2e": {"value": tokens_step / (ms_e2e * 1e-3), "unit": UNIT, "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h},
         "gpu_launches": kernels_per_step * args.steps,
-        "roofline": {"bound": "hbm", "kernel": "k_recur", "achieved": achieved, "peak": peaks["hbm_gbs"],
-                     "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"],
-                     # the DRAM counters were taken with one warp per CTA; the kernel now groups four
-                     # d-range warps of a chain per CTA, so the count is withheld until re-captured
-                     "traffic": None,
-                     "traffic_last_capture": RECUR_DRAM_BYTES_PER_TOKEN_HEAD * B * H * T if cfg.name == "layer_1p4b" else None,
-                     "traffic_source": "ncu dram bytes of the hazard pass + recurrence at B=2 (one warp per CTA), "
-                                       "scaled to B*H*T; not of the current launch shape",
+        "roofline": {"bound": "hbm", "kernel": "k_hazard + k_recur_tw (the recurrence phase)", "achieved": achieved, "peak": peaks["hbm_gbs"],
+                     "unit": "GB/s", "frac": achieved / peaks["hbm_gbs"], "frac_of_8tbs": achieved / 8000.0,
+                     "traffic": RECUR_DRAM_BYTES_PER_TOKEN_HEAD * B * H * T if cfg.name == "layer_1p4b" else None,
+                     "traffic_source": "ncu dram__bytes_read.sum + dram__bytes_write.sum of k_hazard + k_recur_tw, "
+                                       "one launch on this workload (B=8)",
                      "peak_source": peaks["source"], "bytes_per_launch": rec_bytes, "ms_per_launch": rec_ms},
         "phase_ms": ph,
         "lazy_m0": lazy,

@@ -166,10 +166,26 @@ sdm_status sdm_materialize(const sdm_shape* shape, const void* M0, const uint32_
  * x: [B, T, d_model], W_a, W_b: [H, d_model] (storage dtype, 16-byte aligned;
  * d_model * element size a multiple of 16 bytes); b_dt, A: [H] float32; alpha, beta:
  * [B, H, T] storage dtype (the layout sdm_forward takes).  H <= 32.  Uses shape B, H, T
- * and dtype only.  fp32 arithmetic; outputs rounded to nearest. */
+ * and dtype only.  fp32 arithmetic; outputs rounded to nearest.  With bf16 storage, H = 16
+ * or 32 and d_model % 8 == 0 the projections run on the tensor cores ([B*T, d_model] x
+ * [d_model, 2H], bf16 products accumulated in fp32 blocks of 16, see sdm_gates_tensor_cores);
+ * otherwise as fp32 fused multiply-adds. */
 sdm_status sdm_gates(const sdm_shape* shape, int32_t d_model, const void* x, const void* W_a,
                      const void* W_b, const float* b_dt, const float* A, void* alpha, void* beta,
                      sdm_stream_t stream);
+
+/* 1 if sdm_gates takes the tensor-core form for this shape and d_model, else 0 (its error
+ * bound differs: bf16 products summed in fp32 blocks of 16, like the scores). */
+int sdm_gates_tensor_cores(const sdm_shape* shape, int32_t d_model);
+
+/* Head-mixing projection (Sec. 3.1, "Norm, Gating, and Head Mixing") on the tensor cores:
+ *   out[m, n] = sum_k z[m, k] W_o[n, k],   m < B*T, n < d_model, k < H*d_v,
+ * z: [B*T, H*d_v] (sdm_norm_gate's output), W_o: [d_model, H*d_v], out: [B*T, d_model], all
+ * bf16, row-major, 16-byte aligned; fp32 accumulation, out rounded to nearest.  bf16 storage
+ * only (SDM_ERR_UNSUPPORTED otherwise); d_model a multiple of 32, H*d_v a multiple of 8.  out
+ * must not overlap z or W_o. */
+sdm_status sdm_head_mix(const sdm_shape* shape, int32_t d_model, const void* z, const void* W_o,
+                        void* out, sdm_stream_t stream);
 
 /* Output gate of every head (Sec. 3.1, "Norm, Gating, and Head Mixing"):
  *   z[b, t, h, :] = g[b, h, t, :] * gamma * y[b, h, t, :] / sqrt(mean(y[b, h, t, :]^2) + eps).

@@ -9,7 +9,7 @@ from ._binding import (  # noqa: F401
     ADDR_DIRECT, ADDR_PROJECTED, DTYPE_BF16, DTYPE_F32, SdmError, SdmShape, abi_version, address,
     decode_step, device_stats, device_status, forward, forward_m0, init_memory, last_error, lib, lib_path, recur, recur_noalloc,
     recur_workspace_bytes, workspace_bytes, RECUR_NOALLOC_SCRATCH_BYTES, forward_lazy, lazy_workspace_bytes,
-    materialize, touched_words, access_stats, access_stats_workspace_bytes, gates, norm_gate,
+    materialize, touched_words, access_stats, access_stats_workspace_bytes, gates, norm_gate, gates_tensor_cores, head_mix,
     undo_log_bytes, recur_undo, recur_backward, undo_code_bytes, undo_quantize, recur_backward_q, recur_chunkwise, recur_plan, test_recur_wait_timeout,
     RECUR_PLAN_FIELDS, test_scores,
 )

@@ -94,6 +94,10 @@ def lib():
             L.sdm_gates.restype = ctypes.c_int
             L.sdm_norm_gate.argtypes = [_SHP, _VP, _VP, _VP, ctypes.c_float, _VP, _VP]
             L.sdm_norm_gate.restype = ctypes.c_int
+            L.sdm_gates_tensor_cores.argtypes = [_SHP, ctypes.c_int32]
+            L.sdm_gates_tensor_cores.restype = ctypes.c_int
+            L.sdm_head_mix.argtypes = [_SHP, ctypes.c_int32, _VP, _VP, _VP, _VP]
+            L.sdm_head_mix.restype = ctypes.c_int
             L.sdm_access_stats_workspace_bytes.restype = ctypes.c_size_t
             L.sdm_access_stats_workspace_bytes.argtypes = [_SHP]
             L.sdm_access_stats.argtypes = [_SHP, _I32P, _VP, _I32P, _VP, _VP, _VP, _SZ, _VP]
@@ -282,6 +286,16 @@ def gates(shape: SdmShape, d_model: int, x, W_a, W_b, b_dt, A, alpha, beta, stre
     """sdm_gates: alpha, beta [B, H, T] from the layer input x [B, T, d_model]."""
     _check(lib().sdm_gates(ctypes.byref(shape), int(d_model), _ptr(x), _ptr(W_a), _ptr(W_b), _ptr(b_dt), _ptr(A),
                            _ptr(alpha), _ptr(beta), _stream(stream)))
+
+
+def gates_tensor_cores(shape: SdmShape, d_model: int) -> bool:
+    """Whether sdm_gates runs its projections on the tensor cores for this shape."""
+    return bool(lib().sdm_gates_tensor_cores(ctypes.byref(shape), int(d_model)))
+
+
+def head_mix(shape: SdmShape, d_model: int, z, W_o, out, stream=None):
+    """sdm_head_mix: out [B*T, d_model] = z [B*T, H*d_v] W_o^T on the tensor cores (bf16)."""
+    _check(lib().sdm_head_mix(ctypes.byref(shape), int(d_model), _ptr(z), _ptr(W_o), _ptr(out), _stream(stream)))
 
 
 def norm_gate(shape: SdmShape, y, g, gamma, eps: float, z, stream=None):

@@ -48,4 +48,74 @@ cudaError_t launch_init_memory(const void* M0, void* mem, int64_t bytes_per_seq,
     return cudaGetLastError();
 }
 
+// The same broadcast through the bulk-copy (TMA) engine, for the copy that runs beside the
+// addressing: one thread per CTA, one CTA per SM.  The thread loads 16 KB of M0 into shared
+// memory (cp.async.bulk, completion on an mbarrier) and stores that buffer to all B sequences
+// (B cp.async.bulk stores, one bulk group), double-buffered: the load of the next chunk goes
+// out once the stores of the chunk before have read their buffer.  The copy engine keeps the
+// bytes in flight, so the CTA holds one warp, 32 KB of shared memory and few registers, and the
+// addressing kernels keep the rest of the SM.
+constexpr int IB_CHUNK = 16384;
+
+__device__ __forceinline__ bool ib_wait(uint32_t bar, uint32_t parity) {
+    const long long t0 = clock64();
+    for (;;) {
+        uint32_t done;
+        asm volatile("{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+                     : "=r"(done) : "r"(bar), "r"(parity) : "memory");
+        if (done) return true;
+        if (clock64() - t0 > 4000000000LL) return false;
+    }
+}
+
+__global__ void __launch_bounds__(32, 1) k_init_bulk(const char* __restrict__ M0, char* __restrict__ mem,
+                                                     int64_t bytes_per_seq, int B, int* err) {
+    __shared__ __align__(128) unsigned char buf[2][IB_CHUNK];
+    __shared__ __align__(8) unsigned long long bar[2];
+    if (threadIdx.x != 0) return;
+    const uint32_t sb0 = static_cast<uint32_t>(__cvta_generic_to_shared(buf[0]));    // buffer s at sb0 + s * IB_CHUNK
+    const uint32_t mb0 = static_cast<uint32_t>(__cvta_generic_to_shared(&bar[0]));    // barrier s at mb0 + 8 * s
+    for (int i = 0; i < 2; ++i) asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;\n" ::"r"(mb0 + 8 * i) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+    const int64_t nchunks = (bytes_per_seq + IB_CHUNK - 1) / IB_CHUNK;
+    auto load = [&](int64_t c, int s) {
+        const int64_t left = bytes_per_seq - c * IB_CHUNK;
+        const uint32_t n = static_cast<uint32_t>(left < IB_CHUNK ? left : IB_CHUNK);
+        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" ::"r"(mb0 + 8 * s), "r"(n) : "memory");
+        asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];\n"
+                     ::"r"(sb0 + s * IB_CHUNK), "l"(M0 + c * IB_CHUNK), "r"(n), "r"(mb0 + 8 * s) : "memory");
+    };
+    bool ok = true;
+    int64_t c = blockIdx.x;
+    if (c < nchunks) load(c, 0);
+    for (int i = 0; c < nchunks; ++i, c += gridDim.x) {
+        const int s = i & 1;
+        if (!ib_wait(mb0 + 8 * s, static_cast<uint32_t>(i >> 1) & 1u)) { ok = false; break; }
+        const int64_t left = bytes_per_seq - c * IB_CHUNK;
+        const uint32_t n = static_cast<uint32_t>(left < IB_CHUNK ? left : IB_CHUNK);
+        for (int b = 0; b < B; ++b)
+            asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;\n"
+                         ::"l"(mem + b * bytes_per_seq + c * IB_CHUNK), "r"(sb0 + s * IB_CHUNK), "r"(n) : "memory");
+        asm volatile("cp.async.bulk.commit_group;\n" ::: "memory");
+        if (c + gridDim.x < nchunks) {
+            // the other buffer was read by the stores of the chunk before this one
+            asm volatile("cp.async.bulk.wait_group.read 1;\n" ::: "memory");
+            load(c + gridDim.x, s ^ 1);
+        }
+    }
+    asm volatile("cp.async.bulk.wait_group 0;\n" ::: "memory");
+    if (!ok) flag_error(err, ERR_TIMEOUT);
+}
+
+cudaError_t launch_init_bulk(const void* M0, void* mem, int64_t bytes_per_seq, int B, int* err, cudaStream_t stream) {
+    int dev = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    const int64_t nchunks = (bytes_per_seq + IB_CHUNK - 1) / IB_CHUNK;
+    const unsigned grid = static_cast<unsigned>(nchunks < sms ? (nchunks > 0 ? nchunks : 1) : sms);
+    k_init_bulk<<<grid, 32, 0, stream>>>(static_cast<const char*>(M0), static_cast<char*>(mem), bytes_per_seq, B, err);
+    return cudaGetLastError();
+}
+
 }  // namespace sdm

@@ -480,9 +480,46 @@ sdm_status sdm_gates(const sdm_shape* s, int32_t d_model, const void* x, const v
     for (const Range& r : ins)
         if (overlaps(ra, r) || overlaps(rb, r)) return fail(SDM_ERR_INVALID_ARG, "sdm_gates: a gate output overlaps %s", r.name);
     if (overlaps(ra, rb)) return fail(SDM_ERR_INVALID_ARG, "sdm_gates: alpha overlaps beta");
-    cudaError_t e = sdm::launch_gates(s->dtype, x, W_a, W_b, b_dt, A, alpha, beta, s->B, s->T, s->H, d_model,
-                                      reinterpret_cast<cudaStream_t>(stream));
+    cudaError_t e;
+    if (sdm::gates_tc_supported(s->dtype, s->H, d_model)) {
+        int* err = nullptr;
+        SDM_TRY(status_word(&err));
+        e = sdm::launch_gates_tc(x, W_a, W_b, b_dt, A, alpha, beta, s->B, s->T, s->H, d_model, err,
+                                 reinterpret_cast<cudaStream_t>(stream));
+    } else {
+        e = sdm::launch_gates(s->dtype, x, W_a, W_b, b_dt, A, alpha, beta, s->B, s->T, s->H, d_model,
+                              reinterpret_cast<cudaStream_t>(stream));
+    }
     if (e != cudaSuccess) return cuda_fail(e, "gates launch");
+    return ok();
+}
+
+int sdm_gates_tensor_cores(const sdm_shape* s, int32_t d_model) {
+    return s != nullptr && sdm::gates_tc_supported(s->dtype, s->H, d_model) ? 1 : 0;
+}
+
+sdm_status sdm_head_mix(const sdm_shape* s, int32_t d_model, const void* z, const void* W_o, void* out,
+                        sdm_stream_t stream) {
+    SDM_TRY(check_shape(s, false, nullptr));
+    if (s->dtype != SDM_BF16) return fail(SDM_ERR_UNSUPPORTED, "sdm_head_mix: bf16 storage only");
+    const int64_t K = static_cast<int64_t>(s->H) * s->d_v;
+    if (d_model <= 0 || d_model % 32 != 0)
+        return fail(SDM_ERR_UNSUPPORTED, "sdm_head_mix: d_model must be a positive multiple of 32 (d_model=%d)", d_model);
+    if (K % 8 != 0) return fail(SDM_ERR_UNSUPPORTED, "sdm_head_mix: H * d_v must be a multiple of 8");
+    const size_t M = static_cast<size_t>(s->B) * s->T;
+    if (M == 0) return ok();
+    SDM_TRY(check_vec(z, "z", 16));
+    SDM_TRY(check_vec(W_o, "W_o", 16));
+    SDM_TRY(check_vec(out, "out", 16));
+    const Range ro{out, M * d_model * 2, "out"};
+    const Range ins[] = {{z, M * K * 2, "z"}, {W_o, static_cast<size_t>(d_model) * K * 2, "W_o"}};
+    for (const Range& r : ins)
+        if (overlaps(ro, r)) return fail(SDM_ERR_INVALID_ARG, "sdm_head_mix: out overlaps %s", r.name);
+    int* err = nullptr;
+    SDM_TRY(status_word(&err));
+    cudaError_t e = sdm::launch_head_mix(z, W_o, out, static_cast<int64_t>(M), d_model, static_cast<int>(K), err,
+                                         reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "head_mix launch");
     return ok();
 }
 

@@ -13,6 +13,9 @@ namespace sdm {
 // ctas_per_sm: 8 fills the SMs (the copy alone); fewer leave room for kernels running beside it.
 cudaError_t launch_init_memory(const void* M0, void* mem, int64_t bytes_per_seq, int B, cudaStream_t stream,
                                int ctas_per_sm = 8);
+// The same broadcast through the bulk-copy engine (one thread per SM; bytes_per_seq a multiple
+// of 16, both pointers 16-byte aligned); a bounded wait that runs out sets ERR_TIMEOUT.
+cudaError_t launch_init_bulk(const void* M0, void* mem, int64_t bytes_per_seq, int B, int* err, cudaStream_t stream);
 
 // ---------------------------------------------------------------- K-ADDR
 // "which" 0 = read side (q with P_q -> idx_r, w_r), 1 = write side (k with P_k -> idx_w, w_w).
@@ -134,6 +137,14 @@ cudaError_t launch_lazy_bitmap(const int32_t* firstw, uint32_t* touched, int64_t
 // Gate preparation and output epilogue (k_gates.cu).  dtype 0 = fp32, 1 = bf16 storage.
 cudaError_t launch_gates(int dtype, const void* x, const void* W_a, const void* W_b, const float* b_dt, const float* A,
                          void* alpha, void* beta, int B, int T, int H, int d, cudaStream_t stream);
+// Tensor-core forms (k_gemm.cu, bf16 only).  Gates: alpha, beta as launch_gates, for H in
+// {16, 32} and d % 8 == 0.  Head mix: out [M, N] = z [M, K] W_o^T with W_o [N, K], N % 32 == 0,
+// K % 8 == 0.  A bounded wait that runs out sets ERR_TIMEOUT in err.
+bool gates_tc_supported(int dtype, int H, int d);
+cudaError_t launch_gates_tc(const void* x, const void* W_a, const void* W_b, const float* b_dt, const float* A,
+                            void* alpha, void* beta, int B, int T, int H, int d, int* err, cudaStream_t stream);
+cudaError_t launch_head_mix(const void* z, const void* W_o, void* out, int64_t M, int N, int K, int* err,
+                            cudaStream_t stream);
 cudaError_t launch_norm_gate(int dtype, const void* y, const void* g, const float* gamma, float eps, void* z, int B, int H,
                              int T, int dv, cudaStream_t stream);
 // Access diagnostics (k_stats.cu): bits = 2 * chains * ceil(N/32) words of scratch; out =

@@ -872,16 +872,27 @@ _GATE_CFGS = {
                                   dtype="bf16", seed=55, alpha_mu=3.0),
     "dv256_f32": synth.SdmConfig("dv256f", B=1, H=3, T=50, d_k=32, d_v=256, N=1024, k_write=8, k_read=8,
                                  dtype="f32", seed=56, alpha_mu=3.0),
+    "h16_bf16": synth.SdmConfig("h16", B=2, H=16, T=300, d_k=32, d_v=128, N=1024, k_write=8, k_read=8,
+                                dtype="bf16", seed=57, alpha_mu=3.0),
 }
 
 
+def _dot_bound_constant(d: int, tensor_cores: bool) -> float:
+    """Relative bound c of an fp32 dot product of length d against sum |w x|: the classical
+    (d + 2) 2^-24 for sequential fused multiply-adds; for the tensor cores (bf16 products
+    exact in fp32, summed in blocks of 16 into the accumulator) 18 ceil(d / 16) 2^-23, the
+    blocked-accumulation bound of the score kernel."""
+    return 18 * -(-d // 16) * 2.0 ** -23 if tensor_cores else (d + 2) * 2.0 ** -24
+
+
 @pytest.mark.gpu
-@pytest.mark.parametrize("name", ["tiny_fp32", "small_bf16", "h32_bf16"])
+@pytest.mark.parametrize("name", ["tiny_fp32", "small_bf16", "h32_bf16", "h16_bf16"])
 def test_gates_match_the_oracle(sdm, name):
     """sdm_gates against the oracle's gates of the same inputs.  Tolerance from the arithmetic:
-    the fp32 dot products are within (d+2) 2^-24 sum|W x| of the exact ones (gamma_d bound);
-    alpha moves by at most alpha A sigmoid(z) |dz|, beta by beta (1 - beta) |dz|; expf and
-    log1pf add a few ulps; storage rounding may flip one ulp."""
+    the fp32 dot products are within c sum|W x| of the exact ones (``_dot_bound_constant``: the
+    gamma_d bound for fused multiply-adds, the blocked bound on the tensor cores); alpha moves
+    by at most alpha A sigmoid(z) |dz|, beta by beta (1 - beta) |dz|; expf and log1pf add a few
+    ulps; storage rounding may flip one ulp.  h16_bf16 and h32_bf16 take the tensor cores."""
     from synth.gen import layer_inputs
     cfg = _GATE_CFGS[name]
     li = layer_inputs(cfg)
@@ -895,6 +906,10 @@ def test_gates_match_the_oracle(sdm, name):
     beta = torch.empty_like(alpha)
     sdm.gates(G.shape_of(cfg), d, x, Wa, Wb, b_dt, A, alpha, beta)
     torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    tc = sdm.gates_tensor_cores(G.shape_of(cfg), d)
+    assert tc == (name in ("h16_bf16", "h32_bf16"))
+    c = _dot_bound_constant(d, tc)
     ga, gb = G.host(alpha, cfg.dtype), G.host(beta, cfg.dtype)
     f = lambda a: O.to_f64(a, cfg.dtype)
     X, WA, WB = f(li["x"]), f(li["W_a"]), f(li["W_b"])
@@ -903,8 +918,8 @@ def test_gates_match_the_oracle(sdm, name):
         ra, rb = O.gates(X[b], WA, bf, Af, WB)                      # [H, T]
         za = X[b] @ WA.T + bf[None, :]
         zb = X[b] @ WB.T
-        dza = ((d + 2) * 2.0 ** -24 * (np.abs(X[b]) @ np.abs(WA).T) + 2.0 ** -24 * np.abs(za)).T
-        dzb = ((d + 2) * 2.0 ** -24 * (np.abs(X[b]) @ np.abs(WB).T)).T
+        dza = (c * (np.abs(X[b]) @ np.abs(WA).T) + 2.0 ** -24 * np.abs(za)).T
+        dzb = (c * (np.abs(X[b]) @ np.abs(WB).T)).T
         sig = lambda z: 1 / (1 + np.exp(-z))
         tol_a = ra * Af[:, None] * sig(za.T) * dza + 8 * 2.0 ** -24 * (1 + Af[:, None]) * ra + _storage_ulp(ra, cfg.dtype)
         tol_b = rb * (1 - rb) * dzb + 8 * 2.0 ** -24 * rb + _storage_ulp(rb, cfg.dtype)
@@ -942,6 +957,34 @@ def test_norm_gate_matches_the_oracle(sdm, name):
             tol = (cfg.d_v / 2 + 6) * 2.0 ** -24 * np.abs(ref) + _storage_ulp(ref, cfg.dtype)
             err = np.abs(got[b, :, h] - O.round_storage(ref, cfg.dtype))
             assert np.all(err <= tol), (b, h, float(err.max()))
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("B,H,T,dv,d_model", [(2, 16, 300, 128, 2048), (1, 3, 77, 40, 96), (1, 2, 128, 64, 32)])
+def test_head_mix_matches_the_oracle(sdm, B, H, T, dv, d_model):
+    """sdm_head_mix (tensor cores) against the oracle's head mixing of the same z and W_o, element
+    by element: |out - R(o)| <= c sum_k |z_k W_nk| + one bf16 ulp of o, c the blocked-accumulation
+    constant of K = H d_v.  Shapes: the layer's (ragged last row tile: 600 rows), K = 120 (not a
+    multiple of the 64-element K-block: zero-filled tail) with a partial column tile (96 < 256),
+    and a single 32-column output."""
+    rng = np.random.default_rng(92 + H)
+    K = H * dv
+    Z = O.round_storage(rng.standard_normal((B, T, H, dv)), "bf16")
+    W = O.round_storage(rng.standard_normal((d_model, K)) / np.sqrt(K), "bf16")
+    st = lambda x: to_torch(O.to_bf16_bits(x), "bf16")
+    out = torch.empty((B * T, d_model), dtype=torch.bfloat16, device="cuda")
+    shape = sdm.SdmShape.make(B, H, T, 32, dv, 1024, 8, 8, "bf16")
+    sdm.head_mix(shape, d_model, st(Z.reshape(B * T, K)), st(W), out)
+    torch.cuda.synchronize()
+    assert sdm.device_status() == 0
+    got = O.to_f64(G.host(out, "bf16"), "bf16")
+    for b in range(B):
+        ref = O.head_mix(np.transpose(Z[b], (1, 0, 2)), W)                  # [T, d_model]
+        bound = _dot_bound_constant(K, True) * (np.abs(Z[b].reshape(T, K)) @ np.abs(W).T)
+        err = np.abs(got[b * T:(b + 1) * T] - O.round_storage(ref, "bf16"))
+        assert np.all(err <= bound + _storage_ulp(ref, "bf16")), (b, float((err - bound).max()))
+        # most outputs round to the float64 result's bf16 value
+        assert np.mean(err == 0) > 0.9
 
 
 # ------------------------------------------------------------------ access diagnostics
