@@ -40,8 +40,8 @@ UNIT = "tokens/s"
 # DRAM bytes per token-head moved by the recurrence phase (hazard pass + recurrence), from an
 # ncu capture of dram__bytes_read.sum + dram__bytes_write.sum of the hazard pass and the
 # recurrence on the layer_1p4b workload itself (profiles/recurrence_layer_1p4b.md):
-# (134.24 MB + 38.05 MB) + (10.45 GB + 4.35 GB) over 524,288 token-heads.
-RECUR_DRAM_BYTES_PER_TOKEN_HEAD = (134.24e6 + 38.05e6 + 10.45e9 + 4.35e9) / 524288
+# (134.40 MB + 39.86 MB) + (10.37 GB + 4.35 GB) over 524,288 token-heads.
+RECUR_DRAM_BYTES_PER_TOKEN_HEAD = (134.40e6 + 39.86e6 + 10.37e9 + 4.35e9) / 524288
 
 
 def _peaks():

@@ -19,7 +19,11 @@ namespace sdm {
 // strictly ascending within each token (checked: status bit 1).
 //
 // One CTA per (chain, tile of `tile` tokens).  The window's lists are staged in shared memory
-// (write lists [u][kw], read lists [u][kr], u = token - w0); a table entry is 16 bits,
+// (write lists [u][kw], read lists [u][kr], u = token - w0).  A first pass marks every
+// entry's 16-bit hash bucket in a `seen` bitmap and the buckets met twice in a `dup` bitmap;
+// only entries of `dup` buckets can take part in a hazard (a slot met once in the window has
+// none), so only they go into the table and only their accesses probe it -- a few percent at
+// random addressing, which keeps most lookups to one bit test.  A table entry is 16 bits,
 // 1 + (u << 7 | q) with q the position in the token's write list (q < kw) or kw + the position
 // in its read list, 0 marking an empty entry; the slot an entry stands for is read back from
 // the staged lists.  Entries go in with a shared-memory compare-and-swap by linear probing; a
@@ -29,6 +33,8 @@ namespace sdm {
 constexpr int HZ_THREADS = 256;
 constexpr int HZ_WARPS = HZ_THREADS / 32;
 constexpr size_t HZ_SMEM_TARGET = 64 * 1024;       // shared bytes per CTA aimed for
+constexpr int HZ_BUCKET_BITS = 16;                  // hash buckets of the seen / dup bitmaps
+constexpr int HZ_BITMAP_WORDS = (1 << HZ_BUCKET_BITS) / 32;
 
 __host__ __device__ inline int hz_table_log2(int tile, int la, int kw, int kr) {
     const int entries = (tile + la) * (kw + kr);
@@ -37,9 +43,11 @@ __host__ __device__ inline int hz_table_log2(int tile, int la, int kw, int kr) {
     return lg;
 }
 
-// Shared memory of a CTA: the table (16-bit entries), then the window's slot lists as int32.
+// Shared memory of a CTA: the table (16-bit entries), the seen and dup bitmaps, then the
+// window's slot lists as int32.
 __host__ __device__ inline size_t hz_smem_bytes(int tile, int la, int kw, int kr) {
-    return (static_cast<size_t>(2) << hz_table_log2(tile, la, kw, kr)) + static_cast<size_t>(tile + la) * (kw + kr) * 4;
+    return (static_cast<size_t>(2) << hz_table_log2(tile, la, kw, kr)) + 2 * HZ_BITMAP_WORDS * 4 +
+           static_cast<size_t>(tile + la) * (kw + kr) * 4;
 }
 
 // Largest tile (64, 32 or 16 tokens) whose shared memory fits the target size.
@@ -50,6 +58,7 @@ int hz_tile(int la, int kw, int kr) {
 }
 
 __device__ __forceinline__ uint32_t hz_hash(uint32_t s, int lg) { return (s * 0x9E3779B1u) >> (32 - lg); }
+__device__ __forceinline__ uint32_t hz_bucket(uint32_t s) { return ((s ^ (s >> 15)) * 0x85EBCA6Bu) >> (32 - HZ_BUCKET_BITS); }
 
 __global__ void __launch_bounds__(HZ_THREADS, 1) k_hazard(const RecArgs a, int LA, int kmax, int tile, int32_t* hz,
                                                        const int32_t* __restrict__ firstw) {
@@ -65,7 +74,9 @@ __global__ void __launch_bounds__(HZ_THREADS, 1) k_hazard(const RecArgs a, int L
     const int nu = t1 - w0;                                 // window tokens (<= 94 < 128)
     const int64_t tokbase = chain * a.T;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    int32_t* sw = reinterpret_cast<int32_t*>(tab + (mask + 1));     // [nu][kw]
+    uint32_t* seen = reinterpret_cast<uint32_t*>(tab + (mask + 1));  // [HZ_BITMAP_WORDS]
+    uint32_t* dup = seen + HZ_BITMAP_WORDS;                          // [HZ_BITMAP_WORDS]
+    int32_t* sw = reinterpret_cast<int32_t*>(dup + HZ_BITMAP_WORDS); // [nu][kw]
     int32_t* sr = sw + nu * kw;                                      // [nu][kr]
 
     // stage the lists (contiguous per chain: one block of each), clear the table
@@ -81,14 +92,26 @@ __global__ void __launch_bounds__(HZ_THREADS, 1) k_hazard(const RecArgs a, int L
             for (int i = threadIdx.x; i < nw; i += HZ_THREADS) sw[i] = __ldg(gw + i);
             for (int i = threadIdx.x; i < nr; i += HZ_THREADS) sr[i] = __ldg(gr + i);
         }
-        for (int i = threadIdx.x; i < static_cast<int>((mask + 1) / 8); i += HZ_THREADS)
-            reinterpret_cast<uint4*>(tab)[i] = make_uint4(0u, 0u, 0u, 0u);
+        // table and both bitmaps are contiguous: (mask + 1) * 2 + 2 * HZ_BITMAP_WORDS * 4 bytes
+        const int nclr = static_cast<int>(((mask + 1) * 2 + 2 * HZ_BITMAP_WORDS * 4) / 16);
+        for (int i = threadIdx.x; i < nclr; i += HZ_THREADS) reinterpret_cast<uint4*>(tab)[i] = make_uint4(0u, 0u, 0u, 0u);
     }
     __syncthreads();
-    // insert the write and read entries of tokens [w0, t1): warp per token, lane per position
+    // mark the buckets of the window's entries: seen once, then dup
+    for (int uo = warp; uo < nu; uo += HZ_WARPS) {
+        for (int q = lane; q < kk; q += 32) {
+            const uint32_t hb = hz_bucket(static_cast<uint32_t>(q < kw ? sw[uo * kw + q] : sr[uo * kr + (q - kw)]));
+            const uint32_t bit = 1u << (hb & 31);
+            if (atomicOr(seen + (hb >> 5), bit) & bit) atomicOr(dup + (hb >> 5), bit);
+        }
+    }
+    __syncthreads();
+    // insert the entries of dup buckets of tokens [w0, t1): warp per token, lane per position
     for (int uo = warp; uo < nu; uo += HZ_WARPS) {
         for (int q = lane; q < kk; q += 32) {
             const int32_t s = q < kw ? sw[uo * kw + q] : sr[uo * kr + (q - kw)];
+            const uint32_t hb = hz_bucket(static_cast<uint32_t>(s));
+            if (!(dup[hb >> 5] & (1u << (hb & 31)))) continue;
             const unsigned short en = static_cast<unsigned short>(1 + ((uo << 7) | q));
             uint32_t h = hz_hash(static_cast<uint32_t>(s), lg);
             for (uint32_t probe = 0; probe <= mask; ++probe) {      // the table is never full
@@ -114,8 +137,10 @@ __global__ void __launch_bounds__(HZ_THREADS, 1) k_hazard(const RecArgs a, int L
                 if (n > 0 && lst[n - 1] >= s) unsorted = true;
                 const int hi = side ? t : t - 1;                     // writers u in [t - LA, hi]
                 int best_w = -1, best_n = 0, best_r = -1;
+                const uint32_t hb = hz_bucket(static_cast<uint32_t>(s));
+                const bool maybe = (dup[hb >> 5] >> (hb & 31)) & 1u;
                 uint32_t h = hz_hash(static_cast<uint32_t>(s), lg);
-                for (uint32_t probe = 0; probe <= mask; ++probe) {
+                for (uint32_t probe = 0; maybe && probe <= mask; ++probe) {
                     const int en = tab[h];
                     if (en == 0) break;
                     const int uo = (en - 1) >> 7, q = (en - 1) & 127;

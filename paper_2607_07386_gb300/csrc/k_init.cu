@@ -1,7 +1,10 @@
 // K-INIT: broadcast of the learned initial memory (Sec. 3.1, "Learned Initial State M0").
 //   mem[b, h, :, :] = M0[h, :, :] for every sequence b.
-// Pure bandwidth: M0 is read once (streaming, evict-first) and each 16-byte vector is
-// written B times.  Roofline: (1 + B) * H * N * d_v * elem_bytes bytes of HBM traffic.
+// Pure bandwidth: M0 is read once and each byte is written B times.  Roofline:
+// (1 + B) * H * N * d_v * elem_bytes bytes of HBM traffic.  Two forms: k_init_memory, a
+// grid-stride copy by SM threads (sdm_init_memory, the copy alone), and k_init_bulk, a copy
+// driven through the bulk-copy engine by one thread per SM (sdm_forward_m0, the copy beside
+// the addressing).
 #include "sdm_internal.h"
 
 namespace sdm {

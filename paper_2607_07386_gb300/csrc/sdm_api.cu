@@ -67,7 +67,6 @@ struct SideStream {
     cudaEvent_t fork = nullptr, join = nullptr;
 };
 SideStream g_side[kMaxDevices];
-constexpr int kCopyCtasPerSm = 1;     // M0 copy CTAs per SM beside the addressing
 std::mutex g_side_mutex[kMaxDevices];
 
 sdm_status side_stream(int* dev_out, SideStream** out) {
@@ -313,10 +312,10 @@ sdm_status forward_impl(const char* who, const sdm_shape* s, const void* P_q, co
     SDM_TRY(status_word(&err));
     if (run_recurrence && M0 != nullptr) {
         // mem = M0 broadcast on the side stream, running beside the addressing (independent
-        // data) and joined back before the recurrence.  Two CTAs per SM leave room for the
-        // addressing kernels.  (Started after the score kernel instead, beside the finalize
-        // passes, it measured slower: the copy's traffic slows whichever kernel it shares
-        // the SMs with, and the finalize more than the tensor-core kernel.)
+        // data) and joined back before the recurrence.  The copy goes through the bulk-copy
+        // engine from one thread per SM, so it takes almost nothing from the addressing
+        // kernels (an SM-thread copy with one 256-thread CTA per SM measured 0.34 ms slower
+        // per step at layer_1p4b; with more CTAs per SM, slower still).
         int dev = 0;
         SideStream* ss = nullptr;
         SDM_TRY(side_stream(&dev, &ss));
@@ -324,8 +323,8 @@ sdm_status forward_impl(const char* who, const sdm_shape* s, const void* P_q, co
         cudaError_t e = cudaEventRecord(ss->fork, stream);
         if (e == cudaSuccess) e = cudaStreamWaitEvent(ss->stream, ss->fork, 0);
         if (e == cudaSuccess)
-            e = sdm::launch_init_memory(M0, mem, static_cast<int64_t>(static_cast<size_t>(s->H) * s->N * rowb), s->B,
-                                        ss->stream, kCopyCtasPerSm);
+            e = sdm::launch_init_bulk(M0, mem, static_cast<int64_t>(static_cast<size_t>(s->H) * s->N * rowb), s->B,
+                                      err, ss->stream);
         if (e == cudaSuccess) e = cudaEventRecord(ss->join, ss->stream);
         if (e != cudaSuccess) return cuda_fail(e, "M0 broadcast on the side stream");
         SDM_TRY(run_address(s, S, L, P_q, P_k, q, k, iw, ww, ir, wr, ws, err, stream));
