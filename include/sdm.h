@@ -273,9 +273,10 @@ sdm_status sdm_recur_undo(const sdm_shape* shape, const int32_t* idx_w, const fl
  * dtype.  Outputs (float32, written): dv [B, H, T, d_v], dalpha, dbeta [B, H, T], dw_w
  * [B, H, T, k_write], dw_r [B, H, T, k_read]; dM [B, H, N, d_v] float32 must be zero on
  * entry and receives dL/dM_0 per sequence (sum over b for a shared M0).  Other arguments as
- * in sdm_recur.  d_v must be a multiple of 32, at most 256.  Outputs must not overlap each
- * other or the inputs.  Slot lists must be strictly ascending, as in sdm_recur; a violation
- * sets bit 1 of the device status word. */
+ * in sdm_recur.  d_v must be a multiple of 32, at most 256; k_write and k_read at most 32
+ * (SDM_ERR_UNSUPPORTED otherwise).  Outputs must not overlap each other or the inputs.  Slot
+ * lists must be strictly ascending, as in sdm_recur; a violation sets bit 1 of the device
+ * status word. */
 sdm_status sdm_recur_backward(const sdm_shape* shape, const int32_t* idx_w, const float* w_w,
                               const int32_t* idx_r, const float* w_r, const void* v,
                               const void* alpha, const void* beta, void* mem, const void* undo,

@@ -57,12 +57,17 @@ size_t rec_workspace_bytes(int B, int H, int T, int kw, int kr) {
     return static_cast<size_t>(B) * H * T * kmax * sizeof(int32_t);
 }
 
-cudaError_t launch_recur(int dtype, const RecArgs& a_in, int32_t* hz_ws, cudaStream_t stream, const int32_t* firstw) {
+cudaError_t launch_recur(int dtype, const RecArgs& a_in, int32_t* hz_ws, cudaStream_t stream, const int32_t* firstw,
+                         cudaEvent_t mem_ready) {
     RecArgs a = a_in;
     a.firstw = a.M0 ? firstw : nullptr;
     const RecPlan p = rec_plan(dtype, a.B, a.H, a.T, a.dv, a.kw, a.kr);
     if (p.w > 0) {                 // one token per chain needs no hazard table
         cudaError_t e = launch_hazard(a, p.la, p.kmax, hz_ws, stream, a.firstw);
+        if (e != cudaSuccess) return e;
+    }
+    if (mem_ready != nullptr) {    // the hazard pass reads no memory rows: only the recurrence waits
+        cudaError_t e = cudaStreamWaitEvent(stream, mem_ready, 0);
         if (e != cudaSuccess) return e;
     }
     auto al16 = [](const void* q) { return (reinterpret_cast<uintptr_t>(q) & 15) == 0; };

@@ -20,31 +20,15 @@
 // s = max|row| / top (448 for e4m3, 7 for int4) and codes round(row / s), all in float32 with
 // correctly rounded operations; the backward then takes the logged row as the stored value of
 // q * s (rounded to the storage type), for the chain rule and for the undo alike.
-// One warp per (b, h) chain; lane l holds elements l, l + 32, ... of every row.  Plain loads
-// and stores only: no asynchronous copies and no waits.  The forward kernels' prefetch
-// machinery is the next step for this one.
+// Layout of the work: see k_recur_bwd below (one CTA per chain, one warp per 32-element slice
+// of d_v).  Plain loads and stores, no waits.
 #include "sdm_internal.h"
 
 #include <cuda_fp8.h>
 
 namespace sdm {
 
-constexpr int BW_WARPS = 4;
-constexpr int BW_MAXE = 8;          // d_v <= 256
-
-__device__ __forceinline__ float warp_sum(float x) {
-#pragma unroll
-    for (int off = 16; off > 0; off >>= 1) x += __shfl_xor_sync(0xffffffffu, x, off);
-    return x;
-}
-
-template <class D> __device__ __forceinline__ void copy_elem(void* dst, const void* src, int64_t i);
-template <> __device__ __forceinline__ void copy_elem<F32>(void* dst, const void* src, int64_t i) {
-    reinterpret_cast<float*>(dst)[i] = reinterpret_cast<const float*>(src)[i];
-}
-template <> __device__ __forceinline__ void copy_elem<BF16>(void* dst, const void* src, int64_t i) {
-    reinterpret_cast<unsigned short*>(dst)[i] = reinterpret_cast<const unsigned short*>(src)[i];
-}
+constexpr int BW_MAXE = 8;          // d_v <= 256: elements per lane in the one-warp-per-row passes
 
 // The undo log as the backward reads it: Q = 0 the stored rows themselves; Q = 1 fp8 (e4m3)
 // codes, one byte per element; Q = 2 int4 codes, two per byte (element 2i in the low nibble),
@@ -135,118 +119,148 @@ template <> __device__ __forceinline__ void store_elem<BF16>(void* dst, int64_t 
     reinterpret_cast<__nv_bfloat16*>(dst)[i] = __float2bfloat16_rn(x);
 }
 
+// One CTA per (b, h) chain, one warp per 32-element slice of d_v (lane l of warp w holds
+// element 32 w + l of every row).  Every per-element quantity of the chain rule (the rows of M,
+// of G and of the log, pred, delta, d delta, d r) stays in its lane, so the slices walk the
+// tokens independently; only the dot products over d_v (d rho, <G_i, delta>, <r_i, d delta>,
+// <d r_i, M_{t-1}[i]>) need the slices together.  Each warp reduces its 32 lanes' terms of the
+// k_r + 2 k_w products with one butterfly reduce-scatter (lane n ends with the slice's share
+// of product n), writes the shares to shared memory, and after one barrier per token warp 0
+// adds the slices' shares in slice order and writes dw_r, dw_w, dalpha, dbeta (double-buffered
+// by token parity, so one barrier per token suffices).  Row loads of a phase are issued
+// together (32 independent loads per lane) before any is used.
+constexpr int BW_K = 32;           // slots per list handled by the register batches (k <= 32)
+
+// Butterfly reduce-scatter of 32 per-lane vectors x[0..31] over the warp: afterwards lane n
+// holds sum over lanes of x[n] in x[0].
+__device__ __forceinline__ void reduce_scatter32(float (&x)[32], int lane) {
+#pragma unroll
+    for (int lvl = 0; lvl < 5; ++lvl) {
+        const int half = 16 >> lvl;              // values kept after this level: half
+        const bool upper = (lane >> (4 - lvl)) & 1;
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            if (i < half) {
+                const float send = upper ? x[i] : x[i + half];
+                const float keep = upper ? x[i + half] : x[i];
+                x[i] = keep + __shfl_xor_sync(0xffffffffu, send, 16 >> lvl);
+            }
+        }
+    }
+}
+
 template <class D, int Q>
-__global__ void __launch_bounds__(32 * BW_WARPS) k_recur_bwd(const RecArgs a, const UndoLog undo,
-                                                             const void* __restrict__ dy, float* __restrict__ dv_o,
-                                                             float* __restrict__ dalpha, float* __restrict__ dbeta,
-                                                             float* __restrict__ dw_w, float* __restrict__ dw_r,
-                                                             float* __restrict__ dM) {
-    const int lane = threadIdx.x & 31;
-    const int64_t chain = static_cast<int64_t>(blockIdx.x) * BW_WARPS + (threadIdx.x >> 5);
-    if (chain >= static_cast<int64_t>(a.B) * a.H) return;              // whole warps
+__global__ void __launch_bounds__(32 * 8) k_recur_bwd(const RecArgs a, const UndoLog undo,
+                                                      const void* __restrict__ dy, float* __restrict__ dv_o,
+                                                      float* __restrict__ dalpha, float* __restrict__ dbeta,
+                                                      float* __restrict__ dw_w, float* __restrict__ dw_r,
+                                                      float* __restrict__ dM) {
+    // shares [parity][slice][3 * BW_K + 1]: d rho (k_r), <G, delta> (k_w), <r, dd> (k_w), d alpha
+    __shared__ float sh[2][8][3 * BW_K + 1];
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nsl = blockDim.x >> 5;
+    const int64_t chain = blockIdx.x;
     const int dv = a.dv, T = a.T, kw = a.kw, kr = a.kr;
-    const int epl = dv / 32;                                             // elements per lane
+    const int e = w * 32 + lane;                                         // this lane's element
     const uint32_t N = static_cast<uint32_t>(a.N);
-    const int64_t mbase = chain * a.N * dv;                              // element offset of the chain's memory
+    const int64_t mbase = chain * a.N * dv;
     float* G = dM + mbase;
+    char* memc = static_cast<char*>(a.mem) + mbase * D::BYTES;
     bool bad = false, unsorted = false;
-    for (int t = T - 1; t >= 0; --t) {
+    for (int t = T - 1, par = 0; t >= 0; --t, par ^= 1) {
         const int64_t tok = chain * T + t;
         const float alpha = load_elem<D>(a.alpha, tok), beta = load_elem<D>(a.beta, tok);
-        float gy[BW_MAXE];
-#pragma unroll
-        for (int j = 0; j < BW_MAXE; ++j) gy[j] = j < epl ? load_elem<D>(dy, tok * dv + lane + 32 * j) : 0.f;
-        // ---- read of the post-write memory M_t
-        for (int n = 0; n < kr; ++n) {
-            const int32_t s = __ldg(a.idx_r + tok * kr + n);
-            unsorted |= n > 0 && __ldg(a.idx_r + tok * kr + n - 1) >= s;
-            if (static_cast<uint32_t>(s) >= N) { bad = true; continue; }   // warp-uniform
-            const float rho = __ldg(a.w_r + tok * kr + n);
-            const int64_t row = mbase + static_cast<int64_t>(s) * dv;
-            float p = 0.f;
-#pragma unroll
-            for (int j = 0; j < BW_MAXE; ++j) {
-                if (j < epl) {
-                    const int64_t e = static_cast<int64_t>(s) * dv + lane + 32 * j;
-                    p = fmaf(gy[j], load_elem<D>(a.mem, row + lane + 32 * j), p);
-                    G[e] = fmaf(rho, gy[j], G[e]);
-                }
-            }
-            p = warp_sum(p);
-            if (lane == 0) dw_r[tok * kr + n] = p;
+        const float gy = load_elem<D>(dy, tok * dv + e);
+        const float vt = load_elem<D>(a.v, tok * dv + e);
+        // lists: lane n holds entry n
+        const int32_t ir_l = lane < kr ? __ldg(a.idx_r + tok * kr + lane) : 0;
+        const float wr_l = lane < kr ? __ldg(a.w_r + tok * kr + lane) : 0.f;
+        const int32_t iw_l = lane < kw ? __ldg(a.idx_w + tok * kw + lane) : 0;
+        const float ww_l = lane < kw ? __ldg(a.w_w + tok * kw + lane) : 0.f;
+        {
+            const int32_t pr = __shfl_up_sync(0xffffffffu, ir_l, 1), pw = __shfl_up_sync(0xffffffffu, iw_l, 1);
+            unsorted |= (lane > 0 && lane < kr && pr >= ir_l) || (lane > 0 && lane < kw && pw >= iw_l);
+            bad |= (lane < kr && static_cast<uint32_t>(ir_l) >= N) || (lane < kw && static_cast<uint32_t>(iw_l) >= N);
         }
+        // ---- read of the post-write memory M_t: d rho_n = <dy, M_t[r_n]>, G[r_n] += rho_n dy
+        float x[32];
+#pragma unroll
+        for (int n = 0; n < BW_K; ++n) {
+            const int32_t sn = __shfl_sync(0xffffffffu, ir_l, n);
+            const bool ok = n < kr && static_cast<uint32_t>(sn) < N;
+            x[n] = ok ? load_elem<D>(memc, static_cast<int64_t>(sn) * dv + e) : 0.f;
+        }
+        float gr[32];
+#pragma unroll
+        for (int n = 0; n < BW_K; ++n) {
+            const int32_t sn = __shfl_sync(0xffffffffu, ir_l, n);
+            gr[n] = (n < kr && static_cast<uint32_t>(sn) < N) ? G[static_cast<int64_t>(sn) * dv + e] : 0.f;
+        }
+#pragma unroll
+        for (int n = 0; n < BW_K; ++n) {
+            const int32_t sn = __shfl_sync(0xffffffffu, ir_l, n);
+            const float rho = __shfl_sync(0xffffffffu, wr_l, n);
+            if (n < kr && static_cast<uint32_t>(sn) < N) G[static_cast<int64_t>(sn) * dv + e] = fmaf(rho, gy, gr[n]);
+            x[n] *= gy;
+        }
+        reduce_scatter32(x, lane);
+        sh[par][w][lane] = x[0];                                          // share of d rho_lane
         // ---- the write: prediction and delta from the logged rows, d delta from the adjoint
-        float vt[BW_MAXE], pred[BW_MAXE], dd[BW_MAXE];
+        float pv[32], gv[32];
 #pragma unroll
-        for (int j = 0; j < BW_MAXE; ++j) {
-            vt[j] = j < epl ? load_elem<D>(a.v, tok * dv + lane + 32 * j) : 0.f;
-            pred[j] = 0.f;
-            dd[j] = 0.f;
+        for (int m = 0; m < BW_K; ++m) {
+            const int32_t im = __shfl_sync(0xffffffffu, iw_l, m);
+            const bool ok = m < kw && static_cast<uint32_t>(im) < N;
+            pv[m] = ok ? undo_elem<D, Q>(undo, tok * kw + m, dv, e) : 0.f;
+            gv[m] = ok ? G[static_cast<int64_t>(im) * dv + e] : 0.f;
         }
-        for (int m = 0; m < kw; ++m) {
-            const int32_t i = __ldg(a.idx_w + tok * kw + m);
-            // the write slots of a token must be distinct: checked as strictly ascending
-            unsorted |= m > 0 && __ldg(a.idx_w + tok * kw + m - 1) >= i;
-            if (static_cast<uint32_t>(i) >= N) continue;                // no write, no log entry
-            const float w = __ldg(a.w_w + tok * kw + m);
-            const int64_t urow = tok * kw + m;
+        float pred = 0.f, dd = 0.f;
 #pragma unroll
-            for (int j = 0; j < BW_MAXE; ++j) {
-                if (j < epl) {
-                    pred[j] = fmaf(w, alpha * undo_elem<D, Q>(undo, urow, dv, lane + 32 * j), pred[j]);
-                    dd[j] = fmaf(w, G[static_cast<int64_t>(i) * dv + lane + 32 * j], dd[j]);
-                }
+        for (int m = 0; m < BW_K; ++m) {
+            const float wm = __shfl_sync(0xffffffffu, ww_l, m);
+            pred = fmaf(wm, alpha * pv[m], pred);
+            dd = fmaf(wm, gv[m], dd);
+        }
+        const float delta = vt - pred;
+        dd *= beta;
+        dv_o[tok * dv + e] = dd;
+        float gd[32], rd[32], da = 0.f;
+#pragma unroll
+        for (int m = 0; m < BW_K; ++m) {
+            const int32_t im = __shfl_sync(0xffffffffu, iw_l, m);
+            const float wm = __shfl_sync(0xffffffffu, ww_l, m);
+            const bool ok = m < kw && static_cast<uint32_t>(im) < N;
+            gd[m] = gv[m] * delta;
+            rd[m] = alpha * pv[m] * dd;
+            const float dr = gv[m] - wm * dd;
+            da = fmaf(dr, pv[m], da);
+            if (ok) {
+                G[static_cast<int64_t>(im) * dv + e] = alpha * dr;
+                store_elem<D>(memc, static_cast<int64_t>(im) * dv + e, pv[m]);     // the undo
             }
         }
-        float delta[BW_MAXE];
+        reduce_scatter32(gd, lane);
+        reduce_scatter32(rd, lane);
 #pragma unroll
-        for (int j = 0; j < BW_MAXE; ++j) {
-            delta[j] = vt[j] - pred[j];
-            dd[j] *= beta;
-            if (j < epl) dv_o[tok * dv + lane + 32 * j] = dd[j];
-        }
-        float db = 0.f, da = 0.f;
-        for (int m = 0; m < kw; ++m) {
-            const int32_t i = __ldg(a.idx_w + tok * kw + m);
-            if (static_cast<uint32_t>(i) >= N) { bad = true; if (lane == 0) dw_w[tok * kw + m] = 0.f; continue; }
-            const float w = __ldg(a.w_w + tok * kw + m);
-            const int64_t urow = tok * kw + m;
-            float gd = 0.f, rd = 0.f;
-#pragma unroll
-            for (int j = 0; j < BW_MAXE; ++j) {
-                if (j < epl) {
-                    const int64_t e = static_cast<int64_t>(i) * dv + lane + 32 * j;
-                    const float prev = undo_elem<D, Q>(undo, urow, dv, lane + 32 * j);
-                    const float gi = G[e];
-                    gd = fmaf(gi, delta[j], gd);
-                    rd = fmaf(alpha * prev, dd[j], rd);
-                    const float dr = gi - w * dd[j];
-                    da = fmaf(dr, prev, da);
-                    G[e] = alpha * dr;
-                }
+        for (int off = 16; off > 0; off >>= 1) da += __shfl_xor_sync(0xffffffffu, da, off);
+        sh[par][w][BW_K + lane] = gd[0];
+        sh[par][w][2 * BW_K + lane] = rd[0];
+        if (lane == 0) sh[par][w][3 * BW_K] = da;
+        __syncthreads();
+        if (w == 0) {
+            float r = 0.f, g = 0.f, q = 0.f, al = 0.f;
+            for (int s2 = 0; s2 < nsl; ++s2) {                         // slices in order
+                r += sh[par][s2][lane];
+                g += sh[par][s2][BW_K + lane];
+                q += sh[par][s2][2 * BW_K + lane];
+                al += sh[par][s2][3 * BW_K];
             }
-            gd = warp_sum(gd);
-            rd = warp_sum(rd);
-            db = fmaf(w, gd, db);
-            if (lane == 0) dw_w[tok * kw + m] = beta * gd - rd;
-        }
-        da = warp_sum(da);
-        if (lane == 0) { dalpha[tok] = da; dbeta[tok] = db; }
-        // ---- undo: M_t -> M_{t-1} on the written rows (after every read of M_t above)
-        for (int m = 0; m < kw; ++m) {
-            const int32_t i = __ldg(a.idx_w + tok * kw + m);
-            if (static_cast<uint32_t>(i) >= N) continue;
-            const int64_t urow = tok * kw + m;
-            char* mrow = static_cast<char*>(a.mem) + (mbase + static_cast<int64_t>(i) * dv) * D::BYTES;
+            if (lane < kr) dw_r[tok * kr + lane] = r;
+            const bool okw = lane < kw && static_cast<uint32_t>(iw_l) < N;
+            if (lane < kw) dw_w[tok * kw + lane] = okw ? beta * g - q : 0.f;
+            float db = okw ? ww_l * g : 0.f;
 #pragma unroll
-            for (int j = 0; j < BW_MAXE; ++j) {
-                if (j < epl) {
-                    if constexpr (Q == 0)
-                        copy_elem<D>(mrow, static_cast<const char*>(undo.rows) + urow * dv * D::BYTES, lane + 32 * j);
-                    else
-                        store_elem<D>(mrow, lane + 32 * j, undo_elem<D, Q>(undo, urow, dv, lane + 32 * j));
-                }
-            }
+            for (int off = 16; off > 0; off >>= 1) db += __shfl_xor_sync(0xffffffffu, db, off);
+            if (lane == 0) { dalpha[tok] = al; dbeta[tok] = db; }
         }
     }
     if (__any_sync(0xffffffffu, bad) && lane == 0) flag_error(a.err, ERR_BAD_INDEX);
@@ -256,10 +270,11 @@ __global__ void __launch_bounds__(32 * BW_WARPS) k_recur_bwd(const RecArgs a, co
 cudaError_t launch_recur_backward(int dtype, const RecArgs& a, int kind, const void* undo, const void* codes,
                                   const float* scales, const void* dy, float* dv, float* dalpha, float* dbeta,
                                   float* dw_w, float* dw_r, float* dM, cudaStream_t stream) {
-    const int64_t chains = static_cast<int64_t>(a.B) * a.H;
-    const unsigned grid = static_cast<unsigned>((chains + BW_WARPS - 1) / BW_WARPS);
+    if (a.kw > BW_K || a.kr > BW_K || a.dv % 32 != 0 || a.dv > 256) return cudaErrorInvalidValue;
+    const unsigned grid = static_cast<unsigned>(static_cast<int64_t>(a.B) * a.H);
+    const int threads = a.dv;                       // one warp per 32-element slice
     const UndoLog u{undo, static_cast<const uint8_t*>(codes), scales};
-#define SDM_BWD(DT, Q) k_recur_bwd<DT, Q><<<grid, 32 * BW_WARPS, 0, stream>>>(a, u, dy, dv, dalpha, dbeta, dw_w, dw_r, dM)
+#define SDM_BWD(DT, Q) k_recur_bwd<DT, Q><<<grid, threads, 0, stream>>>(a, u, dy, dv, dalpha, dbeta, dw_w, dw_r, dM)
     if (dtype == 0) {
         if (kind == 0) SDM_BWD(F32, 0); else if (kind == 1) SDM_BWD(F32, 1); else SDM_BWD(F32, 2);
     } else {

@@ -310,6 +310,8 @@ sdm_status forward_impl(const char* who, const sdm_shape* s, const void* P_q, co
     float* wr = w_r ? w_r : reinterpret_cast<float*>(ws + L.w_r);
     int* err = nullptr;
     SDM_TRY(status_word(&err));
+    std::unique_lock<std::mutex> side_lock;      // held until the recurrence has waited on the join
+    cudaEvent_t mem_ready = nullptr;
     if (run_recurrence && M0 != nullptr) {
         // mem = M0 broadcast on the side stream, running beside the addressing (independent
         // data) and joined back before the recurrence.  The copy goes through the bulk-copy
@@ -319,7 +321,7 @@ sdm_status forward_impl(const char* who, const sdm_shape* s, const void* P_q, co
         int dev = 0;
         SideStream* ss = nullptr;
         SDM_TRY(side_stream(&dev, &ss));
-        std::lock_guard<std::mutex> lock(g_side_mutex[dev]);
+        side_lock = std::unique_lock<std::mutex>(g_side_mutex[dev]);
         cudaError_t e = cudaEventRecord(ss->fork, stream);
         if (e == cudaSuccess) e = cudaStreamWaitEvent(ss->stream, ss->fork, 0);
         if (e == cudaSuccess)
@@ -328,8 +330,7 @@ sdm_status forward_impl(const char* who, const sdm_shape* s, const void* P_q, co
         if (e == cudaSuccess) e = cudaEventRecord(ss->join, ss->stream);
         if (e != cudaSuccess) return cuda_fail(e, "M0 broadcast on the side stream");
         SDM_TRY(run_address(s, S, L, P_q, P_k, q, k, iw, ww, ir, wr, ws, err, stream));
-        e = cudaStreamWaitEvent(stream, ss->join, 0);
-        if (e != cudaSuccess) return cuda_fail(e, "join of the M0 broadcast");
+        mem_ready = ss->join;                     // joined after the hazard pass, before the recurrence
     } else {
         SDM_TRY(run_address(s, S, L, P_q, P_k, q, k, iw, ww, ir, wr, ws, err, stream));
     }
@@ -351,7 +352,7 @@ sdm_status forward_impl(const char* who, const sdm_shape* s, const void* P_q, co
             if (e != cudaSuccess) return cuda_fail(e, "lazy initial memory launch");
             r.M0 = lazy->M0;
         }
-        cudaError_t e = sdm::launch_recur(s->dtype, r, reinterpret_cast<int32_t*>(ws + L.hz), stream, firstw);
+        cudaError_t e = sdm::launch_recur(s->dtype, r, reinterpret_cast<int32_t*>(ws + L.hz), stream, firstw, mem_ready);
         if (e != cudaSuccess) return cuda_fail(e, "recurrence launch");
     }
     return ok();
@@ -689,6 +690,8 @@ sdm_status backward_impl(const char* who, const sdm_shape* s, const int32_t* idx
     SDM_TRY(check_shape(s, false, nullptr));
     if (s->d_v % 32 != 0 || s->d_v > 256)
         return fail(SDM_ERR_UNSUPPORTED, "%s: d_v must be a multiple of 32, at most 256 (d_v=%d)", who, s->d_v);
+    if (s->k_write > 32 || s->k_read > 32)
+        return fail(SDM_ERR_UNSUPPORTED, "%s: k_write and k_read must be at most 32 (%d, %d)", who, s->k_write, s->k_read);
     const size_t es = elem_bytes(s->dtype);
     const size_t bht = static_cast<size_t>(s->B) * s->H * s->T;
     if (bht == 0) return ok();

@@ -110,8 +110,10 @@ size_t rec_workspace_bytes(int B, int H, int T, int kw, int kr);
 // Runs the hazard pass, then the recurrence.  hz_ws: rec_workspace_bytes() of scratch.
 // firstw (lazy initial memory, with a.M0 set): [B*H, N] first writer of each slot in this
 // call (-1: written by an earlier call; INT_MAX: not written), see k_lazy.cu.
+// mem_ready: when given, the stream waits on it after the hazard pass, before the recurrence
+// (the hazard pass reads only the lists, so it can run while mem is still being written).
 cudaError_t launch_recur(int dtype, const RecArgs& a, int32_t* hz_ws, cudaStream_t stream,
-                         const int32_t* firstw = nullptr);
+                         const int32_t* firstw = nullptr, cudaEvent_t mem_ready = nullptr);
 
 // Backward of the recurrence with in-place undo (k_recur_bwd.cu).  a.mem holds M_T on entry and
 // M_0 on return; dM ([B, H, N, dv] fp32, zero on entry) receives dL/dM_0 per chain.  kind 0:
