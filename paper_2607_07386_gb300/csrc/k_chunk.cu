@@ -170,22 +170,47 @@ __global__ void __launch_bounds__(CK_THREADS) k_recur_chunk(const RecArgs a, int
             }
             __syncthreads();
         }
-        // ---- S4: gathers from the chunk-initial memory
-        for (int e = tid; e < n * dv; e += CK_THREADS) {
-            const int t = e / dv, d = e - t * dv;
-            float rv = 0.f, iv = 0.f;
-            for (int m = 0; m < kw; ++m) {
-                const int s = s_iw[t * kw + m];
-                if (static_cast<uint32_t>(s) < N)
-                    rv = fmaf(s_ww[t * kw + m] * __expf(s_lw[t * kw + m]), load_elem<D>(a.mem, (mrow0 + s) * dv + d), rv);
+        // ---- S4: gathers from the chunk-initial memory: one thread per (token, 16-byte piece of
+        //      the row), 16-byte loads, four rows in flight
+        {
+            constexpr int E = D::E;
+            const int npc = dv / E;                                   // 16-byte pieces per row
+            const char* mrows = static_cast<const char*>(a.mem) + mrow0 * dv * D::BYTES;
+            for (int e = tid; e < n * npc; e += CK_THREADS) {
+                const int t = e / npc, c = e - t * npc;
+                float rv[E], iv[E];
+#pragma unroll
+                for (int j = 0; j < E; ++j) { rv[j] = 0.f; iv[j] = 0.f; }
+                auto acc_rows = [&](const int* sl, const float* sw, const float* slam, int k, float (&out)[E]) {
+                    for (int m0 = 0; m0 < k; m0 += 4) {
+                        uint4 raw[4];
+                        float cf[4];
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            const int m = m0 + q;
+                            const int s = m < k ? sl[t * k + m] : -1;
+                            const bool ok = m < k && static_cast<uint32_t>(s) < N;
+                            cf[q] = ok ? sw[t * k + m] * __expf(slam[t * k + m]) : 0.f;
+                            raw[q] = ok ? __ldg(reinterpret_cast<const uint4*>(mrows + (static_cast<int64_t>(s) * dv) * D::BYTES) + c)
+                                        : make_uint4(0u, 0u, 0u, 0u);
+                        }
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            float f[E];
+                            unpack16<D>(raw[q], f);
+#pragma unroll
+                            for (int j = 0; j < E; ++j) out[j] = fmaf(cf[q], f[j], out[j]);
+                        }
+                    }
+                };
+                acc_rows(s_iw, s_ww, s_lw, kw, rv);
+                acc_rows(s_ir, s_wr, s_lr, kr, iv);
+#pragma unroll
+                for (int j = 0; j < E; ++j) {
+                    s_R[t * dv + c * E + j] = rv[j];
+                    s_I[t * dv + c * E + j] = iv[j];
+                }
             }
-            for (int m = 0; m < kr; ++m) {
-                const int s = s_ir[t * kr + m];
-                if (static_cast<uint32_t>(s) < N)
-                    iv = fmaf(s_wr[t * kr + m] * __expf(s_lr[t * kr + m]), load_elem<D>(a.mem, (mrow0 + s) * dv + d), iv);
-            }
-            s_R[e] = rv;
-            s_I[e] = iv;
         }
         __syncthreads();
         // ---- S5: u = dV + B retrieved (in place, rows descending), then y = inter + QK u
