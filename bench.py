@@ -39,7 +39,7 @@ UNIT = "tokens/s"
 
 # DRAM bytes per token-head moved by the recurrence phase (hazard pass + recurrence), from an
 # ncu capture of dram__bytes_read.sum + dram__bytes_write.sum of the hazard pass and the
-# recurrence on the layer_1p4b workload itself (profiles/recurrence_layer_1p4b.md):
+# recurrence on the layer_1p4b workload itself (one launch, one pass per kernel):
 # (134.40 MB + 39.86 MB) + (10.37 GB + 4.35 GB) over 524,288 token-heads.
 RECUR_DRAM_BYTES_PER_TOKEN_HEAD = (134.40e6 + 39.86e6 + 10.37e9 + 4.35e9) / 524288
 
