@@ -189,6 +189,46 @@ def test_backward_entry_points_reject_bad_arguments(sdm):
     assert bw(s, undo=FAKE + 0x10000000) == 1 and "mem overlaps undo" in sdm.last_error()
 
 
+def test_snapshot_entry_points_size_and_reject_bad_arguments(sdm):
+    s = _shape(sdm)
+    L = sdm.lib()
+    rows = 2 * 2 * 16 * 8
+    assert sdm.undo_code_bytes(s, "fp8") == rows * 32 and sdm.undo_code_bytes(s, "int4") == rows * 16
+    assert L.sdm_undo_code_bytes(ctypes.byref(s), 3) == 0
+    q = lambda shape, kind, **o: L.sdm_undo_quantize(ctypes.byref(shape), o.get("undo", FAKE), kind,
+                                                     o.get("codes", FAKE + 0x100000), o.get("scales", FAKE + 0x200000),
+                                                     None)
+    assert q(s, 3) == 1 and "kind" in sdm.last_error()
+    assert q(_shape(sdm, d_v=48), 1) == 2 and "multiple of 32" in sdm.last_error()
+    assert q(s, 1, codes=FAKE + 0x100) == 1 and "overlap" in sdm.last_error()
+    assert q(s, 2, scales=None) == 1 and "scales is NULL" in sdm.last_error()
+    base = [FAKE, FAKE + 0x100000, FAKE + 0x200000, FAKE + 0x300000, FAKE + 0x400000, FAKE + 0x500000,
+            FAKE + 0x600000, FAKE + 0x10000000]
+    outs = [FAKE + 0x20000000 + i * 0x1000000 for i in range(6)]
+    bq = lambda shape, kind, **o: L.sdm_recur_backward_q(ctypes.byref(shape), *base, kind, o.get("codes", FAKE + 0x800000),
+                                                         o.get("scales", FAKE + 0x880000), FAKE + 0x900000, *outs, None)
+    assert bq(s, 0) == 1 and "kind" in sdm.last_error()
+    assert bq(s, 1, scales=None) == 1 and "scales is NULL" in sdm.last_error()
+    assert bq(s, 2, codes=FAKE + 0x10000000) == 1 and "mem overlaps codes" in sdm.last_error()
+    assert bq(_shape(sdm, N=4096, k_write=40), 1) == 2 and "at most 32" in sdm.last_error()
+
+
+def test_head_mix_and_tensor_core_gates_reject_or_route(sdm):
+    L = sdm.lib()
+    s = _shape(sdm, H=16, d_v=128)
+    hm = lambda shape, d_model, **o: L.sdm_head_mix(ctypes.byref(shape), d_model, o.get("z", FAKE),
+                                                    o.get("W_o", FAKE + 0x1000000), o.get("out", FAKE + 0x2000000), None)
+    assert hm(_shape(sdm, H=16, d_v=128, dtype="f32"), 2048) == 2 and "bf16" in sdm.last_error()
+    assert hm(s, 48) == 2 and "multiple of 32" in sdm.last_error()
+    assert hm(s, 2048, out=FAKE + 0x10) == 1 and "out overlaps z" in sdm.last_error()
+    assert hm(s, 2048, W_o=None) == 1 and "W_o is NULL" in sdm.last_error()
+    # the gates take the tensor cores for bf16 storage with H = 16 or 32 and d_model % 8 == 0
+    assert sdm.gates_tensor_cores(s, 2048) and sdm.gates_tensor_cores(_shape(sdm, H=32), 64)
+    assert not sdm.gates_tensor_cores(_shape(sdm, H=8), 64)
+    assert not sdm.gates_tensor_cores(_shape(sdm, H=16, dtype="f32"), 64)
+    assert not sdm.gates_tensor_cores(s, 2044)
+
+
 def test_chunkwise_rejects_bad_chunks_and_rows(sdm):
     s = _shape(sdm)
     L = sdm.lib()
