@@ -1460,7 +1460,9 @@ __global__ void __launch_bounds__(FT_THREADS, 8) k_addr_finalize_thread(const Ad
 // ------------------------------------------------------------------------------------------
 constexpr int BT_THREADS = 32;
 constexpr int BT_BAND = 8;        // band entries re-ranked here; wider bands go to queue B
-__host__ __device__ constexpr int bt_words(int L) { return 4 * L + 2 * (L - 4) + 2 * L + 4 * BT_BAND; }
+// Shared bytes per thread: values, candidates and band scratch as 32-bit words, the half
+// lists' column indices and the heap positions as 16-bit (one column chunk per half: < 512).
+__host__ __device__ constexpr int bt_bytes(int L) { return 4 * (4 * L + (L - 4) + 4 * BT_BAND) + 2 * (2 * L + (L - 4)); }
 
 // f versus e (compensated values): +1 if f is certainly larger, -1 if certainly smaller, 0 if
 // equal with zero bounds (exact values: the caller breaks the tie); sets unsure when the two
@@ -1484,17 +1486,18 @@ __global__ void __launch_bounds__(BT_THREADS) k_addr_band_thread(const AddrArgs 
     extern __shared__ float bts[];
     const int tid = threadIdx.x;
     float* const A1v = bts + tid;                                              // [L]
-    int* const A1i = reinterpret_cast<int*>(bts) + L * W + tid;                // [L]
-    float* const A2v = bts + 2 * L * W + tid;                                  // [L]
-    int* const A2i = reinterpret_cast<int*>(bts) + 3 * L * W + tid;            // [L]
-    float* const hv = bts + 4 * L * W + tid;                                   // [KM]
-    int* const hp = reinterpret_cast<int*>(bts) + (4 * L + KM) * W + tid;      // [KM]
-    float* const ov = bts + (4 * L + 2 * KM) * W + tid;                        // [L] candidates
-    int* const os = reinterpret_cast<int*>(bts) + (5 * L + 2 * KM) * W + tid;  // [L]
-    float* const bh = bts + (6 * L + 2 * KM) * W + tid;                        // [BT_BAND] band: h
-    float* const bl = bts + (6 * L + 2 * KM + BT_BAND) * W + tid;              //                 l
-    float* const bb = bts + (6 * L + 2 * KM + 2 * BT_BAND) * W + tid;          //                 bound
-    int* const bc = reinterpret_cast<int*>(bts) + (6 * L + 2 * KM + 3 * BT_BAND) * W + tid;   // chosen
+    float* const A2v = bts + L * W + tid;                                      // [L]
+    float* const hv = bts + 2 * L * W + tid;                                   // [KM]
+    float* const ov = bts + (2 * L + KM) * W + tid;                            // [L] candidates
+    int* const os = reinterpret_cast<int*>(bts) + (3 * L + KM) * W + tid;      // [L]
+    float* const bh = bts + (4 * L + KM) * W + tid;                            // [BT_BAND] band: h
+    float* const bl = bts + (4 * L + KM + BT_BAND) * W + tid;                  //                 l
+    float* const bb = bts + (4 * L + KM + 2 * BT_BAND) * W + tid;              //                 bound
+    int* const bc = reinterpret_cast<int*>(bts) + (4 * L + KM + 3 * BT_BAND) * W + tid;   // chosen
+    unsigned short* const h16 = reinterpret_cast<unsigned short*>(bts + (4 * L + KM + 4 * BT_BAND) * W);
+    unsigned short* const A1i = h16 + tid;                                     // [L]
+    unsigned short* const A2i = h16 + L * W + tid;                             // [L]
+    unsigned short* const hp = h16 + 2 * L * W + tid;                          // [KM] row | col << 8
 
     const uint32_t BT = static_cast<uint32_t>(a.B) * static_cast<uint32_t>(a.T);
     const uint32_t nq = static_cast<uint32_t>(*reinterpret_cast<volatile int*>(a.queue));
@@ -1548,7 +1551,7 @@ __global__ void __launch_bounds__(BT_THREADS) k_addr_band_thread(const AddrArgs 
         for (int hf = 0; hf < 2; ++hf) {
             const int64_t base = part_at(static_cast<int>(z), 1, hf, BT, u, L, 0);
             float* Av = hf ? A2v : A1v;
-            int* Ai = hf ? A2i : A1i;
+            unsigned short* Ai = hf ? A2i : A1i;
             const float4* pv = reinterpret_cast<const float4*>(a.part_v + base);   // L % 4 == 0, 16-byte aligned
             const int4* pi = reinterpret_cast<const int4*>(a.part_i + base);
 #pragma unroll
@@ -1556,7 +1559,8 @@ __global__ void __launch_bounds__(BT_THREADS) k_addr_band_thread(const AddrArgs 
                 const float4 v4 = __ldg(pv + q4);
                 const int4 i4 = __ldg(pi + q4);
                 Av[(4 * q4) * W] = v4.x; Av[(4 * q4 + 1) * W] = v4.y; Av[(4 * q4 + 2) * W] = v4.z; Av[(4 * q4 + 3) * W] = v4.w;
-                Ai[(4 * q4) * W] = i4.x; Ai[(4 * q4 + 1) * W] = i4.y; Ai[(4 * q4 + 2) * W] = i4.z; Ai[(4 * q4 + 3) * W] = i4.w;
+                Ai[(4 * q4) * W] = static_cast<unsigned short>(i4.x); Ai[(4 * q4 + 1) * W] = static_cast<unsigned short>(i4.y);
+                Ai[(4 * q4 + 2) * W] = static_cast<unsigned short>(i4.z); Ai[(4 * q4 + 3) * W] = static_cast<unsigned short>(i4.w);
             }
             const float vk = Av[(k - 1) * W], vk1 = Av[k * W];
             if (!(S <= k || __fsub_rd(vk, vk1) > e2)) {
@@ -1596,7 +1600,7 @@ __global__ void __launch_bounds__(BT_THREADS) k_addr_band_thread(const AddrArgs 
                     if (bc[e * W]) {
                         const float v = Av[(cin + e) * W];
                         const int ix = Ai[(cin + e) * W];
-                        Av[q2 * W] = v; Ai[q2 * W] = ix;       // q2 <= cin + e: in-place compaction
+                        Av[q2 * W] = v; Ai[q2 * W] = static_cast<unsigned short>(ix);   // q2 <= cin + e: in place
                         ++q2;
                     }
                 }
@@ -1607,7 +1611,7 @@ __global__ void __launch_bounds__(BT_THREADS) k_addr_band_thread(const AddrArgs 
             const float e2c = __fadd_ru(__fmul_ru(2.f, e2), __fmul_ru(0x1p-21f, __fadd_ru(amax[0], amax[1])));
             // outer-sum candidates by a max-heap of the row heads (k+4 of them, 64 if the band needs)
             const float a20 = A2v[0];
-            for (int i = 0; i < k; ++i) { hv[i * W] = A1v[i * W] + a20; hp[i * W] = i; }
+            for (int i = 0; i < k; ++i) { hv[i * W] = A1v[i * W] + a20; hp[i * W] = static_cast<unsigned short>(i); }
             const int kk2 = k * k;
             int npop = 0;
             auto pops = [&](int upto) {
@@ -1633,7 +1637,7 @@ __global__ void __launch_bounds__(BT_THREADS) k_addr_band_thread(const AddrArgs 
                         else stop = true;
                     }
                     hv[pos * W] = nv;
-                    hp[pos * W] = np;
+                    hp[pos * W] = static_cast<unsigned short>(np);
                 }
             };
             const int len0 = kk2 < L ? kk2 : L;
@@ -1767,7 +1771,7 @@ static cudaError_t launch_finalize(const AddrArgs& a, cudaStream_t stream) {
             // the problem is small (decode): there the queue is short and each item's serial
             // rescoring, not the item count, sets the pass's length
             if (a.ncc == 1 && 2 * a.H * BT >= 32768) {
-                const size_t smb = static_cast<size_t>(bt_words(L)) * BT_THREADS * sizeof(float);
+                const size_t smb = static_cast<size_t>(bt_bytes(L)) * BT_THREADS;
                 e = cudaFuncSetAttribute(k_addr_band_thread<D, L>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          static_cast<int>(smb));
                 if (e != cudaSuccess) return e;
