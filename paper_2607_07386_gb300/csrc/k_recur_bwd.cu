@@ -1,7 +1,7 @@
 // Backward of the sparse gated delta recurrence with in-place undo (App. A.3,
 // "Memory-Efficient Backward").
 //
-// The forward (k_recur with an undo log) updates the memory in place and records, for every
+// The forward (the recurrence kernels with an undo log) updates the memory in place and records, for every
 // token t and write slot n, the row M_{t-1}[I^w_t[n]] its write overwrote.  The backward walks
 // the tokens in reverse with the memory at M_t and an fp32 adjoint G = dL/dM_t of the rows
 // touched so far (dense [N, d_v] per chain, zero elsewhere).  For L = sum_t <dy_t, y_t>:
@@ -20,8 +20,9 @@
 // s = max|row| / top (448 for e4m3, 7 for int4) and codes round(row / s), all in float32 with
 // correctly rounded operations; the backward then takes the logged row as the stored value of
 // q * s (rounded to the storage type), for the chain rule and for the undo alike.
-// Layout of the work: see k_recur_bwd below (one CTA per chain, one warp per 32-element slice
-// of d_v).  Plain loads and stores, no waits.
+//
+// Layout of the work: one CTA per chain, one warp per 32-element slice of d_v (see k_recur_bwd
+// below).  Plain loads and stores, one block barrier per token, no waits on other CTAs.
 #include "sdm_internal.h"
 
 #include <cuda_fp8.h>
